@@ -1,0 +1,444 @@
+"""Benchmark of the pvMVMD hot path on GB300.
+
+A step is one pass of the whole online path over one batch of synthetic
+inputs (the 4096 x 4096 single-projection workload, batch 1):
+    pvmvmd_encode        (100 vectors)
+    pvmvmd_server_mvm    100 times at batch 1 (one GEMV per vector)
+    pvmvmd_decode_verify (100 vectors)
+Preprocessing (P^T and Q) happens once, before timing.  The 100 GEMVs rotate
+over 64 copies of the weights (1 GiB in all), so every timed GEMV streams its
+matrix from HBM rather than from the 126 MB L2.
+
+Prints one JSON line (rank 0).  `--impl reference` times the CPU oracle on the
+same workload instead (a bounded sample of vectors per step).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "field MAC/s and achieved HBM GB/s (batch-1) / int8 tensor-pipe % (batched)"
+UNIT = "field MAC/s"
+M = K = 4096
+VECTORS = 100
+REPLICAS = 64
+SEED_W, SEED_X = 2, 3
+
+
+# --------------------------------------------------------------------------- distributed helpers
+
+def dist_env():
+    return int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)), \
+        int(os.environ.get("LOCAL_RANK", 0))
+
+
+def max_over_ranks(value: float, device=None) -> float:
+    """Max of a float over all ranks (identity without torch.distributed)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()):
+        return value
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(device=None):
+    import torch.distributed as dist
+    if dist.is_available() and dist.is_initialized():
+        if device is not None and dist.get_backend() == "nccl":
+            dist.barrier(device_ids=[device.index])
+        else:
+            dist.barrier()
+
+
+# --------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """Samples nvidia-smi SM clocks and throttle reasons while running."""
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except (OSError, ValueError):
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 7:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                smax.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[3:7]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# --------------------------------------------------------------------------- roofline inputs
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except OSError:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}, "fallback"
+
+
+def gemv_traffic_per_launch():
+    """DRAM bytes per GEMV launch from the committed ncu summary, or None when
+    the kernel source changed since the counters were taken."""
+    path = os.path.join(ROOT, "profiles", "gemv_4096x4096_traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+    except OSError:
+        return None
+    src = os.path.join(ROOT, "paper_2609_10264_gb300", "csrc", "gemv.cu")
+    sha = hashlib.sha256(open(src, "rb").read()).hexdigest()
+    if rec.get("gemv_cu_sha256") != sha:
+        return None
+    return rec.get("dram_bytes_per_launch")
+
+
+# --------------------------------------------------------------------------- CPU oracle (baseline)
+
+class OracleWorkload:
+    """The oracle, as it stands, on this workload (preprocessing done once)."""
+
+    def __init__(self):
+        import oracle
+        from paper_2609_10264_gb300 import workloads as wl
+        self.o = oracle
+        self.W = wl.weights_gaussian(M, K, SEED_W)
+        self.x = oracle.lift(wl.int8_vectors(VECTORS, K, SEED_X))
+        self.pp = oracle.PublicParams(self.W, oracle.key_from_seed(20))
+
+    def client(self, b: int):
+        """Encrypt, server MVM, verify and decrypt of vector b (full vector)."""
+        o, pp = self.o, self.pp
+        xh, s, v = pp.encrypt(self.x[b], o.key_from_seed(21), b)
+        yh = o.server_mvm(self.W, xh)
+        assert pp.verify(xh, yh, o.key_from_seed(22))
+        pp.decrypt(s, v, yh)
+        return xh
+
+    def full_vectors(self, n: int):
+        """Time n full vectors.  Returns (field MACs, seconds)."""
+        t0 = time.perf_counter()
+        for b in range(n):
+            self.client(b % VECTORS)
+        return n * M * K, time.perf_counter() - t0
+
+
+def run_reference(args):
+    """Each step: the server MVM of one vector restricted to R rows, plus that
+    vector's client work (encrypt, verify, decrypt) once every 4096/R steps,
+    so that server and client work keep the proportions of a full vector."""
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    ow = OracleWorkload()
+    o = ow.o
+    xh0 = ow.client(0)
+    t0 = time.perf_counter()
+    o.server_mvm_rows(ow.W, xh0, np.arange(256))
+    t_row = (time.perf_counter() - t0) / 256
+    budget_s = float(os.environ.get("PVMVMD_REF_BUDGET_S", "90"))
+    R = int(max(8, min(M, budget_s / ((args.steps + args.warmup) * t_row))))
+    every = -(-M // R)
+    rng = np.random.default_rng(0)
+
+    def one_step(s):
+        b = s % VECTORS
+        t = time.perf_counter()
+        if s % every == 0:
+            xh = ow.client(b)            # includes the full-vector server MVM: count it
+            macs = M * K
+        else:
+            rows = rng.choice(M, size=R, replace=False)
+            o.server_mvm_rows(ow.W, xh0, rows)
+            macs = R * K
+        return macs, time.perf_counter() - t
+
+    for w in range(args.warmup):
+        one_step(w + 1)
+    total_macs, total_s = 0, 0.0
+    for s in range(args.steps):
+        mac, dt = one_step(s)
+        total_macs += mac
+        total_s += dt
+    value = total_macs / total_s
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total_s / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u32 (F_q, exact)",
+        "data": "synthetic", "config": workload_config(),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": f"per step: server MVM of one vector on {R} sampled rows; every "
+                                   f"{every} steps one full vector (encrypt, MVM, verify, decrypt); "
+                                   "single-threaded C oracle"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def workload_config():
+    return {"workload": "pvMVMD batch-1 round trip: W 4096x4096 int8 (Gaussian sigma 32, clipped), "
+                        "100 int8 vectors per step: encode -> 100 batch-1 GEMVs -> decode+verify",
+            "m": M, "K": K, "vectors_per_step": VECTORS, "w_replicas": REPLICAS,
+            "params": "lambda 128, kappa 40, rate 8, delta 1/2, t_x 157, t_y 31, ell 2",
+            "l2": "inputs larger than L2: 64 weight copies (1 GiB) rotate over the GEMVs; "
+                  "P^T and Q are 0.5 GiB each",
+            "parallelism": "replicas (one independent workload per GPU)"}
+
+
+# --------------------------------------------------------------------------- our arm
+
+def run_ours(args):
+    import torch
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    import paper_2609_10264_gb300 as pv
+    from paper_2609_10264_gb300 import workloads as wl
+
+    W = wl.weights_gaussian(M, K, SEED_W)
+    x = wl.int8_vectors(VECTORS, K, SEED_X)
+    X = np.mod(x, pv.PVMVMD_Q).astype(np.uint32)
+    Wd = torch.from_numpy(W).to(device)
+    Wrep = Wd.repeat(REPLICAS, 1).contiguous()           # 64 distinct copies, 1 GiB
+    Xd = torch.from_numpy(X.view(np.int32)).to(device)
+    params = pv.pvmvmd_params()
+    params.scratch_batch = VECTORS                        # one encode chunk per step
+    ctx = pv.pvmvmd_preprocess(Wd, key=20, params=params)
+    stream = torch.cuda.Stream(device)
+    Xh = torch.empty_like(Xd)
+    st = torch.empty((VECTORS, 2 * ctx.t_x), dtype=torch.int32, device=device)
+    Yh = torch.empty((VECTORS, M), dtype=torch.int32, device=device)
+    Y = torch.empty_like(Yh)
+    acc = torch.empty(VECTORS, dtype=torch.int32, device=device)
+    Wv = [Wrep[(b % REPLICAS) * M:(b % REPLICAS + 1) * M] for b in range(VECTORS)]
+
+    def encode():
+        pv.pvmvmd_encode(ctx, Xd, 21 + rank, Xhat=Xh, st=st, stream=stream)
+
+    def server():
+        for b in range(VECTORS):
+            pv.pvmvmd_server_mvm(Wv[b], Xh[b], Yhat=Yh[b], stream=stream)
+
+    def decode():
+        pv.pvmvmd_decode_verify(ctx, st, Xh, Yh, 22 + rank, Y=Y, accept=acc, stream=stream)
+
+    # eager run once (sets kernel attributes, checks the result), then capture
+    with torch.cuda.stream(stream):
+        encode(); server(); decode()
+    stream.synchronize()
+    pv.pvmvmd_device_status(stream)
+    assert int(acc.sum()) == VECTORS, "honest outputs must be accepted"
+    Yc = pv.as_u32(Y)
+    rows = [0, 1, 2047, 4095]
+    exact = x.astype(np.float64) @ W[rows].astype(np.float64).T
+    assert np.array_equal(np.where(Yc[:, rows] > (pv.PVMVMD_Q - 1) // 2,
+                                   Yc[:, rows].astype(np.int64) - pv.PVMVMD_Q,
+                                   Yc[:, rows].astype(np.int64)), exact.astype(np.int64))
+
+    graphs = []
+    for fn in (encode, server, decode):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            fn()
+        graphs.append(g)
+    g_enc, g_srv, g_dec = graphs
+    launches_per_step = 3 + VECTORS + 5
+
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+
+    def step(record=None):
+        if record is not None:
+            record[0].record(stream)
+        g_enc.replay()
+        if record is not None:
+            record[1].record(stream)
+        g_srv.replay()
+        if record is not None:
+            record[2].record(stream)
+        g_dec.replay()
+        if record is not None:
+            record[3].record(stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            step()
+    stream.synchronize()
+
+    # ---- timed region: whole steps, with per-phase events on the launching stream
+    phase_events = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    clocks = ClockSampler(device.index)
+    barrier(device)
+    torch.cuda.synchronize(device)
+    clocks.start()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_stop = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        t_start.record(stream)
+        for s in range(args.steps):
+            step(phase_events[s])
+        t_stop.record(stream)
+    stream.synchronize()
+    torch.cuda.synchronize(device)
+    clk = clocks.stop()
+    barrier(device)
+    ms_local = t_start.elapsed_time(t_stop)
+    ms = max_over_ranks(ms_local, device)
+    enc_ms = sum(e[0].elapsed_time(e[1]) for e in phase_events) / args.steps
+    srv_ms = sum(e[1].elapsed_time(e[2]) for e in phase_events) / args.steps
+    dec_ms = sum(e[2].elapsed_time(e[3]) for e in phase_events) / args.steps
+
+    macs_per_step = VECTORS * M * K
+    value = world * macs_per_step * args.steps / (ms / 1e3)
+    gemv_s = srv_ms / 1e3 / VECTORS
+    gemv_bytes = M * K + 4 * K + 4 * M                  # W int8 + x_hat + y_hat per launch
+    peaks, peak_kind = measured_peaks()
+    achieved = gemv_bytes / gemv_s / 1e9
+    traffic = gemv_traffic_per_launch()
+
+    # ---- end to end through the public API with pinned host buffers
+    Xhost = torch.from_numpy(X.view(np.int32)).pin_memory()
+    Yhost = torch.empty((VECTORS, M), dtype=torch.int32).pin_memory()
+    Ahost = torch.empty(VECTORS, dtype=torch.int32).pin_memory()
+    Xin = torch.empty_like(Xd)
+
+    def e2e_step():
+        Xin.copy_(Xhost, non_blocking=True)
+        pv.pvmvmd_encode(ctx, Xin, 31 + rank, Xhat=Xh, st=st, stream=stream)
+        server()
+        pv.pvmvmd_decode_verify(ctx, st, Xh, Yh, 32 + rank, Y=Y, accept=acc, stream=stream)
+        Yhost.copy_(Y, non_blocking=True)
+        Ahost.copy_(acc, non_blocking=True)
+
+    with torch.cuda.stream(stream):
+        e2e_step()
+    stream.synchronize()
+    ge = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(ge, stream=stream):
+        e2e_step()
+    e2e_steps = max(1, args.steps // 2)
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            ge.replay()
+    stream.synchronize()
+    barrier(device)
+    t0 = time.perf_counter()
+    with torch.cuda.stream(stream):
+        for _ in range(e2e_steps):
+            ge.replay()
+    stream.synchronize()
+    e2e_s = max_over_ranks(time.perf_counter() - t0, device)
+    assert int(Ahost.sum()) == VECTORS
+    e2e_value = world * macs_per_step * e2e_steps / e2e_s
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        n = args.cpu_vectors
+        macs, dt = OracleWorkload().full_vectors(n)
+        cpu = {"value": macs / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
+               "sample": f"{n} of the {VECTORS} vectors (encrypt, server MVM, verify, decrypt), "
+                         "single-threaded C oracle on the host; preprocessing untimed"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "u32 (F_q exact; int8 weights, dp4a digits)",
+            "data": "synthetic", "config": workload_config(),
+            "hbm_gbs_gemv": achieved,
+            "phases_ms": {"encode": enc_ms, "server_100_gemv": srv_ms, "decode_verify": dec_ms},
+            "roofline": {"bound": "hbm", "kernel": "k_gemv (batch-1 field GEMV)", "achieved": achieved,
+                         "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],
+                         "peak_kind": f"{peak_kind} hbm_gbs", "traffic": traffic,
+                         "algorithmic_bytes_per_launch": gemv_bytes},
+            "cpu_baseline": cpu,
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(Xhost.numel() * 4),
+                    "d2h_bytes_per_step": int(Yhost.numel() * 4 + Ahost.numel() * 4),
+                    "how": "CUDA graph of the public calls with pinned host copies inside, replayed"},
+            "gpu_launches": launches_per_step * args.steps,
+            "clocks": clk,
+        }
+        print(json.dumps(line), flush=True)
+    ctx.destroy()
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-vectors", type=int, default=150)
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        ap.error("--warmup must be at least 3")
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

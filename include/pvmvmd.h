@@ -1,0 +1,172 @@
+/*
+ * pvmvmd.h — C ABI of the GB300 (sm_103a) pvMVMD library.
+ *
+ * The calls follow Protocol 3 (Pi_pvMVMD) of the Maverick paper
+ * (arXiv 2609.10264, Sec. 6.1) and Def. 4.2's algorithm split:
+ *   pvmvmd_preprocess      Preprocess(M) -> pp = (G_x, G_y, P, Q, t_x, t_y, ell)
+ *   pvmvmd_encode          Encrypt(pp, x) -> (x_hat, st)
+ *   pvmvmd_server_mvm      the server's y_hat = M x_hat over F_q
+ *   pvmvmd_decode_verify   Verify(pp, x_hat, y_hat) and Decrypt(pp, st, y_hat)
+ * The codes are the RAA codes of App. B, G = R Pi1 V1 A Pi2 V2 A, with the
+ * parameters of Sec. 7.1 by default.
+ *
+ * Conventions shared by every call
+ *  - Field: BabyBear, q = 15 * 2^27 + 1 = 2013265921 (Sec. 7.1).  Every field
+ *    element crossing the ABI is a uint32 in canonical form [0, q).  Inputs
+ *    outside [0, q) give unspecified (but memory-safe) results.
+ *  - The public matrix M is int8, row-major m x K, embedded in F_q by
+ *    w -> w mod q (Sec. 7.2.1 embeds signed quantised weights the same way).
+ *  - A batch of B vectors of length L is stored vector after vector
+ *    ("B x L row-major"): vector b occupies elements [b*L, (b+1)*L).
+ *  - Pointers named *_dev are CUDA device pointers on the current device;
+ *    the caller owns them.  The library owns only what a context holds.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *    stream).  Every call only enqueues work on that stream and returns;
+ *    results are valid once the stream has been synchronised.  Calls that use
+ *    one context must be ordered on one stream: a context's internal scratch
+ *    is shared by its calls.
+ *  - Return value: PVMVMD_OK (0) or a negative PVMVMD_E_* status.  Nothing
+ *    throws across the ABI.  A device-side bounded wait that expires is
+ *    reported later by pvmvmd_device_status.
+ *  - Randomness: a pvmvmd_key is a 256-bit ChaCha20 key (RFC 8439); each
+ *    sampled object reads its own keystream, selected by the nonce
+ *    (domain tag, index).  Encode keys must never be reused: masks derived
+ *    from a reused key repeat, which voids privacy.
+ */
+#ifndef PVMVMD_H
+#define PVMVMD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define PVMVMD_Q 2013265921u
+
+/* Largest K for which the server product's per-digit int32 sums cannot
+ * overflow for any int8 weight: 128 * 128 * K < 2^31. */
+#define PVMVMD_MAX_K 131071
+
+/* Largest sparsity accepted for t_x and t_y. */
+#define PVMVMD_MAX_T 4096
+
+enum {
+    PVMVMD_OK = 0,
+    PVMVMD_E_ARG = -1,            /* null pointer or invalid argument          */
+    PVMVMD_E_SHAPE = -2,          /* m, K or B outside the supported range      */
+    PVMVMD_E_PARAM = -3,          /* parameters inconsistent (e.g. t > N)       */
+    PVMVMD_E_CUDA = -4,           /* a CUDA runtime call or launch failed       */
+    PVMVMD_E_NOMEM = -5,          /* device or host allocation failed           */
+    PVMVMD_E_DEVICE_TIMEOUT = -6, /* a bounded device-side wait expired         */
+    PVMVMD_E_NODEVICE = -7        /* no sm_103 device is current                */
+};
+
+/* 256-bit ChaCha20 key, eight little-endian 32-bit words. */
+typedef struct { uint32_t k[8]; } pvmvmd_key;
+
+/* Protocol parameters.  A zero field selects the paper's value. */
+typedef struct {
+    int lambda;        /* computational security parameter; 0 -> 128 (Sec. 7.1)        */
+    int kappa;         /* statistical security parameter; 0 -> 40 (Sec. 7.1)           */
+    int rate;          /* N / dimension of both RAA codes; 0 -> 8 (rate 1/8, Sec. 7.1) */
+    double delta;      /* target relative distance; 0 -> 0.5 (Sec. 7.1)                */
+    int t_x;           /* mask sparsity; 0 -> Eq. (1), ceil(ln2 (lambda - log2 N_x)/delta) */
+    int t_y;           /* challenge sparsity; 0 -> Thm 5.2 by its proof's two cases
+                          (31 for BabyBear with kappa = 40, delta = 1/2, as Sec. 7.1 uses) */
+    int ell;           /* challenge repetitions; 0 -> Thm 5.2 (2 with Sec. 7.1's values) */
+    int scratch_batch; /* vectors per internal encode chunk; 0 -> 64 (memory knob only) */
+} pvmvmd_params;
+
+typedef struct pvmvmd_ctx pvmvmd_ctx;
+
+/* Read-only view of a context's public parameters pp (Protocol 3).  All
+ * arrays are device memory owned by the context.  Permutations follow App. B:
+ * pi[j] = pi(j), and Pi_{i,j} = 1 iff pi(j) = i. */
+typedef struct {
+    int m, K;                 /* matrix shape                                   */
+    int rate, N_x, N_y;       /* N_x = rate*K (privacy code), N_y = rate*m (verification code) */
+    int t_x, t_y, ell;
+    const uint32_t *gx_pi1, *gx_pi2, *gx_v1, *gx_v2; /* G_x, each length N_x    */
+    const uint32_t *gy_pi1, *gy_pi2, *gy_v1, *gy_v2; /* G_y, each length N_y    */
+    const uint32_t *PT;       /* P^T = (M G_x)^T, row-major N_x x m              */
+    const uint32_t *Q;        /* Q = G_y^T M, row-major N_y x K                  */
+} pvmvmd_ctx_view;
+
+/* Fill every zero field of *in with the paper's default for an m x K matrix
+ * (Eq. 1, Thm 5.2, Sec. 7.1) and write the result to *out.  Host only; needs
+ * no GPU.  Returns PVMVMD_E_PARAM if the resolved t_x > rate*K,
+ * t_y > rate*m, either t exceeds PVMVMD_MAX_T, or a field is negative. */
+int pvmvmd_params_resolve(const pvmvmd_params *in, int m, int K, pvmvmd_params *out);
+
+/* Preprocess(M) (Protocol 3; P and Q as in Sec. 6.3): samples G_x (dimension
+ * K) and G_y (dimension m) from `key`, computes P^T = G_x^T M^T (m encodings of
+ * the rows of M) and Q = G_y^T M (K encodings of its columns) on the device,
+ * and returns a context owning them.  W_dev: int8 m x K row-major; W need
+ * not stay alive afterwards.  params may be NULL (all defaults).
+ * 1 <= m, 1 <= K <= PVMVMD_MAX_K.  Allocates about 8*rate*m*K bytes of device
+ * memory plus code tables and scratch; the call synchronises `stream` before
+ * returning.  On error *out is NULL. */
+int pvmvmd_preprocess(const int8_t *W_dev, int m, int K, const pvmvmd_params *params,
+                      const pvmvmd_key *key, void *stream, pvmvmd_ctx **out);
+
+/* Bytes of the private state st for B vectors: B * 2 * t_x uint32 (for
+ * vector b, its mask's support in ascending order, then the matching values). */
+int pvmvmd_state_size(const pvmvmd_ctx *ctx, int B, size_t *bytes);
+
+/* Encrypt (Protocol 3): for each of the B vectors x_b (X_dev, B x K), sample
+ * e_x <- E_{t_x}^{N_x} from `key` (vector b reads nonce (9, 2b) for its support
+ * and (9, 2b+1) for its values), write x_hat_b = x_b + G_x e_x to Xhat_dev
+ * (B x K) and st_b = e_x to st_dev (pvmvmd_state_size bytes).  B >= 1.
+ * X_dev and Xhat_dev may alias. */
+int pvmvmd_encode(pvmvmd_ctx *ctx, const uint32_t *X_dev, int B, const pvmvmd_key *key,
+                  uint32_t *Xhat_dev, void *st_dev, void *stream);
+
+/* The server's product Y_hat = M X_hat over F_q (Sec. 6.1: the server's whole
+ * online work).  W_dev int8 m x K row-major, Xhat_dev B x K, Yhat_dev B x m.
+ * Needs no context and no secret.  B == 1 runs the bandwidth-bound GEMV;
+ * B > 1 runs the byte-limb tensor-core product.  1 <= K <= PVMVMD_MAX_K. */
+int pvmvmd_server_mvm(const int8_t *W_dev, int m, int K, const uint32_t *Xhat_dev, int B,
+                      uint32_t *Yhat_dev, void *stream);
+
+/* Verify and Decrypt (Protocol 3).  Verify: ell challenges e_q <- E_{t_y}^{N_y}
+ * are drawn from challenge_key (repetition q reads nonce (10, 2q) and
+ * (10, 2q+1)) and shared by all B vectors of the call, as Sec. 5.4 allows;
+ * vector b is accepted iff (e_q^T Q) x_hat_b == e_q^T (G_y^T y_hat_b) for every q.
+ * The right side is evaluated as (G_y e_q)^T y_hat_b, the same number by
+ * transposition.  Decrypt: Y_b = y_hat_b - P e_x,b.  st_dev as written by
+ * pvmvmd_encode; Xhat_dev B x K; Yhat_dev B x m; Y_dev B x m (may alias
+ * Yhat_dev); accept_dev B int32, each 1 (accept) or 0 (reject).  A rejection
+ * is data, not an error.  Y is written for rejected vectors too. */
+int pvmvmd_decode_verify(pvmvmd_ctx *ctx, const void *st_dev, const uint32_t *Xhat_dev,
+                         const uint32_t *Yhat_dev, int B, const pvmvmd_key *challenge_key,
+                         uint32_t *Y_dev, int32_t *accept_dev, void *stream);
+
+/* Synchronise `stream`, then read and clear the library's device error word:
+ * PVMVMD_E_DEVICE_TIMEOUT if any kernel gave up a bounded wait since the last
+ * call, else PVMVMD_OK (or PVMVMD_E_CUDA if synchronisation failed). */
+int pvmvmd_device_status(void *stream);
+
+/* Fill *view with the context's public parameters. */
+int pvmvmd_ctx_info(const pvmvmd_ctx *ctx, pvmvmd_ctx_view *view);
+
+/* Release every device allocation of the context.  NULL is ignored. */
+void pvmvmd_destroy(pvmvmd_ctx *ctx);
+
+/* Static, human-readable text for a status code. */
+const char *pvmvmd_strerror(int status);
+
+/* Host-side sampling of one RAA generator exactly as pvmvmd_preprocess does
+ * it (App. B): which = 0 for G_x, 1 for G_y; N = rate * dimension.  pi1/pi2
+ * are Fisher-Yates permutations of [N] read from nonces (1+4*which, 0) and
+ * (2+4*which, 0); v1/v2 are N uniform draws from F* read from nonces
+ * (3+4*which, 0) and (4+4*which, 0).  Host arrays of length N.  Needs no GPU. */
+int pvmvmd_code_sample_host(const pvmvmd_key *key, int which, uint32_t N, uint32_t *pi1,
+                            uint32_t *pi2, uint32_t *v1, uint32_t *v2);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PVMVMD_H */

@@ -29,12 +29,12 @@ import threading
 
 import numpy as np
 
-Q = 2013265921  # BabyBear, q = 15 * 2^27 + 1 (Sec. 6.1)
-LAMBDA = 128    # computational security parameter (Sec. 6.1)
-KAPPA = 40      # statistical security parameter (Sec. 6.1)
-RATE = 8        # N / dim for both codes: rate 1/8 (Sec. 6.1)
-DELTA = 0.5     # target relative distance (Sec. 6.1)
-T_Y_PAPER = 31  # verification sparsity used in Sec. 6.1
+Q = 2013265921  # BabyBear, q = 15 * 2^27 + 1 (Sec. 7.1)
+LAMBDA = 128    # computational security parameter (Sec. 7.1)
+KAPPA = 40      # statistical security parameter (Sec. 7.1)
+RATE = 8        # N / dim for both codes: rate 1/8 (Sec. 7.1)
+DELTA = 0.5     # target relative distance (Sec. 7.1)
+T_Y_PAPER = 31  # verification sparsity used in Sec. 7.1
 TAG_MASK = 9
 TAG_CHALLENGE = 10
 

@@ -8,7 +8,7 @@
  * field arithmetic and every protocol step are written out here a second time,
  * in the most direct form the paper's definitions allow.
  *
- * Field: BabyBear, q = 15 * 2^27 + 1 (Sec. 6.1).  Every field element is a
+ * Field: BabyBear, q = 15 * 2^27 + 1 (Sec. 7.1).  Every field element is a
  * uint32 in canonical form [0, q).  Arithmetic is done in uint64 with a
  * reduction after every single operation (no lazy reduction, no tricks).
  *
@@ -25,12 +25,12 @@
 #define ORC_Q 2013265921ULL
 
 /* ---------------------------------------------------------------------- */
-/* Field arithmetic over F_q (Sec. 6.1): one reduction per operation.      */
+/* Field arithmetic over F_q (Sec. 7.1): one reduction per operation.      */
 /* ---------------------------------------------------------------------- */
 static uint64_t f_add(uint64_t a, uint64_t b) { return (a + b) % ORC_Q; }
 static uint64_t f_sub(uint64_t a, uint64_t b) { return (a + ORC_Q - b) % ORC_Q; }
 static uint64_t f_mul(uint64_t a, uint64_t b) { return (a * b) % ORC_Q; }
-/* Embed a signed integer into F_q (the int8 weights of Sec. 6.2.1). */
+/* Embed a signed integer into F_q (the int8 weights of Sec. 7.2.1). */
 static uint64_t f_lift(int64_t v) {
     int64_t r = v % (int64_t)ORC_Q;
     if (r < 0) r += (int64_t)ORC_Q;
@@ -272,7 +272,7 @@ void orc_raa_syndrome(uint32_t n, uint32_t r, const uint32_t *pi1, const uint32_
 }
 
 /* ---------------------------------------------------------------------- */
-/* Parameters (Sec. 5.2 Eq. 1, Thm 5.2 and its proof, Sec. 6.1).           */
+/* Parameters (Eq. 1 of Sec. 6.2, Thm 5.2 and its proof, Sec. 7.1).           */
 /* ---------------------------------------------------------------------- */
 
 /* Mask sparsity, Eq. (1): smallest integer t with t >= ln2 (lambda - log2 N)/delta. */
@@ -300,7 +300,7 @@ void orc_verify_params(int kappa, double delta, int *t_case, int *t_thm, int *el
 }
 
 /* ---------------------------------------------------------------------- */
-/* Server MVM, y_hat = M x_hat over F_q (Sec. 5.1; server's only online work).*/
+/* Server MVM, y_hat = M x_hat over F_q (Sec. 6.1; server's only online work).*/
 /* Textbook: lift each weight, one multiply and one add per MAC, each reduced.*/
 /* ---------------------------------------------------------------------- */
 void orc_server_mvm_rows(const int8_t *W, uint32_t m, uint32_t K, const uint32_t *xhat,
@@ -330,7 +330,7 @@ void orc_server_mvm(const int8_t *W, uint32_t m, uint32_t K, const uint32_t *xha
 /* ---------------------------------------------------------------------- */
 
 /* Preprocess, P = M G_x: P^T = G_x^T M^T is m encodings of the rows of M
- * (Sec. 5.3).  Stored as P^T, row-major N_x x m. */
+ * (Sec. 6.3).  Stored as P^T, row-major N_x x m. */
 void orc_preprocess_PT(const int8_t *W, uint32_t m, uint32_t n, uint32_t r,
                        const uint32_t *pi1, const uint32_t *pi2, const uint32_t *v1,
                        const uint32_t *v2, uint32_t *PT) {
@@ -346,7 +346,7 @@ void orc_preprocess_PT(const int8_t *W, uint32_t m, uint32_t n, uint32_t r,
     free(enc);
 }
 
-/* Preprocess, Q = G_y^T M: n encodings of the columns of M (Sec. 5.3).
+/* Preprocess, Q = G_y^T M: n encodings of the columns of M (Sec. 6.3).
  * Stored row-major N_y x n. */
 void orc_preprocess_Q(const int8_t *W, uint32_t m, uint32_t n, uint32_t r,
                       const uint32_t *pi1, const uint32_t *pi2, const uint32_t *v1,

@@ -1,0 +1,323 @@
+"""Python binding of libpvmvmd (include/pvmvmd.h): argument marshalling only.
+
+Every function has the name of the C entry point it calls.  Device buffers are
+torch CUDA tensors (uint32 field data may be held as torch.int32 or
+torch.uint32; both are passed as raw 32-bit words).  Streams default to
+torch's current stream.  Errors raise PvmvmdError with the library's message.
+
+The library must be built (``python -m paper_2609_10264_gb300.build`` or
+``__graft_entry__.build()``); importing this package without it fails loudly.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libpvmvmd.so")
+
+PVMVMD_Q = 2013265921
+PVMVMD_MAX_K = 131071
+PVMVMD_MAX_T = 4096
+PVMVMD_OK = 0
+PVMVMD_E_ARG = -1
+PVMVMD_E_SHAPE = -2
+PVMVMD_E_PARAM = -3
+PVMVMD_E_CUDA = -4
+PVMVMD_E_NOMEM = -5
+PVMVMD_E_DEVICE_TIMEOUT = -6
+PVMVMD_E_NODEVICE = -7
+
+
+class PvmvmdError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {pvmvmd_strerror(status)} (status {status})")
+
+
+class pvmvmd_key(ctypes.Structure):
+    _fields_ = [("k", ctypes.c_uint32 * 8)]
+
+
+class pvmvmd_params(ctypes.Structure):
+    _fields_ = [("lambda_", ctypes.c_int), ("kappa", ctypes.c_int), ("rate", ctypes.c_int),
+                ("delta", ctypes.c_double), ("t_x", ctypes.c_int), ("t_y", ctypes.c_int),
+                ("ell", ctypes.c_int), ("scratch_batch", ctypes.c_int)]
+
+
+_cu32p = ctypes.POINTER(ctypes.c_uint32)
+
+
+class pvmvmd_ctx_view(ctypes.Structure):
+    _fields_ = [("m", ctypes.c_int), ("K", ctypes.c_int), ("rate", ctypes.c_int),
+                ("N_x", ctypes.c_int), ("N_y", ctypes.c_int), ("t_x", ctypes.c_int),
+                ("t_y", ctypes.c_int), ("ell", ctypes.c_int),
+                ("gx_pi1", ctypes.c_void_p), ("gx_pi2", ctypes.c_void_p), ("gx_v1", ctypes.c_void_p),
+                ("gx_v2", ctypes.c_void_p), ("gy_pi1", ctypes.c_void_p), ("gy_pi2", ctypes.c_void_p),
+                ("gy_v1", ctypes.c_void_p), ("gy_v2", ctypes.c_void_p),
+                ("PT", ctypes.c_void_p), ("Q", ctypes.c_void_p)]
+
+
+# Exported symbols and their ctypes signatures (mirrors include/pvmvmd.h).
+_vp, _i, _sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
+SIGNATURES = {
+    "pvmvmd_params_resolve": (_i, [ctypes.POINTER(pvmvmd_params), _i, _i, ctypes.POINTER(pvmvmd_params)]),
+    "pvmvmd_preprocess": (_i, [_vp, _i, _i, ctypes.POINTER(pvmvmd_params), ctypes.POINTER(pvmvmd_key), _vp,
+                               ctypes.POINTER(_vp)]),
+    "pvmvmd_state_size": (_i, [_vp, _i, ctypes.POINTER(_sz)]),
+    "pvmvmd_encode": (_i, [_vp, _vp, _i, ctypes.POINTER(pvmvmd_key), _vp, _vp, _vp]),
+    "pvmvmd_server_mvm": (_i, [_vp, _i, _i, _vp, _i, _vp, _vp]),
+    "pvmvmd_decode_verify": (_i, [_vp, _vp, _vp, _vp, _i, ctypes.POINTER(pvmvmd_key), _vp, _vp, _vp]),
+    "pvmvmd_device_status": (_i, [_vp]),
+    "pvmvmd_ctx_info": (_i, [_vp, ctypes.POINTER(pvmvmd_ctx_view)]),
+    "pvmvmd_destroy": (None, [_vp]),
+    "pvmvmd_strerror": (ctypes.c_char_p, [_i]),
+    "pvmvmd_code_sample_host": (_i, [ctypes.POINTER(pvmvmd_key), _i, ctypes.c_uint32, _cu32p, _cu32p,
+                                     _cu32p, _cu32p]),
+}
+
+
+def _load():
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(
+            f"{LIB_PATH} is not built: run `python -c 'import __graft_entry__ as g; g.build()'` "
+            "(needs nvcc); this package has no fallback path")
+    lib = ctypes.CDLL(LIB_PATH)
+    for name, (res, args) in SIGNATURES.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    return lib
+
+
+_lib = _load()
+
+
+def _check(status: int, where: str) -> None:
+    if status != PVMVMD_OK:
+        raise PvmvmdError(status, where)
+
+
+def pvmvmd_strerror(status: int) -> str:
+    return _lib.pvmvmd_strerror(int(status)).decode()
+
+
+# --------------------------------------------------------------------------- marshalling
+
+def make_key(seed) -> pvmvmd_key:
+    """A pvmvmd_key from an integer < 2^256 (little-endian 32-bit words), from 32
+    bytes, or from 8 words."""
+    k = pvmvmd_key()
+    if isinstance(seed, pvmvmd_key):
+        return seed
+    if isinstance(seed, (bytes, bytearray)):
+        if len(seed) != 32:
+            raise ValueError("a key is 32 bytes")
+        words = np.frombuffer(bytes(seed), dtype="<u4")
+    elif isinstance(seed, (int, np.integer)):
+        s = int(seed)
+        if s < 0 or s >= 1 << 256:
+            raise ValueError("integer key must be in [0, 2^256)")
+        words = [(s >> (32 * i)) & 0xFFFFFFFF for i in range(8)]
+    else:
+        words = [int(w) for w in seed]
+        if len(words) != 8:
+            raise ValueError("a key is 8 words")
+    for i in range(8):
+        k.k[i] = int(words[i])
+    return k
+
+
+def _stream_ptr(stream):
+    if stream is None:
+        import torch
+        return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, int):
+        return ctypes.c_void_p(stream)
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _dev_ptr(t, name: str, dtypes, numel=None):
+    import torch
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if t.dtype not in dtypes:
+        raise TypeError(f"{name} must have dtype in {dtypes}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if numel is not None and t.numel() != numel:
+        raise ValueError(f"{name} has {t.numel()} elements, expected {numel}")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _u32_types():
+    import torch
+    types = [torch.int32]
+    if hasattr(torch, "uint32"):
+        types.append(torch.uint32)
+    return tuple(types)
+
+
+def _new_u32(shape, like=None):
+    import torch
+    dev = like.device if like is not None else "cuda"
+    return torch.empty(shape, dtype=torch.int32, device=dev)
+
+
+# --------------------------------------------------------------------------- API
+
+def pvmvmd_params_resolve(m: int, K: int, params: pvmvmd_params | None = None) -> pvmvmd_params:
+    out = pvmvmd_params()
+    _check(_lib.pvmvmd_params_resolve(ctypes.byref(params) if params is not None else None, m, K,
+                                      ctypes.byref(out)), "pvmvmd_params_resolve")
+    return out
+
+
+class Ctx:
+    """Owner of a pvmvmd_ctx handle (public parameters pp on the device)."""
+
+    def __init__(self, handle: int, m: int, K: int):
+        self.handle = ctypes.c_void_p(handle)
+        self.m, self.K = m, K
+        v = pvmvmd_ctx_info(self)
+        self.t_x, self.t_y, self.ell = v.t_x, v.t_y, v.ell
+        self.N_x, self.N_y, self.rate = v.N_x, v.N_y, v.rate
+
+    def destroy(self) -> None:
+        if self.handle is not None and self.handle.value:
+            _lib.pvmvmd_destroy(self.handle)
+        self.handle = None
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass
+
+
+def pvmvmd_preprocess(W, key, params: pvmvmd_params | None = None, stream=None) -> Ctx:
+    import torch
+    if W.dim() != 2:
+        raise ValueError("W must be m x K")
+    m, K = W.shape
+    ptr = _dev_ptr(W, "W", (torch.int8,))
+    out = ctypes.c_void_p()
+    k = make_key(key)
+    _check(_lib.pvmvmd_preprocess(ptr, m, K, ctypes.byref(params) if params is not None else None,
+                                  ctypes.byref(k), _stream_ptr(stream), ctypes.byref(out)),
+           "pvmvmd_preprocess")
+    return Ctx(out.value, m, K)
+
+
+def pvmvmd_ctx_info(ctx: Ctx) -> pvmvmd_ctx_view:
+    v = pvmvmd_ctx_view()
+    _check(_lib.pvmvmd_ctx_info(ctx.handle, ctypes.byref(v)), "pvmvmd_ctx_info")
+    return v
+
+
+def pvmvmd_state_size(ctx: Ctx, B: int) -> int:
+    n = ctypes.c_size_t()
+    _check(_lib.pvmvmd_state_size(ctx.handle, B, ctypes.byref(n)), "pvmvmd_state_size")
+    return n.value
+
+
+def _batch(X, L: int, name: str) -> int:
+    if X.dim() == 1:
+        if X.numel() != L:
+            raise ValueError(f"{name} must have {L} entries")
+        return 1
+    if X.dim() != 2 or X.shape[1] != L:
+        raise ValueError(f"{name} must be B x {L}")
+    return X.shape[0]
+
+
+def pvmvmd_encode(ctx: Ctx, X, key, Xhat=None, st=None, stream=None):
+    """Encrypt B vectors: returns (Xhat, st)."""
+    B = _batch(X, ctx.K, "X")
+    xp = _dev_ptr(X, "X", _u32_types())
+    if Xhat is None:
+        Xhat = _new_u32(X.shape, X)
+    if st is None:
+        st = _new_u32((B, 2 * ctx.t_x), X)
+    _check(_lib.pvmvmd_encode(ctx.handle, xp, B, ctypes.byref(make_key(key)),
+                              _dev_ptr(Xhat, "Xhat", _u32_types(), X.numel()),
+                              _dev_ptr(st, "st", _u32_types(), B * 2 * ctx.t_x), _stream_ptr(stream)),
+           "pvmvmd_encode")
+    return Xhat, st
+
+
+def pvmvmd_server_mvm(W, Xhat, Yhat=None, stream=None):
+    """Y_hat = M X_hat over F_q for Xhat of shape (K,) or (B, K)."""
+    import torch
+    m, K = W.shape
+    B = _batch(Xhat, K, "Xhat")
+    if Yhat is None:
+        Yhat = _new_u32((m,) if Xhat.dim() == 1 else (B, m), Xhat)
+    _check(_lib.pvmvmd_server_mvm(_dev_ptr(W, "W", (torch.int8,)), m, K, _dev_ptr(Xhat, "Xhat", _u32_types()),
+                                  B, _dev_ptr(Yhat, "Yhat", _u32_types(), B * m), _stream_ptr(stream)),
+           "pvmvmd_server_mvm")
+    return Yhat
+
+
+def pvmvmd_decode_verify(ctx: Ctx, st, Xhat, Yhat, challenge_key, Y=None, accept=None, stream=None):
+    """Verify and decrypt: returns (Y, accept) with accept an int32 tensor of 0/1."""
+    import torch
+    B = _batch(Xhat, ctx.K, "Xhat")
+    if Y is None:
+        Y = _new_u32(Yhat.shape, Yhat)
+    if accept is None:
+        accept = torch.empty(B, dtype=torch.int32, device=Yhat.device)
+    _check(_lib.pvmvmd_decode_verify(ctx.handle, _dev_ptr(st, "st", _u32_types(), B * 2 * ctx.t_x),
+                                     _dev_ptr(Xhat, "Xhat", _u32_types()),
+                                     _dev_ptr(Yhat, "Yhat", _u32_types(), B * ctx.m), B,
+                                     ctypes.byref(make_key(challenge_key)),
+                                     _dev_ptr(Y, "Y", _u32_types(), B * ctx.m),
+                                     _dev_ptr(accept, "accept", (torch.int32,), B), _stream_ptr(stream)),
+           "pvmvmd_decode_verify")
+    return Y, accept
+
+
+def pvmvmd_device_status(stream=None) -> int:
+    """Synchronise and return the device status (raises on a timeout)."""
+    s = _lib.pvmvmd_device_status(_stream_ptr(stream))
+    _check(s, "pvmvmd_device_status")
+    return s
+
+
+def pvmvmd_destroy(ctx: Ctx) -> None:
+    ctx.destroy()
+
+
+def pvmvmd_code_sample_host(key, which: int, N: int):
+    """Host sampling of one RAA generator: (pi1, pi2, v1, v2) numpy uint32 arrays."""
+    arrs = [np.zeros(N, np.uint32) for _ in range(4)]
+    ptrs = [a.ctypes.data_as(_cu32p) for a in arrs]
+    _check(_lib.pvmvmd_code_sample_host(ctypes.byref(make_key(key)), which, N, *ptrs),
+           "pvmvmd_code_sample_host")
+    return tuple(arrs)
+
+
+def as_u32(t) -> np.ndarray:
+    """Device or host 32-bit tensor -> numpy uint32 (for checks and printing)."""
+    import torch
+    t = t.detach()
+    if t.dtype != torch.int32:
+        t = t.view(torch.int32)
+    return t.cpu().contiguous().numpy().view(np.uint32).reshape(tuple(t.shape))
+
+
+class _CudaArray:
+    def __init__(self, ptr: int, count: int):
+        self.__cuda_array_interface__ = {"shape": (count,), "typestr": "<i4", "data": (int(ptr), True),
+                                         "version": 2, "strides": None}
+
+
+def device_view(ptr, count: int):
+    """A torch.int32 CUDA tensor aliasing `count` 32-bit words at device
+    pointer `ptr` (e.g. a table of pvmvmd_ctx_info); valid while its owner
+    lives."""
+    import torch
+    p = ptr.value if isinstance(ptr, ctypes.c_void_p) else ptr
+    return torch.as_tensor(_CudaArray(p, count), device="cuda")

@@ -1,0 +1,493 @@
+// C ABI of the pvMVMD library (include/pvmvmd.h): parameter resolution, the
+// host-side sampling of the public RAA codes, context management, and the
+// ordering of the device kernels for each protocol call.
+#include <algorithm>
+#include <cmath>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <vector>
+
+#include "common.cuh"
+#include "launch.h"
+
+namespace pv {
+
+// The library's device error word (kErr* bits).
+__device__ uint32_t g_error_word = 0;
+
+namespace {
+
+// Domain tags of the ChaCha20 nonces (tag, index): the two codes, the masks
+// and the challenges each read their own keystream.
+constexpr uint32_t kTagCodeX = 1;       // G_x: pi1 = 1, pi2 = 2, v1 = 3, v2 = 4
+constexpr uint32_t kTagCodeY = 5;       // G_y: pi1 = 5, pi2 = 6, v1 = 7, v2 = 8
+constexpr uint32_t kTagMask = 9;
+constexpr uint32_t kTagChallenge = 10;
+
+// --------------------------------------------------------------------------
+// Host ChaCha20 keystream (RFC 8439 Sec. 2.3) read as 32-bit words.
+// --------------------------------------------------------------------------
+class KeyStream {
+  public:
+    KeyStream(const pvmvmd_key &key, uint32_t tag, uint64_t index) : key_(key) {
+        nonce_[0] = tag;
+        nonce_[1] = (uint32_t)index;
+        nonce_[2] = (uint32_t)(index >> 32);
+    }
+    uint32_t word() {
+        if (used_ == 16) refill();
+        return block_[used_++];
+    }
+    // Uniform in [0, k): top bitlen(k-1) bits, rejected while >= k.
+    uint32_t below(uint32_t k) {
+        if (k <= 1) return 0;
+        int bits = 0;
+        for (uint32_t v = k - 1; v; v >>= 1) ++bits;
+        for (;;) {
+            const uint32_t v = word() >> (32 - bits);
+            if (v < k) return v;
+        }
+    }
+    // Uniform in F* = [1, q): top 31 bits, rejected outside [1, q).
+    uint32_t nonzero_field() {
+        for (;;) {
+            const uint32_t v = word() >> 1;
+            if (v != 0 && v < kQ) return v;
+        }
+    }
+
+  private:
+    static uint32_t rotl(uint32_t v, int c) { return (v << c) | (v >> (32 - c)); }
+    static void quarter(uint32_t *s, int a, int b, int c, int d) {
+        s[a] += s[b]; s[d] = rotl(s[d] ^ s[a], 16);
+        s[c] += s[d]; s[b] = rotl(s[b] ^ s[c], 12);
+        s[a] += s[b]; s[d] = rotl(s[d] ^ s[a], 8);
+        s[c] += s[d]; s[b] = rotl(s[b] ^ s[c], 7);
+    }
+    void refill() {
+        uint32_t in[16] = {0x61707865u, 0x3320646eu, 0x79622d32u, 0x6b206574u};
+        std::memcpy(in + 4, key_.k, sizeof key_.k);
+        in[12] = counter_++;
+        in[13] = nonce_[0];
+        in[14] = nonce_[1];
+        in[15] = nonce_[2];
+        uint32_t s[16];
+        std::memcpy(s, in, sizeof s);
+        for (int i = 0; i < 10; ++i) {
+            quarter(s, 0, 4, 8, 12); quarter(s, 1, 5, 9, 13);
+            quarter(s, 2, 6, 10, 14); quarter(s, 3, 7, 11, 15);
+            quarter(s, 0, 5, 10, 15); quarter(s, 1, 6, 11, 12);
+            quarter(s, 2, 7, 8, 13); quarter(s, 3, 4, 9, 14);
+        }
+        for (int i = 0; i < 16; ++i) block_[i] = s[i] + in[i];
+        used_ = 0;
+    }
+    pvmvmd_key key_;
+    uint32_t nonce_[3];
+    uint32_t counter_ = 0;
+    uint32_t block_[16];
+    int used_ = 16;
+};
+
+void sample_code_host(const pvmvmd_key &key, int which, uint32_t N, uint32_t *pi1, uint32_t *pi2,
+                      uint32_t *v1, uint32_t *v2) {
+    const uint32_t tag0 = which ? kTagCodeY : kTagCodeX;
+    uint32_t *perms[2] = {pi1, pi2};
+    for (int p = 0; p < 2; ++p) {  // Fisher-Yates, last index first
+        KeyStream ks(key, tag0 + p, 0);
+        uint32_t *a = perms[p];
+        for (uint32_t i = 0; i < N; ++i) a[i] = i;
+        for (uint32_t i = N; i-- > 1;) {
+            const uint32_t j = ks.below(i + 1);
+            const uint32_t tmp = a[i];
+            a[i] = a[j];
+            a[j] = tmp;
+        }
+    }
+    uint32_t *scales[2] = {v1, v2};
+    for (int p = 0; p < 2; ++p) {
+        KeyStream ks(key, tag0 + 2 + p, 0);
+        for (uint32_t i = 0; i < N; ++i) scales[p][i] = ks.nonzero_field();
+    }
+}
+
+// --------------------------------------------------------------------------
+// Device helpers
+// --------------------------------------------------------------------------
+int check_device() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return PVMVMD_E_NODEVICE;
+    int major = 0, minor = 0;
+    if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess)
+        return PVMVMD_E_NODEVICE;
+    return (major == 10 && minor == 3) ? PVMVMD_OK : PVMVMD_E_NODEVICE;
+}
+
+uint32_t *error_word() {
+    static std::mutex mu;
+    static uint32_t *addr[64] = {nullptr};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!addr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_error_word) != cudaSuccess) return nullptr;
+        addr[dev] = static_cast<uint32_t *>(p);
+    }
+    return addr[dev];
+}
+
+#define PV_CUDA(expr)                                  \
+    do {                                               \
+        cudaError_t e_ = (expr);                       \
+        if (e_ != cudaSuccess) {                       \
+            (void)cudaGetLastError();                  \
+            return e_ == cudaErrorMemoryAllocation ? PVMVMD_E_NOMEM : PVMVMD_E_CUDA; \
+        }                                              \
+    } while (0)
+
+template <typename T>
+cudaError_t dev_alloc(T **p, size_t count) {
+    *p = nullptr;
+    if (count == 0) count = 1;
+    return cudaMalloc(reinterpret_cast<void **>(p), count * sizeof(T));
+}
+
+struct CodeDev {
+    uint32_t *pi1 = nullptr, *pi2 = nullptr, *v1 = nullptr, *v2 = nullptr;
+    uint32_t *pi1inv = nullptr, *pi2inv = nullptr, *v2p = nullptr;
+};
+
+}  // namespace
+}  // namespace pv
+
+struct pvmvmd_ctx {
+    int device = 0;
+    pvmvmd_params params{};
+    int m = 0, K = 0, rate = 0, Nx = 0, Ny = 0, t_x = 0, t_y = 0, ell = 0, sb = 0;
+    pv::CodeDev gx, gy;
+    uint32_t *PT = nullptr, *Q = nullptr;
+    uint32_t *F = nullptr, *Fy = nullptr, *chal = nullptr, *g = nullptr, *u = nullptr;
+    unsigned long long *status = nullptr;
+    std::vector<void *> owned;
+};
+
+namespace pv {
+namespace {
+
+template <typename T>
+cudaError_t ctx_alloc(pvmvmd_ctx *c, T **p, size_t count) {
+    cudaError_t e = dev_alloc(p, count);
+    if (e == cudaSuccess) c->owned.push_back(*p);
+    return e;
+}
+
+int upload_code(pvmvmd_ctx *c, CodeDev &d, const pvmvmd_key &key, int which, uint32_t N,
+                cudaStream_t s) {
+    std::vector<uint32_t> pi1(N), pi2(N), v1(N), v2(N), pi1inv(N), pi2inv(N), v2p(N);
+    sample_code_host(key, which, N, pi1.data(), pi2.data(), v1.data(), v2.data());
+    for (uint32_t j = 0; j < N; ++j) {
+        pi1inv[pi1[j]] = j;
+        pi2inv[pi2[j]] = j;
+    }
+    for (uint32_t i = 0; i < N; ++i) v2p[i] = v2[pi2inv[i]];
+    uint32_t **dst[7] = {&d.pi1, &d.pi2, &d.v1, &d.v2, &d.pi1inv, &d.pi2inv, &d.v2p};
+    const std::vector<uint32_t> *src[7] = {&pi1, &pi2, &v1, &v2, &pi1inv, &pi2inv, &v2p};
+    for (int i = 0; i < 7; ++i) {
+        PV_CUDA(ctx_alloc(c, dst[i], N));
+        PV_CUDA(cudaMemcpyAsync(*dst[i], src[i]->data(), (size_t)N * 4, cudaMemcpyHostToDevice, s));
+    }
+    // the host vectors are released on return; wait for the copies
+    PV_CUDA(cudaStreamSynchronize(s));
+    return PVMVMD_OK;
+}
+
+// Y (N x L lanes, row stride ldy) = G^T applied to the L lanes of X (n x L,
+// row stride ldx; row i holds message entry i of every lane), in lane chunks.
+int encode_lanes(const CodeDev &d, uint32_t n, uint32_t r, const int8_t *X, size_t ldx,
+                 uint32_t L, uint32_t *Y, size_t ldy, uint32_t *err, cudaStream_t s) {
+    const uint32_t N = n * r;
+    size_t lc = ((size_t)1 << 28) / N;  // lanes per chunk: about 1 GiB of scratch
+    lc = (lc / 256) * 256;
+    if (lc < 256) lc = 256;
+    if (lc > L) lc = L;
+    uint32_t *S = nullptr, *agg = nullptr, *incl = nullptr, *flags = nullptr;
+    const size_t fw = encode_scan_flag_words(N, (uint32_t)lc);
+    const size_t vw = encode_scan_value_words(N, (uint32_t)lc);
+    int status = PVMVMD_OK;
+    if (dev_alloc(&S, (size_t)N * lc) != cudaSuccess || dev_alloc(&agg, vw) != cudaSuccess ||
+        dev_alloc(&incl, vw) != cudaSuccess || dev_alloc(&flags, fw) != cudaSuccess) {
+        status = PVMVMD_E_NOMEM;
+    }
+    for (uint32_t l0 = 0; status == PVMVMD_OK && l0 < L; l0 += (uint32_t)lc) {
+        const uint32_t nl = (uint32_t)((L - l0) < lc ? (L - l0) : lc);
+        cudaError_t e = cudaMemsetAsync(flags, 0, encode_scan_flag_words(N, nl) * 4, s);
+        if (e == cudaSuccess)  // S = A^T V1 Pi1^T R^T X
+            e = launch_encode_scan(X + l0, true, ldx, d.pi1, r, d.v1, N, nl, S, nl, agg, incl,
+                                   flags, err, s);
+        if (e == cudaSuccess) e = cudaMemsetAsync(flags, 0, encode_scan_flag_words(N, nl) * 4, s);
+        if (e == cudaSuccess)  // Y = A^T V2 Pi2^T S
+            e = launch_encode_scan(S, false, nl, d.pi2, 1, d.v2, N, nl, Y + l0, ldy, agg, incl,
+                                   flags, err, s);
+        if (e != cudaSuccess) status = PVMVMD_E_CUDA;
+    }
+    if (cudaStreamSynchronize(s) != cudaSuccess) status = PVMVMD_E_CUDA;
+    cudaFree(S);
+    cudaFree(agg);
+    cudaFree(incl);
+    cudaFree(flags);
+    return status;
+}
+
+int read_and_clear_error() {
+    uint32_t *ew = error_word();
+    if (!ew) return PVMVMD_E_CUDA;
+    uint32_t v = 0;
+    if (cudaMemcpy(&v, ew, 4, cudaMemcpyDeviceToHost) != cudaSuccess) return PVMVMD_E_CUDA;
+    if (v) {
+        const uint32_t zero = 0;
+        if (cudaMemcpy(ew, &zero, 4, cudaMemcpyHostToDevice) != cudaSuccess) return PVMVMD_E_CUDA;
+        return PVMVMD_E_DEVICE_TIMEOUT;
+    }
+    return PVMVMD_OK;
+}
+
+}  // namespace
+}  // namespace pv
+
+using namespace pv;
+
+extern "C" {
+
+const char *pvmvmd_strerror(int status) {
+    switch (status) {
+        case PVMVMD_OK: return "success";
+        case PVMVMD_E_ARG: return "invalid argument (null pointer or bad value)";
+        case PVMVMD_E_SHAPE: return "shape or batch size outside the supported range";
+        case PVMVMD_E_PARAM: return "inconsistent protocol parameters (e.g. t > N)";
+        case PVMVMD_E_CUDA: return "a CUDA runtime call or kernel launch failed";
+        case PVMVMD_E_NOMEM: return "out of memory";
+        case PVMVMD_E_DEVICE_TIMEOUT: return "a bounded device-side wait expired";
+        case PVMVMD_E_NODEVICE: return "no sm_103 (GB300) CUDA device is current";
+        default: return "unknown status";
+    }
+}
+
+int pvmvmd_params_resolve(const pvmvmd_params *in, int m, int K, pvmvmd_params *out) {
+    if (!out || m < 1 || K < 1) return PVMVMD_E_ARG;
+    pvmvmd_params p{};
+    if (in) p = *in;
+    if (p.lambda < 0 || p.kappa < 0 || p.rate < 0 || p.delta < 0 || p.t_x < 0 || p.t_y < 0 ||
+        p.ell < 0 || p.scratch_batch < 0 || p.delta >= 1.0)
+        return PVMVMD_E_PARAM;
+    if (p.lambda == 0) p.lambda = 128;
+    if (p.kappa == 0) p.kappa = 40;
+    if (p.rate == 0) p.rate = 8;
+    if (p.delta == 0) p.delta = 0.5;
+    if (p.scratch_batch == 0) p.scratch_batch = 64;
+    const double Nx = (double)p.rate * K, Ny = (double)p.rate * m;
+    if (Nx > 4294967295.0 || Ny > 4294967295.0) return PVMVMD_E_SHAPE;
+    if (p.t_x == 0) {  // Eq. (1)
+        const double t = std::ceil(std::log(2.0) * ((double)p.lambda - std::log2(Nx)) / p.delta);
+        p.t_x = t < 1 ? 1 : (int)t;
+    }
+    // Thm 5.2, by the two cases of its proof: with lf = log2(|F| - 1),
+    // case 1 (lf >= kappa + 1) needs (1-delta)^t <= 2^-(kappa+1) and ell = 1;
+    // case 2 needs (1-delta)^t <= 1/(|F|-1) and ell = ceil(kappa / (lf - 1)).
+    const double lf = std::log2((double)(kQ - 1));
+    const double per = -std::log2(1.0 - p.delta);
+    const bool case1 = lf >= p.kappa + 1;
+    if (p.t_y == 0) p.t_y = (int)std::ceil((case1 ? (double)(p.kappa + 1) : lf) / per);
+    if (p.ell == 0) p.ell = case1 ? 1 : (int)std::ceil((double)p.kappa / (lf - 1.0));
+    if (p.t_x > Nx || p.t_y > Ny || p.t_x > PVMVMD_MAX_T || p.t_y > PVMVMD_MAX_T || p.ell > 16 ||
+        p.ell < 1)
+        return PVMVMD_E_PARAM;
+    *out = p;
+    return PVMVMD_OK;
+}
+
+int pvmvmd_code_sample_host(const pvmvmd_key *key, int which, uint32_t N, uint32_t *pi1,
+                            uint32_t *pi2, uint32_t *v1, uint32_t *v2) {
+    if (!key || !pi1 || !pi2 || !v1 || !v2 || (which != 0 && which != 1)) return PVMVMD_E_ARG;
+    sample_code_host(*key, which, N, pi1, pi2, v1, v2);
+    return PVMVMD_OK;
+}
+
+void pvmvmd_destroy(pvmvmd_ctx *ctx) {
+    if (!ctx) return;
+    int cur = 0;
+    cudaGetDevice(&cur);
+    cudaSetDevice(ctx->device);
+    for (void *p : ctx->owned) cudaFree(p);
+    cudaSetDevice(cur);
+    delete ctx;
+}
+
+int pvmvmd_preprocess(const int8_t *W_dev, int m, int K, const pvmvmd_params *params,
+                      const pvmvmd_key *key, void *stream, pvmvmd_ctx **out) {
+    if (!out) return PVMVMD_E_ARG;
+    *out = nullptr;
+    if (!W_dev || !key) return PVMVMD_E_ARG;
+    if (m < 1 || K < 1 || K > PVMVMD_MAX_K) return PVMVMD_E_SHAPE;
+    int st = check_device();
+    if (st) return st;
+    pvmvmd_params p;
+    st = pvmvmd_params_resolve(params, m, K, &p);
+    if (st) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    uint32_t *err = error_word();
+    if (!err) return PVMVMD_E_CUDA;
+
+    pvmvmd_ctx *c = new (std::nothrow) pvmvmd_ctx();
+    if (!c) return PVMVMD_E_NOMEM;
+    cudaGetDevice(&c->device);
+    c->params = p;
+    c->m = m;
+    c->K = K;
+    c->rate = p.rate;
+    c->Nx = p.rate * K;
+    c->Ny = p.rate * m;
+    c->t_x = p.t_x;
+    c->t_y = p.t_y;
+    c->ell = p.ell;
+    c->sb = p.scratch_batch;
+
+    auto fail = [&](int code) {
+        pvmvmd_destroy(c);
+        return code;
+    };
+    if ((st = upload_code(c, c->gx, *key, 0, c->Nx, s))) return fail(st);
+    if ((st = upload_code(c, c->gy, *key, 1, c->Ny, s))) return fail(st);
+    const size_t statw = std::max(scan_status_words(c->Nx, c->sb), scan_status_words(c->Ny, c->ell));
+    if (ctx_alloc(c, &c->PT, (size_t)c->Nx * m) != cudaSuccess ||
+        ctx_alloc(c, &c->Q, (size_t)c->Ny * K) != cudaSuccess ||
+        ctx_alloc(c, &c->F, (size_t)c->sb * c->Nx) != cudaSuccess ||
+        ctx_alloc(c, &c->Fy, (size_t)c->ell * c->Ny) != cudaSuccess ||
+        ctx_alloc(c, &c->chal, (size_t)c->ell * 2 * c->t_y) != cudaSuccess ||
+        ctx_alloc(c, &c->g, (size_t)c->ell * m) != cudaSuccess ||
+        ctx_alloc(c, &c->u, (size_t)c->ell * K) != cudaSuccess ||
+        ctx_alloc(c, &c->status, statw) != cudaSuccess)
+        return fail(PVMVMD_E_NOMEM);
+
+    // P^T = G_x^T M^T: the m rows of M are the lanes, so transpose M first.
+    int8_t *MT = nullptr;
+    if (dev_alloc(&MT, (size_t)m * K) != cudaSuccess) return fail(PVMVMD_E_NOMEM);
+    if (launch_transpose_i8(W_dev, m, K, MT, s) != cudaSuccess) {
+        cudaFree(MT);
+        return fail(PVMVMD_E_CUDA);
+    }
+    st = encode_lanes(c->gx, K, c->rate, MT, (size_t)m, m, c->PT, (size_t)m, err, s);
+    cudaFree(MT);
+    if (st) return fail(st);
+    // Q = G_y^T M: the K columns of M are the lanes.
+    st = encode_lanes(c->gy, m, c->rate, W_dev, (size_t)K, K, c->Q, (size_t)K, err, s);
+    if (st) return fail(st);
+    if ((st = read_and_clear_error())) return fail(st);
+    *out = c;
+    return PVMVMD_OK;
+}
+
+int pvmvmd_state_size(const pvmvmd_ctx *ctx, int B, size_t *bytes) {
+    if (!ctx || !bytes || B < 0) return PVMVMD_E_ARG;
+    *bytes = (size_t)B * 2 * ctx->t_x * sizeof(uint32_t);
+    return PVMVMD_OK;
+}
+
+int pvmvmd_encode(pvmvmd_ctx *ctx, const uint32_t *X_dev, int B, const pvmvmd_key *key,
+                  uint32_t *Xhat_dev, void *st_dev, void *stream) {
+    if (!ctx || !X_dev || !key || !Xhat_dev || !st_dev) return PVMVMD_E_ARG;
+    if (B < 1) return PVMVMD_E_SHAPE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    uint32_t *err = error_word();
+    if (!err) return PVMVMD_E_CUDA;
+    uint32_t *stp = static_cast<uint32_t *>(st_dev);
+    const CodeDev &d = ctx->gx;
+    for (int b0 = 0; b0 < B; b0 += ctx->sb) {
+        const uint32_t nb = (uint32_t)(B - b0 < ctx->sb ? B - b0 : ctx->sb);
+        uint32_t *e = stp + (size_t)b0 * 2 * ctx->t_x;
+        PV_CUDA(launch_sample_sparse(*key, kTagMask, (uint64_t)b0, ctx->Nx, ctx->t_x, nb, e,
+                                     ctx->status, scan_status_words(ctx->Nx, nb), s));
+        PV_CUDA(launch_syndrome_scan(d.pi2inv, d.v2p, d.v1, ctx->Nx, e, ctx->t_x, nb, ctx->F,
+                                     ctx->status, err, s));
+        PV_CUDA(launch_syndrome_gather(d.pi1inv, ctx->K, ctx->rate, ctx->F, ctx->Nx,
+                                       X_dev + (size_t)b0 * ctx->K, Xhat_dev + (size_t)b0 * ctx->K,
+                                       nb, s));
+    }
+    return PVMVMD_OK;
+}
+
+int pvmvmd_server_mvm(const int8_t *W_dev, int m, int K, const uint32_t *Xhat_dev, int B,
+                      uint32_t *Yhat_dev, void *stream) {
+    if (!W_dev || !Xhat_dev || !Yhat_dev) return PVMVMD_E_ARG;
+    if (m < 1 || K < 1 || K > PVMVMD_MAX_K || B < 1) return PVMVMD_E_SHAPE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (B == 1) {
+        PV_CUDA(launch_gemv(W_dev, m, K, Xhat_dev, Yhat_dev, s));
+        return PVMVMD_OK;
+    }
+    uint32_t *err = error_word();
+    if (!err) return PVMVMD_E_CUDA;
+    PV_CUDA(launch_batched(W_dev, m, K, Xhat_dev, B, Yhat_dev, err, s));
+    return PVMVMD_OK;
+}
+
+int pvmvmd_decode_verify(pvmvmd_ctx *ctx, const void *st_dev, const uint32_t *Xhat_dev,
+                         const uint32_t *Yhat_dev, int B, const pvmvmd_key *challenge_key,
+                         uint32_t *Y_dev, int32_t *accept_dev, void *stream) {
+    if (!ctx || !st_dev || !Xhat_dev || !Yhat_dev || !challenge_key || !Y_dev || !accept_dev)
+        return PVMVMD_E_ARG;
+    if (B < 1) return PVMVMD_E_SHAPE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    uint32_t *err = error_word();
+    if (!err) return PVMVMD_E_CUDA;
+    const CodeDev &d = ctx->gy;
+    // Challenges e_q <- E_{t_y}^{N_y}, shared by the B vectors; g_q = G_y e_q.
+    PV_CUDA(launch_sample_sparse(*challenge_key, kTagChallenge, 0, ctx->Ny, ctx->t_y, ctx->ell,
+                                 ctx->chal, ctx->status, scan_status_words(ctx->Ny, ctx->ell), s));
+    PV_CUDA(launch_syndrome_scan(d.pi2inv, d.v2p, d.v1, ctx->Ny, ctx->chal, ctx->t_y, ctx->ell,
+                                 ctx->Fy, ctx->status, err, s));
+    PV_CUDA(launch_syndrome_gather(d.pi1inv, ctx->m, ctx->rate, ctx->Fy, ctx->Ny, nullptr, ctx->g,
+                                   ctx->ell, s));
+    // u_q = e_q^T Q.
+    PV_CUDA(launch_verify_u(ctx->Q, ctx->K, ctx->chal, ctx->t_y, ctx->ell, ctx->u, s));
+    PV_CUDA(launch_decode_verify(ctx->PT, ctx->m, ctx->K, static_cast<const uint32_t *>(st_dev),
+                                 ctx->t_x, Xhat_dev, Yhat_dev, ctx->g, ctx->u, ctx->ell, B, Y_dev,
+                                 accept_dev, s));
+    return PVMVMD_OK;
+}
+
+int pvmvmd_device_status(void *stream) {
+    if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) {
+        (void)cudaGetLastError();
+        return PVMVMD_E_CUDA;
+    }
+    return read_and_clear_error();
+}
+
+int pvmvmd_ctx_info(const pvmvmd_ctx *ctx, pvmvmd_ctx_view *v) {
+    if (!ctx || !v) return PVMVMD_E_ARG;
+    v->m = ctx->m;
+    v->K = ctx->K;
+    v->rate = ctx->rate;
+    v->N_x = ctx->Nx;
+    v->N_y = ctx->Ny;
+    v->t_x = ctx->t_x;
+    v->t_y = ctx->t_y;
+    v->ell = ctx->ell;
+    v->gx_pi1 = ctx->gx.pi1;
+    v->gx_pi2 = ctx->gx.pi2;
+    v->gx_v1 = ctx->gx.v1;
+    v->gx_v2 = ctx->gx.v2;
+    v->gy_pi1 = ctx->gy.pi1;
+    v->gy_pi2 = ctx->gy.pi2;
+    v->gy_v1 = ctx->gy.v1;
+    v->gy_v2 = ctx->gy.v2;
+    v->PT = ctx->PT;
+    v->Q = ctx->Q;
+    return PVMVMD_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,81 @@
+// Host-side launchers of the pvMVMD kernels (internal to the library).
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+
+#include <cuda_runtime.h>
+
+#include "pvmvmd.h"
+
+namespace pv {
+
+// Positions per tile of the single-lane syndrome scan.
+constexpr int kScanThreads = 256;
+constexpr int kScanItems = 8;
+constexpr int kScanTile = kScanThreads * kScanItems;
+
+__host__ __device__ inline uint32_t scan_tiles(uint32_t N) { return (N + kScanTile - 1) / kScanTile; }
+
+// Status words a syndrome scan over `count` vectors of length N needs
+// (word 0 is the tile ticket).
+inline size_t scan_status_words(uint32_t N, uint32_t count) {
+    return 1 + (size_t)count * scan_tiles(N);
+}
+
+// Sample `count` vectors of E_t^N: vector j uses index idx0 + j, reading
+// nonces (tag, 2*idx) and (tag, 2*idx + 1).  out: [count][2t] (ascending
+// support, then values).  Also zeroes clear[0 .. clear_words) for the scan
+// that follows in the same stream.
+cudaError_t launch_sample_sparse(const pvmvmd_key &key, uint32_t tag, uint64_t idx0, uint32_t N,
+                                 uint32_t t, uint32_t count, uint32_t *out,
+                                 unsigned long long *clear, size_t clear_words, cudaStream_t s);
+
+// Syndrome scan part of x' = G e for sparse e (App. B, syndrome direction):
+// c_i = v2[pi2^-1(i)] * (A e)_{pi2^-1(i)}, d = A c (suffix sums),
+// F_i = v1_i * d_i.  sparse: [count][2t]; F: [count][N].
+cudaError_t launch_syndrome_scan(const uint32_t *pi2inv, const uint32_t *v2p, const uint32_t *v1,
+                                 uint32_t N, const uint32_t *sparse, uint32_t t, uint32_t count,
+                                 uint32_t *F, unsigned long long *status, uint32_t *err,
+                                 cudaStream_t s);
+
+// Gather part: out_j = addend_j + sum_{c<r} F[pi1^-1(r j + c)], j < n
+// (addend may be null; out may alias addend).
+cudaError_t launch_syndrome_gather(const uint32_t *pi1inv, uint32_t n, uint32_t r,
+                                   const uint32_t *F, uint32_t N, const uint32_t *addend,
+                                   uint32_t *out, uint32_t count, cudaStream_t s);
+
+// One accumulate stage of the encoding G^T w over L lanes (App. B, encoding
+// direction): Y[j][l] = sum_{j' <= j} vscale[j'] * X[perm[j'] / div][l] for
+// j < N.  X is int8 (lifted to F_q) when x_is_i8, else uint32.  The scratch
+// `flags` holds ceil(L/256) * ceil(N/kEncTile) + 1 words and must be zero.
+constexpr int kEncTile = 32;
+size_t encode_scan_flag_words(uint32_t N, uint32_t L);
+size_t encode_scan_value_words(uint32_t N, uint32_t L);
+cudaError_t launch_encode_scan(const void *X, bool x_is_i8, size_t ldx, const uint32_t *perm,
+                               uint32_t div, const uint32_t *vscale, uint32_t N, uint32_t L,
+                               uint32_t *Y, size_t ldy, uint32_t *agg, uint32_t *incl,
+                               uint32_t *flags, uint32_t *err, cudaStream_t s);
+
+// int8 transpose: out[c][r] = in[r][c] for an R x C matrix.
+cudaError_t launch_transpose_i8(const int8_t *in, int R, int C, int8_t *out, cudaStream_t s);
+
+// Batch-1 field GEMV y = M x_hat over F_q.
+cudaError_t launch_gemv(const int8_t *W, int m, int K, const uint32_t *xhat, uint32_t *y,
+                        cudaStream_t s);
+
+// Batched product Y_hat[b] = M x_hat[b] over F_q on the tensor cores.
+cudaError_t launch_batched(const int8_t *W, int m, int K, const uint32_t *Xhat, int B,
+                           uint32_t *Yhat, uint32_t *err, cudaStream_t s);
+
+// Verify part 1: u[q][k] = sum_j e_{q,j} Q[supp_{q,j}][k] (e_q^T Q).
+cudaError_t launch_verify_u(const uint32_t *Qm, int K, const uint32_t *chal, uint32_t t_y,
+                            uint32_t ell, uint32_t *u, cudaStream_t s);
+
+// Fused decrypt and verify reduction for B vectors.
+cudaError_t launch_decode_verify(const uint32_t *PT, int m, int K, const uint32_t *st, uint32_t t_x,
+                                 const uint32_t *Xhat, const uint32_t *Yhat, const uint32_t *g,
+                                 const uint32_t *u, uint32_t ell, int B, uint32_t *Y,
+                                 int32_t *accept, cudaStream_t s);
+
+}  // namespace pv

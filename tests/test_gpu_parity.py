@@ -1,0 +1,275 @@
+"""GPU parity: the CUDA path, called through the C-ABI, against the oracle on
+the same seeded inputs.  Integer (field) results must match bit for bit."""
+import numpy as np
+import pytest
+
+import oracle
+from gpu_util import (Q, ctx_tables, field, pt_columns, q_columns, sample_rows, tamper,
+                      to_dev)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def pv():
+    import torch
+    assert torch.cuda.is_available()
+    import paper_2609_10264_gb300 as pv
+    return pv
+
+
+@pytest.fixture(scope="module")
+def wl():
+    from paper_2609_10264_gb300 import workloads
+    return workloads
+
+
+def _params(pv, **kw):
+    p = pv.pvmvmd_params()
+    for k, v in kw.items():
+        setattr(p, k, v)
+    return p
+
+
+def _full_round_trip(pv, W, x_int, seeds=(11, 12, 13), params=None, oracle_kw=None):
+    """Run preprocess/encode/server/decode_verify on the GPU and the oracle with
+    full tables; compare every intermediate exactly."""
+    import torch
+    m, K = W.shape
+    B = x_int.shape[0]
+    X = field(x_int)
+    Wd = to_dev(W)
+    ctx = pv.pvmvmd_preprocess(Wd, key=seeds[0], params=params)
+    pp = oracle.PublicParams(W, oracle.key_from_seed(seeds[0]), **(oracle_kw or {}))
+    # public codes and tables
+    v, tabs = ctx_tables(pv, ctx)
+    assert (v.t_x, v.t_y, v.ell) == (pp.t_x, pp.t_y, pp.ell)
+    for which, code in (("gx", pp.Gx), ("gy", pp.Gy)):
+        for f in ("pi1", "pi2", "v1", "v2"):
+            assert np.array_equal(tabs[f"{which}_{f}"], getattr(code, f)), f"{which}_{f}"
+    PT = pv.as_u32(pv.device_view(v.PT, v.N_x * m).view(v.N_x, m))
+    Qm = pv.as_u32(pv.device_view(v.Q, v.N_y * K).view(v.N_y, K))
+    assert np.array_equal(PT, pp.PT)
+    assert np.array_equal(Qm, pp.Q)
+    # encode
+    Xd = to_dev(X)
+    Xh, st = pv.pvmvmd_encode(ctx, Xd, key=seeds[1])
+    Xh_h, st_h = pv.as_u32(Xh), pv.as_u32(st)
+    for b in range(B):
+        xh_o, s_o, v_o = pp.encrypt(X[b], oracle.key_from_seed(seeds[1]), b)
+        assert np.array_equal(Xh_h[b], xh_o), f"x_hat {b}"
+        assert np.array_equal(st_h[b], np.concatenate([s_o, v_o])), f"st {b}"
+    # server: batch 1 per vector and the batched call
+    Yh1 = torch.stack([pv.pvmvmd_server_mvm(Wd, Xh[b]) for b in range(B)])
+    YhB = pv.pvmvmd_server_mvm(Wd, Xh)
+    Yh_o = np.stack([oracle.server_mvm(W, Xh_h[b]) for b in range(B)])
+    assert np.array_equal(pv.as_u32(Yh1), Yh_o)
+    assert np.array_equal(pv.as_u32(YhB), Yh_o)
+    # decode + verify
+    Y, acc = pv.pvmvmd_decode_verify(ctx, st, Xh, YhB, challenge_key=seeds[2])
+    Y_h = pv.as_u32(Y)
+    for b in range(B):
+        assert np.array_equal(Y_h[b], pp.decrypt(st_h[b, :pp.t_x], st_h[b, pp.t_x:], Yh_o[b]))
+        assert np.array_equal(oracle.centered(Y_h[b]), W.astype(np.int64) @ x_int[b])
+    assert pv.as_u32(acc).tolist() == [1] * B
+    assert all(pp.verify(Xh_h[b], Yh_o[b], oracle.key_from_seed(seeds[2])) for b in range(B))
+    # tampered outputs: rejected by both
+    bad = YhB.clone()
+    rng = np.random.default_rng(0)
+    for b in range(0, B, 2):
+        tamper(pv, bad, b, int(rng.integers(m)), int(rng.integers(1, Q)))
+    bad_h = pv.as_u32(bad)
+    _, acc_bad = pv.pvmvmd_decode_verify(ctx, st, Xh, bad, challenge_key=seeds[2] + 1)
+    exp = [0 if b % 2 == 0 else 1 for b in range(B)]
+    assert pv.as_u32(acc_bad).tolist() == exp
+    for b in range(0, B, 2):
+        assert not pp.verify(Xh_h[b], bad_h[b], oracle.key_from_seed(seeds[2] + 1))
+    assert pv.pvmvmd_device_status() == 0
+    ctx.destroy()
+
+
+def test_config1_tiny_round_trip(pv, wl):
+    """256 x 256 uniform int8 weights, one int8 vector from seed 0 (config 1)."""
+    W = wl.weights_uniform(256, 256, 0)
+    x = wl.int8_vectors(1, 256, 0)
+    _full_round_trip(pv, W, x, seeds=(0, 0, 0))
+
+
+@pytest.mark.parametrize("m,K,B", [(37, 100, 3), (300, 1000, 5), (129, 48, 2), (4, 40, 1), (513, 33, 4)])
+def test_ragged_round_trip(pv, wl, m, K, B):
+    W = wl.weights_uniform(m, K, m * 7 + K)
+    x = wl.int8_vectors(B, K, m + K)
+    _full_round_trip(pv, W, x, seeds=(m, K, B))
+
+
+def test_small_parameters_round_trip(pv, wl):
+    """Non-default rate and sparsities (rate 3, t_x 5, t_y 3, ell 3)."""
+    W = wl.weights_uniform(20, 12, 5)
+    x = wl.int8_vectors(3, 12, 6)
+    params = _params(pv, rate=3, t_x=5, t_y=3, ell=3)
+    _full_round_trip(pv, W, x, seeds=(3, 4, 5), params=params,
+                     oracle_kw=dict(t_x=5, t_y=3, ell=3, rate=3))
+
+
+def test_encode_chunking_matches(pv, wl):
+    """Encoding in chunks of 3 vectors (scratch_batch) gives the same result."""
+    W = wl.weights_uniform(64, 96, 1)
+    X = field(wl.int8_vectors(8, 96, 2))
+    Wd, Xd = to_dev(W), to_dev(X)
+    a = pv.pvmvmd_preprocess(Wd, key=9)
+    b = pv.pvmvmd_preprocess(Wd, key=9, params=_params(pv, scratch_batch=3))
+    xa, sa = pv.pvmvmd_encode(a, Xd, key=10)
+    xb, sb = pv.pvmvmd_encode(b, Xd, key=10)
+    assert np.array_equal(pv.as_u32(xa), pv.as_u32(xb))
+    assert np.array_equal(pv.as_u32(sa), pv.as_u32(sb))
+    # in place (X and Xhat alias)
+    xc = Xd.clone()
+    pv.pvmvmd_encode(a, xc, key=10, Xhat=xc)
+    assert np.array_equal(pv.as_u32(xc), pv.as_u32(xa))
+
+
+def test_server_mvm_extremes(pv):
+    """Extreme weights and field values: -128, 127, x = 0, 1, (q-1)/2, (q+1)/2, q-1."""
+    rng = np.random.default_rng(1)
+    for m, K in ((64, 4096), (17, 1000), (8, 16)):
+        W = rng.choice(np.array([-128, -127, 127, 0, 1], np.int8), size=(m, K))
+        W[0] = -128
+        W[1] = 127
+        vals = np.array([0, 1, (Q - 1) // 2, (Q + 1) // 2, Q - 1, Q - 2], np.uint32)
+        X = rng.choice(vals, size=(3, K)).astype(np.uint32)
+        X[0] = Q - 1
+        X[1] = (Q + 1) // 2
+        Wd = to_dev(W)
+        Xd = to_dev(X)
+        exp = np.stack([oracle.server_mvm(W, X[b]) for b in range(3)])
+        assert np.array_equal(pv.as_u32(pv.pvmvmd_server_mvm(Wd, Xd)), exp)
+        assert np.array_equal(pv.as_u32(pv.pvmvmd_server_mvm(Wd, Xd[0])), exp[0])
+
+
+def test_server_mvm_long_k_segments(pv):
+    """K beyond one shared-memory segment of digit planes (60000 > 49152)."""
+    rng = np.random.default_rng(2)
+    W = rng.integers(-128, 128, size=(40, 60000), dtype=np.int8)
+    x = rng.integers(0, Q, 60000).astype(np.uint32)
+    got = pv.as_u32(pv.pvmvmd_server_mvm(to_dev(W), to_dev(x)))
+    assert np.array_equal(got, oracle.server_mvm(W, x))
+
+
+def test_config2_gemv_all_vectors(pv, wl):
+    """4096 x 4096 Gaussian(32) int8 weights, 100 vectors uniform in F_q, batch 1."""
+    import torch
+    W = wl.weights_gaussian(4096, 4096, 2)
+    X = wl.field_vectors(100, 4096, 2)
+    Wd, Xd = to_dev(W), to_dev(X)
+    got = torch.stack([pv.pvmvmd_server_mvm(Wd, Xd[b]) for b in range(100)])
+    got = pv.as_u32(got)
+    for b in range(100):
+        assert np.array_equal(got[b], oracle.server_mvm(W, X[b])), b
+
+
+def test_config2_round_trip(pv, wl):
+    """Full pipeline at 4096 x 4096 with 100 int8 vectors; tables compared in full."""
+    import torch
+    W = wl.weights_gaussian(4096, 4096, 2)
+    x = wl.int8_vectors(100, 4096, 3)
+    X = field(x)
+    Wd = to_dev(W)
+    ctx = pv.pvmvmd_preprocess(Wd, key=20)
+    pp = oracle.PublicParams(W, oracle.key_from_seed(20))
+    v = pv.pvmvmd_ctx_info(ctx)
+    assert np.array_equal(pv.as_u32(pv.device_view(v.PT, v.N_x * 4096).view(v.N_x, 4096)), pp.PT)
+    assert np.array_equal(pv.as_u32(pv.device_view(v.Q, v.N_y * 4096).view(v.N_y, 4096)), pp.Q)
+    Xh, st = pv.pvmvmd_encode(ctx, to_dev(X), key=21)
+    Yh = torch.stack([pv.pvmvmd_server_mvm(Wd, Xh[b]) for b in range(100)])
+    Y, acc = pv.pvmvmd_decode_verify(ctx, st, Xh, Yh, challenge_key=22)
+    Xh_h, st_h, Yh_h, Y_h = pv.as_u32(Xh), pv.as_u32(st), pv.as_u32(Yh), pv.as_u32(Y)
+    for b in range(100):
+        xh_o, s_o, v_o = pp.encrypt(X[b], oracle.key_from_seed(21), b)
+        assert np.array_equal(Xh_h[b], xh_o)
+        assert np.array_equal(st_h[b], np.concatenate([s_o, v_o]))
+        assert np.array_equal(Yh_h[b], oracle.server_mvm(W, xh_o))
+        assert np.array_equal(Y_h[b], pp.decrypt(s_o, v_o, Yh_h[b]))
+    # every partial sum is below 2^53, so the float64 product is exact
+    assert np.array_equal(oracle.centered(Y_h), (x.astype(np.float64) @ W.astype(np.float64).T).astype(np.int64))
+    assert pv.as_u32(acc).tolist() == [1] * 100
+    for b in (0, 57, 99):
+        assert pp.verify(Xh_h[b], Yh_h[b], oracle.key_from_seed(22))
+    tamper(pv, Yh, 3, 5, 1)
+    tamper(pv, Yh, 50, 4095, Q - 1)
+    _, acc2 = pv.pvmvmd_decode_verify(ctx, st, Xh, Yh, challenge_key=23)
+    a2 = pv.as_u32(acc2)
+    assert a2[3] == 0 and a2[50] == 0 and a2.sum() == 98
+    assert pv.pvmvmd_device_status() == 0
+
+
+@pytest.mark.parametrize("layer", [0, 31])
+def test_config3_layer_gemv_sampled(pv, wl, layer):
+    """One 8B-class decoder layer at batch 1 (7 projections), sampled rows."""
+    for j, (name, (m, K)) in enumerate(wl.LAYER_8B.items()):
+        W = wl.weights_gaussian(m, K, (3, layer, j))
+        x = wl.field_vectors(1, K, (3, layer, j, 1))[0]
+        got = pv.as_u32(pv.pvmvmd_server_mvm(to_dev(W), to_dev(x)))
+        rows = sample_rows(m, 48, layer * 10 + j)
+        assert np.array_equal(got[rows], oracle.server_mvm_rows(W, x, rows)), name
+
+
+def _batched_pipeline_sampled(pv, W, B, seed, n_rows=24, n_verify=2):
+    """Preprocess/encode/server/decode_verify at a large shape; checks: P^T and
+    Q columns, every x_hat and mask, server outputs on sampled rows for all
+    vectors, decoded rows equal the exact integer product, all accepted, and
+    the oracle's verdict for a few vectors."""
+    m, K = W.shape
+    x = np.random.default_rng(seed).integers(-127, 128, size=(B, K), dtype=np.int64)
+    X = field(x)
+    Wd = to_dev(W)
+    ctx = pv.pvmvmd_preprocess(Wd, key=seed)
+    pp = oracle.PublicParams(W, oracle.key_from_seed(seed), with_tables=False)
+    rows = sample_rows(m, n_rows, seed)
+    cols = sample_rows(K, n_rows, seed + 1)
+    ptc = pt_columns(pv, ctx, rows)
+    for i, r in enumerate(rows):
+        assert np.array_equal(ptc[:, i], pp.Gx.encode(oracle.lift(W[r]))), f"P^T column {r}"
+    qc = q_columns(pv, ctx, cols)
+    for i, c in enumerate(cols):
+        assert np.array_equal(qc[:, i], pp.Gy.encode(oracle.lift(W[:, c]))), f"Q column {c}"
+    Xh, st = pv.pvmvmd_encode(ctx, to_dev(X), key=seed + 1)
+    Xh_h, st_h = pv.as_u32(Xh), pv.as_u32(st)
+    for b in range(B):
+        xh_o, s_o, v_o = pp.encrypt(X[b], oracle.key_from_seed(seed + 1), b)
+        assert np.array_equal(Xh_h[b], xh_o), b
+        assert np.array_equal(st_h[b], np.concatenate([s_o, v_o])), b
+    Yh = pv.pvmvmd_server_mvm(Wd, Xh)
+    Yh_h = pv.as_u32(Yh)
+    for b in range(B):
+        assert np.array_equal(Yh_h[b, rows], oracle.server_mvm_rows(W, Xh_h[b], rows)), b
+    Y, acc = pv.pvmvmd_decode_verify(ctx, st, Xh, Yh, challenge_key=seed + 2)
+    Y_h = pv.as_u32(Y)
+    exact = (x @ W[rows].astype(np.int64).T)
+    assert np.array_equal(oracle.centered(Y_h[:, rows]), exact)
+    assert pv.as_u32(acc).tolist() == [1] * B
+    for b in range(n_verify):
+        assert pp.verify(Xh_h[b], Yh_h[b], oracle.key_from_seed(seed + 2))
+        assert np.array_equal(Y_h[b, rows[:4]], pp.decrypt_rows(st_h[b, :pp.t_x], st_h[b, pp.t_x:],
+                                                                 Yh_h[b, rows[:4]], rows[:4]))
+    tamper(pv, Yh, 1, int(rows[1]), 1)
+    _, acc2 = pv.pvmvmd_decode_verify(ctx, st, Xh, Yh, challenge_key=seed + 3)
+    a2 = pv.as_u32(acc2)
+    assert a2[1] == 0 and a2.sum() == B - 1
+    assert pv.pvmvmd_device_status() == 0
+    ctx.destroy()
+
+
+@pytest.mark.parametrize("name", ["q", "k", "gate", "down"])
+def test_config4_batched_8b(pv, wl, name):
+    """8B-class layer shapes with 64 vectors per call (the batched product)."""
+    m, K = wl.LAYER_8B[name]
+    W = wl.weights_gaussian(m, K, (4, list(wl.LAYER_8B).index(name)))
+    _batched_pipeline_sampled(pv, W, 64, seed=400 + len(name))
+
+
+@pytest.mark.parametrize("name", ["q", "kv", "gate_up", "down"])
+def test_config5_70b(pv, wl, name):
+    """70B-class shapes with 256 vectors per call; the largest K is 28672."""
+    m, K = wl.LAYER_70B[name]
+    W = wl.weights_gaussian(m, K, (5, list(wl.LAYER_70B).index(name)))
+    _batched_pipeline_sampled(pv, W, 256, seed=500 + len(name), n_rows=12, n_verify=1)

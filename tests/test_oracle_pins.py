@@ -279,7 +279,7 @@ def test_preprocess_tables_are_encodings(tiny_pp):
 
 def test_completeness_round_trip(tiny_pp):
     """decode(server(encode(x))) = M x and honest outputs are accepted
-    (Def. 4.2 completeness; Thm 5.4 proof)."""
+    (Def. 4.2 completeness; Thm 6.1 proof)."""
     pp = tiny_pp
     rng = np.random.default_rng(1)
     x_int = rng.integers(-127, 128, pp.n)
@@ -295,7 +295,7 @@ def test_completeness_round_trip(tiny_pp):
 
 
 def test_decrypt_error_identity(tiny_pp):
-    """y - Mx = y_hat - M x_hat (soundness proof of Thm 5.4)."""
+    """y - Mx = y_hat - M x_hat (soundness proof of Thm 6.1)."""
     pp = tiny_pp
     rng = np.random.default_rng(2)
     x = rng.integers(0, Q, pp.n).astype(np.uint32)
@@ -359,7 +359,7 @@ def test_soundness_rate_matches_lemma_5_1(t):
 
 
 def test_masked_vector_looks_uniform(tiny_pp):
-    """Privacy rests on dual-LPN (Thm 5.4): parity unpinned.  Only a sanity
+    """Privacy rests on dual-LPN (Thm 6.1): parity unpinned.  Only a sanity
     check: masked entries spread over F_q even for x = 0."""
     pp = tiny_pp
     vals = np.concatenate([pp.encrypt(np.zeros(pp.n, np.uint32), 9, b)[0] for b in range(40)])
