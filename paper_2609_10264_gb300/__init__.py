@@ -310,7 +310,7 @@ def as_u32(t) -> np.ndarray:
 
 class _CudaArray:
     def __init__(self, ptr: int, count: int):
-        self.__cuda_array_interface__ = {"shape": (count,), "typestr": "<i4", "data": (int(ptr), True),
+        self.__cuda_array_interface__ = {"shape": (count,), "typestr": "<i4", "data": (int(ptr), False),
                                          "version": 2, "strides": None}
 
 
