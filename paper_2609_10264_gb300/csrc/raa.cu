@@ -134,7 +134,8 @@ __global__ void __launch_bounds__(32) k_sample_sparse(pvmvmd_key key, uint32_t t
 __global__ void __launch_bounds__(kScanThreads) k_syndrome_scan(
     const uint32_t *__restrict__ pi2inv, const uint32_t *__restrict__ v2p,
     const uint32_t *__restrict__ v1, uint32_t N, const uint32_t *__restrict__ sparse, uint32_t t,
-    uint32_t *__restrict__ F, unsigned long long *__restrict__ status, uint32_t *__restrict__ err) {
+    uint32_t count, uint32_t *__restrict__ F, unsigned long long *__restrict__ status,
+    uint32_t *__restrict__ err) {
     extern __shared__ uint32_t sm[];
     uint32_t *s_supp = sm;     // t
     uint32_t *s_suf = sm + t;  // t + 1
@@ -146,6 +147,10 @@ __global__ void __launch_bounds__(kScanThreads) k_syndrome_scan(
     __syncthreads();
     const uint32_t ntiles = scan_tiles(N);
     const uint32_t ticket = s_ticket;
+    if (ticket >= count * ntiles) {  // status word not cleared: never index past the data
+        if (tid == 0) record_error(err, kErrScanTimeout);
+        return;
+    }
     const uint32_t vec = ticket / ntiles;
     const uint32_t tile = ntiles - 1 - ticket % ntiles;
     unsigned long long *st = status + 1 + (size_t)vec * ntiles;
@@ -318,6 +323,10 @@ __global__ void __launch_bounds__(256) k_encode_scan(const void *__restrict__ Xv
     if (tid == 0) s_ticket = atomicAdd(flags, 1u);
     __syncthreads();
     const uint32_t ticket = s_ticket;
+    if (ticket >= nlb * ntiles) {  // flags not cleared: never index past the data
+        if (tid == 0) record_error(err, kErrScanTimeout);
+        return;
+    }
     const uint32_t tile = ticket / nlb, lb = ticket % nlb;
     const uint32_t l = lb * 256 + tid;
     const bool lane_ok = l < L;
@@ -428,7 +437,8 @@ cudaError_t launch_syndrome_scan(const uint32_t *pi2inv, const uint32_t *v2p, co
     if (count == 0) return cudaSuccess;
     const size_t smem = (2 * (size_t)t + 1) * sizeof(uint32_t);
     const unsigned grid = count * scan_tiles(N);
-    k_syndrome_scan<<<grid, kScanThreads, smem, s>>>(pi2inv, v2p, v1, N, sparse, t, F, status, err);
+    k_syndrome_scan<<<grid, kScanThreads, smem, s>>>(pi2inv, v2p, v1, N, sparse, t, count, F, status,
+                                                     err);
     return cudaGetLastError();
 }
 
