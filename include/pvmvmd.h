@@ -130,6 +130,24 @@ int pvmvmd_encode(pvmvmd_ctx *ctx, const uint32_t *X_dev, int B, const pvmvmd_ke
 int pvmvmd_server_mvm(const int8_t *W_dev, int m, int K, const uint32_t *Xhat_dev, int B,
                       uint32_t *Yhat_dev, void *stream);
 
+/* One request of pvmvmd_server_mvm_multi: yhat = W xhat over F_q. */
+typedef struct {
+    const int8_t *W_dev;      /* int8 m x K row-major                       */
+    const uint32_t *xhat_dev; /* K field elements                           */
+    uint32_t *yhat_dev;       /* m field elements (output)                  */
+    int m, K;
+} pvmvmd_mvm_job;
+
+/* The server's products for `count` independent batch-1 requests (Sec. 6.1:
+ * the server's online work is one product per masked vector), in as few
+ * launches as possible: jobs[i].yhat_dev = jobs[i].W_dev * jobs[i].xhat_dev
+ * over F_q.  Requests may use different matrices and shapes; each matrix is
+ * streamed once per request (no reuse across requests).  Results equal
+ * `count` calls of pvmvmd_server_mvm with B = 1.  `jobs` is a host array that
+ * may be freed on return; outputs must not overlap any input or each other.
+ * 1 <= count, each 1 <= K <= PVMVMD_MAX_K, 1 <= m. */
+int pvmvmd_server_mvm_multi(const pvmvmd_mvm_job *jobs, int count, void *stream);
+
 /* Verify and Decrypt (Protocol 3).  Verify: ell challenges e_q <- E_{t_y}^{N_y}
  * are drawn from challenge_key (repetition q reads nonce (10, 2q) and
  * (10, 2q+1)) and shared by all B vectors of the call, as Sec. 5.4 allows;

@@ -60,6 +60,11 @@ class pvmvmd_ctx_view(ctypes.Structure):
                 ("PT", ctypes.c_void_p), ("Q", ctypes.c_void_p)]
 
 
+class pvmvmd_mvm_job(ctypes.Structure):
+    _fields_ = [("W_dev", ctypes.c_void_p), ("xhat_dev", ctypes.c_void_p), ("yhat_dev", ctypes.c_void_p),
+                ("m", ctypes.c_int), ("K", ctypes.c_int)]
+
+
 # Exported symbols and their ctypes signatures (mirrors include/pvmvmd.h).
 _vp, _i, _sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
 SIGNATURES = {
@@ -69,6 +74,7 @@ SIGNATURES = {
     "pvmvmd_state_size": (_i, [_vp, _i, ctypes.POINTER(_sz)]),
     "pvmvmd_encode": (_i, [_vp, _vp, _i, ctypes.POINTER(pvmvmd_key), _vp, _vp, _vp]),
     "pvmvmd_server_mvm": (_i, [_vp, _i, _i, _vp, _i, _vp, _vp]),
+    "pvmvmd_server_mvm_multi": (_i, [ctypes.POINTER(pvmvmd_mvm_job), _i, _vp]),
     "pvmvmd_decode_verify": (_i, [_vp, _vp, _vp, _vp, _i, ctypes.POINTER(pvmvmd_key), _vp, _vp, _vp]),
     "pvmvmd_device_status": (_i, [_vp]),
     "pvmvmd_ctx_info": (_i, [_vp, ctypes.POINTER(pvmvmd_ctx_view)]),
@@ -259,6 +265,28 @@ def pvmvmd_server_mvm(W, Xhat, Yhat=None, stream=None):
                                   B, _dev_ptr(Yhat, "Yhat", _u32_types(), B * m), _stream_ptr(stream)),
            "pvmvmd_server_mvm")
     return Yhat
+
+
+def mvm_jobs(triples):
+    """A ctypes job array for pvmvmd_server_mvm_multi from (W, xhat, yhat)
+    tensors; reusable across calls while the tensors live."""
+    import torch
+    arr = (pvmvmd_mvm_job * len(triples))()
+    for i, (W, xh, yh) in enumerate(triples):
+        m, K = W.shape
+        arr[i].W_dev = _dev_ptr(W, "W", (torch.int8,)).value
+        arr[i].xhat_dev = _dev_ptr(xh, "xhat", _u32_types(), K).value
+        arr[i].yhat_dev = _dev_ptr(yh, "yhat", _u32_types(), m).value
+        arr[i].m, arr[i].K = m, K
+    return arr
+
+
+def pvmvmd_server_mvm_multi(jobs, stream=None) -> None:
+    """Independent batch-1 products: `jobs` is a list of (W, xhat, yhat)
+    tensors or an array from mvm_jobs()."""
+    if not isinstance(jobs, ctypes.Array):
+        jobs = mvm_jobs(jobs)
+    _check(_lib.pvmvmd_server_mvm_multi(jobs, len(jobs), _stream_ptr(stream)), "pvmvmd_server_mvm_multi")
 
 
 def pvmvmd_decode_verify(ctx: Ctx, st, Xhat, Yhat, challenge_key, Y=None, accept=None, stream=None):

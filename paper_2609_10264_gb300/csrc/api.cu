@@ -424,13 +424,37 @@ int pvmvmd_server_mvm(const int8_t *W_dev, int m, int K, const uint32_t *Xhat_de
     if (!W_dev || !Xhat_dev || !Yhat_dev) return PVMVMD_E_ARG;
     if (m < 1 || K < 1 || K > PVMVMD_MAX_K || B < 1) return PVMVMD_E_SHAPE;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    if (B == 1) {
-        PV_CUDA(launch_gemv(W_dev, m, K, Xhat_dev, Yhat_dev, s));
-        return PVMVMD_OK;
-    }
     uint32_t *err = error_word();
     if (!err) return PVMVMD_E_CUDA;
+    if (B == 1) {
+        PV_CUDA(launch_gemv(W_dev, m, K, Xhat_dev, Yhat_dev, err, s));
+        return PVMVMD_OK;
+    }
     PV_CUDA(launch_batched(W_dev, m, K, Xhat_dev, B, Yhat_dev, err, s));
+    return PVMVMD_OK;
+}
+
+int pvmvmd_server_mvm_multi(const pvmvmd_mvm_job *jobs, int count, void *stream) {
+    if (!jobs || count < 1) return count < 1 ? PVMVMD_E_SHAPE : PVMVMD_E_ARG;
+    for (int i = 0; i < count; ++i) {
+        const pvmvmd_mvm_job &j = jobs[i];
+        if (!j.W_dev || !j.xhat_dev || !j.yhat_dev) return PVMVMD_E_ARG;
+        if (j.m < 1 || j.K < 1 || j.K > PVMVMD_MAX_K) return PVMVMD_E_SHAPE;
+    }
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    uint32_t *err = error_word();
+    if (!err) return PVMVMD_E_CUDA;
+    std::vector<MvmJob> grouped;
+    grouped.reserve(count);
+    for (int i = 0; i < count; ++i) {
+        const pvmvmd_mvm_job &j = jobs[i];
+        MvmJob t{j.W_dev, j.xhat_dev, j.yhat_dev, j.m, j.K, (size_t)j.K, 0};
+        if (multi_eligible(t))
+            grouped.push_back(t);
+        else
+            PV_CUDA(launch_gemv(j.W_dev, j.m, j.K, j.xhat_dev, j.yhat_dev, err, s));
+    }
+    if (!grouped.empty()) PV_CUDA(launch_gemv_multi(grouped.data(), (int)grouped.size(), s));
     return PVMVMD_OK;
 }
 

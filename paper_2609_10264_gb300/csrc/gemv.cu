@@ -14,6 +14,10 @@
 //  * Per row: a transposed butterfly reduces the 4*ROWS lane partials in
 //    4*ROWS - 1 + log2(32/(4*ROWS)) shuffles, the four limb sums are combined
 //    in int64 and reduced mod q once.
+#include <algorithm>
+#include <mutex>
+#include <vector>
+
 #include "common.cuh"
 #include "launch.h"
 
@@ -190,6 +194,191 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
     }
 }
 
+// ---------------------------------------------------------------------------
+// Grouped persistent variant (K % 16 == 0, 16-byte aligned rows): one launch
+// computes a list of independent batch-1 products (jobs), each streaming its
+// own matrix once.  The bytes of all matrices are split evenly over the CTAs
+// (whole rows); a CTA walks its share job by job, splitting that job's x_hat
+// into digit planes once, and its warps stream row pairs with the loads of
+// the next batch issued before the arithmetic of the current one.  A single
+// launch over many matrices keeps every SM's loads in flight for the whole
+// stream instead of paying the ramp-up and drain of one launch per matrix.
+// Launched with programmatic dependent launch; it waits for the preceding
+// kernel (griddepcontrol.wait) before reading anything.
+// ---------------------------------------------------------------------------
+constexpr int kMultiThreads = 256;
+constexpr int kMultiWarps = kMultiThreads / 32;
+
+struct MultiArgs {
+    int count;
+    long long base[kMultiMaxJobs + 1];  // prefix sums of m_j * K_j (bytes of M)
+    MvmJob job[kMultiMaxJobs];
+};
+
+template <int ROWS, int UNROLL>
+__global__ void __launch_bounds__(kMultiThreads, 2) k_gemv_multi(const __grid_constant__ MultiArgs args) {
+    extern __shared__ uint4 s_planes[];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    constexpr int V = ROWS * 4;
+    const long long total = args.base[args.count];
+    const long long lo = total * blockIdx.x / gridDim.x;
+    const long long hi = total * (blockIdx.x + 1) / gridDim.x;
+
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+
+    for (int j = 0; j < args.count; ++j) {
+        const long long b0 = args.base[j], b1 = args.base[j + 1];
+        if (b1 <= lo || b0 >= hi) continue;
+        const MvmJob &job = args.job[j];
+        const int K = job.K, m = job.m, nchunks = K / 16;
+        // rows whose first byte lies in [lo, hi)
+        const int row_a = lo > b0 ? (int)((lo - b0 + K - 1) / K) : 0;
+        const int row_b = (int)min((long long)m, (hi - b0 + K - 1) / K);
+        if (row_a >= row_b) continue;
+        const int ngroups = (row_b - row_a + ROWS - 1) / ROWS;
+
+        uint4 wbuf[UNROLL][ROWS];
+        auto issue = [&](int grp, int c) {
+#pragma unroll
+            for (int u = 0; u < UNROLL; ++u)
+#pragma unroll
+                for (int r = 0; r < ROWS; ++r) {
+                    const int cc = c + 32 * u, row = row_a + grp * ROWS + r;
+                    wbuf[u][r] = (cc < nchunks && row < row_b)
+                                     ? ldg_stream(job.W + (size_t)row * job.ldw + (size_t)cc * 16)
+                                     : make_uint4(0u, 0u, 0u, 0u);
+                }
+        };
+        int g = warp;
+        if (g < ngroups) issue(g, lane);
+
+        __syncthreads();  // the previous job's planes are no longer read
+        uint32_t *planes = reinterpret_cast<uint32_t *>(s_planes);
+        const int pstride = K / 4;
+        for (int q4 = tid; q4 < pstride; q4 += kMultiThreads) {
+            const uint4 xv = __ldg(reinterpret_cast<const uint4 *>(job.xhat) + q4);
+            const uint32_t xs[4] = {xv.x, xv.y, xv.z, xv.w};
+            uint32_t p0 = 0, p1 = 0, p2 = 0, p3 = 0;
+#pragma unroll
+            for (int b = 0; b < 4; ++b) {
+                int d0, d1, d2, d3;
+                limb_split(xs[b], d0, d1, d2, d3);
+                p0 |= (uint32_t)(d0 & 0xff) << (8 * b);
+                p1 |= (uint32_t)(d1 & 0xff) << (8 * b);
+                p2 |= (uint32_t)(d2 & 0xff) << (8 * b);
+                p3 |= (uint32_t)(d3 & 0xff) << (8 * b);
+            }
+            planes[q4] = p0;
+            planes[pstride + q4] = p1;
+            planes[2 * pstride + q4] = p2;
+            planes[3 * pstride + q4] = p3;
+        }
+        __syncthreads();
+        const uint4 *P0 = s_planes, *P1 = s_planes + nchunks, *P2 = s_planes + 2 * nchunks,
+                    *P3 = s_planes + 3 * nchunks;
+
+        for (; g < ngroups; g += kMultiWarps) {
+            int acc[ROWS][4];
+#pragma unroll
+            for (int r = 0; r < ROWS; ++r) acc[r][0] = acc[r][1] = acc[r][2] = acc[r][3] = 0;
+            for (int c = lane; c < nchunks; c += 32 * UNROLL) {
+                uint4 cur[UNROLL][ROWS];
+#pragma unroll
+                for (int u = 0; u < UNROLL; ++u)
+#pragma unroll
+                    for (int r = 0; r < ROWS; ++r) cur[u][r] = wbuf[u][r];
+                const int cn = c + 32 * UNROLL;
+                if (cn < nchunks) issue(g, cn);
+                else if (g + kMultiWarps < ngroups) issue(g + kMultiWarps, lane);
+#pragma unroll
+                for (int u = 0; u < UNROLL; ++u) {
+                    const int cc = c + 32 * u;
+                    if (cc < nchunks) {
+                        const uint4 l0 = P0[cc], l1 = P1[cc], l2 = P2[cc], l3 = P3[cc];
+#pragma unroll
+                        for (int r = 0; r < ROWS; ++r) {
+                            const uint4 w = cur[u][r];
+                            acc[r][0] = __dp4a((int)w.x, (int)l0.x, acc[r][0]);
+                            acc[r][1] = __dp4a((int)w.x, (int)l1.x, acc[r][1]);
+                            acc[r][2] = __dp4a((int)w.x, (int)l2.x, acc[r][2]);
+                            acc[r][3] = __dp4a((int)w.x, (int)l3.x, acc[r][3]);
+                            acc[r][0] = __dp4a((int)w.y, (int)l0.y, acc[r][0]);
+                            acc[r][1] = __dp4a((int)w.y, (int)l1.y, acc[r][1]);
+                            acc[r][2] = __dp4a((int)w.y, (int)l2.y, acc[r][2]);
+                            acc[r][3] = __dp4a((int)w.y, (int)l3.y, acc[r][3]);
+                            acc[r][0] = __dp4a((int)w.z, (int)l0.z, acc[r][0]);
+                            acc[r][1] = __dp4a((int)w.z, (int)l1.z, acc[r][1]);
+                            acc[r][2] = __dp4a((int)w.z, (int)l2.z, acc[r][2]);
+                            acc[r][3] = __dp4a((int)w.z, (int)l3.z, acc[r][3]);
+                            acc[r][0] = __dp4a((int)w.w, (int)l0.w, acc[r][0]);
+                            acc[r][1] = __dp4a((int)w.w, (int)l1.w, acc[r][1]);
+                            acc[r][2] = __dp4a((int)w.w, (int)l2.w, acc[r][2]);
+                            acc[r][3] = __dp4a((int)w.w, (int)l3.w, acc[r][3]);
+                        }
+                    }
+                }
+            }
+            int v[V];
+#pragma unroll
+            for (int r = 0; r < ROWS; ++r)
+#pragma unroll
+                for (int p = 0; p < 4; ++p) v[r * 4 + p] = acc[r][p];
+            const int tot = transposed_reduce<V>(v, lane);
+            constexpr int span = 32 / V;
+            const int a1 = __shfl_down_sync(kFull, tot, span);
+            const int a2 = __shfl_down_sync(kFull, tot, 2 * span);
+            const int a3 = __shfl_down_sync(kFull, tot, 3 * span);
+            const int entry = lane / span;
+            if ((lane % span) == 0 && (entry & 3) == 0) {
+                const int row = row_a + g * ROWS + (entry >> 2);
+                if (row < row_b) {
+                    const int64_t sum = (int64_t)tot + ((int64_t)a1 << 8) + ((int64_t)a2 << 16) +
+                                        ((int64_t)a3 << 24);
+                    const uint32_t part = fred_signed(sum);
+                    job.y[row] = job.accumulate ? fadd(job.y[row], part) : part;
+                }
+            }
+        }
+    }
+}
+
+cudaError_t run_gemv_multi(const MvmJob *jobs, int count, cudaStream_t s) {
+    static MultiArgs args;  // host staging of the kernel parameters (copied at launch)
+    static std::mutex mu;
+    std::lock_guard<std::mutex> lock(mu);
+    args.count = count;
+    args.base[0] = 0;
+    int kmax = 16;
+    for (int j = 0; j < count; ++j) {
+        args.job[j] = jobs[j];
+        args.base[j + 1] = args.base[j] + (long long)jobs[j].m * jobs[j].K;
+        if (jobs[j].K > kmax) kmax = jobs[j].K;
+    }
+    long long rows = 0;
+    for (int j = 0; j < count; ++j) rows += jobs[j].m;
+    if (rows == 0) return cudaSuccess;
+    static const cudaError_t attr = cudaFuncSetAttribute(
+        k_gemv_multi<2, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, 4 * kMultiMaxK);
+    if (attr != cudaSuccess) return attr;
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    long long grid = 2LL * sms;
+    if (grid > rows) grid = rows;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid, 1, 1);
+    cfg.blockDim = dim3(kMultiThreads, 1, 1);
+    cfg.dynamicSmemBytes = (size_t)4 * kmax;
+    cfg.stream = s;
+    cudaLaunchAttribute attrs[1];
+    attrs[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attrs[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attrs;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, k_gemv_multi<2, 4>, args);
+}
+
 template <int ROWS, int UNROLL, bool kVec>
 cudaError_t run_gemv(const int8_t *W, size_t ldw, int m, int K, const uint32_t *xhat, uint32_t *y,
                      bool accumulate, cudaStream_t s) {
@@ -211,14 +400,44 @@ cudaError_t run_gemv(const int8_t *W, size_t ldw, int m, int K, const uint32_t *
 
 }  // namespace
 
+bool multi_eligible(const MvmJob &j) {
+    return j.K % 16 == 0 && j.ldw % 16 == 0 && (reinterpret_cast<uintptr_t>(j.W) & 15u) == 0 &&
+           (reinterpret_cast<uintptr_t>(j.xhat) & 15u) == 0;
+}
+
+cudaError_t launch_gemv_multi(const MvmJob *jobs, int count, cudaStream_t s) {
+    // Jobs with K beyond one shared-memory segment are split into K segments;
+    // segment k of every job goes into launch k, later launches accumulate.
+    std::vector<MvmJob> seg;
+    for (int k0 = 0;; k0 += kMultiMaxK) {
+        seg.clear();
+        for (int j = 0; j < count; ++j) {
+            if (jobs[j].K <= k0) continue;
+            MvmJob t = jobs[j];
+            t.W = jobs[j].W + k0;
+            t.xhat = jobs[j].xhat + k0;
+            t.K = jobs[j].K - k0 < kMultiMaxK ? jobs[j].K - k0 : kMultiMaxK;
+            t.accumulate = k0 > 0 ? 1 : jobs[j].accumulate;
+            seg.push_back(t);
+        }
+        if (seg.empty()) return cudaSuccess;
+        for (size_t a = 0; a < seg.size(); a += kMultiMaxJobs) {
+            const int n = (int)std::min(seg.size() - a, (size_t)kMultiMaxJobs);
+            cudaError_t e = run_gemv_multi(seg.data() + a, n, s);
+            if (e != cudaSuccess) return e;
+        }
+    }
+}
+
 cudaError_t launch_gemv(const int8_t *W, int m, int K, const uint32_t *xhat, uint32_t *y,
-                        cudaStream_t s) {
+                        uint32_t *err, cudaStream_t s) {
+    (void)err;
     if (m <= 0 || K <= 0) return cudaSuccess;
-    const bool vec = (K % 16 == 0) && ((reinterpret_cast<uintptr_t>(W) & 15u) == 0);
+    MvmJob j{W, xhat, y, m, K, (size_t)K, 0};
+    if (multi_eligible(j)) return launch_gemv_multi(&j, 1, s);
     for (int k0 = 0; k0 < K; k0 += kGemvMaxK) {
         const int kl = K - k0 < kGemvMaxK ? K - k0 : kGemvMaxK;
-        cudaError_t e = vec ? run_gemv<2, 4, true>(W + k0, (size_t)K, m, kl, xhat + k0, y, k0 > 0, s)
-                            : run_gemv<2, 2, false>(W + k0, (size_t)K, m, kl, xhat + k0, y, k0 > 0, s);
+        cudaError_t e = run_gemv<2, 2, false>(W + k0, (size_t)K, m, kl, xhat + k0, y, k0 > 0, s);
         if (e != cudaSuccess) return e;
     }
     return cudaSuccess;

@@ -60,9 +60,26 @@ cudaError_t launch_encode_scan(const void *X, bool x_is_i8, size_t ldx, const ui
 // int8 transpose: out[c][r] = in[r][c] for an R x C matrix.
 cudaError_t launch_transpose_i8(const int8_t *in, int R, int C, int8_t *out, cudaStream_t s);
 
+// One independent batch-1 product y = M x_hat over F_q (M row stride ldw).
+struct MvmJob {
+    const int8_t *W;
+    const uint32_t *xhat;
+    uint32_t *y;
+    int m, K;
+    size_t ldw;
+    int accumulate;  // y += M x_hat instead of y = M x_hat
+};
+constexpr int kMultiMaxJobs = 256;  // jobs per grouped launch
+constexpr int kMultiMaxK = 16384;   // K per grouped launch (longer K is segmented)
+
+// Eligible for the grouped kernel: K % 16 == 0 and 16-byte aligned rows.
+bool multi_eligible(const MvmJob &j);
+// Any number of eligible jobs, in as few launches as K allows.
+cudaError_t launch_gemv_multi(const MvmJob *jobs, int count, cudaStream_t s);
+
 // Batch-1 field GEMV y = M x_hat over F_q.
 cudaError_t launch_gemv(const int8_t *W, int m, int K, const uint32_t *xhat, uint32_t *y,
-                        cudaStream_t s);
+                        uint32_t *err, cudaStream_t s);
 
 // Batched product Y_hat[b] = M x_hat[b] over F_q on the tensor cores.
 cudaError_t launch_batched(const int8_t *W, int m, int K, const uint32_t *Xhat, int B,

@@ -1,17 +1,495 @@
-// Batched field product Y_hat[b] = M x_hat[b] over F_q.
+// Batched field product Y_hat[b] = M x_hat[b] over F_q on the tcgen05 tensor
+// cores (the server's online work at batch > 1, Sec. 6.1).
+//
+// Arithmetic.  Each centred x_hat entry is split into four signed base-256
+// digits d_k in [-128, 127] (x = sum_k 2^(8k) d_k), so
+//     (M x_hat)_i = sum_k 2^(8k) sum_j M_ij d_k[j]        (exact over Z).
+// The inner sums run on the tensor cores as a bf16 GEMM (every int8 weight and
+// every digit is an exact bf16 value) with fp32 accumulation in TMEM.  A
+// product is at most 128 * 128 = 2^14 in magnitude, so a chunk of 1024
+// K-elements sums to at most 2^24: every partial sum is an integer that fp32
+// holds exactly.  After each chunk the epilogue warps read the accumulator,
+// convert it to integers, combine the four digits in int64 and add to a
+// running int64 per output; the result is reduced mod q once at the end.
+// (This GPU generation has no int8 tcgen05 kind, hence bf16 digits.)
+//
+// Tiles.  A CTA owns 128 rows of M (MMA M = 128) and 64 vectors (MMA N = 256:
+// 64 vectors x 4 digits, the digit rows of vector v at N-rows 4v..4v+3).
+// K is split over the CTAs of a thread-block cluster; their int64 partial
+// sums are added through distributed shared memory.
+//
+// Warp roles (320 threads):
+//   warps 0-3  convert the int8 M tile to bf16 in the 128-byte-swizzled
+//              K-major layout the MMA reads (one row per thread);
+//   warps 4-7  epilogue (TMEM lanes 32(w-4)..32(w-4)+31);
+//   warp 8     bulk-copies the pre-tiled digit operand (cp.async.bulk);
+//   warp 9     allocates TMEM and issues the MMAs (one elected lane).
+#include <cooperative_groups.h>
+
 #include "common.cuh"
 #include "launch.h"
 
+namespace cg = cooperative_groups;
+
 namespace pv {
+namespace {
+
+constexpr int kBM = 128;            // rows of M per CTA
+constexpr int kBV = 64;             // vectors per CTA
+constexpr int kBN = 4 * kBV;        // MMA N (digit rows)
+constexpr int kBK = 64;             // K-elements per stage (128 bytes of bf16)
+constexpr int kStages = 4;
+constexpr int kChunkBlocks = 16;    // 16 x 64 = 1024 K-elements per exact chunk
+constexpr int kATile = kBM * kBK * 2;   // 16 KiB
+constexpr int kBTile = kBN * kBK * 2;   // 32 KiB
+constexpr int kStageBytes = kATile + kBTile;
+constexpr int kThreads = 320;
+constexpr int kMmaSmem = kStages * kStageBytes + 1024;  // + alignment slack
+constexpr uint32_t kWaitLimit = 1u << 24;
+
+__device__ __forceinline__ uint32_t smem_addr(const void *p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+// ---------------------------------------------------------------- mbarrier
+__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count));
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
+    uint64_t state;
+    asm volatile("mbarrier.arrive.shared::cta.b64 %0, [%1];"
+                 : "=l"(state)
+                 : "r"(smem_addr(bar))
+                 : "memory");
+    (void)state;
+}
+__device__ __forceinline__ void mbar_arrive_tx(uint64_t *bar, uint32_t bytes) {
+    uint64_t state;
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 %0, [%1], %2;"
+                 : "=l"(state)
+                 : "r"(smem_addr(bar)), "r"(bytes)
+                 : "memory");
+    (void)state;
+}
+__device__ __forceinline__ bool mbar_test(uint64_t *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        " selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(smem_addr(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Bounded wait for the phase of parity `parity`; false (and an error bit) on
+// expiry.
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, uint32_t *err) {
+    for (uint32_t i = 0; i < kWaitLimit; ++i) {
+        if (mbar_test(bar, parity)) return true;
+        if (i > 32) __nanosleep(64);
+    }
+    record_error(err, kErrMmaTimeout);
+    return false;
+}
+
+// ---------------------------------------------------------------- async copies, fences
+__device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+            smem_addr(dst)),
+        "l"(src), "r"(bytes), "r"(smem_addr(bar))
+        : "memory");
+}
+__device__ __forceinline__ void fence_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// ---------------------------------------------------------------- tcgen05
+// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups
+// 1024 bytes apart (stride byte offset), start address in 16-byte units.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
+    d |= (uint64_t)1u << 16;                      // leading byte offset (unused here)
+    d |= (uint64_t)(1024u >> 4) << 32;            // stride byte offset
+    d |= (uint64_t)1u << 46;                      // descriptor version
+    d |= (uint64_t)2u << 61;                      // 128-byte swizzle
+    return d;
+}
+// Instruction descriptor, kind::f16: bf16 A and B, f32 D, both K-major.
+constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kBN >> 3) << 17) |
+                            ((uint32_t)(kBM >> 4) << 24);
+
+__device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                         uint32_t accumulate) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+        "l"(adesc), "l"(bdesc), "r"(kIdesc), "r"(accumulate));
+}
+__device__ __forceinline__ void mma_commit(uint64_t *bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                     smem_addr(bar))
+                 : "memory");
+}
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
+        "%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+          "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+          "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+          "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Byte offset of (row, 16-byte chunk) inside a K-major 128-byte-swizzled tile.
+__device__ __forceinline__ uint32_t sw128_off(uint32_t row, uint32_t chunk) {
+    return (row >> 3) * 1024u + (row & 7u) * 128u + ((chunk ^ (row & 7u)) << 4);
+}
+
+__device__ __forceinline__ uint32_t bf16x2_of_i8(int lo, int hi) {
+    const __nv_bfloat162 v = __floats2bfloat162_rn((float)lo, (float)hi);
+    return *reinterpret_cast<const uint32_t *>(&v);
+}
+
+// ---------------------------------------------------------------- digit operand
+// X_hat (B x K u32) -> pre-tiled bf16 digit operand: for vector tile nt and
+// K-block kb, a 32 KiB block laid out exactly as the MMA's B tile in shared
+// memory.  Zero for vectors >= B and K-elements >= K.  One thread per
+// (vector, 8 K-elements).
+__global__ void __launch_bounds__(256) k_digit_tiles(const uint32_t *__restrict__ Xhat, int B, int K,
+                                                    int nkb, int nvt, uint8_t *__restrict__ D) {
+    const size_t gid = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const size_t per_vec = (size_t)nkb * 8;  // 8-element groups per vector
+    const size_t total = (size_t)nvt * kBV * per_vec;
+    if (gid >= total) return;
+    const int v = (int)(gid / per_vec);
+    const int grp = (int)(gid % per_vec);
+    const int kb = grp >> 3, chunk = grp & 7;
+    const int k0 = kb * kBK + chunk * 8;
+    int d[4][8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+        const int k = k0 + e;
+        if (v < B && k < K) {
+            limb_split(Xhat[(size_t)v * K + k], d[0][e], d[1][e], d[2][e], d[3][e]);
+        } else {
+            d[0][e] = d[1][e] = d[2][e] = d[3][e] = 0;
+        }
+    }
+    const int nt = v / kBV, vl = v % kBV;
+    uint8_t *blk = D + ((size_t)nt * nkb + kb) * kBTile;
+#pragma unroll
+    for (int l = 0; l < 4; ++l) {
+        const uint32_t row = 4 * vl + l;
+        uint4 q;
+        q.x = bf16x2_of_i8(d[l][0], d[l][1]);
+        q.y = bf16x2_of_i8(d[l][2], d[l][3]);
+        q.z = bf16x2_of_i8(d[l][4], d[l][5]);
+        q.w = bf16x2_of_i8(d[l][6], d[l][7]);
+        *reinterpret_cast<uint4 *>(blk + sw128_off(row, chunk)) = q;
+    }
+}
+
+// ---------------------------------------------------------------- main kernel
+template <bool kVec>
+__global__ void __launch_bounds__(kThreads, 1)
+    k_batched(const int8_t *__restrict__ W, int m, int K, const uint8_t *__restrict__ D, int nkb,
+              int B, uint32_t *__restrict__ Yhat, uint32_t *__restrict__ err) {
+    cg::cluster_group cluster = cg::this_cluster();
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ __align__(8) uint64_t full_a[kStages], full_b[kStages], empty_bar[kStages];
+    __shared__ __align__(8) uint64_t acc_full[2], acc_empty[2], mma_done;
+    __shared__ uint32_t s_tmem;
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const uint32_t base = (smem_addr(smem_raw) + 1023u) & ~1023u;
+    uint8_t *smem = smem_raw + (base - smem_addr(smem_raw));
+
+    const int m0 = blockIdx.x * kBM;
+    const int nt = blockIdx.y;
+    const int split = (int)cluster.num_blocks();
+    const int rank = (int)cluster.block_rank();
+    const int per = (nkb + split - 1) / split;
+    const int kb0 = rank * per;
+    const int kb1 = min(nkb, kb0 + per);
+    const int nblk = max(0, kb1 - kb0);
+    const int nchunks = (nblk + kChunkBlocks - 1) / kChunkBlocks;
+
+    if (tid == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(&full_a[s], 128);
+            mbar_init(&full_b[s], 1);
+            mbar_init(&empty_bar[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&acc_full[b], 1);
+            mbar_init(&acc_empty[b], 128);
+        }
+        mbar_init(&mma_done, 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 9) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 512;" ::"r"(
+                         smem_addr(&s_tmem)));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = s_tmem;
+
+    // running int64 sums of the epilogue threads (row = lane of TMEM)
+    long long run[kBV];
+#pragma unroll
+    for (int v = 0; v < kBV; ++v) run[v] = 0;
+
+    if (warp < 4) {
+        // ------------------------------------------------ A: int8 M tile -> bf16 swizzled
+        const int r = tid;  // tile row
+        const int grow = m0 + r;
+        const bool row_ok = grow < m;
+        const int8_t *wrow = W + (size_t)(row_ok ? grow : 0) * K;
+        constexpr int PF = 4;
+        uint4 buf[PF][4];
+        auto load = [&](int i, uint4 (&dst)[4]) {
+            const int k0 = (kb0 + i) * kBK;
+            if (kVec && row_ok && k0 + kBK <= K) {
+#pragma unroll
+                for (int c = 0; c < 4; ++c)
+                    dst[c] = __ldg(reinterpret_cast<const uint4 *>(wrow + k0) + c);
+            } else {
+                uint32_t w[16];
+#pragma unroll
+                for (int q = 0; q < 16; ++q) w[q] = 0;
+                if (row_ok)
+                    for (int e = 0; e < kBK && k0 + e < K; ++e)
+                        w[e >> 2] |= (uint32_t)(uint8_t)wrow[k0 + e] << (8 * (e & 3));
+#pragma unroll
+                for (int c = 0; c < 4; ++c) dst[c] = make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]);
+            }
+        };
+#pragma unroll
+        for (int u = 0; u < PF; ++u)
+            if (u < nblk) load(u, buf[u]);
+        bool ok = true;
+        for (int i0 = 0; i0 < nblk && ok; i0 += PF) {
+#pragma unroll
+            for (int u = 0; u < PF; ++u) {
+                const int i = i0 + u;
+                if (i >= nblk || !ok) break;
+                const int s = i % kStages;
+                const uint32_t ph = (uint32_t)(i / kStages) & 1u;
+                if (!mbar_wait(&empty_bar[s], ph ^ 1u, err)) { ok = false; break; }
+                uint8_t *a = smem + s * kStageBytes;
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {  // 16 int8 -> two 16-byte bf16 chunks
+                    const uint32_t w4[4] = {buf[u][c].x, buf[u][c].y, buf[u][c].z, buf[u][c].w};
+                    uint32_t o[8];
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const int b0 = (int)(int8_t)(w4[q] & 0xff), b1 = (int)(int8_t)((w4[q] >> 8) & 0xff);
+                        const int b2 = (int)(int8_t)((w4[q] >> 16) & 0xff), b3 = (int)(int8_t)(w4[q] >> 24);
+                        o[2 * q] = bf16x2_of_i8(b0, b1);
+                        o[2 * q + 1] = bf16x2_of_i8(b2, b3);
+                    }
+                    *reinterpret_cast<uint4 *>(a + sw128_off(r, 2 * c)) = make_uint4(o[0], o[1], o[2], o[3]);
+                    *reinterpret_cast<uint4 *>(a + sw128_off(r, 2 * c + 1)) = make_uint4(o[4], o[5], o[6], o[7]);
+                }
+                fence_async_smem();
+                mbar_arrive(&full_a[s]);
+                if (i + PF < nblk) load(i + PF, buf[u]);
+            }
+        }
+    } else if (warp < 8) {
+        // ------------------------------------------------ epilogue: TMEM -> int64 sums
+        const int q = warp - 4;  // TMEM lane quadrant
+        for (int c = 0; c < nchunks; ++c) {
+            const int bsel = c & 1;
+            if (!mbar_wait(&acc_full[bsel], (uint32_t)(c >> 1) & 1u, err)) break;
+            tc_fence_after();
+#pragma unroll
+            for (int j = 0; j < kBN / 32; ++j) {
+                uint32_t r[32];
+                tmem_ld32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(bsel * kBN + 32 * j), r);
+#pragma unroll
+                for (int v = 0; v < 8; ++v) {
+                    const long long d0 = __float2int_rn(__uint_as_float(r[4 * v]));
+                    const long long d1 = __float2int_rn(__uint_as_float(r[4 * v + 1]));
+                    const long long d2 = __float2int_rn(__uint_as_float(r[4 * v + 2]));
+                    const long long d3 = __float2int_rn(__uint_as_float(r[4 * v + 3]));
+                    run[8 * j + v] += d0 + (d1 << 8) + (d2 << 16) + (d3 << 24);
+                }
+            }
+            tc_fence_before();
+            mbar_arrive(&acc_empty[bsel]);
+        }
+    } else if (warp == 8) {
+        // ------------------------------------------------ B: bulk copies of digit tiles
+        if (lane == 0) {
+            const uint8_t *src = D + ((size_t)nt * nkb + kb0) * kBTile;
+            int issued = 0;
+            for (int i = 0; i < nblk; ++i) {
+                const int s = i % kStages;
+                const uint32_t ph = (uint32_t)(i / kStages) & 1u;
+                if (!mbar_wait(&empty_bar[s], ph ^ 1u, err)) break;
+                uint8_t *b = smem + s * kStageBytes + kATile;
+                mbar_arrive_tx(&full_b[s], kBTile);
+                bulk_g2s(b, src + (size_t)i * kBTile, kBTile, &full_b[s]);
+                issued = i + 1;
+            }
+            // copies in flight complete before the CTA may exit
+            for (int i = max(0, issued - kStages); i < issued; ++i)
+                mbar_wait(&full_b[i % kStages], (uint32_t)(i / kStages) & 1u, err);
+        }
+    } else {
+        // ------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            bool ok = true;
+            for (int c = 0; c < nchunks && ok; ++c) {
+                const int bsel = c & 1;
+                if (!mbar_wait(&acc_empty[bsel], ((uint32_t)(c >> 1) & 1u) ^ 1u, err)) break;
+                tc_fence_after();
+                const uint32_t dcol = tmem + (uint32_t)(bsel * kBN);
+                const int i_end = min(nblk, (c + 1) * kChunkBlocks);
+                for (int i = c * kChunkBlocks; i < i_end; ++i) {
+                    const int s = i % kStages;
+                    const uint32_t ph = (uint32_t)(i / kStages) & 1u;
+                    if (!mbar_wait(&full_a[s], ph, err) || !mbar_wait(&full_b[s], ph, err)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t a_addr = base + (uint32_t)(s * kStageBytes);
+                    const uint32_t b_addr = a_addr + kATile;
+#pragma unroll
+                    for (int k = 0; k < kBK / 16; ++k) {
+                        mma_bf16(dcol, sw128_desc(a_addr + 32u * k), sw128_desc(b_addr + 32u * k),
+                                 (i > c * kChunkBlocks || k > 0) ? 1u : 0u);
+                    }
+                    mma_commit(&empty_bar[s]);
+                }
+                mma_commit(&acc_full[bsel]);
+            }
+            // all issued MMAs have finished before TMEM is released
+            mma_commit(&mma_done);
+            mbar_wait(&mma_done, 0, err);
+        }
+    }
+
+    // ---------------------------------------------------- split-K reduction and store
+    tc_fence_before();
+    __syncthreads();  // every stage is consumed: the stage memory is reused below
+    long long *part = reinterpret_cast<long long *>(smem);  // [kBV][kBM]
+    if (warp >= 4 && warp < 8) {
+        const int row = tid - 128;
+#pragma unroll
+        for (int v = 0; v < kBV; ++v) part[v * kBM + row] = run[v];
+    }
+    cluster.sync();
+    if (rank == 0 && warp >= 4 && warp < 8) {
+        const int row = tid - 128;
+        const int grow = m0 + row;
+        for (int v = 0; v < kBV; ++v) {
+            long long s = part[v * kBM + row];
+            for (int r = 1; r < split; ++r) s += cluster.map_shared_rank(part, r)[v * kBM + row];
+            const int b = nt * kBV + v;
+            if (grow < m && b < B) Yhat[(size_t)b * m + grow] = fred_signed(s);
+        }
+    }
+    cluster.sync();
+    if (warp == 9) {
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem));
+    }
+}
+
+// ---------------------------------------------------------------- scratch for the digit operand
+struct Scratch {
+    uint8_t *ptr = nullptr;
+    size_t bytes = 0;
+};
+
+cudaError_t digit_scratch(size_t need, uint8_t **out) {
+    static Scratch per_dev[64];
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    Scratch &s = per_dev[dev];
+    if (s.bytes < need) {
+        if (s.ptr) {
+            e = cudaDeviceSynchronize();  // the old buffer may still be in use
+            if (e != cudaSuccess) return e;
+            cudaFree(s.ptr);
+            s.ptr = nullptr;
+            s.bytes = 0;
+        }
+        e = cudaMalloc(&s.ptr, need);
+        if (e != cudaSuccess) return e;
+        s.bytes = need;
+    }
+    *out = s.ptr;
+    return cudaSuccess;
+}
+
+}  // namespace
 
 cudaError_t launch_batched(const int8_t *W, int m, int K, const uint32_t *Xhat, int B,
                            uint32_t *Yhat, uint32_t *err, cudaStream_t s) {
-    (void)err;
-    for (int b = 0; b < B; ++b) {
-        cudaError_t e = launch_gemv(W, m, K, Xhat + (size_t)b * K, Yhat + (size_t)b * m, s);
-        if (e != cudaSuccess) return e;
+    if (m <= 0 || K <= 0 || B <= 0) return cudaSuccess;
+    const int nkb = (K + kBK - 1) / kBK;
+    const int nvt = (B + kBV - 1) / kBV;
+    const size_t need = (size_t)nvt * nkb * kBTile;
+    uint8_t *D = nullptr;
+    cudaError_t e = digit_scratch(need, &D);
+    if (e != cudaSuccess) return e;
+    {
+        const size_t threads = (size_t)nvt * kBV * nkb * 8;
+        k_digit_tiles<<<(unsigned)((threads + 255) / 256), 256, 0, s>>>(Xhat, B, K, nkb, nvt, D);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
-    return cudaSuccess;
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int mt = (m + kBM - 1) / kBM;
+    const int tiles = mt * nvt;
+    // split K over a cluster until the grid covers the GPU (and each CTA keeps
+    // at least one exact 1024-element chunk of work)
+    int split = 1;
+    while (split < 8 && tiles * split < sms && nkb / (2 * split) >= kChunkBlocks / 2) split *= 2;
+
+    const bool vec = (K % 16 == 0) && ((reinterpret_cast<uintptr_t>(W) & 15u) == 0);
+    auto kern = vec ? k_batched<true> : k_batched<false>;
+    static const cudaError_t a1 =
+        cudaFuncSetAttribute(k_batched<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
+    static const cudaError_t a2 =
+        cudaFuncSetAttribute(k_batched<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
+    if (a1 != cudaSuccess) return a1;
+    if (a2 != cudaSuccess) return a2;
+
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(mt, nvt, split);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = kMmaSmem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 1;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = split;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, W, m, K, (const uint8_t *)D, nkb, B, Yhat, err);
 }
 
 }  // namespace pv

@@ -273,3 +273,32 @@ def test_config5_70b(pv, wl, name):
     m, K = wl.LAYER_70B[name]
     W = wl.weights_gaussian(m, K, (5, list(wl.LAYER_70B).index(name)))
     _batched_pipeline_sampled(pv, W, 256, seed=500 + len(name), n_rows=12, n_verify=1)
+
+
+def test_server_mvm_multi_mixed_jobs(pv, wl):
+    """Grouped batch-1 products over mixed shapes, including K beyond one
+    segment (20000), a K that is not a multiple of 16 (1001) and tiny matrices; equal to the
+    single calls and to the oracle."""
+    import torch
+    rng = np.random.default_rng(7)
+    shapes = [(4096, 4096), (1024, 4096), (300, 20000), (17, 1001), (5, 16), (64, 48), (2048, 14336)]
+    W = [rng.integers(-128, 128, size=s, dtype=np.int8) for s in shapes]
+    X = [rng.integers(0, Q, size=s[1]).astype(np.uint32) for s in shapes]
+    Wd = [to_dev(w) for w in W]
+    Xd = [to_dev(x) for x in X]
+    Yd = [torch.empty(s[0], dtype=torch.int32, device="cuda") for s in shapes]
+    pv.pvmvmd_server_mvm_multi(list(zip(Wd, Xd, Yd)))
+    for i, s in enumerate(shapes):
+        single = pv.as_u32(pv.pvmvmd_server_mvm(Wd[i], Xd[i]))
+        got = pv.as_u32(Yd[i])
+        assert np.array_equal(got, single), s
+        rows = sample_rows(s[0], 32, i)
+        assert np.array_equal(got[rows], oracle.server_mvm_rows(W[i], X[i], rows)), s
+    # many jobs (more than one launch's worth) on replicas of one matrix
+    Wr = Wd[4]
+    Xs = to_dev(rng.integers(0, Q, size=(300, 16)).astype(np.uint32))
+    Ys = torch.empty((300, 5), dtype=torch.int32, device="cuda")
+    pv.pvmvmd_server_mvm_multi([(Wr, Xs[b], Ys[b]) for b in range(300)])
+    Xs_h = pv.as_u32(Xs)
+    assert np.array_equal(pv.as_u32(Ys), np.stack([oracle.server_mvm(W[4], Xs_h[b]) for b in range(300)]))
+    assert pv.pvmvmd_device_status() == 0
