@@ -148,6 +148,32 @@ typedef struct {
  * 1 <= count, each 1 <= K <= PVMVMD_MAX_K, 1 <= m. */
 int pvmvmd_server_mvm_multi(const pvmvmd_mvm_job *jobs, int count, void *stream);
 
+/* Size of the fixed device buffer behind pvmvmd_server_mvm_noalloc. */
+#define PVMVMD_NOALLOC_SCRATCH_BYTES (16u << 20)
+
+/* The server's product Y_hat = M X_hat over F_q, like pvmvmd_server_mvm, but
+ * without any memory allocation inside the call.  The paper has no
+ * counterpart: this entry point exists for callers that cannot let the
+ * library call cudaMalloc -- for instance a serving process whose device
+ * memory is reserved up front by its own allocator or pool (a cudaMalloc
+ * from inside the library could fail or fragment that pool), or a
+ * latency-critical loop that cannot afford the regular call's first-use
+ * allocation, or the device-wide synchronisation of replacing an outgrown
+ * buffer.  It always runs the tensor-core digit product (also for B = 1),
+ * whose bf16 digit tiles then live in one file-scope __device__ array of
+ * PVMVMD_NOALLOC_SCRATCH_BYTES (16 MiB) that every GPU which loads the
+ * library holds until the process exits.  The tiles take
+ * ceil(B/64) * ceil(K/64) * 32 KiB, so for example B <= 64 allows
+ * K <= 32768 and B <= 256 allows K <= 8192; a larger problem returns
+ * PVMVMD_E_SHAPE and does nothing.  The first call on each device looks up
+ * the array's device address (cudaGetSymbolAddress) with that device
+ * current; make that first call before any stream capture.  All calls share
+ * the one array, so calls that overlap on the GPU (e.g. on two streams) race
+ * and give wrong results; order them on one stream.  Arguments and results
+ * are those of pvmvmd_server_mvm. */
+int pvmvmd_server_mvm_noalloc(const int8_t *W_dev, int m, int K, const uint32_t *Xhat_dev, int B,
+                              uint32_t *Yhat_dev, void *stream);
+
 /* Verify and Decrypt (Protocol 3).  Verify: ell challenges e_q <- E_{t_y}^{N_y}
  * are drawn from challenge_key (repetition q reads nonce (10, 2q) and
  * (10, 2q+1)) and shared by all B vectors of the call, as Sec. 5.4 allows;

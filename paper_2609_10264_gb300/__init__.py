@@ -21,6 +21,7 @@ LIB_PATH = os.path.join(_PKG, "libpvmvmd.so")
 PVMVMD_Q = 2013265921
 PVMVMD_MAX_K = 131071
 PVMVMD_MAX_T = 4096
+PVMVMD_NOALLOC_SCRATCH_BYTES = 16 << 20
 PVMVMD_OK = 0
 PVMVMD_E_ARG = -1
 PVMVMD_E_SHAPE = -2
@@ -75,6 +76,7 @@ SIGNATURES = {
     "pvmvmd_encode": (_i, [_vp, _vp, _i, ctypes.POINTER(pvmvmd_key), _vp, _vp, _vp]),
     "pvmvmd_server_mvm": (_i, [_vp, _i, _i, _vp, _i, _vp, _vp]),
     "pvmvmd_server_mvm_multi": (_i, [ctypes.POINTER(pvmvmd_mvm_job), _i, _vp]),
+    "pvmvmd_server_mvm_noalloc": (_i, [_vp, _i, _i, _vp, _i, _vp, _vp]),
     "pvmvmd_decode_verify": (_i, [_vp, _vp, _vp, _vp, _i, ctypes.POINTER(pvmvmd_key), _vp, _vp, _vp]),
     "pvmvmd_device_status": (_i, [_vp]),
     "pvmvmd_ctx_info": (_i, [_vp, ctypes.POINTER(pvmvmd_ctx_view)]),
@@ -265,6 +267,20 @@ def pvmvmd_server_mvm(W, Xhat, Yhat=None, stream=None):
                                   B, _dev_ptr(Yhat, "Yhat", _u32_types(), B * m), _stream_ptr(stream)),
            "pvmvmd_server_mvm")
     return Yhat
+
+
+def pvmvmd_server_mvm_noalloc(W, Xhat, Yhat, stream=None) -> None:
+    """Y_hat = M X_hat like pvmvmd_server_mvm, for callers that cannot let the
+    library allocate device memory: the call allocates nothing (the caller
+    passes the output) and uses the library's fixed 16 MiB device buffer,
+    shared by all such calls (order them on one stream)."""
+    import torch
+    m, K = W.shape
+    B = _batch(Xhat, K, "Xhat")
+    _check(_lib.pvmvmd_server_mvm_noalloc(_dev_ptr(W, "W", (torch.int8,)), m, K,
+                                          _dev_ptr(Xhat, "Xhat", _u32_types()), B,
+                                          _dev_ptr(Yhat, "Yhat", _u32_types(), B * m), _stream_ptr(stream)),
+           "pvmvmd_server_mvm_noalloc")
 
 
 def mvm_jobs(triples):

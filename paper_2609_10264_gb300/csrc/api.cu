@@ -256,6 +256,9 @@ int read_and_clear_error() {
 }
 
 }  // namespace
+
+uint32_t *library_error_word() { return error_word(); }
+
 }  // namespace pv
 
 using namespace pv;

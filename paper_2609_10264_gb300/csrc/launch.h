@@ -85,6 +85,9 @@ cudaError_t launch_gemv(const int8_t *W, int m, int K, const uint32_t *xhat, uin
 cudaError_t launch_batched(const int8_t *W, int m, int K, const uint32_t *Xhat, int B,
                            uint32_t *Yhat, uint32_t *err, cudaStream_t s);
 
+// The library's device error word on the current device (null on failure).
+uint32_t *library_error_word();
+
 // Verify part 1: u[q][k] = sum_j e_{q,j} Q[supp_{q,j}][k] (e_q^T Q).
 cudaError_t launch_verify_u(const uint32_t *Qm, int K, const uint32_t *chal, uint32_t t_y,
                             uint32_t ell, uint32_t *u, cudaStream_t s);

@@ -26,6 +26,8 @@
 //   warp 9     allocates TMEM and issues the MMAs (one elected lane).
 #include <cooperative_groups.h>
 
+#include <mutex>
+
 #include "common.cuh"
 #include "launch.h"
 
@@ -493,3 +495,93 @@ cudaError_t launch_batched(const int8_t *W, int m, int K, const uint32_t *Xhat, 
 }
 
 }  // namespace pv
+
+// ---------------------------------------------------------------------------
+// pvmvmd_server_mvm_noalloc: the batched product with its digit tiles in a
+// fixed file-scope device array instead of a buffer the library allocates.
+// ---------------------------------------------------------------------------
+namespace pv {
+namespace {
+
+constexpr size_t kNoAllocBytes = PVMVMD_NOALLOC_SCRATCH_BYTES;
+static __device__ __align__(256) uint8_t g_noalloc_tiles[kNoAllocBytes];
+
+// Device address of g_noalloc_tiles on the current device.  Host code may
+// not use the symbol itself (its host-side name is only a stand-in), so it is
+// looked up once per device, with that device current.
+cudaError_t noalloc_tiles(uint8_t **out) {
+    static std::mutex mu;
+    static uint8_t *addr[64] = {nullptr};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!addr[dev]) {
+        void *p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_noalloc_tiles);
+        if (e != cudaSuccess) return e;
+        addr[dev] = static_cast<uint8_t *>(p);
+    }
+    *out = addr[dev];
+    return cudaSuccess;
+}
+
+}  // namespace
+}  // namespace pv
+
+extern "C" int pvmvmd_server_mvm_noalloc(const int8_t *W_dev, int m, int K, const uint32_t *Xhat_dev,
+                                         int B, uint32_t *Yhat_dev, void *stream) {
+    using namespace pv;
+    if (!W_dev || !Xhat_dev || !Yhat_dev) return PVMVMD_E_ARG;
+    if (m < 1 || K < 1 || K > PVMVMD_MAX_K || B < 1) return PVMVMD_E_SHAPE;
+    const int nkb = (K + kBK - 1) / kBK;
+    const int nvt = (B + kBV - 1) / kBV;
+    const size_t need = (size_t)nvt * nkb * kBTile;
+    if (need > kNoAllocBytes) return PVMVMD_E_SHAPE;  // beyond the fixed buffer
+    uint8_t *D = nullptr;
+    if (noalloc_tiles(&D) != cudaSuccess) return PVMVMD_E_CUDA;
+    uint32_t *err = library_error_word();
+    if (!err) return PVMVMD_E_CUDA;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+
+    // every byte of the tiles in use is rewritten: nothing left by an
+    // earlier call is read
+    const size_t threads = (size_t)nvt * kBV * nkb * 8;
+    k_digit_tiles<<<(unsigned)((threads + 255) / 256), 256, 0, s>>>(Xhat_dev, B, K, nkb, nvt, D);
+    if (cudaGetLastError() != cudaSuccess) return PVMVMD_E_CUDA;
+
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return PVMVMD_E_CUDA;
+    const int mt = (m + kBM - 1) / kBM;
+    const int tiles = mt * nvt;
+    int split = 1;
+    while (split < 8 && tiles * split < sms && nkb / (2 * split) >= kChunkBlocks / 2) split *= 2;
+    const bool vec = (K % 16 == 0) && ((reinterpret_cast<uintptr_t>(W_dev) & 15u) == 0);
+    auto kern = vec ? k_batched<true> : k_batched<false>;
+    static const cudaError_t a1 =
+        cudaFuncSetAttribute(k_batched<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
+    static const cudaError_t a2 =
+        cudaFuncSetAttribute(k_batched<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
+    if (a1 != cudaSuccess || a2 != cudaSuccess) return PVMVMD_E_CUDA;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(mt, nvt, split);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = kMmaSmem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 1;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = split;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (cudaLaunchKernelEx(&cfg, kern, W_dev, m, K, (const uint8_t *)D, nkb, B, Yhat_dev, err) !=
+        cudaSuccess) {
+        (void)cudaGetLastError();
+        return PVMVMD_E_CUDA;
+    }
+    return PVMVMD_OK;
+}
