@@ -159,6 +159,7 @@ cudaError_t dev_alloc(T **p, size_t count) {
 struct CodeDev {
     uint32_t *pi1 = nullptr, *pi2 = nullptr, *v1 = nullptr, *v2 = nullptr;
     uint32_t *pi1inv = nullptr, *pi2inv = nullptr, *v2p = nullptr;
+    uint32_t *v2m = nullptr, *v1pm = nullptr;  // Montgomery-scaled v2 and v1 o pi1^-1
 };
 
 }  // namespace
@@ -187,16 +188,20 @@ cudaError_t ctx_alloc(pvmvmd_ctx *c, T **p, size_t count) {
 
 int upload_code(pvmvmd_ctx *c, CodeDev &d, const pvmvmd_key &key, int which, uint32_t N,
                 cudaStream_t s) {
-    std::vector<uint32_t> pi1(N), pi2(N), v1(N), v2(N), pi1inv(N), pi2inv(N), v2p(N);
+    std::vector<uint32_t> pi1(N), pi2(N), v1(N), v2(N), pi1inv(N), pi2inv(N), v2p(N), v2m(N), v1pm(N);
     sample_code_host(key, which, N, pi1.data(), pi2.data(), v1.data(), v2.data());
     for (uint32_t j = 0; j < N; ++j) {
         pi1inv[pi1[j]] = j;
         pi2inv[pi2[j]] = j;
     }
-    for (uint32_t i = 0; i < N; ++i) v2p[i] = v2[pi2inv[i]];
-    uint32_t **dst[7] = {&d.pi1, &d.pi2, &d.v1, &d.v2, &d.pi1inv, &d.pi2inv, &d.v2p};
-    const std::vector<uint32_t> *src[7] = {&pi1, &pi2, &v1, &v2, &pi1inv, &pi2inv, &v2p};
-    for (int i = 0; i < 7; ++i) {
+    for (uint32_t i = 0; i < N; ++i) {
+        v2p[i] = v2[pi2inv[i]];
+        v2m[i] = to_mont(v2[i]);
+        v1pm[i] = to_mont(v1[pi1inv[i]]);
+    }
+    uint32_t **dst[9] = {&d.pi1, &d.pi2, &d.v1, &d.v2, &d.pi1inv, &d.pi2inv, &d.v2p, &d.v2m, &d.v1pm};
+    const std::vector<uint32_t> *src[9] = {&pi1, &pi2, &v1, &v2, &pi1inv, &pi2inv, &v2p, &v2m, &v1pm};
+    for (int i = 0; i < 9; ++i) {
         PV_CUDA(ctx_alloc(c, dst[i], N));
         PV_CUDA(cudaMemcpyAsync(*dst[i], src[i]->data(), (size_t)N * 4, cudaMemcpyHostToDevice, s));
     }
@@ -408,6 +413,16 @@ int pvmvmd_encode(pvmvmd_ctx *ctx, const uint32_t *X_dev, int B, const pvmvmd_ke
     if (!err) return PVMVMD_E_CUDA;
     uint32_t *stp = static_cast<uint32_t *>(st_dev);
     const CodeDev &d = ctx->gx;
+    int C;
+    uint32_t slice;
+    size_t smem;
+    if (syndrome_fused_plan(ctx->Nx, ctx->t_x, &C, &slice, &smem)) {
+        // sample, scan and gather in one launch per batch, no scratch
+        PV_CUDA(launch_syndrome_fused(*key, kTagMask, 0, ctx->Nx, ctx->t_x, (uint32_t)B, d.pi2inv,
+                                      d.v2p, d.v1, d.pi1inv, d.pi2, d.v2m, d.v1pm, ctx->K, ctx->rate,
+                                      stp, X_dev, Xhat_dev, s));
+        return PVMVMD_OK;
+    }
     for (int b0 = 0; b0 < B; b0 += ctx->sb) {
         const uint32_t nb = (uint32_t)(B - b0 < ctx->sb ? B - b0 : ctx->sb);
         uint32_t *e = stp + (size_t)b0 * 2 * ctx->t_x;
@@ -472,12 +487,21 @@ int pvmvmd_decode_verify(pvmvmd_ctx *ctx, const void *st_dev, const uint32_t *Xh
     if (!err) return PVMVMD_E_CUDA;
     const CodeDev &d = ctx->gy;
     // Challenges e_q <- E_{t_y}^{N_y}, shared by the B vectors; g_q = G_y e_q.
-    PV_CUDA(launch_sample_sparse(*challenge_key, kTagChallenge, 0, ctx->Ny, ctx->t_y, ctx->ell,
-                                 ctx->chal, ctx->status, scan_status_words(ctx->Ny, ctx->ell), s));
-    PV_CUDA(launch_syndrome_scan(d.pi2inv, d.v2p, d.v1, ctx->Ny, ctx->chal, ctx->t_y, ctx->ell,
-                                 ctx->Fy, ctx->status, err, s));
-    PV_CUDA(launch_syndrome_gather(d.pi1inv, ctx->m, ctx->rate, ctx->Fy, ctx->Ny, nullptr, ctx->g,
-                                   ctx->ell, s));
+    int C;
+    uint32_t slice;
+    size_t smem;
+    if (syndrome_fused_plan(ctx->Ny, ctx->t_y, &C, &slice, &smem)) {
+        PV_CUDA(launch_syndrome_fused(*challenge_key, kTagChallenge, 0, ctx->Ny, ctx->t_y,
+                                      (uint32_t)ctx->ell, d.pi2inv, d.v2p, d.v1, d.pi1inv, d.pi2,
+                                      d.v2m, d.v1pm, ctx->m, ctx->rate, ctx->chal, nullptr, ctx->g, s));
+    } else {
+        PV_CUDA(launch_sample_sparse(*challenge_key, kTagChallenge, 0, ctx->Ny, ctx->t_y, ctx->ell,
+                                     ctx->chal, ctx->status, scan_status_words(ctx->Ny, ctx->ell), s));
+        PV_CUDA(launch_syndrome_scan(d.pi2inv, d.v2p, d.v1, ctx->Ny, ctx->chal, ctx->t_y, ctx->ell,
+                                     ctx->Fy, ctx->status, err, s));
+        PV_CUDA(launch_syndrome_gather(d.pi1inv, ctx->m, ctx->rate, ctx->Fy, ctx->Ny, nullptr, ctx->g,
+                                       ctx->ell, s));
+    }
     // u_q = e_q^T Q.
     PV_CUDA(launch_verify_u(ctx->Q, ctx->K, ctx->chal, ctx->t_y, ctx->ell, ctx->u, s));
     PV_CUDA(launch_decode_verify(ctx->PT, ctx->m, ctx->K, static_cast<const uint32_t *>(st_dev),

@@ -33,10 +33,45 @@ __host__ __device__ __forceinline__ uint32_t fadd(uint32_t a, uint32_t b) {
 __host__ __device__ __forceinline__ uint32_t fsub(uint32_t a, uint32_t b) {
     return a >= b ? a - b : a + (kQ - b);
 }
-__host__ __device__ __forceinline__ uint32_t fred(uint64_t v) { return (uint32_t)(v % kQ); }
+// x mod q for any 64-bit x.  On the device by Barrett reduction (Barrett,
+// CRYPTO 1986): with mu = floor(2^64 / q), est = floor(x mu / 2^64) is
+// floor(x / q) or one less (the error x (2^64/q - mu) / 2^64 is below 1), so
+// x - est q lies in [0, 2q) and one conditional subtraction finishes.
+constexpr uint64_t kBarrettMu = 0xFFFFFFFFFFFFFFFFull / PVMVMD_Q;  // = floor(2^64 / q), q odd
+__host__ __device__ __forceinline__ uint32_t fred(uint64_t v) {
+#ifdef __CUDA_ARCH__
+    const uint64_t est = __umul64hi(v, kBarrettMu);
+    const uint64_t r = v - est * kQ;
+    return (uint32_t)(r >= kQ ? r - kQ : r);
+#else
+    return (uint32_t)(v % kQ);
+#endif
+}
 __host__ __device__ __forceinline__ uint32_t fmul(uint32_t a, uint32_t b) {
     return fred((uint64_t)a * b);
 }
+// Montgomery multiplication with R = 2^32 (Montgomery, Math. Comp. 1985):
+// for a < q and b < q, mont(a, b) = a b R^-1 mod q.  With b_m = b R mod q
+// stored in a table, mont(a, b_m) = a b, the canonical product, in a few
+// integer instructions: t = a b_m; m = -t q^-1 mod 2^32; (t + m q) / 2^32 < 2q.
+constexpr uint32_t qinv_mod_2_32() {
+    uint32_t x = PVMVMD_Q;  // Newton: each step doubles the correct low bits
+    for (int i = 0; i < 5; ++i) x *= 2u - PVMVMD_Q * x;
+    return x;
+}
+constexpr uint32_t kQInvNeg = 0u - qinv_mod_2_32();
+static_assert(PVMVMD_Q * qinv_mod_2_32() == 1u, "q^-1 mod 2^32");
+__host__ __device__ __forceinline__ uint32_t fmul_mont(uint32_t a, uint32_t b_m) {
+    const uint64_t t = (uint64_t)a * b_m;
+    const uint32_t m = (uint32_t)t * kQInvNeg;
+    const uint64_t u = (t + (uint64_t)m * kQ) >> 32;  // t + m q < 2^62 + 2^63
+    return (uint32_t)(u >= kQ ? u - kQ : u);
+}
+// b -> b R mod q (host table preparation).
+__host__ __device__ __forceinline__ uint32_t to_mont(uint32_t b) {
+    return (uint32_t)(((uint64_t)b << 32) % kQ);
+}
+
 // Signed 64-bit integer -> canonical representative.
 __host__ __device__ __forceinline__ uint32_t fred_signed(int64_t v) {
     int64_t r = v % (int64_t)kQ;

@@ -30,35 +30,31 @@ __device__ __forceinline__ uint4 ldg4(const uint32_t *p) {
 
 __global__ void __launch_bounds__(256) k_verify_u(const uint32_t *__restrict__ Qm, int K,
                                                  const uint32_t *__restrict__ chal, uint32_t t,
-                                                 uint32_t *__restrict__ u, bool vec) {
+                                                 uint32_t *__restrict__ u) {
     extern __shared__ uint32_t sm[];
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    asm volatile("griddepcontrol.wait;" ::: "memory");  // the challenges come from the kernel before
     const uint32_t q = blockIdx.y;
     const uint32_t *c = chal + (size_t)q * 2 * t;
     for (uint32_t j = threadIdx.x; j < 2 * t; j += blockDim.x) sm[j] = c[j];
     __syncthreads();
-    const int k0 = (blockIdx.x * blockDim.x + threadIdx.x) * 4;
-    if (k0 >= K) return;
-    uint64_t a0 = 0, a1 = 0, a2 = 0, a3 = 0;
-    for (uint32_t j = 0; j < t; ++j) {
-        const uint32_t *row = Qm + (size_t)sm[j] * K + k0;
-        const uint64_t e = sm[t + j];
-        uint4 v;
-        if (vec) {
-            v = ldg4(row);
-        } else {
-            v.x = row[0];
-            v.y = k0 + 1 < K ? row[1] : 0u;
-            v.z = k0 + 2 < K ? row[2] : 0u;
-            v.w = k0 + 3 < K ? row[3] : 0u;
-        }
-        a0 += e * v.x; a1 += e * v.y; a2 += e * v.z; a3 += e * v.w;
-        if ((j & 3) == 3) { a0 %= kQ; a1 %= kQ; a2 %= kQ; a3 %= kQ; }
+    const int k = blockIdx.x * blockDim.x + threadIdx.x;
+    if (k >= K) return;
+    uint64_t acc = 0;
+    uint32_t j = 0;
+    for (; j + 8 <= t; j += 8) {
+        uint32_t v[8];
+#pragma unroll
+        for (int s2 = 0; s2 < 8; ++s2) v[s2] = __ldg(Qm + (size_t)sm[j + s2] * K + k);
+#pragma unroll
+        for (int s2 = 0; s2 < 4; ++s2) acc += (uint64_t)sm[t + j + s2] * v[s2];
+        acc = fred(acc);
+#pragma unroll
+        for (int s2 = 4; s2 < 8; ++s2) acc += (uint64_t)sm[t + j + s2] * v[s2];
+        acc = fred(acc);
     }
-    uint32_t *uo = u + (size_t)q * K + k0;
-    uo[0] = fred(a0);
-    if (k0 + 1 < K) uo[1] = fred(a1);
-    if (k0 + 2 < K) uo[2] = fred(a2);
-    if (k0 + 3 < K) uo[3] = fred(a3);
+    for (; j < t; ++j) acc = fred(acc + (uint64_t)sm[t + j] * __ldg(Qm + (size_t)sm[j] * K + k));
+    u[(size_t)q * K + k] = (uint32_t)acc;
 }
 
 __device__ __forceinline__ uint32_t warp_fsum(uint32_t v) {
@@ -81,8 +77,13 @@ __global__ void __launch_bounds__(kDecThreads) k_decode_verify(
     const uint32_t C = cluster.num_blocks();
     const size_t b = blockIdx.y;
 
+    // Inputs of this kernel (P^T, st, x_hat, y_hat) were written before the
+    // challenge kernels that precede it in the stream; g and u come from
+    // those kernels, so they are read only after griddepcontrol.wait.
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const uint32_t *stb = st + b * 2 * t_x;
     for (uint32_t j = tid; j < 2 * t_x; j += kDecThreads) sm[j] = stb[j];
+    uint32_t *ystage = sm + 2 * t_x;  // this CTA's y_hat columns (y may alias y_hat)
     __syncthreads();
     const uint32_t *supp = sm, *vals = sm + t_x;
 
@@ -99,6 +100,30 @@ __global__ void __launch_bounds__(kDecThreads) k_decode_verify(
     for (int i = c0 + tid * 4; i < c1; i += kDecThreads * 4) {
         uint64_t a0 = 0, a1 = 0, a2 = 0, a3 = 0;
         uint32_t j = 0;
+        for (; j + 8 <= t_x; j += 8) {
+            uint4 v[8];
+#pragma unroll
+            for (int s = 0; s < 8; ++s) {
+                const uint32_t *row = PT + (size_t)supp[j + s] * m + i;
+                if (vec) {
+                    v[s] = ldg4(row);
+                } else {
+                    v[s].x = row[0];
+                    v[s].y = i + 1 < c1 ? row[1] : 0u;
+                    v[s].z = i + 2 < c1 ? row[2] : 0u;
+                    v[s].w = i + 3 < c1 ? row[3] : 0u;
+                }
+            }
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+#pragma unroll
+                for (int s = 4 * h; s < 4 * h + 4; ++s) {
+                    const uint64_t e = vals[j + s];
+                    a0 += e * v[s].x; a1 += e * v[s].y; a2 += e * v[s].z; a3 += e * v[s].w;
+                }
+                a0 = fred(a0); a1 = fred(a1); a2 = fred(a2); a3 = fred(a3);
+            }
+        }
         for (; j + 4 <= t_x; j += 4) {
             uint4 v[4];
 #pragma unroll
@@ -118,7 +143,7 @@ __global__ void __launch_bounds__(kDecThreads) k_decode_verify(
                 const uint64_t e = vals[j + s];
                 a0 += e * v[s].x; a1 += e * v[s].y; a2 += e * v[s].z; a3 += e * v[s].w;
             }
-            a0 %= kQ; a1 %= kQ; a2 %= kQ; a3 %= kQ;
+            a0 = fred(a0); a1 = fred(a1); a2 = fred(a2); a3 = fred(a3);
         }
         for (; j < t_x; ++j) {
             const uint32_t *row = PT + (size_t)supp[j] * m + i;
@@ -134,11 +159,21 @@ __global__ void __launch_bounds__(kDecThreads) k_decode_verify(
             const int col = i + s;
             if (col < c1) {
                 const uint32_t yv = yh[col];
+                ystage[col - c0] = yv;
                 yo[col] = fsub(yv, pe[s]);
-                for (uint32_t q = 0; q < ell; ++q) racc[q] += (uint64_t)g[(size_t)q * m + col] * yv;
             }
         }
-        for (uint32_t q = 0; q < ell; ++q) racc[q] %= kQ;
+    }
+    __syncthreads();
+    asm volatile("griddepcontrol.wait;" ::: "memory");  // g and u are complete from here on
+    int cnty = 0;
+    for (int col = c0 + tid; col < c1; col += kDecThreads) {
+        const uint64_t yv = ystage[col - c0];
+        for (uint32_t q = 0; q < ell; ++q) racc[q] += (uint64_t)g[(size_t)q * m + col] * yv;
+        if (++cnty == 4) {
+            cnty = 0;
+            for (uint32_t q = 0; q < ell; ++q) racc[q] = fred(racc[q]);
+        }
     }
 
     // ---- the x_hat side over this CTA's slice of K
@@ -151,7 +186,7 @@ __global__ void __launch_bounds__(kDecThreads) k_decode_verify(
         for (uint32_t q = 0; q < ell; ++q) lacc[q] += (uint64_t)u[(size_t)q * K + k] * xv;
         if (++cnt == 4) {
             cnt = 0;
-            for (uint32_t q = 0; q < ell; ++q) lacc[q] %= kQ;
+            for (uint32_t q = 0; q < ell; ++q) lacc[q] = fred(lacc[q]);
         }
     }
 
@@ -191,10 +226,17 @@ __global__ void __launch_bounds__(kDecThreads) k_decode_verify(
 cudaError_t launch_verify_u(const uint32_t *Qm, int K, const uint32_t *chal, uint32_t t_y,
                             uint32_t ell, uint32_t *u, cudaStream_t s) {
     if (K <= 0 || ell == 0) return cudaSuccess;
-    const bool vec = (K % 4 == 0) && ((reinterpret_cast<uintptr_t>(Qm) & 15u) == 0);
-    dim3 grid((K + 1023) / 1024, ell);
-    k_verify_u<<<grid, 256, 2 * (size_t)t_y * sizeof(uint32_t), s>>>(Qm, K, chal, t_y, u, vec);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((K + 255) / 256, ell, 1);
+    cfg.blockDim = dim3(256, 1, 1);
+    cfg.dynamicSmemBytes = 2 * (size_t)t_y * sizeof(uint32_t);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, k_verify_u, Qm, K, chal, t_y, u);
 }
 
 cudaError_t launch_decode_verify(const uint32_t *PT, int m, int K, const uint32_t *st, uint32_t t_x,
@@ -206,20 +248,27 @@ cudaError_t launch_decode_verify(const uint32_t *PT, int m, int K, const uint32_
     const bool vec = (m % 4 == 0) && ((reinterpret_cast<uintptr_t>(PT) & 15u) == 0);
     int C = (m + 1023) / 1024;
     C = C < 1 ? 1 : (C > 8 ? 8 : C);
+    const int chunk = (((m + C - 1) / C) + 3) & ~3;  // y_hat columns per CTA (staged in smem)
+    if ((2 * (size_t)t_x + (size_t)chunk) * sizeof(uint32_t) > 200 * 1024) return cudaErrorInvalidValue;
+    static const cudaError_t smem_attr = cudaFuncSetAttribute(
+        k_decode_verify, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+    if (smem_attr != cudaSuccess) return smem_attr;
     for (int b0 = 0; b0 < B; b0 += 65535) {
         const int nb = B - b0 < 65535 ? B - b0 : 65535;
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(C, nb, 1);
         cfg.blockDim = dim3(kDecThreads, 1, 1);
-        cfg.dynamicSmemBytes = 2 * (size_t)t_x * sizeof(uint32_t);
+        cfg.dynamicSmemBytes = (2 * (size_t)t_x + (size_t)chunk) * sizeof(uint32_t);
         cfg.stream = s;
-        cudaLaunchAttribute attr[1];
+        cudaLaunchAttribute attr[2];
         attr[0].id = cudaLaunchAttributeClusterDimension;
         attr[0].val.clusterDim.x = C;
         attr[0].val.clusterDim.y = 1;
         attr[0].val.clusterDim.z = 1;
+        attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[1].val.programmaticStreamSerializationAllowed = 1;
         cfg.attrs = attr;
-        cfg.numAttrs = 1;
+        cfg.numAttrs = 2;
         cudaError_t e = cudaLaunchKernelEx(&cfg, k_decode_verify, PT, m, K, st + (size_t)b0 * 2 * t_x,
                                            t_x, Xhat + (size_t)b0 * K, Yhat + (size_t)b0 * m, g, u,
                                            ell, Y + (size_t)b0 * m, accept + b0, vec);

@@ -39,6 +39,21 @@ cudaError_t launch_syndrome_scan(const uint32_t *pi2inv, const uint32_t *v2p, co
                                  uint32_t *F, unsigned long long *status, uint32_t *err,
                                  cudaStream_t s);
 
+// Fused syndrome for `count` freshly sampled sparse vectors (as
+// launch_sample_sparse, then out = addend + G e) in one launch with the
+// intermediate in cluster shared memory.  sparse_out: [count][2t];
+// out (and addend, may alias): [count][n].  cudaErrorNotSupported when N is
+// too long for one cluster (use the three-kernel path).
+bool syndrome_fused_plan(uint32_t N, uint32_t t, int *C, uint32_t *slice, size_t *smem);
+// Tables: pi2inv, v2p = v2 o pi2^-1, v1 (cluster form); pi2, v2m = v2 R,
+// v1pm = (v1 o pi1^-1) R (single-CTA form, Montgomery-scaled, R = 2^32).
+cudaError_t launch_syndrome_fused(const pvmvmd_key &key, uint32_t tag, uint64_t idx0, uint32_t N,
+                                  uint32_t t, uint32_t count, const uint32_t *pi2inv,
+                                  const uint32_t *v2p, const uint32_t *v1, const uint32_t *pi1inv,
+                                  const uint32_t *pi2, const uint32_t *v2m, const uint32_t *v1pm,
+                                  uint32_t n, uint32_t r, uint32_t *sparse_out,
+                                  const uint32_t *addend, uint32_t *out, cudaStream_t s);
+
 // Gather part: out_j = addend_j + sum_{c<r} F[pi1^-1(r j + c)], j < n
 // (addend may be null; out may alias addend).
 cudaError_t launch_syndrome_gather(const uint32_t *pi1inv, uint32_t n, uint32_t r,

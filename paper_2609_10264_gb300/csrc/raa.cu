@@ -8,8 +8,12 @@
 //                         block sums of R, fused with x_hat = x + x'.
 //  * k_encode_scan        one accumulate stage of the encoding G^T w over many
 //                         lanes (preprocessing of P^T and Q, Sec. 6.3).
+#include <cooperative_groups.h>
+
 #include "common.cuh"
 #include "launch.h"
+
+namespace cg = cooperative_groups;
 
 namespace pv {
 namespace {
@@ -25,34 +29,17 @@ __device__ __forceinline__ int bitlen32(uint32_t v) { return v ? 32 - __clz(v) :
 // whose top 31 bits lie in [1, q); the k-th one goes to the k-th smallest
 // support index.
 // -----------------------------------------------------------------------------
-__global__ void __launch_bounds__(32) k_sample_sparse(pvmvmd_key key, uint32_t tag, uint64_t idx0,
-                                                     uint32_t N, uint32_t t,
-                                                     uint32_t *__restrict__ out,
-                                                     unsigned long long *__restrict__ clear,
-                                                     size_t clear_words) {
-    extern __shared__ uint32_t sm[];
-    const uint32_t nbw = (N + 31) / 32;
-    uint32_t *bitmap = sm;
-    uint32_t *words = sm + nbw;  // 512 keystream words = 32 blocks
-    const int lane = threadIdx.x;
-
-    for (size_t i = (size_t)blockIdx.x * 32 + lane; i < clear_words; i += (size_t)gridDim.x * 32)
-        clear[i] = 0ull;
-
-    const uint64_t idx = idx0 + blockIdx.x;
-    uint32_t *supp = out + (size_t)blockIdx.x * 2 * t;
-    uint32_t *vals = supp + t;
-    for (uint32_t w = lane; w < nbw; w += 32) bitmap[w] = 0u;
-    __syncwarp();
-
-    // ---- support
-    const uint64_t sidx = 2 * idx;
+// Warp: mark the support of e <- E_t^N in `bitmap` (N bits, cleared by the
+// caller) from stream (tag, sidx), using `words` (512 words) as keystream buffer.
+__device__ void warp_sample_support(const pvmvmd_key &key, uint32_t tag, uint64_t sidx, uint32_t N,
+                                    uint32_t t, uint32_t *bitmap, uint32_t *words, int lane) {
     uint32_t have = 0;
     if (N <= 1) {  // below(1) = 0 reads no word
         if (t >= 1 && lane == 0) bitmap[0] = 1u;
-        have = t;
+        __syncwarp();
+        return;
     }
-    const int shift = 32 - (N > 1 ? bitlen32(N - 1) : 1);
+    const int shift = 32 - bitlen32(N - 1);
     for (uint64_t wpos = 0; have < t; wpos += 512) {
         uint32_t blk[16];
         chacha20_block_dev(key, (uint32_t)(wpos / 16 + lane), tag, (uint32_t)sidx,
@@ -78,8 +65,52 @@ __global__ void __launch_bounds__(32) k_sample_sparse(pvmvmd_key key, uint32_t t
         }
         __syncwarp();  // words are read before the next refill
     }
+}
 
-    // ---- ascending support from the bitmap
+// Warp: as warp_sample_support, and also writes the accepted indices, in the
+// order they were accepted, to list[0..t).
+__device__ void warp_sample_support_list(const pvmvmd_key &key, uint32_t tag, uint64_t sidx,
+                                         uint32_t N, uint32_t t, uint32_t *bitmap, uint32_t *words,
+                                         uint32_t *list, int lane) {
+    uint32_t have = 0;
+    if (N <= 1) {
+        if (t >= 1 && lane == 0) list[0] = 0u;
+        __syncwarp();
+        return;
+    }
+    const int shift = 32 - bitlen32(N - 1);
+    for (uint64_t wpos = 0; have < t; wpos += 512) {
+        uint32_t blk[16];
+        chacha20_block_dev(key, (uint32_t)(wpos / 16 + lane), tag, (uint32_t)sidx,
+                           (uint32_t)(sidx >> 32), blk);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) words[lane * 16 + i] = blk[i];
+        __syncwarp();
+        for (int batch = 0; batch < 16 && have < t; ++batch) {
+            const uint32_t v = words[batch * 32 + lane] >> shift;
+            const bool valid = v < N;
+            const bool inset = valid && ((bitmap[v >> 5] >> (v & 31)) & 1u);
+            const uint32_t vmask = __ballot_sync(kFull, valid);
+            const uint32_t same = __match_any_sync(kFull, valid ? v : 0xffffffffu);
+            const bool dup = (same & vmask & lanemask_lt()) != 0u;
+            const bool cand = valid && !inset && !dup;
+            const uint32_t cmask = __ballot_sync(kFull, cand);
+            const uint32_t need = t - have;
+            const uint32_t rk = __popc(cmask & lanemask_lt());
+            __syncwarp();
+            if (cand && rk < need) {
+                atomicOr(&bitmap[v >> 5], 1u << (v & 31));
+                list[have + rk] = v;
+            }
+            have += min((uint32_t)__popc(cmask), need);
+            __syncwarp();
+        }
+        __syncwarp();
+    }
+}
+
+// Warp: the set bits of `bitmap` (nbw words) in ascending order -> dst.
+__device__ void warp_bitmap_to_support(const uint32_t *bitmap, uint32_t nbw, uint32_t *dst, int lane) {
     uint32_t written = 0;
     for (uint32_t base = 0; base < nbw; base += 32) {
         uint32_t w = (base + lane < nbw) ? bitmap[base + lane] : 0u;
@@ -93,15 +124,17 @@ __global__ void __launch_bounds__(32) k_sample_sparse(pvmvmd_key key, uint32_t t
         uint32_t pos = written + incl - c;
         while (w) {
             const int b = __ffs(w) - 1;
-            supp[pos++] = (base + lane) * 32 + b;
+            dst[pos++] = (base + lane) * 32 + b;
             w &= w - 1;
         }
         written += __shfl_sync(kFull, incl, 31);
     }
+}
 
-    // ---- values in F*
-    const uint64_t vidx = 2 * idx + 1;
-    have = 0;
+// Warp: the first t draws of F* from stream (tag, vidx) -> dst.
+__device__ void warp_sample_values(const pvmvmd_key &key, uint32_t tag, uint64_t vidx, uint32_t t,
+                                   uint32_t *words, uint32_t *dst, int lane) {
+    uint32_t have = 0;
     for (uint64_t wpos = 0; have < t; wpos += 512) {
         uint32_t blk[16];
         chacha20_block_dev(key, (uint32_t)(wpos / 16 + lane), tag, (uint32_t)vidx,
@@ -115,10 +148,35 @@ __global__ void __launch_bounds__(32) k_sample_sparse(pvmvmd_key key, uint32_t t
             const bool valid = v != 0u && v < kQ;
             const uint32_t m = __ballot_sync(kFull, valid);
             const uint32_t r = __popc(m & lanemask_lt());
-            if (valid && have + r < t) vals[have + r] = v;
+            if (valid && have + r < t) dst[have + r] = v;
             have = min(have + (uint32_t)__popc(m), t);
         }
     }
+    __syncwarp();
+}
+
+// One warp per vector (the path for codes too long for one cluster).
+__global__ void __launch_bounds__(32) k_sample_sparse(pvmvmd_key key, uint32_t tag, uint64_t idx0,
+                                                     uint32_t N, uint32_t t,
+                                                     uint32_t *__restrict__ out,
+                                                     unsigned long long *__restrict__ clear,
+                                                     size_t clear_words) {
+    extern __shared__ uint32_t sm[];
+    const uint32_t nbw = (N + 31) / 32;
+    uint32_t *bitmap = sm;
+    uint32_t *words = sm + nbw;  // 512 keystream words = 32 blocks
+    const int lane = threadIdx.x;
+
+    for (size_t i = (size_t)blockIdx.x * 32 + lane; i < clear_words; i += (size_t)gridDim.x * 32)
+        clear[i] = 0ull;
+
+    const uint64_t idx = idx0 + blockIdx.x;
+    uint32_t *supp = out + (size_t)blockIdx.x * 2 * t;
+    for (uint32_t w = lane; w < nbw; w += 32) bitmap[w] = 0u;
+    __syncwarp();
+    warp_sample_support(key, tag, 2 * idx, N, t, bitmap, words, lane);
+    warp_bitmap_to_support(bitmap, nbw, supp, lane);
+    warp_sample_values(key, tag, 2 * idx + 1, t, words, supp + t, lane);
 }
 
 // -----------------------------------------------------------------------------
@@ -302,6 +360,323 @@ __global__ void __launch_bounds__(256) k_syndrome_gather(const uint32_t *__restr
 }
 
 // -----------------------------------------------------------------------------
+// Fused syndrome: x' = G e for a freshly sampled sparse e, in one kernel per
+// vector, with the length-N intermediate held in shared memory: one CTA of
+// 1024 threads when it fits, else a thread-block cluster whose CTAs each hold
+// a slice (CTA `rank` owns positions [rank*slice, (rank+1)*slice)) and read
+// each other's through DSMEM.  Steps (App. B, syndrome direction):
+//   sample e (warp 0: support; warp 1: values; every CTA of a cluster draws
+//     the same keystream, rank 0 writes the state), sort the support by rank;
+//   c_i = v2[pi2^-1(i)] * (A e)_{pi2^-1(i)}, the step function (A e)_k found
+//     through a bucket index over the sorted support;
+//   d = A c: a block suffix scan plus the aggregates of later CTAs;
+//   F_i = v1_i * d_i;  out_j = addend_j + sum_{c<r} F[pi1^-1(r j + c)].
+// No global scratch and no look-back.
+// -----------------------------------------------------------------------------
+constexpr int kFusedThreads = 1024;
+constexpr int kFusedBuckets = 512;   // index over the sorted support
+constexpr int kFusedBatch = 16;      // loads in flight per thread
+
+__device__ __forceinline__ uint32_t fpad(uint32_t i) { return i + (i >> 5); }  // bank padding
+
+__global__ void __launch_bounds__(kFusedThreads) k_syndrome_fused(
+    pvmvmd_key key, uint32_t tag, uint64_t idx0, uint32_t N, uint32_t t, uint32_t slice,
+    const uint32_t *__restrict__ pi2inv, const uint32_t *__restrict__ v2p,
+    const uint32_t *__restrict__ v1, const uint32_t *__restrict__ pi1inv, uint32_t n, uint32_t r,
+    uint32_t *__restrict__ sparse_out, const uint32_t *addend, uint32_t *out,
+    const uint32_t *__restrict__ pi2, const uint32_t *__restrict__ v2m,
+    const uint32_t *__restrict__ v1pm) {
+    cg::cluster_group cluster = cg::this_cluster();
+    extern __shared__ uint32_t sm[];
+    __shared__ uint32_t s_wsum[kFusedThreads / 32];
+    __shared__ uint32_t s_texcl[kFusedThreads];
+    __shared__ uint32_t s_first[kFusedBuckets];
+    __shared__ uint32_t s_agg;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const uint32_t C = cluster.num_blocks(), rank = cluster.block_rank();
+    const uint32_t vec = blockIdx.y;
+    const uint64_t idx = idx0 + vec;
+    const uint32_t fwords = fpad(slice);
+    uint32_t *F = sm;                 // padded slice (bitmap while sampling)
+    uint32_t *supp = sm + fwords;     // t
+    uint32_t *suf = supp + t;         // t + 1
+    uint32_t *words0 = suf + t + 1;   // 512
+    uint32_t *words1 = words0 + 512;  // 512 (then the unsorted support list)
+    uint32_t *list = words1 + 512;    // t
+    const uint32_t nbw = (N + 31) / 32;
+
+    // the kernels that follow may launch now; they wait for this one before
+    // reading anything it writes
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    // ---- sample e: warp 0 the support, warp 1 the values
+    for (uint32_t w = tid; w < nbw; w += kFusedThreads) F[w] = 0u;
+    __syncthreads();
+    if (warp == 0)
+        warp_sample_support_list(key, tag, 2 * idx, N, t, F, words0, list, lane);
+    else if (warp == 1)
+        warp_sample_values(key, tag, 2 * idx + 1, t, words1, suf, lane);
+    __syncthreads();
+    for (uint32_t i = tid; i < t; i += kFusedThreads) {  // ascending support by rank
+        const uint32_t v = list[i];
+        uint32_t rk = 0;
+        for (uint32_t j = 0; j < t; ++j) rk += list[j] < v;
+        supp[rk] = v;
+    }
+    __syncthreads();
+    if (rank == 0) {
+        uint32_t *st = sparse_out + (size_t)vec * 2 * t;
+        for (uint32_t j = tid; j < t; j += kFusedThreads) {
+            st[j] = supp[j];
+            st[t + j] = suf[j];
+        }
+    }
+    __syncthreads();
+    if (warp == 0) {  // suf[j] <- sum_{j' >= j} e_{j'}; suf[t] = 0
+        const uint32_t per = (t + 31) / 32;
+        const uint32_t lo = min(t, lane * per), hi = min(t, lo + per);
+        uint32_t sum = 0;
+        for (uint32_t j = hi; j-- > lo;) sum = fadd(sum, suf[j]);
+        uint32_t incl = sum;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t y = __shfl_down_sync(kFull, incl, o);
+            if (lane + o < 32) incl = fadd(incl, y);
+        }
+        uint32_t run = fsub(incl, sum);
+        for (uint32_t j = hi; j-- > lo;) {
+            run = fadd(run, suf[j]);
+            suf[j] = run;
+        }
+        if (lane == 0) suf[t] = 0;
+    }
+    if (C == 1) {
+        // ---- the whole vector in this CTA.  Thread tid walks positions k of
+        // its own range in order, so (A e)_k is a running pointer into the
+        // sorted support, and scatters c_{pi2(k)} = v2_k (A e)_k.
+        __syncthreads();
+        const uint32_t items = slice / kFusedThreads;
+        for (uint32_t i = N + tid; i < slice; i += kFusedThreads) F[fpad(i)] = 0u;  // padding
+        const uint32_t k0 = tid * items, k1 = min(N, k0 + items);
+        uint32_t j = 0;
+        if (k0 < k1) {
+            uint32_t lo = 0, hi = t;  // first support index >= k0
+            while (lo < hi) {
+                const uint32_t mid = (lo + hi) >> 1;
+                if (supp[mid] < k0) lo = mid + 1; else hi = mid;
+            }
+            j = lo;
+        }
+        for (uint32_t k = k0; k < k1; k += 4) {
+            uint32_t pk[4], vk[4];
+            if (k + 4 <= k1 && (k & 3) == 0) {
+                const uint4 a = __ldg(reinterpret_cast<const uint4 *>(pi2 + k));
+                const uint4 b = __ldg(reinterpret_cast<const uint4 *>(v2m + k));
+                pk[0] = a.x; pk[1] = a.y; pk[2] = a.z; pk[3] = a.w;
+                vk[0] = b.x; vk[1] = b.y; vk[2] = b.z; vk[3] = b.w;
+            } else {
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    pk[u] = k + u < k1 ? __ldg(pi2 + k + u) : 0u;
+                    vk[u] = k + u < k1 ? __ldg(v2m + k + u) : 0u;
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                if (k + u < k1) {
+                    while (j < t && supp[j] < k + u) ++j;
+                    F[fpad(pk[u])] = fmul_mont(suf[j], vk[u]);
+                }
+            }
+        }
+        __syncthreads();
+        // d = A c: thread tid owns positions [tid*items, (tid+1)*items)
+        uint32_t run = 0;
+        for (uint32_t u = items; u-- > 0;) {
+            const uint32_t li = tid * items + u;
+            run = fadd(run, F[fpad(li)]);
+            F[fpad(li)] = run;
+        }
+        uint32_t incl = run;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t y = __shfl_down_sync(kFull, incl, o);
+            if (lane + o < 32) incl = fadd(incl, y);
+        }
+        if (lane == 0) s_wsum[warp] = incl;
+        __syncthreads();
+        if (warp == 0) {
+            constexpr int nw = kFusedThreads / 32;
+            const uint32_t wv = lane < nw ? s_wsum[lane] : 0u;
+            uint32_t winc = wv;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const uint32_t y = __shfl_down_sync(kFull, winc, o);
+                if (lane + o < 32) winc = fadd(winc, y);
+            }
+            __syncwarp();
+            if (lane < nw) s_wsum[lane] = fsub(winc, wv);
+        }
+        __syncthreads();
+        const uint32_t add = fadd(fsub(incl, run), s_wsum[warp]);
+        for (uint32_t u = 0; u < items; ++u) {
+            const uint32_t li = tid * items + u;
+            F[fpad(li)] = fadd(F[fpad(li)], add);
+        }
+        __syncthreads();
+        // out_j = addend_j + sum_c v1[pi1^-1(r j + c)] d[pi1^-1(r j + c)]
+        for (uint32_t jo = tid; jo < n; jo += kFusedThreads) {
+            const uint32_t *p = pi1inv + (size_t)jo * r;
+            const uint32_t *w = v1pm + (size_t)jo * r;
+            uint32_t acc = 0;
+            if (r == 8) {
+                const uint4 a = __ldg(reinterpret_cast<const uint4 *>(p));
+                const uint4 b = __ldg(reinterpret_cast<const uint4 *>(p + 4));
+                const uint4 c = __ldg(reinterpret_cast<const uint4 *>(w));
+                const uint4 d = __ldg(reinterpret_cast<const uint4 *>(w + 4));
+                acc = fadd(fadd(fadd(fmul_mont(F[fpad(a.x)], c.x), fmul_mont(F[fpad(a.y)], c.y)),
+                                fadd(fmul_mont(F[fpad(a.z)], c.z), fmul_mont(F[fpad(a.w)], c.w))),
+                           fadd(fadd(fmul_mont(F[fpad(b.x)], d.x), fmul_mont(F[fpad(b.y)], d.y)),
+                                fadd(fmul_mont(F[fpad(b.z)], d.z), fmul_mont(F[fpad(b.w)], d.w))));
+            } else {
+                for (uint32_t cc = 0; cc < r; ++cc) acc = fadd(acc, fmul_mont(F[fpad(__ldg(p + cc))], __ldg(w + cc)));
+            }
+            const size_t o = (size_t)vec * n + jo;
+            out[o] = addend ? fadd(addend[o], acc) : acc;
+        }
+        return;
+    }
+
+    // bucket index: position k lies in bucket k >> bshift; s_first[b] is the
+    // first support index >= b << bshift
+    int bshift = 0;
+    while ((N >> bshift) > (uint32_t)kFusedBuckets - 1) ++bshift;
+    const uint32_t nbk = (N >> bshift) + 1;
+    for (uint32_t b = tid; b < nbk; b += kFusedThreads) {
+        const uint32_t start = b << bshift;
+        uint32_t lo = 0, hi = t;
+        while (lo < hi) {
+            const uint32_t mid = (lo + hi) >> 1;
+            if (supp[mid] < start) lo = mid + 1; else hi = mid;
+        }
+        s_first[b] = lo;
+    }
+    __syncthreads();
+
+    // ---- c over this CTA's slice (coalesced positions, loads batched)
+    const uint32_t base = rank * slice;
+    const uint32_t items = slice / kFusedThreads;
+    for (uint32_t u0 = 0; u0 < items; u0 += kFusedBatch) {
+        uint32_t kk[kFusedBatch], sc[kFusedBatch];
+#pragma unroll
+        for (int u = 0; u < kFusedBatch; ++u) {
+            const uint32_t i = base + (u0 + u) * kFusedThreads + tid;
+            const bool ok = u0 + u < items && i < N;
+            kk[u] = ok ? __ldg(pi2inv + i) : 0u;
+            sc[u] = ok ? __ldg(v2p + i) : 0u;
+        }
+#pragma unroll
+        for (int u = 0; u < kFusedBatch; ++u) {
+            if (u0 + u < items) {
+                uint32_t j = s_first[kk[u] >> bshift];  // first support index >= kk[u]
+                while (j < t && supp[j] < kk[u]) ++j;
+                F[fpad((u0 + u) * kFusedThreads + tid)] = fmul(sc[u], suf[j]);
+            }
+        }
+    }
+    __syncthreads();
+    // ---- suffix sums: thread tid owns [tid*items, (tid+1)*items)
+    uint32_t run = 0;
+    for (uint32_t u = items; u-- > 0;) {
+        const uint32_t li = tid * items + u;
+        run = fadd(run, F[fpad(li)]);
+        F[fpad(li)] = run;
+    }
+    uint32_t incl = run;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_down_sync(kFull, incl, o);
+        if (lane + o < 32) incl = fadd(incl, y);
+    }
+    if (lane == 0) s_wsum[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+        constexpr int nw = kFusedThreads / 32;
+        const uint32_t wv = lane < nw ? s_wsum[lane] : 0u;
+        uint32_t winc = wv;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t y = __shfl_down_sync(kFull, winc, o);
+            if (lane + o < 32) winc = fadd(winc, y);
+        }
+        __syncwarp();
+        if (lane < nw) s_wsum[lane] = fsub(winc, wv);
+        if (lane == 0) s_agg = winc;
+    }
+    __syncthreads();
+    s_texcl[tid] = fadd(fsub(incl, run), s_wsum[warp]);
+    uint32_t after = 0;  // sum over the positions owned by later CTAs
+    if (C > 1) {
+        cluster.sync();
+        for (uint32_t rr = rank + 1; rr < C; ++rr)
+            after = fadd(after, *cluster.map_shared_rank(&s_agg, rr));
+    } else {
+        __syncthreads();
+    }
+    for (uint32_t u0 = 0; u0 < items; u0 += kFusedBatch) {
+        uint32_t sc[kFusedBatch];
+#pragma unroll
+        for (int u = 0; u < kFusedBatch; ++u) {
+            const uint32_t i = base + (u0 + u) * kFusedThreads + tid;
+            sc[u] = (u0 + u < items && i < N) ? __ldg(v1 + i) : 0u;
+        }
+#pragma unroll
+        for (int u = 0; u < kFusedBatch; ++u) {
+            if (u0 + u < items) {
+                const uint32_t li = (u0 + u) * kFusedThreads + tid;
+                const uint32_t d = fadd(F[fpad(li)], fadd(s_texcl[li / items], after));
+                F[fpad(li)] = fmul(sc[u], d);
+            }
+        }
+    }
+    if (C > 1) cluster.sync(); else __syncthreads();
+
+    // ---- gather: out_j = addend_j + sum_c F[pi1^-1(r j + c)]
+    const uint32_t nsl = (n + C - 1) / C;
+    const uint32_t j0 = rank * nsl, j1 = min(n, j0 + nsl);
+    for (uint32_t j = j0 + tid; j < j1; j += kFusedThreads) {
+        const uint32_t *p = pi1inv + (size_t)j * r;
+        uint32_t acc = 0;
+        if (r == 8) {
+            const uint4 a = __ldg(reinterpret_cast<const uint4 *>(p));
+            const uint4 b = __ldg(reinterpret_cast<const uint4 *>(p + 4));
+            const uint32_t gi[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+            uint32_t v[8];
+            if (C == 1) {
+#pragma unroll
+                for (int c = 0; c < 8; ++c) v[c] = F[fpad(gi[c])];
+            } else {
+#pragma unroll
+                for (int c = 0; c < 8; ++c) {
+                    const uint32_t owner = gi[c] / slice;
+                    v[c] = cluster.map_shared_rank(F, owner)[fpad(gi[c] - owner * slice)];
+                }
+            }
+#pragma unroll
+            for (int c = 0; c < 8; ++c) acc = fadd(acc, v[c]);
+        } else {
+            for (uint32_t c = 0; c < r; ++c) {
+                const uint32_t gi = __ldg(p + c);
+                const uint32_t owner = gi / slice, off = gi - owner * slice;
+                acc = fadd(acc, C == 1 ? F[fpad(off)] : cluster.map_shared_rank(F, owner)[fpad(off)]);
+            }
+        }
+        const size_t o = (size_t)vec * n + j;
+        out[o] = addend ? fadd(addend[o], acc) : acc;
+    }
+    if (C > 1) cluster.sync();  // peers may still read this CTA's F
+}
+
+// -----------------------------------------------------------------------------
 // One accumulate stage of G^T w (App. B, encoding direction) over L lanes:
 //   Y[j][l] = sum_{j' <= j} vscale[j'] * X[perm[j'] / div][l]
 // With (perm, div, vscale) = (pi1, r, v1) this is A^T V1 Pi1^T R^T; with
@@ -480,6 +855,62 @@ cudaError_t launch_transpose_i8(const int8_t *in, int R, int C, int8_t *out, cud
     if (grid.y > 65535u) return cudaErrorInvalidValue;
     k_transpose_i8<<<grid, block, 0, s>>>(in, R, C, out);
     return cudaGetLastError();
+}
+
+
+// Cluster size and slice for the fused syndrome; false if N is too long for
+// one cluster of at most 8 CTAs.
+bool syndrome_fused_plan(uint32_t N, uint32_t t, int *C_out, uint32_t *slice_out, size_t *smem_out) {
+    // one CTA when the padded intermediate fits, else the smallest cluster
+    for (int C = 1; C <= 8; C *= 2) {
+        const uint32_t slice = (uint32_t)(((N + C - 1) / C + kFusedThreads - 1) / kFusedThreads) * kFusedThreads;
+        const size_t smem = ((size_t)slice + slice / 32 + 3 * (size_t)t + 1 + 1024) * sizeof(uint32_t);
+        if (smem <= (size_t)180 * 1024) {
+            *C_out = C;
+            *slice_out = slice;
+            *smem_out = smem;
+            return true;
+        }
+    }
+    return false;
+}
+
+cudaError_t launch_syndrome_fused(const pvmvmd_key &key, uint32_t tag, uint64_t idx0, uint32_t N,
+                                  uint32_t t, uint32_t count, const uint32_t *pi2inv,
+                                  const uint32_t *v2p, const uint32_t *v1, const uint32_t *pi1inv,
+                                  const uint32_t *pi2, const uint32_t *v2m, const uint32_t *v1pm,
+                                  uint32_t n, uint32_t r, uint32_t *sparse_out,
+                                  const uint32_t *addend, uint32_t *out, cudaStream_t s) {
+    if (count == 0) return cudaSuccess;
+    int C = 0;
+    uint32_t slice = 0;
+    size_t smem = 0;
+    if (!syndrome_fused_plan(N, t, &C, &slice, &smem)) return cudaErrorNotSupported;
+    static const cudaError_t attr = cudaFuncSetAttribute(
+        k_syndrome_fused, cudaFuncAttributeMaxDynamicSharedMemorySize, 180 * 1024);
+    if (attr != cudaSuccess) return attr;
+    for (uint32_t c0 = 0; c0 < count; c0 += 65535) {
+        const uint32_t nb = count - c0 < 65535 ? count - c0 : 65535;
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(C, nb, 1);
+        cfg.blockDim = dim3(kFusedThreads, 1, 1);
+        cfg.dynamicSmemBytes = smem;
+        cfg.stream = s;
+        cudaLaunchAttribute attr1[1];
+        attr1[0].id = cudaLaunchAttributeClusterDimension;
+        attr1[0].val.clusterDim.x = C;
+        attr1[0].val.clusterDim.y = 1;
+        attr1[0].val.clusterDim.z = 1;
+        cfg.attrs = attr1;
+        cfg.numAttrs = 1;
+        cudaError_t e = cudaLaunchKernelEx(&cfg, k_syndrome_fused, key, tag, idx0 + c0, N, t, slice,
+                                           pi2inv, v2p, v1, pi1inv, n, r,
+                                           sparse_out + (size_t)c0 * 2 * t,
+                                           addend ? addend + (size_t)c0 * n : nullptr,
+                                           out + (size_t)c0 * n, pi2, v2m, v1pm);
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
 }
 
 }  // namespace pv

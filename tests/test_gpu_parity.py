@@ -302,3 +302,12 @@ def test_server_mvm_multi_mixed_jobs(pv, wl):
     Xs_h = pv.as_u32(Xs)
     assert np.array_equal(pv.as_u32(Ys), np.stack([oracle.server_mvm(W[4], Xs_h[b]) for b in range(300)]))
     assert pv.pvmvmd_device_status() == 0
+
+
+def test_long_code_uses_three_kernel_path(pv, wl):
+    """K = 50000 gives N_x = 400000, too long for one cluster's shared memory,
+    so encode takes the sample / look-back scan / gather kernels; the result
+    must still equal the oracle."""
+    W = wl.weights_uniform(16, 50000, 9)
+    x = wl.int8_vectors(2, 50000, 10)
+    _full_round_trip(pv, W, x, seeds=(31, 32, 33))
