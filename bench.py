@@ -461,8 +461,8 @@ BATCHED = {
 def run_batched(args):
     """Step = for every projection of the layer: encode B vectors, the
     batched server product, decode+verify.  The server phase (tcgen05 digit
-    GEMM) is reported against the bf16 tensor peak: it executes
-    2 * m * K * 4 * B bf16 flops (four digit planes per field MAC)."""
+    GEMM) is reported against the 16-bit tensor peak: it executes
+    2 * m * K * 4 * B fp16 flops (four digit planes per field MAC)."""
     import torch
     rank, world, local = dist_env()
     if world > 1:
@@ -550,7 +550,7 @@ def run_batched(args):
             "metric": METRIC, "value": world * macs * args.steps / (ms / 1e3), "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-            "dtype": "u32 (F_q exact; bf16 digit MMAs, fp32 TMEM accumulation)", "data": "synthetic",
+            "dtype": "u32 (F_q exact; fp16 digit MMAs, fp32 TMEM accumulation)", "data": "synthetic",
             "config": {"workload": args.workload, "B": B, "projections": [[p["name"], p["m"], p["K"]] for p in projs]},
             "phases_ms": {"encode": ph[0], "server_batched": ph[2 - 1], "decode_verify": ph[2]},
             "roofline": {"bound": "tensor", "kernel": "k_batched (tcgen05 kind::f16 digit GEMM)",
@@ -564,6 +564,71 @@ def run_batched(args):
     return 0
 
 
+def run_server_shape(args):
+    """The batched server product Y_hat = M X_hat alone on one m x K x B
+    shape (``--shape MxKxB``), timed over --steps launches after --warmup.
+    Each step rotates over enough independent weight copies that the weights
+    read per step exceed the L2 cache."""
+    import torch
+    rank, world, local = dist_env()
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    import paper_2609_10264_gb300 as pv
+    from paper_2609_10264_gb300 import workloads as wl
+    m, K, B = (int(v) for v in args.shape.lower().split("x"))
+    copies = max(1, -(-256 * 2**20 // (m * K)))  # > 2x the 129 MB L2 in rotation
+    Wh = wl.weights_gaussian(m, K, (9, 0))
+    W0 = torch.from_numpy(Wh).to(device)
+    W = [W0] + [W0.clone() for _ in range(copies - 1)]
+    x = wl.int8_vectors(B, K, (10, 0))
+    Xd = torch.from_numpy(np.mod(x, pv.PVMVMD_Q).astype(np.uint32).view(np.int32)).to(device)
+    Y = torch.empty((B, m), dtype=torch.int32, device=device)
+    stream = torch.cuda.Stream(device)
+    with torch.cuda.stream(stream):
+        pv.pvmvmd_server_mvm(W0, Xd, Yhat=Y, stream=stream)
+    stream.synchronize()
+    pv.pvmvmd_device_status(stream)
+    rows = [0, m // 2, m - 1]
+    got = pv.as_u32(Y)[:, rows].astype(np.int64)
+    got = np.where(got > (pv.PVMVMD_Q - 1) // 2, got - pv.PVMVMD_Q, got)
+    assert np.array_equal(got, x @ Wh[rows].astype(np.int64).T), "server product mismatch"
+    with torch.cuda.stream(stream):
+        for s in range(args.warmup):
+            pv.pvmvmd_server_mvm(W[s % copies], Xd, Yhat=Y, stream=stream)
+    stream.synchronize()
+    clocks = ClockSampler(device.index)
+    clocks.start()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        t0.record(stream)
+        for s in range(args.steps):
+            pv.pvmvmd_server_mvm(W[s % copies], Xd, Yhat=Y, stream=stream)
+        t1.record(stream)
+    stream.synchronize()
+    clk = clocks.stop()
+    pv.pvmvmd_device_status(stream)
+    ms = t0.elapsed_time(t1) / args.steps
+    macs = m * K * B
+    flops = 2 * 4 * macs
+    peaks, kind = measured_peaks()
+    peak = peaks.get("bf16_tflops", 0.0)
+    achieved = flops / (ms / 1e3) / 1e12
+    if rank == 0:
+        print(json.dumps({
+            "metric": "server_field_mac_per_s", "value": macs / (ms / 1e3), "unit": "field-MAC/s",
+            "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "u32 (F_q exact; fp16 digit MMAs, fp32 TMEM accumulation)", "data": "synthetic",
+            "config": {"workload": "server-shape", "m": m, "K": K, "B": B, "weight_copies": copies,
+                       "l2": "weights rotated over copies larger than L2"},
+            "roofline": {"bound": "tensor", "kernel": "k_batched (tcgen05 kind::f16 digit GEMM) + k_digit_tiles",
+                         "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak if peak else None,
+                         "peak_kind": f"{kind} bf16_tflops (burst)"},
+            "gpu_launches": 2 * args.steps, "clocks": clk}), flush=True)
+    return 0
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
@@ -573,7 +638,9 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-vectors", type=int, default=150)
     ap.add_argument("--server-mode", choices=["multi", "calls"], default="multi")
-    ap.add_argument("--workload", choices=["batch1-4096"] + sorted(BATCHED), default="batch1-4096")
+    ap.add_argument("--workload", choices=["batch1-4096", "server-shape"] + sorted(BATCHED),
+                    default="batch1-4096")
+    ap.add_argument("--shape", default="4096x4096x64", help="m x K x B for --workload server-shape")
     ap.add_argument("--server-streams", type=int, default=2)
     args = ap.parse_args(argv)
     if args.warmup < 3:
@@ -582,6 +649,8 @@ def main(argv=None):
         return run_reference(args)
     if args.workload in BATCHED:
         return run_batched(args)
+    if args.workload == "server-shape":
+        return run_server_shape(args)
     return run_ours(args)
 
 

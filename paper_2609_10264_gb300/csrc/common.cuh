@@ -74,8 +74,14 @@ __host__ __device__ __forceinline__ uint32_t to_mont(uint32_t b) {
 
 // Signed 64-bit integer -> canonical representative.
 __host__ __device__ __forceinline__ uint32_t fred_signed(int64_t v) {
+#ifdef __CUDA_ARCH__
+    if (v >= 0) return fred((uint64_t)v);
+    const uint32_t r = fred(0ull - (uint64_t)v);  // |v|, exact also for INT64_MIN
+    return r ? kQ - r : 0u;
+#else
     int64_t r = v % (int64_t)kQ;
     return (uint32_t)(r < 0 ? r + (int64_t)kQ : r);
+#endif
 }
 __host__ __device__ __forceinline__ uint32_t flift_i8(int8_t w) {
     return w < 0 ? kQ + (uint32_t)(int32_t)w : (uint32_t)w;

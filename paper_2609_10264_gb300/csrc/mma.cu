@@ -4,27 +4,31 @@
 // Arithmetic.  Each centred x_hat entry is split into four signed base-256
 // digits d_k in [-128, 127] (x = sum_k 2^(8k) d_k), so
 //     (M x_hat)_i = sum_k 2^(8k) sum_j M_ij d_k[j]        (exact over Z).
-// The inner sums run on the tensor cores as a bf16 GEMM (every int8 weight and
-// every digit is an exact bf16 value) with fp32 accumulation in TMEM.  A
+// The inner sums run on the tensor cores as an fp16 GEMM (every int8 weight
+// and every digit is an exact fp16 value) with fp32 accumulation in TMEM.  A
 // product is at most 128 * 128 = 2^14 in magnitude, so a chunk of 1024
 // K-elements sums to at most 2^24: every partial sum is an integer that fp32
 // holds exactly.  After each chunk the epilogue warps read the accumulator,
-// convert it to integers, combine the four digits in int64 and add to a
-// running int64 per output; the result is reduced mod q once at the end.
-// (This GPU generation has no int8 tcgen05 kind, hence bf16 digits.)
+// convert it to integers, combine the four digits in int64, reduce mod q and
+// add to a running sum per output.  (This GPU generation has no int8 tcgen05
+// kind; fp16 and bf16 run at the same rate, and int8 -> fp16 is one byte
+// permute and one packed add per two elements.)
 //
 // Tiles.  A CTA owns 128 rows of M (MMA M = 128) and 64 vectors (MMA N = 256:
 // 64 vectors x 4 digits, the digit rows of vector v at N-rows 4v..4v+3).
-// K is split over the CTAs of a thread-block cluster; their int64 partial
-// sums are added through distributed shared memory.
+// K may be split over the CTAs of a thread-block cluster; their mod-q partial
+// sums are added through distributed shared memory, each rank finishing a
+// slice of the vectors.
 //
-// Warp roles (320 threads):
-//   warps 0-3  convert the int8 M tile to bf16 in the 128-byte-swizzled
-//              K-major layout the MMA reads (one row per thread);
-//   warps 4-7  epilogue (TMEM lanes 32(w-4)..32(w-4)+31);
-//   warp 8     bulk-copies the pre-tiled digit operand (cp.async.bulk);
-//   warp 9     allocates TMEM and issues the MMAs (one elected lane).
+// Warp roles (576 threads):
+//   warps 0-7    convert the int8 M tile to fp16 in the 128-byte-swizzled
+//                K-major layout the MMA reads (two threads per row);
+//   warps 8-11   epilogue for vectors 0-31, warps 12-15 for vectors 32-63
+//                (TMEM lanes 32 (w mod 4) .. +31);
+//   warp 16      bulk-copies the pre-tiled digit operand (cp.async.bulk);
+//   warp 17      allocates TMEM and issues the MMAs (one elected lane).
 #include <cooperative_groups.h>
+#include <cuda_fp16.h>
 
 #include <mutex>
 
@@ -45,7 +49,10 @@ constexpr int kChunkBlocks = 16;    // 16 x 64 = 1024 K-elements per exact chunk
 constexpr int kATile = kBM * kBK * 2;   // 16 KiB
 constexpr int kBTile = kBN * kBK * 2;   // 32 KiB
 constexpr int kStageBytes = kATile + kBTile;
-constexpr int kThreads = 320;
+constexpr int kThreads = 576;
+constexpr int kConvThreads = 256;   // warps 0-7
+constexpr int kEpiThreads = 256;    // warps 8-15
+constexpr int kWarpLoader = 16, kWarpMma = 17;
 constexpr int kMmaSmem = kStages * kStageBytes + 1024;  // + alignment slack
 constexpr uint32_t kWaitLimit = 1u << 24;
 
@@ -124,8 +131,9 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
     d |= (uint64_t)2u << 61;                      // 128-byte swizzle
     return d;
 }
-// Instruction descriptor, kind::f16: bf16 A and B, f32 D, both K-major.
-constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kBN >> 3) << 17) |
+// Instruction descriptor, kind::f16: fp16 A and B (format 0), f32 D (1),
+// both K-major, N = 256, M = 128.
+constexpr uint32_t kIdesc = (1u << 4) | (0u << 7) | (0u << 10) | ((uint32_t)(kBN >> 3) << 17) |
                             ((uint32_t)(kBM >> 4) << 24);
 
 __device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
@@ -158,13 +166,26 @@ __device__ __forceinline__ uint32_t sw128_off(uint32_t row, uint32_t chunk) {
     return (row >> 3) * 1024u + (row & 7u) * 128u + ((chunk ^ (row & 7u)) << 4);
 }
 
-__device__ __forceinline__ uint32_t bf16x2_of_i8(int lo, int hi) {
-    const __nv_bfloat162 v = __floats2bfloat162_rn((float)lo, (float)hi);
+// Four signed bytes -> two fp16x2 words holding the same integers: with
+// u = b + 128 (the byte xor 0x80), the fp16 pattern 0x6400 | u is 1024 + u,
+// and subtracting 1152 leaves b exactly.
+__device__ __forceinline__ void i8x4_to_f16x4(uint32_t w, uint32_t &lo, uint32_t &hi) {
+    const uint32_t u = w ^ 0x80808080u;
+    const uint32_t a = __byte_perm(u, 0x64646464u, 0x5150);  // bytes u0, 0x64, u1, 0x64
+    const uint32_t b = __byte_perm(u, 0x64646464u, 0x5352);  // bytes u2, 0x64, u3, 0x64
+    const __half2 off = __halves2half2(__ushort_as_half(0xE480u), __ushort_as_half(0xE480u));  // -1152
+    const __half2 ha = __hadd2(*reinterpret_cast<const __half2 *>(&a), off);
+    const __half2 hb = __hadd2(*reinterpret_cast<const __half2 *>(&b), off);
+    lo = *reinterpret_cast<const uint32_t *>(&ha);
+    hi = *reinterpret_cast<const uint32_t *>(&hb);
+}
+__device__ __forceinline__ uint32_t f16x2_of_int(int lo, int hi) {
+    const __half2 v = __halves2half2(__int2half_rn(lo), __int2half_rn(hi));
     return *reinterpret_cast<const uint32_t *>(&v);
 }
 
 // ---------------------------------------------------------------- digit operand
-// X_hat (B x K u32) -> pre-tiled bf16 digit operand: for vector tile nt and
+// X_hat (B x K u32) -> pre-tiled fp16 digit operand: for vector tile nt and
 // K-block kb, a 32 KiB block laid out exactly as the MMA's B tile in shared
 // memory.  Zero for vectors >= B and K-elements >= K.  One thread per
 // (vector, 8 K-elements).
@@ -194,10 +215,10 @@ __global__ void __launch_bounds__(256) k_digit_tiles(const uint32_t *__restrict_
     for (int l = 0; l < 4; ++l) {
         const uint32_t row = 4 * vl + l;
         uint4 q;
-        q.x = bf16x2_of_i8(d[l][0], d[l][1]);
-        q.y = bf16x2_of_i8(d[l][2], d[l][3]);
-        q.z = bf16x2_of_i8(d[l][4], d[l][5]);
-        q.w = bf16x2_of_i8(d[l][6], d[l][7]);
+        q.x = f16x2_of_int(d[l][0], d[l][1]);
+        q.y = f16x2_of_int(d[l][2], d[l][3]);
+        q.z = f16x2_of_int(d[l][4], d[l][5]);
+        q.w = f16x2_of_int(d[l][6], d[l][7]);
         *reinterpret_cast<uint4 *>(blk + sw128_off(row, chunk)) = q;
     }
 }
@@ -229,18 +250,18 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     if (tid == 0) {
         for (int s = 0; s < kStages; ++s) {
-            mbar_init(&full_a[s], 128);
+            mbar_init(&full_a[s], kConvThreads);
             mbar_init(&full_b[s], 1);
             mbar_init(&empty_bar[s], 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&acc_full[b], 1);
-            mbar_init(&acc_empty[b], 128);
+            mbar_init(&acc_empty[b], kEpiThreads);
         }
         mbar_init(&mma_done, 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
-    if (warp == 9) {
+    if (warp == kWarpMma) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 512;" ::"r"(
                          smem_addr(&s_tmem)));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
@@ -250,34 +271,32 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     const uint32_t tmem = s_tmem;
 
-    // running int64 sums of the epilogue threads (row = lane of TMEM)
-    long long run[kBV];
+    uint32_t run[32];  // epilogue: running mod-q sums of 32 vectors for one row
 #pragma unroll
-    for (int v = 0; v < kBV; ++v) run[v] = 0;
+    for (int v = 0; v < 32; ++v) run[v] = 0u;
 
-    if (warp < 4) {
-        // ------------------------------------------------ A: int8 M tile -> bf16 swizzled
-        const int r = tid;  // tile row
+    if (warp < 8) {
+        // ------------------------------------------------ A: int8 M tile -> fp16 swizzled
+        const int r = tid >> 1, half = tid & 1;  // row, and which 32 K-elements of the block
         const int grow = m0 + r;
         const bool row_ok = grow < m;
         const int8_t *wrow = W + (size_t)(row_ok ? grow : 0) * K;
         constexpr int PF = 4;
-        uint4 buf[PF][4];
-        auto load = [&](int i, uint4 (&dst)[4]) {
-            const int k0 = (kb0 + i) * kBK;
-            if (kVec && row_ok && k0 + kBK <= K) {
-#pragma unroll
-                for (int c = 0; c < 4; ++c)
-                    dst[c] = __ldg(reinterpret_cast<const uint4 *>(wrow + k0) + c);
+        uint4 buf[PF][2];
+        auto load = [&](int i, uint4 (&dst)[2]) {
+            const int k0 = (kb0 + i) * kBK + 32 * half;
+            if (kVec && row_ok && k0 + 32 <= K) {
+                dst[0] = __ldg(reinterpret_cast<const uint4 *>(wrow + k0));
+                dst[1] = __ldg(reinterpret_cast<const uint4 *>(wrow + k0) + 1);
             } else {
-                uint32_t w[16];
+                uint32_t w[8];
 #pragma unroll
-                for (int q = 0; q < 16; ++q) w[q] = 0;
+                for (int q = 0; q < 8; ++q) w[q] = 0;
                 if (row_ok)
-                    for (int e = 0; e < kBK && k0 + e < K; ++e)
+                    for (int e = 0; e < 32 && k0 + e < K; ++e)
                         w[e >> 2] |= (uint32_t)(uint8_t)wrow[k0 + e] << (8 * (e & 3));
-#pragma unroll
-                for (int c = 0; c < 4; ++c) dst[c] = make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]);
+                dst[0] = make_uint4(w[0], w[1], w[2], w[3]);
+                dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
             }
         };
 #pragma unroll
@@ -294,48 +313,47 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!mbar_wait(&empty_bar[s], ph ^ 1u, err)) { ok = false; break; }
                 uint8_t *a = smem + s * kStageBytes;
 #pragma unroll
-                for (int c = 0; c < 4; ++c) {  // 16 int8 -> two 16-byte bf16 chunks
-                    const uint32_t w4[4] = {buf[u][c].x, buf[u][c].y, buf[u][c].z, buf[u][c].w};
+                for (int c = 0; c < 2; ++c) {  // 16 int8 -> two 16-byte fp16 chunks
                     uint32_t o[8];
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const int b0 = (int)(int8_t)(w4[q] & 0xff), b1 = (int)(int8_t)((w4[q] >> 8) & 0xff);
-                        const int b2 = (int)(int8_t)((w4[q] >> 16) & 0xff), b3 = (int)(int8_t)(w4[q] >> 24);
-                        o[2 * q] = bf16x2_of_i8(b0, b1);
-                        o[2 * q + 1] = bf16x2_of_i8(b2, b3);
-                    }
-                    *reinterpret_cast<uint4 *>(a + sw128_off(r, 2 * c)) = make_uint4(o[0], o[1], o[2], o[3]);
-                    *reinterpret_cast<uint4 *>(a + sw128_off(r, 2 * c + 1)) = make_uint4(o[4], o[5], o[6], o[7]);
+                    i8x4_to_f16x4(buf[u][c].x, o[0], o[1]);
+                    i8x4_to_f16x4(buf[u][c].y, o[2], o[3]);
+                    i8x4_to_f16x4(buf[u][c].z, o[4], o[5]);
+                    i8x4_to_f16x4(buf[u][c].w, o[6], o[7]);
+                    const int chunk = 4 * half + 2 * c;
+                    *reinterpret_cast<uint4 *>(a + sw128_off(r, chunk)) = make_uint4(o[0], o[1], o[2], o[3]);
+                    *reinterpret_cast<uint4 *>(a + sw128_off(r, chunk + 1)) = make_uint4(o[4], o[5], o[6], o[7]);
                 }
                 fence_async_smem();
                 mbar_arrive(&full_a[s]);
                 if (i + PF < nblk) load(i + PF, buf[u]);
             }
         }
-    } else if (warp < 8) {
-        // ------------------------------------------------ epilogue: TMEM -> int64 sums
-        const int q = warp - 4;  // TMEM lane quadrant
+    } else if (warp < 16) {
+        // ------------------------------------------------ epilogue: TMEM -> mod-q sums
+        const int q = warp & 3;            // TMEM lane quadrant
+        const int grp = (warp - 8) >> 2;   // vectors 32 grp .. 32 grp + 31
         for (int c = 0; c < nchunks; ++c) {
             const int bsel = c & 1;
             if (!mbar_wait(&acc_full[bsel], (uint32_t)(c >> 1) & 1u, err)) break;
             tc_fence_after();
 #pragma unroll
-            for (int j = 0; j < kBN / 32; ++j) {
+            for (int j = 0; j < 4; ++j) {
                 uint32_t r[32];
-                tmem_ld32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(bsel * kBN + 32 * j), r);
+                tmem_ld32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(bsel * kBN + 128 * grp + 32 * j), r);
 #pragma unroll
                 for (int v = 0; v < 8; ++v) {
                     const long long d0 = __float2int_rn(__uint_as_float(r[4 * v]));
                     const long long d1 = __float2int_rn(__uint_as_float(r[4 * v + 1]));
                     const long long d2 = __float2int_rn(__uint_as_float(r[4 * v + 2]));
                     const long long d3 = __float2int_rn(__uint_as_float(r[4 * v + 3]));
-                    run[8 * j + v] += d0 + (d1 << 8) + (d2 << 16) + (d3 << 24);
+                    run[8 * j + v] = fadd(run[8 * j + v],
+                                          fred_signed(d0 + (d1 << 8) + (d2 << 16) + (d3 << 24)));
                 }
             }
             tc_fence_before();
             mbar_arrive(&acc_empty[bsel]);
         }
-    } else if (warp == 8) {
+    } else if (warp == kWarpLoader) {
         // ------------------------------------------------ B: bulk copies of digit tiles
         if (lane == 0) {
             const uint8_t *src = D + ((size_t)nt * nkb + kb0) * kBTile;
@@ -391,28 +409,81 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ---------------------------------------------------- split-K reduction and store
     tc_fence_before();
     __syncthreads();  // every stage is consumed: the stage memory is reused below
-    long long *part = reinterpret_cast<long long *>(smem);  // [kBV][kBM]
-    if (warp >= 4 && warp < 8) {
-        const int row = tid - 128;
+    uint32_t *part = reinterpret_cast<uint32_t *>(smem);  // [kBV][kBM] mod-q partial sums
+    if (warp >= 8 && warp < 16) {
+        const int row = 32 * (warp & 3) + lane;
+        const int v0 = 32 * ((warp - 8) >> 2);
 #pragma unroll
-        for (int v = 0; v < kBV; ++v) part[v * kBM + row] = run[v];
+        for (int v = 0; v < 32; ++v) part[(v0 + v) * kBM + row] = run[v];
     }
     cluster.sync();
-    if (rank == 0 && warp >= 4 && warp < 8) {
-        const int row = tid - 128;
-        const int grow = m0 + row;
-        for (int v = 0; v < kBV; ++v) {
-            long long s = part[v * kBM + row];
-            for (int r = 1; r < split; ++r) s += cluster.map_shared_rank(part, r)[v * kBM + row];
-            const int b = nt * kBV + v;
-            if (grow < m && b < B) Yhat[(size_t)b * m + grow] = fred_signed(s);
-        }
+    // rank r finishes vectors [r * 64 / split, (r + 1) * 64 / split)
+    const int vper = kBV / split;
+    for (int idx = tid; idx < vper * kBM; idx += kThreads) {
+        const int v = rank * vper + idx / kBM, row = idx % kBM;
+        uint32_t sum = 0;
+        for (int rr = 0; rr < split; ++rr) sum = fadd(sum, cluster.map_shared_rank(part, rr)[v * kBM + row]);
+        const int b = nt * kBV + v, grow = m0 + row;
+        if (grow < m && b < B) Yhat[(size_t)b * m + grow] = sum;
     }
     cluster.sync();
-    if (warp == 9) {
+    if (warp == kWarpMma) {
         tc_fence_after();
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem));
     }
+}
+
+// Cluster split of K: the fewest CTAs per tile that still give the fewest
+// waves per unit of work, with at least 4 K-blocks per CTA.
+int choose_split(int tiles, int nkb, int sms) {
+    int best = 1;
+    double best_cost = 1e30;
+    for (int split = 1; split <= 8; split *= 2) {
+        if (split > 1 && nkb < 4 * split) break;
+        const int waves = (tiles * split + sms - 1) / sms;
+        const double cost = (double)waves / split + 0.02 * (split - 1);
+        if (cost < best_cost - 1e-9) {
+            best_cost = cost;
+            best = split;
+        }
+    }
+    return best;
+}
+
+cudaError_t batched_launch(const int8_t *W, int m, int K, const uint32_t *Xhat, int B, uint32_t *Yhat,
+                           uint32_t *err, uint8_t *D, cudaStream_t s) {
+    const int nkb = (K + kBK - 1) / kBK;
+    const int nvt = (B + kBV - 1) / kBV;
+    const size_t threads = (size_t)nvt * kBV * nkb * 8;
+    k_digit_tiles<<<(unsigned)((threads + 255) / 256), 256, 0, s>>>(Xhat, B, K, nkb, nvt, D);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int mt = (m + kBM - 1) / kBM;
+    const int split = choose_split(mt * nvt, nkb, sms);
+    const bool vec = (K % 16 == 0) && ((reinterpret_cast<uintptr_t>(W) & 15u) == 0);
+    auto kern = vec ? k_batched<true> : k_batched<false>;
+    static const cudaError_t a1 =
+        cudaFuncSetAttribute(k_batched<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
+    static const cudaError_t a2 =
+        cudaFuncSetAttribute(k_batched<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
+    if (a1 != cudaSuccess) return a1;
+    if (a2 != cudaSuccess) return a2;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(mt, nvt, split);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = kMmaSmem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 1;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = split;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, W, m, K, (const uint8_t *)D, nkb, B, Yhat, err);
 }
 
 // ---------------------------------------------------------------- scratch for the digit operand
@@ -451,47 +522,10 @@ cudaError_t launch_batched(const int8_t *W, int m, int K, const uint32_t *Xhat, 
     if (m <= 0 || K <= 0 || B <= 0) return cudaSuccess;
     const int nkb = (K + kBK - 1) / kBK;
     const int nvt = (B + kBV - 1) / kBV;
-    const size_t need = (size_t)nvt * nkb * kBTile;
     uint8_t *D = nullptr;
-    cudaError_t e = digit_scratch(need, &D);
+    cudaError_t e = digit_scratch((size_t)nvt * nkb * kBTile, &D);
     if (e != cudaSuccess) return e;
-    {
-        const size_t threads = (size_t)nvt * kBV * nkb * 8;
-        k_digit_tiles<<<(unsigned)((threads + 255) / 256), 256, 0, s>>>(Xhat, B, K, nkb, nvt, D);
-        if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    }
-    int dev = 0, sms = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    const int mt = (m + kBM - 1) / kBM;
-    const int tiles = mt * nvt;
-    // split K over a cluster until the grid covers the GPU (and each CTA keeps
-    // at least one exact 1024-element chunk of work)
-    int split = 1;
-    while (split < 8 && tiles * split < sms && nkb / (2 * split) >= kChunkBlocks / 2) split *= 2;
-
-    const bool vec = (K % 16 == 0) && ((reinterpret_cast<uintptr_t>(W) & 15u) == 0);
-    auto kern = vec ? k_batched<true> : k_batched<false>;
-    static const cudaError_t a1 =
-        cudaFuncSetAttribute(k_batched<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
-    static const cudaError_t a2 =
-        cudaFuncSetAttribute(k_batched<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
-    if (a1 != cudaSuccess) return a1;
-    if (a2 != cudaSuccess) return a2;
-
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(mt, nvt, split);
-    cfg.blockDim = dim3(kThreads, 1, 1);
-    cfg.dynamicSmemBytes = kMmaSmem;
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = 1;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = split;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kern, W, m, K, (const uint8_t *)D, nkb, B, Yhat, err);
+    return batched_launch(W, m, K, Xhat, B, Yhat, err, D, s);
 }
 
 }  // namespace pv
@@ -547,39 +581,7 @@ extern "C" int pvmvmd_server_mvm_noalloc(const int8_t *W_dev, int m, int K, cons
 
     // every byte of the tiles in use is rewritten: nothing left by an
     // earlier call is read
-    const size_t threads = (size_t)nvt * kBV * nkb * 8;
-    k_digit_tiles<<<(unsigned)((threads + 255) / 256), 256, 0, s>>>(Xhat_dev, B, K, nkb, nvt, D);
-    if (cudaGetLastError() != cudaSuccess) return PVMVMD_E_CUDA;
-
-    int dev = 0, sms = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-        return PVMVMD_E_CUDA;
-    const int mt = (m + kBM - 1) / kBM;
-    const int tiles = mt * nvt;
-    int split = 1;
-    while (split < 8 && tiles * split < sms && nkb / (2 * split) >= kChunkBlocks / 2) split *= 2;
-    const bool vec = (K % 16 == 0) && ((reinterpret_cast<uintptr_t>(W_dev) & 15u) == 0);
-    auto kern = vec ? k_batched<true> : k_batched<false>;
-    static const cudaError_t a1 =
-        cudaFuncSetAttribute(k_batched<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
-    static const cudaError_t a2 =
-        cudaFuncSetAttribute(k_batched<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
-    if (a1 != cudaSuccess || a2 != cudaSuccess) return PVMVMD_E_CUDA;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(mt, nvt, split);
-    cfg.blockDim = dim3(kThreads, 1, 1);
-    cfg.dynamicSmemBytes = kMmaSmem;
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = 1;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = split;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    if (cudaLaunchKernelEx(&cfg, kern, W_dev, m, K, (const uint8_t *)D, nkb, B, Yhat_dev, err) !=
-        cudaSuccess) {
+    if (batched_launch(W_dev, m, K, Xhat_dev, B, Yhat_dev, err, D, s) != cudaSuccess) {
         (void)cudaGetLastError();
         return PVMVMD_E_CUDA;
     }
