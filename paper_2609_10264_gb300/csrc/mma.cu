@@ -14,22 +14,35 @@
 // kind; fp16 and bf16 run at the same rate, and int8 -> fp16 is one byte
 // permute and one packed add per two elements.)
 //
-// Tiles.  A CTA owns 128 rows of M (MMA M = 128) and 64 vectors (MMA N = 256:
-// 64 vectors x 4 digits, the digit rows of vector v at N-rows 4v..4v+3).
-// K may be split over the CTAs of a thread-block cluster; their mod-q partial
-// sums are added through distributed shared memory, each rank finishing a
-// slice of the vectors.
+// Tiles.  Two CTAs on two SMs (a CTA pair of a cluster) run one MMA of
+// M = 256 rows of M by N = 256 digit rows (64 vectors x 4 digits, the digit
+// rows of vector v at N-rows 4v..4v+3) with tcgen05 cta_group::2: each CTA
+// holds its own 128 rows of M and half of the digit rows (vectors 0-31 in the
+// even CTA, 32-63 in the odd one), and each CTA's TMEM receives the full
+// 128 x 256 accumulator of its own rows.  The even CTA issues the MMAs.
+// K may further be split over pairs of the cluster; their mod-q partial sums
+// are added through distributed shared memory, each rank finishing a slice
+// of the vectors.
 //
-// Warp roles (576 threads):
+// Warp roles (576 threads per CTA):
 //   warps 0-7    convert the int8 M tile to fp16 in the 128-byte-swizzled
-//                K-major layout the MMA reads (two threads per row);
+//                K-major layout the MMA reads: warps 0-3 take the even
+//                K-blocks, warps 4-7 the odd ones (four threads per row);
 //   warps 8-11   epilogue for vectors 0-31, warps 12-15 for vectors 32-63
 //                (TMEM lanes 32 (w mod 4) .. +31);
-//   warp 16      bulk-copies the pre-tiled digit operand (cp.async.bulk);
-//   warp 17      allocates TMEM and issues the MMAs (one elected lane).
+//   warp 16      bulk-copies this CTA's half of the digit operand;
+//   warp 17      allocates TMEM; in the even CTA one lane issues the MMAs, in
+//                the odd CTA one lane tells the even CTA when a stage of
+//                its own shared memory is filled;
+//   warp 18      streams 128 x 64 int8 tiles of M into a ring of raw tiles
+//                with the tensor memory accelerator (TMA), far ahead of the
+//                converter.
 #include <cooperative_groups.h>
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_fp16.h>
 
+#include <cstring>
 #include <mutex>
 
 #include "common.cuh"
@@ -44,16 +57,20 @@ constexpr int kBM = 128;            // rows of M per CTA
 constexpr int kBV = 64;             // vectors per CTA
 constexpr int kBN = 4 * kBV;        // MMA N (digit rows)
 constexpr int kBK = 64;             // K-elements per stage (128 bytes of bf16)
-constexpr int kStages = 4;
+constexpr int kStages = 5;
+constexpr int kRaw = 8;                 // raw int8 tiles of M in flight
 constexpr int kChunkBlocks = 16;    // 16 x 64 = 1024 K-elements per exact chunk
 constexpr int kATile = kBM * kBK * 2;   // 16 KiB
 constexpr int kBTile = kBN * kBK * 2;   // 32 KiB
-constexpr int kStageBytes = kATile + kBTile;
-constexpr int kThreads = 576;
+constexpr int kBHalf = kBTile / 2;     // 16 KiB: the digit rows one CTA of a pair holds
+constexpr int kStageBytes = kATile + kBHalf;
+constexpr int kThreads = 608;
 constexpr int kConvThreads = 256;   // warps 0-7
 constexpr int kEpiThreads = 256;    // warps 8-15
-constexpr int kWarpLoader = 16, kWarpMma = 17;
-constexpr int kMmaSmem = kStages * kStageBytes + 1024;  // + alignment slack
+constexpr int kWarpLoader = 16, kWarpMma = 17, kWarpWLoad = 18;
+constexpr int kRawTile = kBM * kBK;     // 8 KiB: rows of 64 bytes, unswizzled
+constexpr int kRawOff = kStages * kStageBytes;
+constexpr int kMmaSmem = kRawOff + kRaw * kRawTile + 1024;  // + alignment slack
 constexpr uint32_t kWaitLimit = 1u << 24;
 
 __device__ __forceinline__ uint32_t smem_addr(const void *p) {
@@ -64,41 +81,62 @@ __device__ __forceinline__ uint32_t smem_addr(const void *p) {
 __device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count));
 }
+// Arrivals discard the barrier state (sink `_`): the thread does not wait
+// for it.
 __device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
-    uint64_t state;
-    asm volatile("mbarrier.arrive.shared::cta.b64 %0, [%1];"
-                 : "=l"(state)
-                 : "r"(smem_addr(bar))
-                 : "memory");
-    (void)state;
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
 }
 __device__ __forceinline__ void mbar_arrive_tx(uint64_t *bar, uint32_t bytes) {
-    uint64_t state;
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 %0, [%1], %2;"
-                 : "=l"(state)
-                 : "r"(smem_addr(bar)), "r"(bytes)
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
                  : "memory");
-    (void)state;
 }
-__device__ __forceinline__ bool mbar_test(uint64_t *bar, uint32_t parity) {
+// mbarrier.try_wait suspends the thread until the phase completes or a
+// hardware time limit passes, so a waiting warp costs no issue slots and
+// resumes as soon as the phase flips.
+__device__ __forceinline__ bool mbar_try(uint64_t *bar, uint32_t parity) {
     uint32_t ok;
     asm volatile(
-        "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
         " selp.u32 %0, 1, 0, p;\n}\n"
         : "=r"(ok)
         : "r"(smem_addr(bar)), "r"(parity)
         : "memory");
     return ok != 0;
 }
-// Bounded wait for the phase of parity `parity`; false (and an error bit) on
-// expiry.
+__device__ __forceinline__ uint64_t global_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+// Bounded wait for the phase of parity `parity`: false (and an error bit)
+// after kWaitNs nanoseconds or kWaitLimit attempts, whichever comes first.
+constexpr uint64_t kWaitNs = 1000000000ull;
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, uint32_t *err) {
+    if (mbar_try(bar, parity)) return true;
+    const uint64_t t0 = global_ns();
     for (uint32_t i = 0; i < kWaitLimit; ++i) {
-        if (mbar_test(bar, parity)) return true;
-        if (i > 32) __nanosleep(64);
+        if (mbar_try(bar, parity)) return true;
+        if (global_ns() - t0 > kWaitNs) break;
     }
     record_error(err, kErrMmaTimeout);
     return false;
+}
+
+// The same wait taken by a whole warp: every lane polls, and the warp goes on
+// only if every lane saw the phase, so the lanes stay converged for the
+// .sync.aligned tcgen05 instructions and the warp-level arrivals that follow.
+__device__ __forceinline__ bool mbar_wait_warp(uint64_t *bar, uint32_t parity, uint32_t *err) {
+    return __all_sync(kFull, mbar_wait(bar, parity, err));
+}
+
+// Arrival on a barrier of any CTA of the cluster (address from mapa).
+__device__ __forceinline__ uint32_t cluster_addr(const void *p, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_addr(p)), "r"(rank));
+    return r;
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t addr) {
+    asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(addr) : "memory");
 }
 
 // ---------------------------------------------------------------- async copies, fences
@@ -107,6 +145,15 @@ __device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t by
         "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
             smem_addr(dst)),
         "l"(src), "r"(bytes), "r"(smem_addr(bar))
+        : "memory");
+}
+// 2-D tiled TMA load of box {x .. x+63, y .. y+127} into shared memory;
+// elements outside the tensor arrive as zeros.
+__device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, int x, int y, uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+            smem_addr(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
         : "memory");
 }
 __device__ __forceinline__ void fence_async_smem() {
@@ -132,21 +179,25 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
     return d;
 }
 // Instruction descriptor, kind::f16: fp16 A and B (format 0), f32 D (1),
-// both K-major, N = 256, M = 128.
+// both K-major, N = 256, M = 256 (the pair's two 128-row halves).
 constexpr uint32_t kIdesc = (1u << 4) | (0u << 7) | (0u << 10) | ((uint32_t)(kBN >> 3) << 17) |
-                            ((uint32_t)(kBM >> 4) << 24);
+                            ((uint32_t)(2 * kBM >> 4) << 24);
 
-__device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+__device__ __forceinline__ void mma_pair(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
                                          uint32_t accumulate) {
     asm volatile(
         "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+        " tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
         "l"(adesc), "l"(bdesc), "r"(kIdesc), "r"(accumulate));
 }
-__device__ __forceinline__ void mma_commit(uint64_t *bar) {
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-                     smem_addr(bar))
-                 : "memory");
+// Arrive on `bar` (same offset) in every CTA of `mask` once all MMAs issued
+// so far have completed.
+__device__ __forceinline__ void mma_commit_pair(uint64_t *bar, uint16_t mask) {
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+            smem_addr(bar)),
+        "h"(mask)
+        : "memory");
 }
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
     asm volatile(
@@ -183,6 +234,27 @@ __device__ __forceinline__ uint32_t f16x2_of_int(int lo, int hi) {
     const __half2 v = __halves2half2(__int2half_rn(lo), __int2half_rn(hi));
     return *reinterpret_cast<const uint32_t *>(&v);
 }
+
+// ---------------------------------------------------------------- epilogue arithmetic
+// Four exact digit-plane sums s_l (|s_l| <= 2^24, one chunk) -> 
+//     (s_0 + 2^8 s_1 + 2^16 s_2 + 2^24 s_3) * 2^-32 mod q,
+// in [0, q).  The combination is formed in int64 (|.| < 2^48.01) and shifted
+// by K0 = 2^18 q (> 2^48.01, a multiple of q) to u in (0, 2^50); Montgomery's
+// REDC with R = 2^32 then gives (u + m q) / 2^32 < 2^18 + q < 2q, where
+// m = -u q^-1 mod 2^32, and one conditional subtraction finishes.  The factor
+// 2^-32 is the same for every term of an output's sum and is removed once,
+// after the last chunk (kR2 below).
+constexpr int64_t kK0 = (int64_t)PVMVMD_Q << 18;
+__device__ __forceinline__ uint32_t digits_redc(int s0, int s1, int s2, int s3) {
+    const uint64_t u = (uint64_t)((int64_t)s0 + kK0 + (int64_t)s1 * 256 + (int64_t)s2 * 65536 +
+                                  (int64_t)s3 * 16777216);
+    const uint32_t m = (uint32_t)u * kQInvNeg;
+    const uint32_t r = (uint32_t)((u + (uint64_t)m * kQ) >> 32);
+    return r >= kQ ? r - kQ : r;
+}
+// R^2 mod q for R = 2^32: fmul_mont(x, kR2) = x R mod q undoes the 2^-32.
+constexpr uint32_t kRmodQ = (uint32_t)((1ull << 32) % PVMVMD_Q);
+constexpr uint32_t kR2 = (uint32_t)(((uint64_t)kRmodQ * kRmodQ) % PVMVMD_Q);
 
 // ---------------------------------------------------------------- digit operand
 // X_hat (B x K u32) -> pre-tiled fp16 digit operand: for vector tile nt and
@@ -226,12 +298,20 @@ __global__ void __launch_bounds__(256) k_digit_tiles(const uint32_t *__restrict_
 // ---------------------------------------------------------------- main kernel
 template <bool kVec>
 __global__ void __launch_bounds__(kThreads, 1)
-    k_batched(const int8_t *__restrict__ W, int m, int K, const uint8_t *__restrict__ D, int nkb,
-              int B, uint32_t *__restrict__ Yhat, uint32_t *__restrict__ err) {
+    k_batched(const __grid_constant__ CUtensorMap tmap_w, const int8_t *__restrict__ W, int m, int K,
+              const uint8_t *__restrict__ D, int nkb, int B, uint32_t *__restrict__ Yhat,
+              uint32_t *__restrict__ err) {
     cg::cluster_group cluster = cg::this_cluster();
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t full_a[kStages], full_b[kStages], empty_bar[kStages];
+    // full: this CTA's stage is complete -- the converter group's warps have
+    // arrived, the digit half has landed (transaction bytes) and, in the even
+    // CTA, the odd CTA has reported its own stage complete;
+    // empty: the pair's MMAs on the stage finished (commit from the even CTA);
+    // acc_full / acc_empty: the accumulator buffer is ready / drained by the
+    // epilogue warps of both CTAs (arrivals land in the even CTA).
+    __shared__ __align__(8) uint64_t full[kStages], empty_bar[kStages];
     __shared__ __align__(8) uint64_t acc_full[2], acc_empty[2], mma_done;
+    __shared__ __align__(8) uint64_t raw_full[kRaw], raw_empty[kRaw];  // raw int8 tile ring
     __shared__ uint32_t s_tmem;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -240,101 +320,123 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     const int m0 = blockIdx.x * kBM;
     const int nt = blockIdx.y;
-    const int split = (int)cluster.num_blocks();
-    const int rank = (int)cluster.block_rank();
+    const uint32_t rank = cluster.block_rank();  // = (blockIdx.x & 1) + 2 * blockIdx.z
+    const uint32_t half = rank & 1u;             // 0: the even CTA, which issues the MMAs
+    const uint32_t leader = rank & ~1u;
+    const uint16_t pair_mask = (uint16_t)(3u << leader);
+    const int split = (int)cluster.num_blocks() / 2;
+    const int zr = (int)(rank >> 1);
     const int per = (nkb + split - 1) / split;
-    const int kb0 = rank * per;
+    const int kb0 = zr * per;
     const int kb1 = min(nkb, kb0 + per);
     const int nblk = max(0, kb1 - kb0);
     const int nchunks = (nblk + kChunkBlocks - 1) / kChunkBlocks;
 
     if (tid == 0) {
         for (int s = 0; s < kStages; ++s) {
-            mbar_init(&full_a[s], kConvThreads);
-            mbar_init(&full_b[s], 1);
+            // the warps of one converter group + the digit copy's arrival
+            // (+ the odd CTA's report, in the even CTA)
+            mbar_init(&full[s], kConvThreads / 64 + 1 + (half == 0 ? 1 : 0));
             mbar_init(&empty_bar[s], 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&acc_full[b], 1);
-            mbar_init(&acc_empty[b], kEpiThreads);
+            mbar_init(&acc_empty[b], 2 * kEpiThreads / 32);  // epilogue warps of both CTAs
         }
         mbar_init(&mma_done, 1);
+        for (int r = 0; r < kRaw; ++r) {
+            mbar_init(&raw_full[r], 1);
+            mbar_init(&raw_empty[r], kConvThreads / 64);
+        }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
-    if (warp == kWarpMma) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 512;" ::"r"(
+    if (warp == kWarpMma) {  // one warp of each CTA of the pair allocates together
+        asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], 512;" ::"r"(
                          smem_addr(&s_tmem)));
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;");
     }
     tc_fence_before();
-    __syncthreads();
+    cluster.sync();  // barriers initialised and TMEM allocated in every CTA
     tc_fence_after();
     const uint32_t tmem = s_tmem;
 
-    uint32_t run[32];  // epilogue: running mod-q sums of 32 vectors for one row
+    uint32_t run[32];  // epilogue: running sums of 32 vectors for one row, times 2^-32 mod q
 #pragma unroll
     for (int v = 0; v < 32; ++v) run[v] = 0u;
 
     if (warp < 8) {
         // ------------------------------------------------ A: int8 M tile -> fp16 swizzled
-        const int r = tid >> 1, half = tid & 1;  // row, and which 32 K-elements of the block
-        const int grow = m0 + r;
-        const bool row_ok = grow < m;
-        const int8_t *wrow = W + (size_t)(row_ok ? grow : 0) * K;
-        constexpr int PF = 4;
-        uint4 buf[PF][2];
-        auto load = [&](int i, uint4 (&dst)[2]) {
-            const int k0 = (kb0 + i) * kBK + 32 * half;
-            if (kVec && row_ok && k0 + 32 <= K) {
-                dst[0] = __ldg(reinterpret_cast<const uint4 *>(wrow + k0));
-                dst[1] = __ldg(reinterpret_cast<const uint4 *>(wrow + k0) + 1);
-            } else {
-                uint32_t w[8];
+        // Two groups of four warps take alternate K-blocks.  In a block,
+        // thread t of a group converts 16 K-elements (two 16-byte fp16
+        // chunks) of rows t/4 + 32 j, j = 0..3: a quarter-warp covers one
+        // row's 64 bytes.
+        const int grp = warp >> 2;
+        const int t = tid & 127;
+        const int r0 = t >> 2, qk = t & 3;
+        auto convert_store = [&](uint8_t *a, const uint4 (&v)[4]) {
 #pragma unroll
-                for (int q = 0; q < 8; ++q) w[q] = 0;
-                if (row_ok)
-                    for (int e = 0; e < 32 && k0 + e < K; ++e)
-                        w[e >> 2] |= (uint32_t)(uint8_t)wrow[k0 + e] << (8 * (e & 3));
-                dst[0] = make_uint4(w[0], w[1], w[2], w[3]);
-                dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
+            for (int j = 0; j < 4; ++j) {  // 16 int8 -> two 16-byte fp16 chunks
+                uint32_t o[8];
+                i8x4_to_f16x4(v[j].x, o[0], o[1]);
+                i8x4_to_f16x4(v[j].y, o[2], o[3]);
+                i8x4_to_f16x4(v[j].z, o[4], o[5]);
+                i8x4_to_f16x4(v[j].w, o[6], o[7]);
+                const int row = r0 + 32 * j;
+                *reinterpret_cast<uint4 *>(a + sw128_off(row, 2 * qk)) = make_uint4(o[0], o[1], o[2], o[3]);
+                *reinterpret_cast<uint4 *>(a + sw128_off(row, 2 * qk + 1)) = make_uint4(o[4], o[5], o[6], o[7]);
             }
         };
+        if constexpr (kVec) {
+            // the int8 tile arrives by TMA (warp 18)
+            for (int i = grp; i < nblk; i += 2) {
+                const int s = i % kStages, rs = i % kRaw;
+                const uint32_t ph = (uint32_t)(i / kStages) & 1u, rph = (uint32_t)(i / kRaw) & 1u;
+                if (!mbar_wait_warp(&raw_full[rs], rph, err) || !mbar_wait_warp(&empty_bar[s], ph ^ 1u, err))
+                    break;
+                const uint8_t *raw = smem + kRawOff + rs * kRawTile;
+                uint4 v[4];
 #pragma unroll
-        for (int u = 0; u < PF; ++u)
-            if (u < nblk) load(u, buf[u]);
-        bool ok = true;
-        for (int i0 = 0; i0 < nblk && ok; i0 += PF) {
-#pragma unroll
-            for (int u = 0; u < PF; ++u) {
-                const int i = i0 + u;
-                if (i >= nblk || !ok) break;
+                for (int j = 0; j < 4; ++j)
+                    v[j] = *reinterpret_cast<const uint4 *>(raw + (r0 + 32 * j) * kBK + 16 * qk);
+                convert_store(smem + s * kStageBytes, v);
+                fence_async_smem();  // this thread's stores -> visible to the tensor cores
+                __syncwarp();
+                if (lane == 0) {
+                    mbar_arrive(&full[s]);
+                    mbar_arrive(&raw_empty[rs]);
+                }
+            }
+        } else {
+            // rows of any length and alignment: plain byte loads
+            for (int i = grp; i < nblk; i += 2) {
                 const int s = i % kStages;
                 const uint32_t ph = (uint32_t)(i / kStages) & 1u;
-                if (!mbar_wait(&empty_bar[s], ph ^ 1u, err)) { ok = false; break; }
-                uint8_t *a = smem + s * kStageBytes;
+                const int k0 = (kb0 + i) * kBK + 16 * qk;
+                uint4 v[4];
 #pragma unroll
-                for (int c = 0; c < 2; ++c) {  // 16 int8 -> two 16-byte fp16 chunks
-                    uint32_t o[8];
-                    i8x4_to_f16x4(buf[u][c].x, o[0], o[1]);
-                    i8x4_to_f16x4(buf[u][c].y, o[2], o[3]);
-                    i8x4_to_f16x4(buf[u][c].z, o[4], o[5]);
-                    i8x4_to_f16x4(buf[u][c].w, o[6], o[7]);
-                    const int chunk = 4 * half + 2 * c;
-                    *reinterpret_cast<uint4 *>(a + sw128_off(r, chunk)) = make_uint4(o[0], o[1], o[2], o[3]);
-                    *reinterpret_cast<uint4 *>(a + sw128_off(r, chunk + 1)) = make_uint4(o[4], o[5], o[6], o[7]);
+                for (int j = 0; j < 4; ++j) {
+                    const int grow = m0 + r0 + 32 * j;
+                    uint32_t w[4] = {0u, 0u, 0u, 0u};
+                    if (grow < m)
+                        for (int e = 0; e < 16 && k0 + e < K; ++e)
+                            w[e >> 2] |= (uint32_t)(uint8_t)W[(size_t)grow * K + k0 + e] << (8 * (e & 3));
+                    v[j] = make_uint4(w[0], w[1], w[2], w[3]);
                 }
+                if (!mbar_wait_warp(&empty_bar[s], ph ^ 1u, err)) break;
+                convert_store(smem + s * kStageBytes, v);
                 fence_async_smem();
-                mbar_arrive(&full_a[s]);
-                if (i + PF < nblk) load(i + PF, buf[u]);
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&full[s]);
             }
         }
     } else if (warp < 16) {
         // ------------------------------------------------ epilogue: TMEM -> mod-q sums
         const int q = warp & 3;            // TMEM lane quadrant
         const int grp = (warp - 8) >> 2;   // vectors 32 grp .. 32 grp + 31
+        const uint32_t acc_empty_leader = cluster_addr(&acc_empty[0], leader);
         for (int c = 0; c < nchunks; ++c) {
             const int bsel = c & 1;
-            if (!mbar_wait(&acc_full[bsel], (uint32_t)(c >> 1) & 1u, err)) break;
+            if (!mbar_wait_warp(&acc_full[bsel], (uint32_t)(c >> 1) & 1u, err)) break;
             tc_fence_after();
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
@@ -342,37 +444,53 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tmem_ld32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(bsel * kBN + 128 * grp + 32 * j), r);
 #pragma unroll
                 for (int v = 0; v < 8; ++v) {
-                    const long long d0 = __float2int_rn(__uint_as_float(r[4 * v]));
-                    const long long d1 = __float2int_rn(__uint_as_float(r[4 * v + 1]));
-                    const long long d2 = __float2int_rn(__uint_as_float(r[4 * v + 2]));
-                    const long long d3 = __float2int_rn(__uint_as_float(r[4 * v + 3]));
                     run[8 * j + v] = fadd(run[8 * j + v],
-                                          fred_signed(d0 + (d1 << 8) + (d2 << 16) + (d3 << 24)));
+                                          digits_redc(__float2int_rn(__uint_as_float(r[4 * v])),
+                                                      __float2int_rn(__uint_as_float(r[4 * v + 1])),
+                                                      __float2int_rn(__uint_as_float(r[4 * v + 2])),
+                                                      __float2int_rn(__uint_as_float(r[4 * v + 3]))));
                 }
             }
             tc_fence_before();
-            mbar_arrive(&acc_empty[bsel]);
+            __syncwarp();
+            if (lane == 0) mbar_arrive_cluster(acc_empty_leader + 8u * (uint32_t)bsel);
         }
     } else if (warp == kWarpLoader) {
-        // ------------------------------------------------ B: bulk copies of digit tiles
+        // ------------------------------------------------ B: this CTA's digit half
         if (lane == 0) {
-            const uint8_t *src = D + ((size_t)nt * nkb + kb0) * kBTile;
+            const uint8_t *src = D + ((size_t)nt * nkb + kb0) * kBTile + (size_t)half * kBHalf;
             int issued = 0;
             for (int i = 0; i < nblk; ++i) {
                 const int s = i % kStages;
                 const uint32_t ph = (uint32_t)(i / kStages) & 1u;
                 if (!mbar_wait(&empty_bar[s], ph ^ 1u, err)) break;
                 uint8_t *b = smem + s * kStageBytes + kATile;
-                mbar_arrive_tx(&full_b[s], kBTile);
-                bulk_g2s(b, src + (size_t)i * kBTile, kBTile, &full_b[s]);
+                mbar_arrive_tx(&full[s], kBHalf);
+                bulk_g2s(b, src + (size_t)i * kBTile, kBHalf, &full[s]);
                 issued = i + 1;
             }
             // copies in flight complete before the CTA may exit
             for (int i = max(0, issued - kStages); i < issued; ++i)
-                mbar_wait(&full_b[i % kStages], (uint32_t)(i / kStages) & 1u, err);
+                mbar_wait(&full[i % kStages], (uint32_t)(i / kStages) & 1u, err);
         }
-    } else {
-        // ------------------------------------------------ MMA issuer
+    } else if (warp == kWarpWLoad) {
+        // ------------------------------------------------ raw int8 tiles of M by TMA
+        if (kVec && lane == 0) {
+            int issued = 0;
+            for (int i = 0; i < nblk; ++i) {
+                const int rs = i % kRaw;
+                const uint32_t rph = (uint32_t)(i / kRaw) & 1u;
+                if (!mbar_wait(&raw_empty[rs], rph ^ 1u, err)) break;
+                mbar_arrive_tx(&raw_full[rs], kRawTile);
+                tma_load_2d(smem + kRawOff + rs * kRawTile, &tmap_w, (kb0 + i) * kBK, m0, &raw_full[rs]);
+                issued = i + 1;
+            }
+            // copies in flight complete before the CTA may exit
+            for (int i = max(0, issued - kRaw); i < issued; ++i)
+                mbar_wait(&raw_full[i % kRaw], (uint32_t)(i / kRaw) & 1u, err);
+        }
+    } else if (half == 0) {
+        // ------------------------------------------------ MMA issuer (even CTA)
         if (lane == 0) {
             bool ok = true;
             for (int c = 0; c < nchunks && ok; ++c) {
@@ -384,7 +502,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int i = c * kChunkBlocks; i < i_end; ++i) {
                     const int s = i % kStages;
                     const uint32_t ph = (uint32_t)(i / kStages) & 1u;
-                    if (!mbar_wait(&full_a[s], ph, err) || !mbar_wait(&full_b[s], ph, err)) {
+                    if (!mbar_wait(&full[s], ph, err)) {
                         ok = false;
                         break;
                     }
@@ -393,22 +511,34 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const uint32_t b_addr = a_addr + kATile;
 #pragma unroll
                     for (int k = 0; k < kBK / 16; ++k) {
-                        mma_bf16(dcol, sw128_desc(a_addr + 32u * k), sw128_desc(b_addr + 32u * k),
+                        mma_pair(dcol, sw128_desc(a_addr + 32u * k), sw128_desc(b_addr + 32u * k),
                                  (i > c * kChunkBlocks || k > 0) ? 1u : 0u);
                     }
-                    mma_commit(&empty_bar[s]);
+                    mma_commit_pair(&empty_bar[s], pair_mask);
                 }
-                mma_commit(&acc_full[bsel]);
+                mma_commit_pair(&acc_full[bsel], pair_mask);
             }
             // all issued MMAs have finished before TMEM is released
-            mma_commit(&mma_done);
+            mma_commit_pair(&mma_done, (uint16_t)(1u << leader));
             mbar_wait(&mma_done, 0, err);
+        }
+    } else {
+        // ------------------------------------------------ stage relay (odd CTA)
+        if (lane == 0) {
+            const uint32_t full_leader = cluster_addr(&full[0], leader);
+            for (int i = 0; i < nblk; ++i) {
+                const int s = i % kStages;
+                const uint32_t ph = (uint32_t)(i / kStages) & 1u;
+                if (!mbar_wait(&full[s], ph, err)) break;
+                mbar_arrive_cluster(full_leader + 8u * (uint32_t)s);
+            }
         }
     }
 
     // ---------------------------------------------------- split-K reduction and store
     tc_fence_before();
-    __syncthreads();  // every stage is consumed: the stage memory is reused below
+    __syncthreads();  // this CTA's roles are done
+    cluster.sync();   // ... and the peer's: no MMA reads this CTA's stages any more
     uint32_t *part = reinterpret_cast<uint32_t *>(smem);  // [kBV][kBM] mod-q partial sums
     if (warp >= 8 && warp < 16) {
         const int row = 32 * (warp & 3) + lane;
@@ -417,30 +547,66 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int v = 0; v < 32; ++v) part[(v0 + v) * kBM + row] = run[v];
     }
     cluster.sync();
-    // rank r finishes vectors [r * 64 / split, (r + 1) * 64 / split)
+    // the CTA at K-rank zr finishes vectors [zr * 64 / split, (zr + 1) * 64 / split)
     const int vper = kBV / split;
     for (int idx = tid; idx < vper * kBM; idx += kThreads) {
-        const int v = rank * vper + idx / kBM, row = idx % kBM;
+        const int v = zr * vper + idx / kBM, row = idx % kBM;
         uint32_t sum = 0;
-        for (int rr = 0; rr < split; ++rr) sum = fadd(sum, cluster.map_shared_rank(part, rr)[v * kBM + row]);
+        for (int rr = 0; rr < split; ++rr)
+            sum = fadd(sum, cluster.map_shared_rank(part, (unsigned)(2 * rr) + half)[v * kBM + row]);
+        sum = fmul_mont(sum, kR2);
         const int b = nt * kBV + v, grow = m0 + row;
         if (grow < m && b < B) Yhat[(size_t)b * m + grow] = sum;
     }
     cluster.sync();
     if (warp == kWarpMma) {
         tc_fence_after();
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem));
+        asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, 512;" ::"r"(tmem));
     }
 }
 
-// Cluster split of K: the fewest CTAs per tile that still give the fewest
-// waves per unit of work, with at least 4 K-blocks per CTA.
-int choose_split(int tiles, int nkb, int sms) {
+// Resident clusters of (2, 1, split) CTAs of the kernel, from the occupancy
+// calculator (a cluster must fit in one GPC), cached per split.
+int resident_clusters(const void *kern, int split) {
+    static int cache[8] = {0};
+    static std::mutex mu;
+    std::lock_guard<std::mutex> lock(mu);
+    int &c = cache[split];
+    if (c == 0) {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(2, 1, split);
+        cfg.blockDim = dim3(kThreads, 1, 1);
+        cfg.dynamicSmemBytes = kMmaSmem;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = 2;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = split;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        int n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess || n <= 0) {
+            (void)cudaGetLastError();
+            int dev = 0, sms = 0;
+            cudaGetDevice(&dev);
+            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+            n = max(1, sms / (2 * split));
+        }
+        c = n;
+    }
+    return c;
+}
+
+// Cluster split of K: the fewest pairs per tile that still give the fewest
+// waves per unit of work, with at least 4 K-blocks per pair.
+int choose_split(const void *kern, int pairs, int nkb) {
     int best = 1;
     double best_cost = 1e30;
-    for (int split = 1; split <= 8; split *= 2) {
+    for (int split = 1; split <= 4; split *= 2) {
         if (split > 1 && nkb < 4 * split) break;
-        const int waves = (tiles * split + sms - 1) / sms;
+        const int clusters = pairs;  // one cluster of `split` pairs per tile pair
+        const int cap = resident_clusters(kern, split);
+        const int waves = (clusters + cap - 1) / cap;
         const double cost = (double)waves / split + 0.02 * (split - 1);
         if (cost < best_cost - 1e-9) {
             best_cost = cost;
@@ -448,6 +614,22 @@ int choose_split(int tiles, int nkb, int sms) {
         }
     }
     return best;
+}
+
+// cuTensorMapEncodeTiled from the driver, looked up once.
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) !=
+                cudaSuccess ||
+            q != cudaDriverEntryPointSuccess) {
+            (void)cudaGetLastError();
+            p = nullptr;
+        }
+        return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    }();
+    return fn;
 }
 
 cudaError_t batched_launch(const int8_t *W, int m, int K, const uint32_t *Xhat, int B, uint32_t *Yhat,
@@ -458,12 +640,23 @@ cudaError_t batched_launch(const int8_t *W, int m, int K, const uint32_t *Xhat, 
     k_digit_tiles<<<(unsigned)((threads + 255) / 256), 256, 0, s>>>(Xhat, B, K, nkb, nvt, D);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    int dev = 0, sms = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    const int mt = (m + kBM - 1) / kBM;
-    const int split = choose_split(mt * nvt, nkb, sms);
+    const int mp = (m + 2 * kBM - 1) / (2 * kBM);  // CTA pairs along M
+    // M as a K x m tensor of bytes for TMA: needs 16-byte aligned rows
     const bool vec = (K % 16 == 0) && ((reinterpret_cast<uintptr_t>(W) & 15u) == 0);
+    CUtensorMap tmap;
+    memset(&tmap, 0, sizeof(tmap));
+    if (vec) {
+        PFN_cuTensorMapEncodeTiled_v12000 encode = tensor_map_encoder();
+        if (!encode) return cudaErrorNotSupported;
+        const cuuint64_t gdim[2] = {(cuuint64_t)K, (cuuint64_t)m};
+        const cuuint64_t gstride[1] = {(cuuint64_t)K};
+        const cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)kBM};
+        const cuuint32_t estride[2] = {1, 1};
+        if (encode(&tmap, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<int8_t *>(W), gdim, gstride, box, estride,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+    }
     auto kern = vec ? k_batched<true> : k_batched<false>;
     static const cudaError_t a1 =
         cudaFuncSetAttribute(k_batched<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
@@ -471,19 +664,20 @@ cudaError_t batched_launch(const int8_t *W, int m, int K, const uint32_t *Xhat, 
         cudaFuncSetAttribute(k_batched<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
     if (a1 != cudaSuccess) return a1;
     if (a2 != cudaSuccess) return a2;
+    const int split = choose_split((const void *)kern, mp * nvt, nkb);
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(mt, nvt, split);
+    cfg.gridDim = dim3(2 * mp, nvt, split);
     cfg.blockDim = dim3(kThreads, 1, 1);
     cfg.dynamicSmemBytes = kMmaSmem;
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = 1;
+    attr[0].val.clusterDim.x = 2;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = split;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kern, W, m, K, (const uint8_t *)D, nkb, B, Yhat, err);
+    return cudaLaunchKernelEx(&cfg, kern, tmap, W, m, K, (const uint8_t *)D, nkb, B, Yhat, err);
 }
 
 // ---------------------------------------------------------------- scratch for the digit operand
