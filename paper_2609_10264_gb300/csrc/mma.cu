@@ -263,6 +263,9 @@ constexpr uint32_t kR2 = (uint32_t)(((uint64_t)kRmodQ * kRmodQ) % PVMVMD_Q);
 // (vector, 8 K-elements).
 __global__ void __launch_bounds__(256) k_digit_tiles(const uint32_t *__restrict__ Xhat, int B, int K,
                                                     int nkb, int nvt, uint8_t *__restrict__ D) {
+    // the product kernel may start its set-up now; it reads these tiles only
+    // after griddepcontrol.wait
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const size_t gid = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
     const size_t per_vec = (size_t)nkb * 8;  // 8-element groups per vector
     const size_t total = (size_t)nvt * kBV * per_vec;
@@ -459,6 +462,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ------------------------------------------------ B: this CTA's digit half
         if (lane == 0) {
             const uint8_t *src = D + ((size_t)nt * nkb + kb0) * kBTile + (size_t)half * kBHalf;
+            // the digit tiles come from the kernel launched just before this one
+            asm volatile("griddepcontrol.wait;" ::: "memory");
             int issued = 0;
             for (int i = 0; i < nblk; ++i) {
                 const int s = i % kStages;
@@ -670,13 +675,17 @@ cudaError_t batched_launch(const int8_t *W, int m, int K, const uint32_t *Xhat, 
     cfg.blockDim = dim3(kThreads, 1, 1);
     cfg.dynamicSmemBytes = kMmaSmem;
     cfg.stream = s;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = 2;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = split;
+    // programmatic dependent launch: barrier set-up, TMEM allocation and the
+    // first weight tiles overlap the digit-tile kernel
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     return cudaLaunchKernelEx(&cfg, kern, tmap, W, m, K, (const uint8_t *)D, nkb, B, Yhat, err);
 }
 
