@@ -25,6 +25,10 @@ constexpr uint32_t kTagCodeX = 1;       // G_x: pi1 = 1, pi2 = 2, v1 = 3, v2 = 4
 constexpr uint32_t kTagCodeY = 5;       // G_y: pi1 = 5, pi2 = 6, v1 = 7, v2 = 8
 constexpr uint32_t kTagMask = 9;
 constexpr uint32_t kTagChallenge = 10;
+// Encode batches of at least this many vectors as the lanes of N x B arrays
+// (launch_lane_syndrome) when the code needs a cluster per vector; smaller
+// batches and codes that fit one CTA use the fused kernel.
+constexpr int kLaneMinBatch = 32;
 
 // --------------------------------------------------------------------------
 // Host ChaCha20 keystream (RFC 8439 Sec. 2.3) read as 32-bit words.
@@ -173,6 +177,8 @@ struct pvmvmd_ctx {
     uint32_t *PT = nullptr, *Q = nullptr;
     uint32_t *F = nullptr, *Fy = nullptr, *chal = nullptr, *g = nullptr, *u = nullptr;
     unsigned long long *status = nullptr;
+    // lane-parallel encode scratch (null when scratch_batch < kLaneMinBatch)
+    uint32_t *S = nullptr, *laux = nullptr;
     std::vector<void *> owned;
 };
 
@@ -372,12 +378,16 @@ int pvmvmd_preprocess(const int8_t *W_dev, int m, int K, const pvmvmd_params *pa
     const size_t statw = std::max(scan_status_words(c->Nx, c->sb), scan_status_words(c->Ny, c->ell));
     if (ctx_alloc(c, &c->PT, (size_t)c->Nx * m) != cudaSuccess ||
         ctx_alloc(c, &c->Q, (size_t)c->Ny * K) != cudaSuccess ||
-        ctx_alloc(c, &c->F, (size_t)c->sb * c->Nx) != cudaSuccess ||
+        ctx_alloc(c, &c->F, (size_t)((c->sb + 3) & ~3) * c->Nx) != cudaSuccess ||  // lanes padded to 4
         ctx_alloc(c, &c->Fy, (size_t)c->ell * c->Ny) != cudaSuccess ||
         ctx_alloc(c, &c->chal, (size_t)c->ell * 2 * c->t_y) != cudaSuccess ||
         ctx_alloc(c, &c->g, (size_t)c->ell * m) != cudaSuccess ||
         ctx_alloc(c, &c->u, (size_t)c->ell * K) != cudaSuccess ||
         ctx_alloc(c, &c->status, statw) != cudaSuccess)
+        return fail(PVMVMD_E_NOMEM);
+    if (c->sb >= kLaneMinBatch &&
+        (ctx_alloc(c, &c->S, (size_t)c->sb * (c->t_x + 1)) != cudaSuccess ||
+         ctx_alloc(c, &c->laux, lane_aux_words(c->Nx, c->sb)) != cudaSuccess))
         return fail(PVMVMD_E_NOMEM);
 
     // P^T = G_x^T M^T: the m rows of M are the lanes, so transpose M first.
@@ -416,7 +426,21 @@ int pvmvmd_encode(pvmvmd_ctx *ctx, const uint32_t *X_dev, int B, const pvmvmd_ke
     int C;
     uint32_t slice;
     size_t smem;
-    if (syndrome_fused_plan(ctx->Nx, ctx->t_x, &C, &slice, &smem)) {
+    const bool fused = syndrome_fused_plan(ctx->Nx, ctx->t_x, &C, &slice, &smem);
+    if (B >= kLaneMinBatch && ctx->laux && !(fused && C == 1)) {
+        // vectors as lanes: every permutation step moves whole rows (a code
+        // that fits one CTA's shared memory stays on chip in the fused kernel)
+        for (int b0 = 0; b0 < B; b0 += ctx->sb) {
+            const uint32_t L = (uint32_t)(B - b0 < ctx->sb ? B - b0 : ctx->sb);
+            PV_CUDA(launch_lane_syndrome(*key, kTagMask, (uint64_t)b0, ctx->Nx, ctx->t_x, L, d.pi2,
+                                         d.v2m, d.v1, d.pi1inv, ctx->K, ctx->rate,
+                                         stp + (size_t)b0 * 2 * ctx->t_x, ctx->S, ctx->F, ctx->laux,
+                                         X_dev + (size_t)b0 * ctx->K, Xhat_dev + (size_t)b0 * ctx->K,
+                                         s));
+        }
+        return PVMVMD_OK;
+    }
+    if (fused) {
         // sample, scan and gather in one launch per batch, no scratch
         PV_CUDA(launch_syndrome_fused(*key, kTagMask, 0, ctx->Nx, ctx->t_x, (uint32_t)B, d.pi2inv,
                                       d.v2p, d.v1, d.pi1inv, d.pi2, d.v2m, d.v1pm, ctx->K, ctx->rate,

@@ -8,6 +8,8 @@
 //                         block sums of R, fused with x_hat = x + x'.
 //  * k_encode_scan        one accumulate stage of the encoding G^T w over many
 //                         lanes (preprocessing of P^T and Q, Sec. 6.3).
+//  * k_lane_*             the syndrome for a batch of vectors held as the lanes
+//                         of an N x B array (sample, step function, scan, gather).
 #include <cooperative_groups.h>
 
 #include "common.cuh"
@@ -787,6 +789,300 @@ __global__ void k_transpose_i8(const int8_t *__restrict__ in, int R, int C, int8
     }
 }
 
+// -----------------------------------------------------------------------------
+// Lane-parallel syndrome x' = G e for a batch of L vectors (Encrypt at large
+// batch).  The vectors are the lanes of an N x Lp array C (Lp = L rounded up
+// to a multiple of 4, lane index contiguous), so every permutation step of
+// G = R Pi1 V1 A Pi2 V2 A moves whole rows:
+//   C[pi2(k)][b] = v2_k (A e_b)_k,  (A e_b)_k = sum_{j: s_j >= k} e_j
+//                                                   (k_lane_expand)
+//   agg[tau][b]  = sum of C[i][b] over tile tau     (k_lane_tile_sum)
+//   carry[tau][b] = sum_{tau' > tau} agg[tau'][b]   (k_lane_carry)
+//   C[i][b] <- v1_i (carry + sum_{i' >= i in the tile} C[i'][b])
+//                                                   (k_lane_scan, in place)
+//   out[b][j] = addend[b][j] + sum_{c<r} C[pi1^-1(r j + c)][b]
+//                                                   (k_lane_gather)
+// A thread owns four consecutive lanes (16-byte accesses) of one tile or
+// span; a CTA of 256 threads covers `cols` lane quads (Lp/4 rounded up to 32,
+// at most 64) of 256 / cols tiles or spans.
+// -----------------------------------------------------------------------------
+constexpr int kLaneTile = 32;      // positions per tile (one thread walks them)
+constexpr int kLaneCta = 256;      // threads per lane CTA
+constexpr int kLaneQuadsMax = 64;  // lane quads per CTA (256 lanes)
+constexpr int kExpandSpan = 32;    // positions per expand thread (a multiple of 4)
+constexpr int kGatherJ = 16;       // outputs per gather CTA
+constexpr int kCarryChunks = 128;  // tile chunks per lane quad in the carry kernel
+
+__host__ __device__ inline uint32_t lane_pad(uint32_t L) { return (L + 3) & ~3u; }
+__host__ __device__ inline uint32_t lane_cols(uint32_t L) {  // lane quads per CTA
+    const uint32_t q = lane_pad(L) / 4, q32 = (q + 31) / 32 * 32;
+    return q32 < (uint32_t)kLaneQuadsMax ? q32 : (uint32_t)kLaneQuadsMax;
+}
+__device__ __forceinline__ uint4 fadd4(uint4 a, uint4 b) {
+    return make_uint4(fadd(a.x, b.x), fadd(a.y, b.y), fadd(a.z, b.z), fadd(a.w, b.w));
+}
+
+// e_b for vector idx0 + blockIdx.x as in k_sample_sparse (warp 0 the
+// support, warp 1 the values), written as st[b] = (ascending support,
+// values), and S[b][j] = sum_{j' >= j} values[j'], S[b][t] = 0.
+__global__ void __launch_bounds__(128) k_lane_sample(pvmvmd_key key, uint32_t tag, uint64_t idx0,
+                                                    uint32_t N, uint32_t t, uint32_t *__restrict__ st,
+                                                    uint32_t *__restrict__ S) {
+    extern __shared__ uint32_t sm[];
+    const uint32_t nbw = (N + 31) / 32;
+    uint32_t *bitmap = sm;
+    uint32_t *words = sm + nbw;      // 512 keystream words (support)
+    uint32_t *words2 = words + 512;  // 512 keystream words (values)
+    uint32_t *list = words2 + 512;   // t, in the order accepted
+    uint32_t *vals = list + t;       // t
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const uint64_t idx = idx0 + blockIdx.x;
+    uint32_t *supp = st + (size_t)blockIdx.x * 2 * t;
+    for (uint32_t w = tid; w < nbw; w += 128) bitmap[w] = 0u;
+    __syncthreads();
+    if (warp == 0) warp_sample_support_list(key, tag, 2 * idx, N, t, bitmap, words, list, lane);
+    else if (warp == 1) warp_sample_values(key, tag, 2 * idx + 1, t, words2, vals, lane);
+    __syncthreads();
+    for (uint32_t i = tid; i < t; i += 128) {  // ascending support by rank (entries distinct)
+        const uint32_t v = list[i];
+        uint32_t rk = 0;
+        for (uint32_t j = 0; j < t; ++j) rk += list[j] < v;
+        supp[rk] = v;
+        supp[t + i] = vals[i];
+    }
+    if (warp != 0) return;
+    uint32_t *Sb = S + (size_t)blockIdx.x * (t + 1);
+    // suffix sums: lane owns a contiguous chunk, chunks combined by shuffles
+    const uint32_t per = (t + 31) / 32;
+    const uint32_t lo = min(t, lane * per), hi = min(t, lo + per);
+    uint32_t sum = 0;
+    for (uint32_t j = hi; j-- > lo;) sum = fadd(sum, vals[j]);
+    uint32_t incl = sum;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_down_sync(kFull, incl, o);
+        if (lane + o < 32) incl = fadd(incl, y);
+    }
+    uint32_t run = fsub(incl, sum);  // sum over the chunks after this lane's
+    for (uint32_t j = hi; j-- > lo;) {
+        run = fadd(run, vals[j]);
+        Sb[j] = run;
+    }
+    if (lane == 0) Sb[t] = 0u;
+}
+
+// C[pi2(k)][b] = v2_k (A e_b)_k: a thread walks kExpandSpan positions k of
+// four lanes in order with a pointer per lane into the sorted support, and
+// writes the four lanes of row pi2(k) with one 16-byte store.
+__global__ void __launch_bounds__(kLaneCta) k_lane_expand(const uint32_t *__restrict__ st,
+                                                         const uint32_t *__restrict__ S, uint32_t t,
+                                                         uint32_t N, uint32_t L,
+                                                         const uint32_t *__restrict__ pi2,
+                                                         const uint32_t *__restrict__ v2m,
+                                                         uint4 *__restrict__ C) {
+    const uint32_t cols = lane_cols(L), Lq = lane_pad(L) / 4;
+    const uint32_t g = blockIdx.y * cols + threadIdx.x % cols;
+    const uint32_t k0 = (blockIdx.x * (kLaneCta / cols) + threadIdx.x / cols) * kExpandSpan;
+    const uint32_t k1 = min(N, k0 + kExpandSpan);
+    if (g >= Lq || k0 >= k1) return;
+    uint32_t j[4], next[4], cur[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const uint32_t b = 4 * g + q;
+        next[q] = 0xffffffffu;
+        cur[q] = 0u;
+        j[q] = 0u;
+        if (b < L) {
+            const uint32_t *supp = st + (size_t)b * 2 * t;
+            uint32_t lo = 0, hi = t;  // first support index with s_j >= k0
+            while (lo < hi) {
+                const uint32_t mid = (lo + hi) >> 1;
+                if (__ldg(supp + mid) < k0) lo = mid + 1; else hi = mid;
+            }
+            j[q] = lo;
+            next[q] = lo < t ? __ldg(supp + lo) : 0xffffffffu;
+            cur[q] = __ldg(S + (size_t)b * (t + 1) + lo);
+        }
+    }
+    for (uint32_t kb = k0; kb < k1; kb += 4) {  // k0 is a multiple of 4: 16-byte table loads
+        uint32_t pk[4], vk[4];
+        if (kb + 4 <= N) {
+            const uint4 a = __ldg(reinterpret_cast<const uint4 *>(pi2 + kb));
+            const uint4 c = __ldg(reinterpret_cast<const uint4 *>(v2m + kb));
+            pk[0] = a.x; pk[1] = a.y; pk[2] = a.z; pk[3] = a.w;
+            vk[0] = c.x; vk[1] = c.y; vk[2] = c.z; vk[3] = c.w;
+        } else {
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                pk[u] = kb + u < N ? __ldg(pi2 + kb + u) : 0u;
+                vk[u] = kb + u < N ? __ldg(v2m + kb + u) : 0u;
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const uint32_t k = kb + u;
+            if (k >= k1) break;
+            uint32_t o[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const uint32_t b = 4 * g + q;
+                while (next[q] < k) {
+                    ++j[q];
+                    next[q] = j[q] < t ? __ldg(st + (size_t)b * 2 * t + j[q]) : 0xffffffffu;
+                    cur[q] = __ldg(S + (size_t)b * (t + 1) + j[q]);
+                }
+                o[q] = fmul_mont(cur[q], vk[u]);
+            }
+            C[(size_t)pk[u] * Lq + g] = make_uint4(o[0], o[1], o[2], o[3]);
+        }
+    }
+}
+
+// agg[tau][b] = sum over the tile's positions of C[i][b].
+__global__ void __launch_bounds__(kLaneCta) k_lane_tile_sum(const uint4 *__restrict__ C, uint32_t N,
+                                                           uint32_t L, uint4 *__restrict__ agg) {
+    const uint32_t cols = lane_cols(L), Lq = lane_pad(L) / 4, ntiles = (N + kLaneTile - 1) / kLaneTile;
+    const uint32_t g = blockIdx.y * cols + threadIdx.x % cols;
+    const uint32_t tau = blockIdx.x * (kLaneCta / cols) + threadIdx.x / cols;
+    if (g >= Lq || tau >= ntiles) return;
+    const uint32_t i0 = tau * kLaneTile, i1 = min(N, i0 + kLaneTile);
+    uint4 sum = make_uint4(0u, 0u, 0u, 0u);
+    for (uint32_t i = i0; i < i1; i += 8) {
+        uint4 v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+            v[u] = i + u < i1 ? C[(size_t)(i + u) * Lq + g] : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) sum = fadd4(sum, v[u]);
+    }
+    agg[(size_t)tau * Lq + g] = sum;
+}
+
+// carry[tau][b] = sum_{tau' > tau} agg[tau'][b]: a CTA takes 8 lane quads;
+// thread (chunk c, quad) sums its chunk of tiles, the chunk sums are
+// combined in shared memory, then each thread writes its chunk's carries
+// walking down.
+__global__ void __launch_bounds__(8 * kCarryChunks) k_lane_carry(const uint4 *__restrict__ agg,
+                                                                uint32_t ntiles, uint32_t Lq,
+                                                                uint4 *__restrict__ carry) {
+    __shared__ uint4 part[kCarryChunks][8];
+    const uint32_t l = threadIdx.x & 7, c = threadIdx.x >> 3;
+    const uint32_t g = blockIdx.x * 8 + l;
+    const uint32_t per = (ntiles + kCarryChunks - 1) / kCarryChunks;
+    const uint32_t t0 = min(ntiles, c * per), t1 = min(ntiles, t0 + per);
+    uint4 sum = make_uint4(0u, 0u, 0u, 0u);
+    if (g < Lq) {
+        for (uint32_t tau = t0; tau < t1; tau += 8) {
+            uint4 v[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u)
+                v[u] = tau + u < t1 ? agg[(size_t)(tau + u) * Lq + g] : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+            for (int u = 0; u < 8; ++u) sum = fadd4(sum, v[u]);
+        }
+    }
+    part[c][l] = sum;
+    __syncthreads();
+    uint4 run = make_uint4(0u, 0u, 0u, 0u);  // sum over the chunks after this one
+    for (uint32_t cc = c + 1; cc < (uint32_t)kCarryChunks; ++cc) run = fadd4(run, part[cc][l]);
+    if (g >= Lq) return;
+    for (uint32_t hi = t1; hi > t0;) {  // eight tiles at a time, loads first
+        const uint32_t cnt = hi - t0 < 8u ? hi - t0 : 8u;
+        uint4 v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+            v[u] = (uint32_t)u < cnt ? agg[(size_t)(hi - 1 - u) * Lq + g] : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            if ((uint32_t)u < cnt) {
+                carry[(size_t)(hi - 1 - u) * Lq + g] = run;
+                run = fadd4(run, v[u]);
+            }
+        }
+        hi -= cnt;
+    }
+}
+
+// In place: C[i][b] <- v1_i (carry[tau][b] + sum_{i' >= i in tile tau} C[i'][b]).
+__global__ void __launch_bounds__(kLaneCta) k_lane_scan(uint4 *__restrict__ C, uint32_t N, uint32_t L,
+                                                       const uint4 *__restrict__ carry,
+                                                       const uint32_t *__restrict__ v1) {
+    const uint32_t cols = lane_cols(L), Lq = lane_pad(L) / 4, ntiles = (N + kLaneTile - 1) / kLaneTile;
+    const uint32_t g = blockIdx.y * cols + threadIdx.x % cols;
+    const uint32_t tau = blockIdx.x * (kLaneCta / cols) + threadIdx.x / cols;
+    if (g >= Lq || tau >= ntiles) return;
+    const uint32_t i0 = tau * kLaneTile, i1 = min(N, i0 + kLaneTile);
+    uint4 run = carry[(size_t)tau * Lq + g];
+    for (uint32_t hi = i1; hi > i0;) {
+        const uint32_t cnt = hi - i0 < 8u ? hi - i0 : 8u;  // positions hi-1 .. hi-cnt
+        uint4 v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+            v[u] = (uint32_t)u < cnt ? C[(size_t)(hi - 1 - u) * Lq + g] : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            if ((uint32_t)u < cnt) {
+                const uint32_t i = hi - 1 - u, w = __ldg(v1 + i);
+                run = fadd4(run, v[u]);
+                C[(size_t)i * Lq + g] = make_uint4(fmul(w, run.x), fmul(w, run.y), fmul(w, run.z), fmul(w, run.w));
+            }
+        }
+        hi -= cnt;
+    }
+}
+
+// out[b][j] = addend[b][j] + sum_{c<r} C[pi1^-1(r j + c)][b] for kGatherJ
+// outputs and the CTA's lanes, transposed through shared memory so that out
+// rows are written 128 bytes at a time.  addend may be null or alias out.
+__global__ void __launch_bounds__(kLaneCta) k_lane_gather(const uint4 *__restrict__ C,
+                                                         const uint32_t *__restrict__ pi1inv,
+                                                         uint32_t r, uint32_t n, uint32_t L,
+                                                         const uint32_t *addend, uint32_t *out) {
+    __shared__ uint32_t tile[kGatherJ][4 * kLaneQuadsMax + 1];
+    const uint32_t cols = lane_cols(L), subs = kLaneCta / cols, Lq = lane_pad(L) / 4;
+    const uint32_t tid = threadIdx.x, gl = tid % cols, sub = tid / cols;
+    const uint32_t g = blockIdx.y * cols + gl;
+    const uint32_t j0 = blockIdx.x * kGatherJ;
+    // thread (sub, quad) takes outputs jj = sub, sub + subs, ... two at a time
+    for (uint32_t jj0 = sub; jj0 < (uint32_t)kGatherJ; jj0 += 2 * subs) {
+        uint4 v[2][8];
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+            const uint32_t jj = jj0 + q * subs, j = j0 + jj;
+            const bool ok = jj < (uint32_t)kGatherJ && j < n && g < Lq;
+#pragma unroll
+            for (int c = 0; c < 8; ++c)
+                v[q][c] = ok && (uint32_t)c < r ? C[(size_t)__ldg(pi1inv + (size_t)j * r + c) * Lq + g]
+                                              : make_uint4(0u, 0u, 0u, 0u);
+        }
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+            const uint32_t jj = jj0 + q * subs, j = j0 + jj;
+            if (jj >= (uint32_t)kGatherJ) continue;
+            uint4 acc = make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+            for (int c = 0; c < 8; ++c) acc = fadd4(acc, v[q][c]);
+            if (r > 8 && j < n && g < Lq)
+                for (uint32_t c = 8; c < r; ++c)
+                    acc = fadd4(acc, C[(size_t)__ldg(pi1inv + (size_t)j * r + c) * Lq + g]);
+            tile[jj][4 * gl] = acc.x;
+            tile[jj][4 * gl + 1] = acc.y;
+            tile[jj][4 * gl + 2] = acc.z;
+            tile[jj][4 * gl + 3] = acc.w;
+        }
+    }
+    __syncthreads();
+    // consecutive threads write consecutive outputs of one vector's row
+    for (uint32_t idx = tid; idx < 4 * cols * (uint32_t)kGatherJ; idx += kLaneCta) {
+        const uint32_t bb = idx / kGatherJ, jj = idx % kGatherJ;
+        const uint32_t vb = blockIdx.y * 4 * cols + bb, j = j0 + jj;
+        if (vb < L && j < n) {
+            const size_t o = (size_t)vb * n + j;
+            out[o] = addend ? fadd(addend[o], tile[jj][bb]) : tile[jj][bb];
+        }
+    }
+}
+
 }  // namespace
 
 // Bitmap of N bits plus 512 keystream words; covers N up to 8 * PVMVMD_MAX_K.
@@ -911,6 +1207,44 @@ cudaError_t launch_syndrome_fused(const pvmvmd_key &key, uint32_t tag, uint64_t 
         if (e != cudaSuccess) return e;
     }
     return cudaSuccess;
+}
+
+size_t lane_aux_words(uint32_t N, uint32_t L) {
+    return 2 * (size_t)((N + kLaneTile - 1) / kLaneTile) * lane_pad(L);
+}
+
+cudaError_t launch_lane_syndrome(const pvmvmd_key &key, uint32_t tag, uint64_t idx0, uint32_t N,
+                                 uint32_t t, uint32_t L, const uint32_t *pi2, const uint32_t *v2m,
+                                 const uint32_t *v1, const uint32_t *pi1inv, uint32_t n, uint32_t r,
+                                 uint32_t *sparse_out, uint32_t *S, uint32_t *C, uint32_t *aux,
+                                 const uint32_t *addend, uint32_t *out, cudaStream_t s) {
+    if (L == 0) return cudaSuccess;
+    const size_t smem = ((size_t)(N + 31) / 32 + 1024 + 2 * (size_t)t) * sizeof(uint32_t);
+    if (smem > kSampleMaxSmem) return cudaErrorInvalidValue;
+    static const cudaError_t a1 = cudaFuncSetAttribute(
+        k_lane_sample, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSampleMaxSmem);
+    if (a1 != cudaSuccess) return a1;
+    if ((reinterpret_cast<uintptr_t>(C) | reinterpret_cast<uintptr_t>(aux)) & 15u)
+        return cudaErrorInvalidValue;
+    const uint32_t Lp = lane_pad(L), cols = lane_cols(L), per_cta = kLaneCta / cols;
+    const unsigned gy = (Lp / 4 + cols - 1) / cols;
+    const uint32_t ntiles = (N + kLaneTile - 1) / kLaneTile;
+    const uint32_t nspans = (N + kExpandSpan - 1) / kExpandSpan;
+    if (gy > 65535u || L > 0x7fffffffu) return cudaErrorInvalidValue;
+    uint32_t *agg = aux, *carry = aux + (size_t)ntiles * Lp;
+    uint4 *C4 = reinterpret_cast<uint4 *>(C);
+    k_lane_sample<<<L, 128, smem, s>>>(key, tag, idx0, N, t, sparse_out, S);
+    k_lane_expand<<<dim3((nspans + per_cta - 1) / per_cta, gy), kLaneCta, 0, s>>>(sparse_out, S, t, N, L,
+                                                                                 pi2, v2m, C4);
+    k_lane_tile_sum<<<dim3((ntiles + per_cta - 1) / per_cta, gy), kLaneCta, 0, s>>>(
+        C4, N, L, reinterpret_cast<uint4 *>(agg));
+    k_lane_carry<<<(Lp / 4 + 7) / 8, 8 * kCarryChunks, 0, s>>>(reinterpret_cast<const uint4 *>(agg), ntiles,
+                                                             Lp / 4, reinterpret_cast<uint4 *>(carry));
+    k_lane_scan<<<dim3((ntiles + per_cta - 1) / per_cta, gy), kLaneCta, 0, s>>>(
+        C4, N, L, reinterpret_cast<const uint4 *>(carry), v1);
+    k_lane_gather<<<dim3((n + kGatherJ - 1) / kGatherJ, gy), kLaneCta, 0, s>>>(C4, pi1inv, r, n, L,
+                                                                              addend, out);
+    return cudaGetLastError();
 }
 
 }  // namespace pv

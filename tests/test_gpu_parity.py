@@ -128,6 +128,37 @@ def test_encode_chunking_matches(pv, wl):
     assert np.array_equal(pv.as_u32(xc), pv.as_u32(xa))
 
 
+def test_lane_encode_ragged_groups_and_chunks(pv, wl):
+    """Batches large enough for the lane-parallel encode, on a code too long for
+    one CTA (K = 6000, N_x = 48000): 300 vectors in chunks of 270 (two lane
+    groups of 256 and 14 lanes, then a 30-lane chunk) and a ragged 33-vector
+    batch; every x_hat and mask equals the oracle, and the chunked and
+    unchunked contexts agree."""
+    W = wl.weights_uniform(40, 6000, 21)
+    x = wl.int8_vectors(300, 6000, 22)
+    X = field(x)
+    Wd, Xd = to_dev(W), to_dev(X)
+    pp = oracle.PublicParams(W, oracle.key_from_seed(23), with_tables=False)
+    a = pv.pvmvmd_preprocess(Wd, key=23, params=_params(pv, scratch_batch=270))
+    b = pv.pvmvmd_preprocess(Wd, key=23, params=_params(pv, scratch_batch=300))
+    xa, sa = pv.pvmvmd_encode(a, Xd, key=24)
+    xb, sb = pv.pvmvmd_encode(b, Xd, key=24)
+    xa_h, sa_h = pv.as_u32(xa), pv.as_u32(sa)
+    for i in range(300):
+        xh_o, s_o, v_o = pp.encrypt(X[i], oracle.key_from_seed(24), i)
+        assert np.array_equal(xa_h[i], xh_o), i
+        assert np.array_equal(sa_h[i], np.concatenate([s_o, v_o])), i
+    assert np.array_equal(pv.as_u32(xb), xa_h)
+    assert np.array_equal(pv.as_u32(sb), sa_h)
+    # 33 vectors (one lane group, a ragged warp), in place
+    xc = Xd[:33].clone()
+    pv.pvmvmd_encode(a, xc, key=24, Xhat=xc)
+    assert np.array_equal(pv.as_u32(xc), xa_h[:33])
+    assert pv.pvmvmd_device_status() == 0
+    a.destroy()
+    b.destroy()
+
+
 def test_server_mvm_extremes(pv):
     """Extreme weights and field values: -128, 127, x = 0, 1, (q-1)/2, (q+1)/2, q-1."""
     rng = np.random.default_rng(1)
