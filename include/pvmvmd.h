@@ -187,6 +187,31 @@ int pvmvmd_decode_verify(pvmvmd_ctx *ctx, const void *st_dev, const uint32_t *Xh
                          const uint32_t *Yhat_dev, int B, const pvmvmd_key *challenge_key,
                          uint32_t *Y_dev, int32_t *accept_dev, void *stream);
 
+/* Boost mode (Sec. 7.2): the masks of a batch prepared ahead of the online
+ * phase, while the client is idle, like preprocessed triples in MPC.
+ *
+ * pvmvmd_boost_prepare (offline) draws e_x for vectors numbered 0 .. B-1
+ * under `key`, exactly as pvmvmd_encode would for the same key, and writes
+ * the input masks Mask_in_b = G_x e_x,b (B x K), the output masks
+ * Mask_out_b = P e_x,b (B x m) and st_b = e_x,b (pvmvmd_state_size bytes;
+ * not needed online).  The online calls then cost one pass over the
+ * vectors each:
+ *   pvmvmd_boost_encode:  Xhat = X + Mask_in (B x K; Xhat may alias X or
+ *                         Mask_in), the same Xhat pvmvmd_encode gives;
+ *   pvmvmd_boost_decode_verify: as pvmvmd_decode_verify (fresh shared
+ *                         challenges, same accept rule), with
+ *                         Y = Yhat - Mask_out instead of the t_x rows of P.
+ * A mask pair must be used for one vector only (Sec. 4.2 multi-query
+ * privacy needs fresh masks per query). */
+int pvmvmd_boost_prepare(pvmvmd_ctx *ctx, int B, const pvmvmd_key *key, uint32_t *mask_in_dev,
+                         uint32_t *mask_out_dev, void *st_dev, void *stream);
+int pvmvmd_boost_encode(const uint32_t *X_dev, const uint32_t *mask_in_dev, int B, int K,
+                        uint32_t *Xhat_dev, void *stream);
+int pvmvmd_boost_decode_verify(pvmvmd_ctx *ctx, const uint32_t *mask_out_dev,
+                               const uint32_t *Xhat_dev, const uint32_t *Yhat_dev, int B,
+                               const pvmvmd_key *challenge_key, uint32_t *Y_dev,
+                               int32_t *accept_dev, void *stream);
+
 /* Synchronise `stream`, then read and clear the library's device error word:
  * PVMVMD_E_DEVICE_TIMEOUT if any kernel gave up a bounded wait since the last
  * call, else PVMVMD_OK (or PVMVMD_E_CUDA if synchronisation failed). */

@@ -78,6 +78,10 @@ SIGNATURES = {
     "pvmvmd_server_mvm_multi": (_i, [ctypes.POINTER(pvmvmd_mvm_job), _i, _vp]),
     "pvmvmd_server_mvm_noalloc": (_i, [_vp, _i, _i, _vp, _i, _vp, _vp]),
     "pvmvmd_decode_verify": (_i, [_vp, _vp, _vp, _vp, _i, ctypes.POINTER(pvmvmd_key), _vp, _vp, _vp]),
+    "pvmvmd_boost_prepare": (_i, [_vp, _i, ctypes.POINTER(pvmvmd_key), _vp, _vp, _vp, _vp]),
+    "pvmvmd_boost_encode": (_i, [_vp, _vp, _i, _i, _vp, _vp]),
+    "pvmvmd_boost_decode_verify": (_i, [_vp, _vp, _vp, _vp, _i, ctypes.POINTER(pvmvmd_key), _vp, _vp,
+                                        _vp]),
     "pvmvmd_device_status": (_i, [_vp]),
     "pvmvmd_ctx_info": (_i, [_vp, ctypes.POINTER(pvmvmd_ctx_view)]),
     "pvmvmd_destroy": (None, [_vp]),
@@ -320,6 +324,64 @@ def pvmvmd_decode_verify(ctx: Ctx, st, Xhat, Yhat, challenge_key, Y=None, accept
                                      _dev_ptr(Y, "Y", _u32_types(), B * ctx.m),
                                      _dev_ptr(accept, "accept", (torch.int32,), B), _stream_ptr(stream)),
            "pvmvmd_decode_verify")
+    return Y, accept
+
+
+def pvmvmd_boost_prepare(ctx: Ctx, B: int, key, mask_in=None, mask_out=None, st=None, device=None,
+                         stream=None):
+    """Boost mode, offline: the masks of vectors 0 .. B-1 under `key`.
+    Returns (mask_in [B x K] = G_x e_x, mask_out [B x m] = P e_x, st)."""
+    like = None
+    for t in (mask_in, mask_out, st):
+        if t is not None:
+            like = t
+            break
+    dev = like.device if like is not None else (device or "cuda")
+    import torch
+    if mask_in is None:
+        mask_in = torch.empty((B, ctx.K), dtype=torch.int32, device=dev)
+    if mask_out is None:
+        mask_out = torch.empty((B, ctx.m), dtype=torch.int32, device=dev)
+    if st is None:
+        st = torch.empty((B, 2 * ctx.t_x), dtype=torch.int32, device=dev)
+    _check(_lib.pvmvmd_boost_prepare(ctx.handle, B, ctypes.byref(make_key(key)),
+                                     _dev_ptr(mask_in, "mask_in", _u32_types(), B * ctx.K),
+                                     _dev_ptr(mask_out, "mask_out", _u32_types(), B * ctx.m),
+                                     _dev_ptr(st, "st", _u32_types(), B * 2 * ctx.t_x), _stream_ptr(stream)),
+           "pvmvmd_boost_prepare")
+    return mask_in, mask_out, st
+
+
+def pvmvmd_boost_encode(X, mask_in, Xhat=None, stream=None):
+    """Boost mode, online: Xhat = X + mask_in over F_q (X and mask_in B x K)."""
+    if X.shape != mask_in.shape:
+        raise ValueError("X and mask_in must have the same shape")
+    K = X.shape[-1]
+    B = X.numel() // K
+    if Xhat is None:
+        Xhat = _new_u32(X.shape, X)
+    _check(_lib.pvmvmd_boost_encode(_dev_ptr(X, "X", _u32_types()), _dev_ptr(mask_in, "mask_in", _u32_types()),
+                                    B, K, _dev_ptr(Xhat, "Xhat", _u32_types(), X.numel()), _stream_ptr(stream)),
+           "pvmvmd_boost_encode")
+    return Xhat
+
+
+def pvmvmd_boost_decode_verify(ctx: Ctx, mask_out, Xhat, Yhat, challenge_key, Y=None, accept=None,
+                               stream=None):
+    """Boost mode, online: verify and Y = Yhat - mask_out; returns (Y, accept)."""
+    import torch
+    B = _batch(Xhat, ctx.K, "Xhat")
+    if Y is None:
+        Y = _new_u32(Yhat.shape, Yhat)
+    if accept is None:
+        accept = torch.empty(B, dtype=torch.int32, device=Yhat.device)
+    _check(_lib.pvmvmd_boost_decode_verify(ctx.handle, _dev_ptr(mask_out, "mask_out", _u32_types(), B * ctx.m),
+                                           _dev_ptr(Xhat, "Xhat", _u32_types()),
+                                           _dev_ptr(Yhat, "Yhat", _u32_types(), B * ctx.m), B,
+                                           ctypes.byref(make_key(challenge_key)),
+                                           _dev_ptr(Y, "Y", _u32_types(), B * ctx.m),
+                                           _dev_ptr(accept, "accept", (torch.int32,), B), _stream_ptr(stream)),
+           "pvmvmd_boost_decode_verify")
     return Y, accept
 
 

@@ -414,11 +414,48 @@ int pvmvmd_state_size(const pvmvmd_ctx *ctx, int B, size_t *bytes) {
     return PVMVMD_OK;
 }
 
+namespace pv {
+namespace {
+// Xhat = X + G_x e_x for the B vectors (X null: Xhat = G_x e_x alone).
+int encode_batch(pvmvmd_ctx *ctx, const uint32_t *X_dev, int B, const pvmvmd_key *key,
+                 uint32_t *Xhat_dev, void *st_dev, cudaStream_t s);
+}  // namespace
+}  // namespace pv
+
 int pvmvmd_encode(pvmvmd_ctx *ctx, const uint32_t *X_dev, int B, const pvmvmd_key *key,
                   uint32_t *Xhat_dev, void *st_dev, void *stream) {
     if (!ctx || !X_dev || !key || !Xhat_dev || !st_dev) return PVMVMD_E_ARG;
     if (B < 1) return PVMVMD_E_SHAPE;
+    return pv::encode_batch(ctx, X_dev, B, key, Xhat_dev, st_dev, static_cast<cudaStream_t>(stream));
+}
+
+int pvmvmd_boost_prepare(pvmvmd_ctx *ctx, int B, const pvmvmd_key *key, uint32_t *mask_in_dev,
+                         uint32_t *mask_out_dev, void *st_dev, void *stream) {
+    using namespace pv;
+    if (!ctx || !key || !mask_in_dev || !mask_out_dev || !st_dev) return PVMVMD_E_ARG;
+    if (B < 1) return PVMVMD_E_SHAPE;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const int st = encode_batch(ctx, nullptr, B, key, mask_in_dev, st_dev, s);
+    if (st != PVMVMD_OK) return st;
+    PV_CUDA(launch_output_mask(ctx->PT, ctx->m, static_cast<const uint32_t *>(st_dev), ctx->t_x, B,
+                               mask_out_dev, s));
+    return PVMVMD_OK;
+}
+
+int pvmvmd_boost_encode(const uint32_t *X_dev, const uint32_t *mask_in_dev, int B, int K,
+                        uint32_t *Xhat_dev, void *stream) {
+    using namespace pv;
+    if (!X_dev || !mask_in_dev || !Xhat_dev) return PVMVMD_E_ARG;
+    if (B < 1 || K < 1) return PVMVMD_E_SHAPE;
+    PV_CUDA(launch_field_add(X_dev, mask_in_dev, (size_t)B * K, Xhat_dev,
+                             static_cast<cudaStream_t>(stream)));
+    return PVMVMD_OK;
+}
+
+namespace pv {
+namespace {
+int encode_batch(pvmvmd_ctx *ctx, const uint32_t *X_dev, int B, const pvmvmd_key *key,
+                 uint32_t *Xhat_dev, void *st_dev, cudaStream_t s) {
     uint32_t *err = error_word();
     if (!err) return PVMVMD_E_CUDA;
     uint32_t *stp = static_cast<uint32_t *>(st_dev);
@@ -435,8 +472,8 @@ int pvmvmd_encode(pvmvmd_ctx *ctx, const uint32_t *X_dev, int B, const pvmvmd_ke
             PV_CUDA(launch_lane_syndrome(*key, kTagMask, (uint64_t)b0, ctx->Nx, ctx->t_x, L, d.pi2,
                                          d.v2m, d.v1, d.pi1inv, ctx->K, ctx->rate,
                                          stp + (size_t)b0 * 2 * ctx->t_x, ctx->S, ctx->F, ctx->laux,
-                                         X_dev + (size_t)b0 * ctx->K, Xhat_dev + (size_t)b0 * ctx->K,
-                                         s));
+                                         X_dev ? X_dev + (size_t)b0 * ctx->K : nullptr,
+                                         Xhat_dev + (size_t)b0 * ctx->K, s));
         }
         return PVMVMD_OK;
     }
@@ -455,11 +492,13 @@ int pvmvmd_encode(pvmvmd_ctx *ctx, const uint32_t *X_dev, int B, const pvmvmd_ke
         PV_CUDA(launch_syndrome_scan(d.pi2inv, d.v2p, d.v1, ctx->Nx, e, ctx->t_x, nb, ctx->F,
                                      ctx->status, err, s));
         PV_CUDA(launch_syndrome_gather(d.pi1inv, ctx->K, ctx->rate, ctx->F, ctx->Nx,
-                                       X_dev + (size_t)b0 * ctx->K, Xhat_dev + (size_t)b0 * ctx->K,
-                                       nb, s));
+                                       X_dev ? X_dev + (size_t)b0 * ctx->K : nullptr,
+                                       Xhat_dev + (size_t)b0 * ctx->K, nb, s));
     }
     return PVMVMD_OK;
 }
+}  // namespace
+}  // namespace pv
 
 int pvmvmd_server_mvm(const int8_t *W_dev, int m, int K, const uint32_t *Xhat_dev, int B,
                       uint32_t *Yhat_dev, void *stream) {
@@ -500,13 +539,14 @@ int pvmvmd_server_mvm_multi(const pvmvmd_mvm_job *jobs, int count, void *stream)
     return PVMVMD_OK;
 }
 
-int pvmvmd_decode_verify(pvmvmd_ctx *ctx, const void *st_dev, const uint32_t *Xhat_dev,
-                         const uint32_t *Yhat_dev, int B, const pvmvmd_key *challenge_key,
-                         uint32_t *Y_dev, int32_t *accept_dev, void *stream) {
-    if (!ctx || !st_dev || !Xhat_dev || !Yhat_dev || !challenge_key || !Y_dev || !accept_dev)
-        return PVMVMD_E_ARG;
-    if (B < 1) return PVMVMD_E_SHAPE;
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
+namespace pv {
+namespace {
+// Challenges, u and g, then decrypt + verify: Y = Yhat - P e_x from st, or
+// Y = Yhat - mask_out when mask_out is given (boost mode).
+int decode_verify_batch(pvmvmd_ctx *ctx, const void *st_dev, const uint32_t *mask_out_dev,
+                        const uint32_t *Xhat_dev, const uint32_t *Yhat_dev, int B,
+                        const pvmvmd_key *challenge_key, uint32_t *Y_dev, int32_t *accept_dev,
+                        cudaStream_t s) {
     uint32_t *err = error_word();
     if (!err) return PVMVMD_E_CUDA;
     const CodeDev &d = ctx->gy;
@@ -530,8 +570,31 @@ int pvmvmd_decode_verify(pvmvmd_ctx *ctx, const void *st_dev, const uint32_t *Xh
     PV_CUDA(launch_verify_u(ctx->Q, ctx->K, ctx->chal, ctx->t_y, ctx->ell, ctx->u, s));
     PV_CUDA(launch_decode_verify(ctx->PT, ctx->m, ctx->K, static_cast<const uint32_t *>(st_dev),
                                  ctx->t_x, Xhat_dev, Yhat_dev, ctx->g, ctx->u, ctx->ell, B, Y_dev,
-                                 accept_dev, s));
+                                 accept_dev, s, mask_out_dev));
     return PVMVMD_OK;
+}
+}  // namespace
+}  // namespace pv
+
+int pvmvmd_decode_verify(pvmvmd_ctx *ctx, const void *st_dev, const uint32_t *Xhat_dev,
+                         const uint32_t *Yhat_dev, int B, const pvmvmd_key *challenge_key,
+                         uint32_t *Y_dev, int32_t *accept_dev, void *stream) {
+    if (!ctx || !st_dev || !Xhat_dev || !Yhat_dev || !challenge_key || !Y_dev || !accept_dev)
+        return PVMVMD_E_ARG;
+    if (B < 1) return PVMVMD_E_SHAPE;
+    return pv::decode_verify_batch(ctx, st_dev, nullptr, Xhat_dev, Yhat_dev, B, challenge_key, Y_dev,
+                                   accept_dev, static_cast<cudaStream_t>(stream));
+}
+
+int pvmvmd_boost_decode_verify(pvmvmd_ctx *ctx, const uint32_t *mask_out_dev,
+                               const uint32_t *Xhat_dev, const uint32_t *Yhat_dev, int B,
+                               const pvmvmd_key *challenge_key, uint32_t *Y_dev,
+                               int32_t *accept_dev, void *stream) {
+    if (!ctx || !mask_out_dev || !Xhat_dev || !Yhat_dev || !challenge_key || !Y_dev || !accept_dev)
+        return PVMVMD_E_ARG;
+    if (B < 1) return PVMVMD_E_SHAPE;
+    return pv::decode_verify_batch(ctx, nullptr, mask_out_dev, Xhat_dev, Yhat_dev, B, challenge_key,
+                                   Y_dev, accept_dev, static_cast<cudaStream_t>(stream));
 }
 
 int pvmvmd_device_status(void *stream) {

@@ -11,6 +11,10 @@
 //                       the CTAs of the cluster reduce their partial dot
 //                       products through distributed shared memory and
 //                       rank 0 writes accept_b = AND_q (L_q == R_q).
+//                       In boost mode (Sec. 7.2) P e_x,b was prepared ahead
+//                       and is read instead of the t_x rows of P^T.
+//  * k_output_mask      the output masks P e_x,b alone (boost mode's
+//                       offline step).
 #include <cooperative_groups.h>
 
 #include "common.cuh"
@@ -63,11 +67,78 @@ __device__ __forceinline__ uint32_t warp_fsum(uint32_t v) {
     return v;
 }
 
+// pe[s] = sum_j vals[j] P^T[supp[j]][i + s] mod q for the four columns
+// i .. i+3 (columns at or past c1 read as 0); 16-byte loads when vec.
+__device__ __forceinline__ void pe_cols(const uint32_t *__restrict__ PT, int m, const uint32_t *supp,
+                                    const uint32_t *vals, uint32_t t_x, int i, int c1, bool vec,
+                                    uint32_t pe[4]) {
+    uint64_t a0 = 0, a1 = 0, a2 = 0, a3 = 0;
+    uint32_t j = 0;
+    for (; j + 8 <= t_x; j += 8) {
+        uint4 v[8];
+#pragma unroll
+        for (int s = 0; s < 8; ++s) {
+            const uint32_t *row = PT + (size_t)supp[j + s] * m + i;
+            if (vec) {
+                v[s] = ldg4(row);
+            } else {
+                v[s].x = row[0];
+                v[s].y = i + 1 < c1 ? row[1] : 0u;
+                v[s].z = i + 2 < c1 ? row[2] : 0u;
+                v[s].w = i + 3 < c1 ? row[3] : 0u;
+            }
+        }
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+#pragma unroll
+            for (int s = 4 * h; s < 4 * h + 4; ++s) {
+                const uint64_t e = vals[j + s];
+                a0 += e * v[s].x; a1 += e * v[s].y; a2 += e * v[s].z; a3 += e * v[s].w;
+            }
+            a0 = fred(a0); a1 = fred(a1); a2 = fred(a2); a3 = fred(a3);
+        }
+    }
+    for (; j + 4 <= t_x; j += 4) {
+        uint4 v[4];
+#pragma unroll
+        for (int s = 0; s < 4; ++s) {
+            const uint32_t *row = PT + (size_t)supp[j + s] * m + i;
+            if (vec) {
+                v[s] = ldg4(row);
+            } else {
+                v[s].x = row[0];
+                v[s].y = i + 1 < c1 ? row[1] : 0u;
+                v[s].z = i + 2 < c1 ? row[2] : 0u;
+                v[s].w = i + 3 < c1 ? row[3] : 0u;
+            }
+        }
+#pragma unroll
+        for (int s = 0; s < 4; ++s) {
+            const uint64_t e = vals[j + s];
+            a0 += e * v[s].x; a1 += e * v[s].y; a2 += e * v[s].z; a3 += e * v[s].w;
+        }
+        a0 = fred(a0); a1 = fred(a1); a2 = fred(a2); a3 = fred(a3);
+    }
+    for (; j < t_x; ++j) {
+        const uint32_t *row = PT + (size_t)supp[j] * m + i;
+        const uint64_t e = vals[j];
+        a0 += e * row[0];
+        if (i + 1 < c1) a1 += e * row[1];
+        if (i + 2 < c1) a2 += e * row[2];
+        if (i + 3 < c1) a3 += e * row[3];
+    }
+    pe[0] = fred(a0);
+    pe[1] = fred(a1);
+    pe[2] = fred(a2);
+    pe[3] = fred(a3);
+}
+
+template <bool kBoost>
 __global__ void __launch_bounds__(kDecThreads) k_decode_verify(
     const uint32_t *__restrict__ PT, int m, int K, const uint32_t *__restrict__ st, uint32_t t_x,
     const uint32_t *__restrict__ Xhat, const uint32_t *Yhat, const uint32_t *__restrict__ g,
     const uint32_t *__restrict__ u, uint32_t ell, uint32_t *Y, int32_t *__restrict__ accept,
-    bool vec) {
+    bool vec, const uint32_t *__restrict__ mask) {
     cg::cluster_group cluster = cg::this_cluster();
     extern __shared__ uint32_t sm[];  // support[t_x], values[t_x]
     __shared__ uint32_t s_part[2 * kMaxEll];
@@ -81,8 +152,10 @@ __global__ void __launch_bounds__(kDecThreads) k_decode_verify(
     // challenge kernels that precede it in the stream; g and u come from
     // those kernels, so they are read only after griddepcontrol.wait.
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-    const uint32_t *stb = st + b * 2 * t_x;
-    for (uint32_t j = tid; j < 2 * t_x; j += kDecThreads) sm[j] = stb[j];
+    if (!kBoost) {
+        const uint32_t *stb = st + b * 2 * t_x;
+        for (uint32_t j = tid; j < 2 * t_x; j += kDecThreads) sm[j] = stb[j];
+    }
     uint32_t *ystage = sm + 2 * t_x;  // this CTA's y_hat columns (y may alias y_hat)
     __syncthreads();
     const uint32_t *supp = sm, *vals = sm + t_x;
@@ -98,62 +171,14 @@ __global__ void __launch_bounds__(kDecThreads) k_decode_verify(
     const uint32_t *yh = Yhat + b * m;
     uint32_t *yo = Y + b * m;
     for (int i = c0 + tid * 4; i < c1; i += kDecThreads * 4) {
-        uint64_t a0 = 0, a1 = 0, a2 = 0, a3 = 0;
-        uint32_t j = 0;
-        for (; j + 8 <= t_x; j += 8) {
-            uint4 v[8];
+        uint32_t pe[4];
+        if (kBoost) {
 #pragma unroll
-            for (int s = 0; s < 8; ++s) {
-                const uint32_t *row = PT + (size_t)supp[j + s] * m + i;
-                if (vec) {
-                    v[s] = ldg4(row);
-                } else {
-                    v[s].x = row[0];
-                    v[s].y = i + 1 < c1 ? row[1] : 0u;
-                    v[s].z = i + 2 < c1 ? row[2] : 0u;
-                    v[s].w = i + 3 < c1 ? row[3] : 0u;
-                }
-            }
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-#pragma unroll
-                for (int s = 4 * h; s < 4 * h + 4; ++s) {
-                    const uint64_t e = vals[j + s];
-                    a0 += e * v[s].x; a1 += e * v[s].y; a2 += e * v[s].z; a3 += e * v[s].w;
-                }
-                a0 = fred(a0); a1 = fred(a1); a2 = fred(a2); a3 = fred(a3);
-            }
+            for (int q2 = 0; q2 < 4; ++q2) pe[q2] = i + q2 < c1 ? mask[b * m + i + q2] : 0u;
+        } else {
+            pe_cols(PT, m, supp, vals, t_x, i, c1, vec, pe);
         }
-        for (; j + 4 <= t_x; j += 4) {
-            uint4 v[4];
-#pragma unroll
-            for (int s = 0; s < 4; ++s) {
-                const uint32_t *row = PT + (size_t)supp[j + s] * m + i;
-                if (vec) {
-                    v[s] = ldg4(row);
-                } else {
-                    v[s].x = row[0];
-                    v[s].y = i + 1 < c1 ? row[1] : 0u;
-                    v[s].z = i + 2 < c1 ? row[2] : 0u;
-                    v[s].w = i + 3 < c1 ? row[3] : 0u;
-                }
-            }
-#pragma unroll
-            for (int s = 0; s < 4; ++s) {
-                const uint64_t e = vals[j + s];
-                a0 += e * v[s].x; a1 += e * v[s].y; a2 += e * v[s].z; a3 += e * v[s].w;
-            }
-            a0 = fred(a0); a1 = fred(a1); a2 = fred(a2); a3 = fred(a3);
-        }
-        for (; j < t_x; ++j) {
-            const uint32_t *row = PT + (size_t)supp[j] * m + i;
-            const uint64_t e = vals[j];
-            a0 += e * row[0];
-            if (i + 1 < c1) a1 += e * row[1];
-            if (i + 2 < c1) a2 += e * row[2];
-            if (i + 3 < c1) a3 += e * row[3];
-        }
-        const uint32_t pe[4] = {fred(a0), fred(a1), fred(a2), fred(a3)};
+
 #pragma unroll
         for (int s = 0; s < 4; ++s) {
             const int col = i + s;
@@ -221,7 +246,63 @@ __global__ void __launch_bounds__(kDecThreads) k_decode_verify(
     cluster.sync();
 }
 
+// out[b][col] = (P e_x,b)_col for the columns of this CTA (1024 per CTA).
+__global__ void __launch_bounds__(kDecThreads) k_output_mask(const uint32_t *__restrict__ PT, int m,
+                                                            const uint32_t *__restrict__ st, uint32_t t_x,
+                                                            uint32_t *__restrict__ out, bool vec) {
+    extern __shared__ uint32_t sm[];  // support[t_x], values[t_x]
+    const size_t b = blockIdx.y;
+    const uint32_t *stb = st + b * 2 * t_x;
+    for (uint32_t j = threadIdx.x; j < 2 * t_x; j += kDecThreads) sm[j] = stb[j];
+    __syncthreads();
+    const int i = (int)blockIdx.x * kDecThreads * 4 + (int)threadIdx.x * 4;
+    if (i >= m) return;
+    uint32_t pe[4];
+    pe_cols(PT, m, sm, sm + t_x, t_x, i, m, vec, pe);
+#pragma unroll
+    for (int s = 0; s < 4; ++s)
+        if (i + s < m) out[b * m + i + s] = pe[s];
+}
+
+// out = a + b over F_q, n elements, 16 bytes per thread where aligned.
+__global__ void __launch_bounds__(256) k_field_add(const uint32_t *a, const uint32_t *b, size_t n,
+                                                  uint32_t *out, bool vec) {
+    const size_t i = ((size_t)blockIdx.x * 256 + threadIdx.x) * 4;
+    if (i >= n) return;
+    if (vec && i + 4 <= n) {
+        const uint4 x = *reinterpret_cast<const uint4 *>(a + i);
+        const uint4 y = *reinterpret_cast<const uint4 *>(b + i);
+        *reinterpret_cast<uint4 *>(out + i) = make_uint4(fadd(x.x, y.x), fadd(x.y, y.y), fadd(x.z, y.z), fadd(x.w, y.w));
+    } else {
+        for (size_t k = i; k < n && k < i + 4; ++k) out[k] = fadd(a[k], b[k]);
+    }
+}
+
 }  // namespace
+
+cudaError_t launch_field_add(const uint32_t *a, const uint32_t *b, size_t n, uint32_t *out,
+                             cudaStream_t s) {
+    if (n == 0) return cudaSuccess;
+    const bool vec = ((reinterpret_cast<uintptr_t>(a) | reinterpret_cast<uintptr_t>(b) |
+                       reinterpret_cast<uintptr_t>(out)) & 15u) == 0;
+    const size_t blocks = (n + 1023) / 1024;
+    if (blocks > 0x7fffffffu) return cudaErrorInvalidValue;
+    k_field_add<<<(unsigned)blocks, 256, 0, s>>>(a, b, n, out, vec);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_output_mask(const uint32_t *PT, int m, const uint32_t *st, uint32_t t_x, int B,
+                               uint32_t *out, cudaStream_t s) {
+    if (B <= 0 || m <= 0) return cudaSuccess;
+    const bool vec = (m % 4 == 0) && ((reinterpret_cast<uintptr_t>(PT) & 15u) == 0);
+    for (int b0 = 0; b0 < B; b0 += 65535) {
+        const int nb = B - b0 < 65535 ? B - b0 : 65535;
+        dim3 grid((m + kDecThreads * 4 - 1) / (kDecThreads * 4), nb);
+        k_output_mask<<<grid, kDecThreads, 2 * (size_t)t_x * sizeof(uint32_t), s>>>(
+            PT, m, st + (size_t)b0 * 2 * t_x, t_x, out + (size_t)b0 * m, vec);
+    }
+    return cudaGetLastError();
+}
 
 cudaError_t launch_verify_u(const uint32_t *Qm, int K, const uint32_t *chal, uint32_t t_y,
                             uint32_t ell, uint32_t *u, cudaStream_t s) {
@@ -242,7 +323,7 @@ cudaError_t launch_verify_u(const uint32_t *Qm, int K, const uint32_t *chal, uin
 cudaError_t launch_decode_verify(const uint32_t *PT, int m, int K, const uint32_t *st, uint32_t t_x,
                                  const uint32_t *Xhat, const uint32_t *Yhat, const uint32_t *g,
                                  const uint32_t *u, uint32_t ell, int B, uint32_t *Y,
-                                 int32_t *accept, cudaStream_t s) {
+                                 int32_t *accept, cudaStream_t s, const uint32_t *mask) {
     if (B <= 0) return cudaSuccess;
     if (ell > (uint32_t)kMaxEll) return cudaErrorInvalidValue;
     const bool vec = (m % 4 == 0) && ((reinterpret_cast<uintptr_t>(PT) & 15u) == 0);
@@ -251,8 +332,11 @@ cudaError_t launch_decode_verify(const uint32_t *PT, int m, int K, const uint32_
     const int chunk = (((m + C - 1) / C) + 3) & ~3;  // y_hat columns per CTA (staged in smem)
     if ((2 * (size_t)t_x + (size_t)chunk) * sizeof(uint32_t) > 200 * 1024) return cudaErrorInvalidValue;
     static const cudaError_t smem_attr = cudaFuncSetAttribute(
-        k_decode_verify, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+        k_decode_verify<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+    static const cudaError_t smem_attr2 = cudaFuncSetAttribute(
+        k_decode_verify<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
     if (smem_attr != cudaSuccess) return smem_attr;
+    if (smem_attr2 != cudaSuccess) return smem_attr2;
     for (int b0 = 0; b0 < B; b0 += 65535) {
         const int nb = B - b0 < 65535 ? B - b0 : 65535;
         cudaLaunchConfig_t cfg = {};
@@ -269,9 +353,14 @@ cudaError_t launch_decode_verify(const uint32_t *PT, int m, int K, const uint32_
         attr[1].val.programmaticStreamSerializationAllowed = 1;
         cfg.attrs = attr;
         cfg.numAttrs = 2;
-        cudaError_t e = cudaLaunchKernelEx(&cfg, k_decode_verify, PT, m, K, st + (size_t)b0 * 2 * t_x,
-                                           t_x, Xhat + (size_t)b0 * K, Yhat + (size_t)b0 * m, g, u,
-                                           ell, Y + (size_t)b0 * m, accept + b0, vec);
+        cudaError_t e = mask ? cudaLaunchKernelEx(&cfg, k_decode_verify<true>, PT, m, K, st, t_x,
+                                                  Xhat + (size_t)b0 * K, Yhat + (size_t)b0 * m, g, u,
+                                                  ell, Y + (size_t)b0 * m, accept + b0, vec,
+                                                  mask + (size_t)b0 * m)
+                             : cudaLaunchKernelEx(&cfg, k_decode_verify<false>, PT, m, K,
+                                                  st + (size_t)b0 * 2 * t_x, t_x, Xhat + (size_t)b0 * K,
+                                                  Yhat + (size_t)b0 * m, g, u, ell, Y + (size_t)b0 * m,
+                                                  accept + b0, vec, (const uint32_t *)nullptr);
         if (e != cudaSuccess) return e;
     }
     return cudaGetLastError();

@@ -120,10 +120,20 @@ uint32_t *library_error_word();
 cudaError_t launch_verify_u(const uint32_t *Qm, int K, const uint32_t *chal, uint32_t t_y,
                             uint32_t ell, uint32_t *u, cudaStream_t s);
 
-// Fused decrypt and verify reduction for B vectors.
+// Fused decrypt and verify reduction for B vectors.  With mask non-null
+// (boost mode) Y = Y_hat - mask, mask [B][m] = P e_x per vector, and st is
+// not read.
 cudaError_t launch_decode_verify(const uint32_t *PT, int m, int K, const uint32_t *st, uint32_t t_x,
                                  const uint32_t *Xhat, const uint32_t *Yhat, const uint32_t *g,
                                  const uint32_t *u, uint32_t ell, int B, uint32_t *Y,
-                                 int32_t *accept, cudaStream_t s);
+                                 int32_t *accept, cudaStream_t s, const uint32_t *mask = nullptr);
+
+// out = a + b over F_q (n elements; out may alias a or b).
+cudaError_t launch_field_add(const uint32_t *a, const uint32_t *b, size_t n, uint32_t *out,
+                             cudaStream_t s);
+
+// Output masks out[b] = P e_x,b (m values) from st [B][2t_x].
+cudaError_t launch_output_mask(const uint32_t *PT, int m, const uint32_t *st, uint32_t t_x, int B,
+                               uint32_t *out, cudaStream_t s);
 
 }  // namespace pv

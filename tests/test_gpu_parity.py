@@ -159,6 +159,44 @@ def test_lane_encode_ragged_groups_and_chunks(pv, wl):
     b.destroy()
 
 
+@pytest.mark.parametrize("m,K,B", [(300, 1000, 5), (64, 6000, 40), (4096, 4096, 3)])
+def test_boost_mode_matches_standard_mode(pv, wl, m, K, B):
+    """Boost mode (masks prepared ahead) gives the same x_hat, y and verdicts
+    as the standard calls with the same keys; the masks equal the oracle's
+    G_x e_x and P e_x; a tampered output is rejected."""
+    W = wl.weights_uniform(m, K, m + K)
+    x = wl.int8_vectors(B, K, m + 2 * K)
+    X = field(x)
+    Wd, Xd = to_dev(W), to_dev(X)
+    ctx = pv.pvmvmd_preprocess(Wd, key=41)
+    pp = oracle.PublicParams(W, oracle.key_from_seed(41), with_tables=False)
+    mi, mo, st = pv.pvmvmd_boost_prepare(ctx, B, key=42)
+    mi_h, mo_h, st_h = pv.as_u32(mi), pv.as_u32(mo), pv.as_u32(st)
+    zeros = np.zeros(K, np.uint32)
+    for b in range(B):
+        xp, s_o, v_o = pp.encrypt(zeros, oracle.key_from_seed(42), b)
+        assert np.array_equal(mi_h[b], xp), b
+        assert np.array_equal(st_h[b], np.concatenate([s_o, v_o])), b
+        rows = sample_rows(m, 16, b)
+        y0 = np.zeros(len(rows), np.uint32)
+        neg = pp.decrypt_rows(s_o, v_o, y0, rows)  # 0 - P e_x on the sampled rows
+        assert np.array_equal((Q - neg.astype(np.int64)) % Q, mo_h[b, rows].astype(np.int64)), b
+    Xh = pv.pvmvmd_boost_encode(Xd, mi)
+    Xs, sts = pv.pvmvmd_encode(ctx, Xd, key=42)
+    assert np.array_equal(pv.as_u32(Xh), pv.as_u32(Xs))
+    Yh = pv.pvmvmd_server_mvm(Wd, Xh)
+    Yb, ab = pv.pvmvmd_boost_decode_verify(ctx, mo, Xh, Yh, challenge_key=43)
+    Ys, as_ = pv.pvmvmd_decode_verify(ctx, sts, Xs, Yh, challenge_key=43)
+    assert np.array_equal(pv.as_u32(Yb), pv.as_u32(Ys))
+    assert np.array_equal(oracle.centered(pv.as_u32(Yb)), x.astype(np.int64) @ W.astype(np.int64).T)
+    assert pv.as_u32(ab).tolist() == [1] * B and pv.as_u32(as_).tolist() == [1] * B
+    tamper(pv, Yh, B - 1, m // 2, 7)
+    _, ab2 = pv.pvmvmd_boost_decode_verify(ctx, mo, Xh, Yh, challenge_key=44)
+    assert pv.as_u32(ab2).tolist() == [1] * (B - 1) + [0]
+    assert pv.pvmvmd_device_status() == 0
+    ctx.destroy()
+
+
 def test_server_mvm_extremes(pv):
     """Extreme weights and field values: -128, 127, x = 0, 1, (q-1)/2, (q+1)/2, q-1."""
     rng = np.random.default_rng(1)
