@@ -624,6 +624,104 @@ def run_batched(args):
     return 0
 
 
+def run_token(args):
+    """One token of 32 independent 8B-class layers at batch 1 (the server's
+    side): the 7 projections of each layer as one grouped product call,
+    32 calls per token in one CUDA graph.  Weights are seeded int8 (Gaussian,
+    sigma 32, rounded and clipped), 6.98 GB per token, so every token streams
+    them from HBM; x_hat is uniform in F_q."""
+    import torch
+    rank, world, local = dist_env()
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    import paper_2609_10264_gb300 as pv
+    from paper_2609_10264_gb300 import workloads as wl
+    Q = pv.PVMVMD_Q
+    nlayers = 32
+    gen = torch.Generator(device=device)
+    layers = []
+    for l in range(nlayers):
+        trip = []
+        for j, (name, (m, K)) in enumerate(wl.LAYER_8B.items()):
+            gen.manual_seed(1000 + 7 * l + j)
+            W = (torch.randn((m, K), generator=gen, device=device) * 32.0).round_().clamp_(-127, 127).to(torch.int8)
+            xh = torch.randint(0, Q, (K,), generator=gen, device=device, dtype=torch.int64).to(torch.int32)
+            trip.append((W, xh, torch.empty(m, dtype=torch.int32, device=device)))
+        layers.append(trip)
+    jobs = [pv.mvm_jobs(t) for t in layers]
+    stream = torch.cuda.Stream(device)
+
+    def token():
+        for l in range(nlayers):
+            pv.pvmvmd_server_mvm_multi(jobs[l], stream=stream)
+
+    with torch.cuda.stream(stream):
+        token()
+    stream.synchronize()
+    pv.pvmvmd_device_status(stream)
+    # exact check of sampled rows of one projection per layer (int64 numpy)
+    for l in (0, nlayers - 1):
+        W, xh, yh = layers[l][6]
+        rows = [0, 1, W.shape[0] // 2, W.shape[0] - 1]
+        Wr = W[rows].cpu().numpy().astype(np.int64)
+        x = pv.as_u32(xh).astype(np.int64)
+        assert np.array_equal(pv.as_u32(yh)[rows].astype(np.int64), (Wr @ x) % Q), f"layer {l}"
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        token()
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            g.replay()
+    stream.synchronize()
+    clocks = ClockSampler(device.index)
+    clocks.start()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        t0.record(stream)
+        for _ in range(args.steps):
+            g.replay()
+        t1.record(stream)
+    stream.synchronize()
+    clk = clocks.stop()
+    pv.pvmvmd_device_status(stream)
+    ms = t0.elapsed_time(t1) / args.steps
+    # the same 224 requests as one grouped call (the server's view when the
+    # layers' inputs are all known, e.g. when it replays a finished token)
+    all_jobs = pv.mvm_jobs([t for trip in layers for t in trip])
+    g1 = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g1, stream=stream):
+        pv.pvmvmd_server_mvm_multi(all_jobs, stream=stream)
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            g1.replay()
+        t0.record(stream)
+        for _ in range(args.steps):
+            g1.replay()
+        t1.record(stream)
+    stream.synchronize()
+    ms_one = t0.elapsed_time(t1) / args.steps
+    macs = nlayers * sum(m * K for (m, K) in wl.LAYER_8B.values())
+    nbytes = nlayers * sum(m * K + 4 * K + 4 * m for (m, K) in wl.LAYER_8B.values())
+    peaks, kind = measured_peaks()
+    achieved = nbytes / (ms / 1e3) / 1e9
+    if rank == 0:
+        print(json.dumps({
+            "metric": METRIC, "value": macs / (ms / 1e3), "unit": UNIT, "n_gpus": 1, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "u32 (F_q exact; int8 weights, dp4a digits)", "data": "synthetic",
+            "config": {"workload": "token8b-b1", "layers": nlayers, "projections": list(wl.LAYER_8B),
+                       "calls_per_token": nlayers, "weight_bytes_per_token": nbytes,
+                       "l2": "6.98 GB of distinct weights per token (larger than L2)"},
+            "one_call_per_token": {"ms": ms_one, "hbm_gbs": nbytes / (ms_one / 1e3) / 1e9,
+                                   "value": macs / (ms_one / 1e3)},
+            "roofline": {"bound": "hbm", "kernel": "k_gemv_multi (7 requests per launch)", "achieved": achieved,
+                         "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],
+                         "peak_kind": f"{kind} hbm_gbs", "traffic": None},
+            "gpu_launches": nlayers * args.steps, "clocks": clk}), flush=True)
+    return 0
+
+
 def run_server_shape(args):
     """The batched server product Y_hat = M X_hat alone on one m x K x B
     shape (``--shape MxKxB``), timed over --steps launches after --warmup.
@@ -698,7 +796,7 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-vectors", type=int, default=150)
     ap.add_argument("--server-mode", choices=["multi", "calls"], default="multi")
-    ap.add_argument("--workload", choices=["batch1-4096", "server-shape"] + sorted(BATCHED),
+    ap.add_argument("--workload", choices=["batch1-4096", "server-shape", "token8b-b1"] + sorted(BATCHED),
                     default="batch1-4096")
     ap.add_argument("--shape", default="4096x4096x64", help="m x K x B for --workload server-shape")
     ap.add_argument("--server-streams", type=int, default=2)
@@ -715,6 +813,8 @@ def main(argv=None):
         return run_batched(args)
     if args.workload == "server-shape":
         return run_server_shape(args)
+    if args.workload == "token8b-b1":
+        return run_token(args)
     return run_ours(args)
 
 
