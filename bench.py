@@ -512,6 +512,10 @@ BATCHED = {
     "layer8b-b64": {"B": 64, "shapes": [("q", 4096, 4096), ("k", 1024, 4096), ("v", 1024, 4096),
                                         ("o", 4096, 4096), ("gate", 14336, 4096), ("up", 14336, 4096),
                                         ("down", 4096, 14336)]},
+    # one Qwen3-4B block (the paper's evaluation model) with an eight-token prompt
+    "layerqwen4b-b8": {"B": 8, "shapes": [("q", 4096, 2560), ("k", 1024, 2560), ("v", 1024, 2560),
+                                          ("o", 2560, 4096), ("gate", 9728, 2560), ("up", 9728, 2560),
+                                          ("down", 2560, 9728)]},
     # 70B-class projections, 256 vectors each
     "layer70b-b256": {"B": 256, "shapes": [("q", 8192, 8192), ("kv", 1024, 8192), ("gate_up", 28672, 8192),
                                            ("down", 8192, 28672)]},

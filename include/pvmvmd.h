@@ -126,7 +126,9 @@ int pvmvmd_encode(pvmvmd_ctx *ctx, const uint32_t *X_dev, int B, const pvmvmd_ke
 /* The server's product Y_hat = M X_hat over F_q (Sec. 6.1: the server's whole
  * online work).  W_dev int8 m x K row-major, Xhat_dev B x K, Yhat_dev B x m.
  * Needs no context and no secret.  B == 1 runs the bandwidth-bound GEMV;
- * B > 1 runs the byte-limb tensor-core product.  1 <= K <= PVMVMD_MAX_K. */
+ * 2 <= B <= 16 (K a multiple of 16, 16-byte aligned W and Xhat) a GEMV that
+ * reads M once per four vectors; larger B the byte-limb tensor-core product.
+ * 1 <= K <= PVMVMD_MAX_K. */
 int pvmvmd_server_mvm(const int8_t *W_dev, int m, int K, const uint32_t *Xhat_dev, int B,
                       uint32_t *Yhat_dev, void *stream);
 

@@ -29,6 +29,8 @@ constexpr uint32_t kTagChallenge = 10;
 // (launch_lane_syndrome) when the code needs a cluster per vector; smaller
 // batches and codes that fit one CTA use the fused kernel.
 constexpr int kLaneMinBatch = 32;
+// Server products of at most this many vectors use the small-batch GEMV.
+constexpr int kSmallBatchMax = 16;
 
 // --------------------------------------------------------------------------
 // Host ChaCha20 keystream (RFC 8439 Sec. 2.3) read as 32-bit words.
@@ -509,6 +511,13 @@ int pvmvmd_server_mvm(const int8_t *W_dev, int m, int K, const uint32_t *Xhat_de
     if (!err) return PVMVMD_E_CUDA;
     if (B == 1) {
         PV_CUDA(launch_gemv(W_dev, m, K, Xhat_dev, Yhat_dev, err, s));
+        return PVMVMD_OK;
+    }
+    // a few vectors: one pass over M per four vectors (the tensor-core
+    // product's tiles hold 64 vectors)
+    if (B <= kSmallBatchMax && K % 16 == 0 &&
+        ((reinterpret_cast<uintptr_t>(W_dev) | reinterpret_cast<uintptr_t>(Xhat_dev)) & 15u) == 0) {
+        PV_CUDA(launch_gemv_small_batch(W_dev, m, K, Xhat_dev, B, Yhat_dev, s));
         return PVMVMD_OK;
     }
     PV_CUDA(launch_batched(W_dev, m, K, Xhat_dev, B, Yhat_dev, err, s));

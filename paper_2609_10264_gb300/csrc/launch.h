@@ -100,6 +100,11 @@ struct MvmJob {
 constexpr int kMultiMaxJobs = 256;  // jobs per grouped launch
 constexpr int kMultiMaxK = 16384;   // K per grouped launch (longer K is segmented)
 
+// Y_hat = M X_hat for a few vectors (2 <= B <= 16): one pass over M per group
+// of four vectors.  Needs K % 16 == 0 and 16-byte aligned W and X_hat.
+cudaError_t launch_gemv_small_batch(const int8_t *W, int m, int K, const uint32_t *Xhat, int B,
+                                    uint32_t *Yhat, cudaStream_t s);
+
 // Eligible for the grouped kernel: K % 16 == 0 and 16-byte aligned rows.
 bool multi_eligible(const MvmJob &j);
 // Any number of eligible jobs, in as few launches as K allows.

@@ -16,6 +16,10 @@ Q = 2013265921
 LAYER_8B = {"q": (4096, 4096), "k": (1024, 4096), "v": (1024, 4096), "o": (4096, 4096),
             "gate": (14336, 4096), "up": (14336, 4096), "down": (4096, 14336)}
 LAYER_70B = {"q": (8192, 8192), "kv": (1024, 8192), "gate_up": (28672, 8192), "down": (8192, 28672)}
+# Qwen3-4B transformer block (the paper's evaluation model, Sec. 7.3 table
+# of projection dimensions), as (output m, input K); weights stay synthetic
+LAYER_QWEN3_4B = {"q": (4096, 2560), "k": (1024, 2560), "v": (1024, 2560), "o": (2560, 4096),
+                  "gate": (9728, 2560), "up": (9728, 2560), "down": (2560, 9728)}
 
 
 def _rng(seed) -> np.random.Generator:

@@ -344,6 +344,37 @@ def test_config5_70b(pv, wl, name):
     _batched_pipeline_sampled(pv, W, 256, seed=500 + len(name), n_rows=12, n_verify=1)
 
 
+@pytest.mark.parametrize("m,K,B", [(4096, 2560, 8), (37, 6144 + 96, 5), (300, 16, 2), (2560, 9728, 16),
+                                   (1000, 4096, 3)])
+def test_small_batch_server_product(pv, wl, m, K, B):
+    """2 <= B <= 16 runs the small-batch GEMV (one pass over M per four
+    vectors, K in segments of 6144): equal to the per-vector GEMV and to the
+    oracle on sampled rows, with full-range x_hat and extreme weights."""
+    import torch
+    rng = np.random.default_rng(m + K + B)
+    W = rng.integers(-128, 128, size=(m, K), dtype=np.int8)
+    W[0, :] = -128
+    X = rng.integers(0, Q, size=(B, K)).astype(np.uint32)
+    X[0, :] = (Q - 1) // 2 + 1
+    Wd, Xd = to_dev(W), to_dev(X)
+    Y = pv.as_u32(pv.pvmvmd_server_mvm(Wd, Xd))
+    Y1 = np.stack([pv.as_u32(pv.pvmvmd_server_mvm(Wd, Xd[b])) for b in range(B)])
+    assert np.array_equal(Y, Y1)
+    rows = sample_rows(m, 24, B)
+    for b in range(B):
+        assert np.array_equal(Y[b, rows], oracle.server_mvm_rows(W, X[b], rows)), b
+    assert pv.pvmvmd_device_status() == 0
+
+
+@pytest.mark.parametrize("name", ["q", "o", "down"])
+def test_qwen3_4b_block_8_tokens(pv, wl, name):
+    """Qwen3-4B projection shapes (the paper's evaluation table) with an
+    eight-token batch, synthetic weights."""
+    m, K = wl.LAYER_QWEN3_4B[name]
+    W = wl.weights_gaussian(m, K, (6, list(wl.LAYER_QWEN3_4B).index(name)))
+    _batched_pipeline_sampled(pv, W, 8, seed=600 + len(name))
+
+
 def test_server_mvm_multi_mixed_jobs(pv, wl):
     """Grouped batch-1 products over mixed shapes, including K beyond one
     segment (20000), a K that is not a multiple of 16 (1001) and tiny matrices; equal to the
