@@ -17,6 +17,10 @@ Parity status of each function (what pins it is listed in the tests):
   raa_encode / raa_syndrome ........ pinned (dense App. B matrices, adjoint)
   server_mvm ....................... pinned (Python big-int brute force)
   encrypt / decrypt / verify ....... pinned (completeness, Lemma 5.1 rate)
+  BatchParams (Protocol 2) ......... pinned (dense Q~^T G' product, the
+                                      bilinear identity, completeness,
+                                      rejection of wrong outputs and of a
+                                      wrong server projection)
   privacy of x_hat ................. parity unpinned (computational assumption)
 """
 from __future__ import annotations
@@ -37,6 +41,12 @@ DELTA = 0.5     # target relative distance (Sec. 7.1)
 T_Y_PAPER = 31  # verification sparsity used in Sec. 7.1
 TAG_MASK = 9
 TAG_CHALLENGE = 10
+# Batch verification (Protocol 2): code numbers for the sampler (tags
+# 4 which + 1 .. 4 which + 4) and challenge tags.
+BV_CODE_PRIMARY = 3     # G over the outputs, dimension m
+BV_CODE_SECONDARY = 4   # G' over the stacked inputs, dimension B n
+TAG_BV_PRIMARY = 21
+TAG_BV_SECONDARY = 22
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "pvmvmd_oracle.c")
@@ -313,3 +323,77 @@ def hypergeom_miss(N: int, w: int, t: int) -> float:
         return 0.0
     return math.exp(math.lgamma(N - w + 1) - math.lgamma(N - w - t + 1)
                     - math.lgamma(N + 1) + math.lgamma(N - t + 1))
+
+
+# --------------------------------------------------------------------------- Protocol 2
+
+def _dot(a, b) -> int:
+    """sum a_i b_i mod q with Python integers."""
+    return int(sum(int(x) * int(y) for x, y in zip(a, b)) % Q)
+
+
+class BatchParams:
+    """Batch verification Pi_Batch-vMVMD (Protocol 2) for B matrices of one
+    shape m x n, written out step by step.
+
+    Preprocess: G <- primary code (dimension m, N = rate m), G' <- secondary
+    code (dimension B n, N' = rate B n); Q_b = G^T M_b (N x n);
+    Qt = (Q_1, ..., Q_B)^T (B n x N, row b n + k = column k of Q_b);
+    Qaux = Qt^T G' (N x N', row i = the code word G'^T (column i of Qt)).
+    Verify: z_b = G^T y_b; primary challenges e^(q) <- E_t^N shared by the
+    B claims; server u^(q) = Qt e^(q); secondary challenges
+    e'^(j) <- E_t'^N' drawn after the responses; r^(j) = G' e'^(j); accept
+    iff e^(q)^T Qaux e'^(j) = r^(j)^T u^(q) for all q, j and
+    u_b^(q)^T x_b = e^(q)^T z_b for all b, q."""
+
+    def __init__(self, Ws, key, t: int = T_Y_PAPER, ell: int | None = None, t2: int = T_Y_PAPER,
+                 ell2: int | None = None, rate: int = RATE):
+        self.Ws = [np.ascontiguousarray(W, dtype=np.int8) for W in Ws]
+        self.B = len(self.Ws)
+        self.m, self.n = self.Ws[0].shape
+        self.rate = rate
+        self.t, self.t2 = int(t), int(t2)
+        self.ell = verify_params()[2] if ell is None else int(ell)
+        self.ell2 = verify_params()[2] if ell2 is None else int(ell2)
+        self.G = Code.sample(key, BV_CODE_PRIMARY, self.m, rate)
+        self.G2 = Code.sample(key, BV_CODE_SECONDARY, self.B * self.n, rate)
+        self.N, self.N2 = self.G.N, self.G2.N
+        # Q_b = G^T M_b: column k of Q_b encodes column k of M_b
+        self.Qb = [np.stack([self.G.encode(lift(W[:, k])) for k in range(self.n)], axis=1) for W in self.Ws]
+        self.Qt = np.concatenate([Q.T for Q in self.Qb], axis=0)            # B n x N
+        self.Qaux = np.stack([self.G2.encode(self.Qt[:, i]) for i in range(self.N)], axis=0)  # N x N'
+
+    def challenges(self, key):
+        """Primary challenges e^(q), q < ell, as (support, values) pairs."""
+        return [sample_sparse(key, TAG_BV_PRIMARY, q, self.N, self.t) for q in range(self.ell)]
+
+    def server_project(self, chals) -> np.ndarray:
+        """u^(q) = Qt e^(q) for every q: ell x B n."""
+        out = np.zeros((len(chals), self.B * self.n), np.uint32)
+        for q, (s, v) in enumerate(chals):
+            for p in range(self.B * self.n):
+                out[q, p] = _dot(self.Qt[p, s], v)
+        return out
+
+    def secondary(self, key):
+        return [sample_sparse(key, TAG_BV_SECONDARY, j, self.N2, self.t2) for j in range(self.ell2)]
+
+    def check(self, xs, ys, chals, us, key2) -> bool:
+        """The client's checks of Protocol 2 on claims y_b = M_b x_b."""
+        sec = self.secondary(key2)
+        for (s2, v2) in sec:
+            dense = np.zeros(self.N2, np.uint32)
+            dense[s2] = v2
+            r = self.G2.syndrome(dense)                                    # G' e'
+            for q, (s, v) in enumerate(chals):
+                lhs = int(sum(int(v[a]) * _dot(self.Qaux[s[a], s2], v2) for a in range(len(s))) % Q)
+                if lhs != _dot(r, us[q]):
+                    return False
+        for b in range(self.B):
+            z = self.G.encode(_u32a(ys[b]))                                # G^T y_b
+            for q, (s, v) in enumerate(chals):
+                ub = us[q][b * self.n:(b + 1) * self.n]
+                if _dot(ub, xs[b]) != _dot(z[s], v):
+                    return False
+        return True
+

@@ -201,7 +201,7 @@ enum { TAG_PI1 = 1, TAG_PI2 = 2, TAG_V1 = 3, TAG_V2 = 4, TAG_MASK = 9, TAG_CHALL
  * which = 1 for G_y. */
 void orc_code_sample(const uint32_t key[8], int which, uint32_t N,
                      uint32_t *pi1, uint32_t *pi2, uint32_t *v1, uint32_t *v2) {
-    uint32_t base = which ? 4u : 0u;
+    uint32_t base = 4u * (uint32_t)which;  /* code `which` reads tags 4 which + 1 .. 4 which + 4 */
     orc_sample_permutation(key, base + TAG_PI1, 0, N, pi1);
     orc_sample_permutation(key, base + TAG_PI2, 0, N, pi2);
     orc_sample_field_vector(key, base + TAG_V1, 0, N, 1, v1);

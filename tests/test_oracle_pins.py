@@ -383,3 +383,91 @@ def test_verify_noQ_identity_agrees(tiny_pp):
     rows = [0, 9, 255]
     assert np.array_equal(small.decrypt_rows(supp, vals, yhat[rows], rows),
                           pp.decrypt(supp, vals, yhat)[rows])
+
+
+# --------------------------------------------------------------------------- Protocol 2
+
+def _bv_claims(rng, B, m, n):
+    Ws = [rng.integers(-128, 128, size=(m, n), dtype=np.int8) for _ in range(B)]
+    xs = [rng.integers(0, Q, n).astype(np.uint32) for _ in range(B)]
+    ys = [oracle.server_mvm(Ws[b], xs[b]) for b in range(B)]
+    return Ws, xs, ys
+
+
+def test_bv_tables_match_dense_definitions():
+    """Q_b = G^T M_b and Qaux = Qt^T G' equal the products with the dense App. B
+    generators built entry by entry (Protocol 2 preprocessing)."""
+    rng = np.random.default_rng(3)
+    B, m, n = 2, 3, 2
+    Ws, _, _ = _bv_claims(rng, B, m, n)
+    bp = oracle.BatchParams(Ws, oracle.key_from_seed(4), t=3, t2=3)
+    G, G2 = _dense_G(bp.G), _dense_G(bp.G2)                  # m x N, B n x N'
+    GT = [list(col) for col in zip(*G)]                       # N x m
+    for b in range(B):
+        Mb = [[int(v) % Q for v in row] for row in Ws[b]]     # lifted, m x n
+        assert np.array_equal(np.array(_mm(GT, Mb), dtype=np.uint32), bp.Qb[b])
+    QtT = [[int(v) for v in row] for row in bp.Qt.T]          # N x B n
+    assert np.array_equal(np.array(_mm(QtT, G2), dtype=np.uint32), bp.Qaux)
+
+
+def test_bv_bilinear_identity():
+    """e^T Qaux e' = (G' e')^T (Qt e) for arbitrary e, e' (the identity the
+    secondary check relies on), with the syndrome computed independently."""
+    rng = np.random.default_rng(5)
+    Ws, _, _ = _bv_claims(rng, 3, 4, 3)
+    bp = oracle.BatchParams(Ws, oracle.key_from_seed(6), t=5, t2=5)
+    for _ in range(5):
+        e = rng.integers(0, Q, bp.N).astype(np.uint32)
+        e2 = rng.integers(0, Q, bp.N2).astype(np.uint32)
+        lhs = sum(int(e[i]) * oracle._dot(bp.Qaux[i], e2) for i in range(bp.N)) % Q
+        u = [oracle._dot(bp.Qt[p], e) for p in range(bp.B * bp.n)]
+        assert lhs == oracle._dot(bp.G2.syndrome(e2), u)
+
+
+def test_bv_completeness():
+    """Honest outputs and an honest server projection are always accepted."""
+    rng = np.random.default_rng(7)
+    Ws, xs, ys = _bv_claims(rng, 4, 6, 5)
+    bp = oracle.BatchParams(Ws, oracle.key_from_seed(8))
+    for s in range(6):
+        ch = bp.challenges(oracle.key_from_seed(100 + s))
+        assert bp.check(xs, ys, ch, bp.server_project(ch), oracle.key_from_seed(200 + s))
+
+
+def test_bv_rejects_wrong_outputs_and_projections():
+    """A wrong entry in any y_b fails an original check; a server projection
+    off by a nonzero vector fails a secondary check (paper parameters)."""
+    rng = np.random.default_rng(9)
+    Ws, xs, ys = _bv_claims(rng, 3, 5, 4)
+    bp = oracle.BatchParams(Ws, oracle.key_from_seed(10))
+    for s in range(6):
+        ch = bp.challenges(oracle.key_from_seed(300 + s))
+        us = bp.server_project(ch)
+        bad = [y.copy() for y in ys]
+        b, i = s % 3, (2 * s) % 5
+        bad[b][i] = (int(bad[b][i]) + 1 + s) % Q
+        assert not bp.check(xs, bad, ch, us, oracle.key_from_seed(400 + s))
+        ub = us.copy()
+        ub[s % bp.ell, (3 * s) % (bp.B * bp.n)] ^= 1
+        assert not bp.check(xs, ys, ch, ub, oracle.key_from_seed(500 + s))
+
+
+@pytest.mark.parametrize("t2", [1, 3])
+def test_bv_secondary_rate_matches_lemma_5_1(t2):
+    """With a weak secondary challenge (t' small, ell' = 1) a fixed wrong
+    projection u = Qt e + Gamma is accepted at the rate
+    C(N' - w, t')/C(N', t'), w = wt(G'^T Gamma) (Lemma 5.1 applied to G')."""
+    rng = np.random.default_rng(11 + t2)
+    Ws, xs, ys = _bv_claims(rng, 2, 3, 3)
+    bp = oracle.BatchParams(Ws, oracle.key_from_seed(12), t=4, ell=1, t2=t2, ell2=1)
+    ch = bp.challenges(oracle.key_from_seed(13))
+    us = bp.server_project(ch)
+    gamma = np.zeros(bp.B * bp.n, np.uint64)
+    gamma[2] = 777
+    bad = ((us + gamma[None, :]) % Q).astype(np.uint32)
+    w = int(np.count_nonzero(bp.G2.encode(gamma.astype(np.uint32))))
+    p = oracle.hypergeom_miss(bp.N2, w, t2)
+    trials = 3000
+    acc = sum(bp.check(xs, ys, ch, bad, oracle.key_from_seed(10 ** 6 + s)) for s in range(trials))
+    sigma = math.sqrt(p * (1 - p) / trials)
+    assert abs(acc / trials - p) <= 4 * sigma + 1e-9, (acc / trials, p, w)
