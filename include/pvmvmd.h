@@ -214,6 +214,47 @@ int pvmvmd_boost_decode_verify(pvmvmd_ctx *ctx, const uint32_t *mask_out_dev,
                                const pvmvmd_key *challenge_key, uint32_t *Y_dev,
                                int32_t *accept_dev, void *stream);
 
+/* ---------------------------------------------------------------------
+ * Batch verification, Protocol 2 (Pi_Batch-vMVMD, Sec. 5): B claims
+ * y_b = M_b x_b for B matrices of one shape m x n, checked together.  The
+ * primary code G (dimension m, N = rate m) and the secondary code G'
+ * (dimension B n, N' = rate B n) are sampled as code numbers 3 and 4 of
+ * pvmvmd_code_sample_host.  Preprocess computes Q_b = G^T M_b, stored side
+ * by side as Qs (N x B n, row i = (Q_1[i], ..., Q_B[i]) = Qt^T, the matrix
+ * the server needs), and Qaux = Qt^T G' (stored transposed, N' x N).
+ * A round:
+ *   client pvmvmd_bv_challenge     once every y_b is fixed: ell primary
+ *                                   challenges e^(q) <- E_t^N (tag 21),
+ *                                   chal_dev ell x 2t (support, values);
+ *   server pvmvmd_bv_server_project u^(q) = Qt e^(q), u_dev ell x B n;
+ *   client pvmvmd_bv_check          draws ell' secondary challenges
+ *                                   e'^(j) <- E_t'^N' (tag 22, key2) and
+ *                                   sets *accept_dev (int32) to 1 iff
+ *                                   e^(q)^T Qaux e'^(j) = (G' e'^(j))^T u^(q)
+ *                                   for all q, j and
+ *                                   u_b^(q)^T x_b = e^(q)^T G^T y_b for all
+ *                                   b, q; else 0.
+ * W_dev: B x m x n int8 (matrix b at W_dev + b m n); X_dev B x n; Y_dev
+ * B x m.  Defaults (0 fields): rate 8, t = t' = 31, ell = ell' = 2. */
+typedef struct pvmvmd_bv_ctx pvmvmd_bv_ctx;
+typedef struct {
+    int rate, t, ell, t2, ell2;
+} pvmvmd_bv_params;
+typedef struct {
+    int B, m, n, rate, N, N2, t, ell, t2, ell2;
+    const uint32_t *Qs, *QauxT, *chal2; /* device pointers owned by the context */
+} pvmvmd_bv_view;
+int pvmvmd_bv_preprocess(const int8_t *W_dev, int B, int m, int n, const pvmvmd_bv_params *params,
+                         const pvmvmd_key *key, void *stream, pvmvmd_bv_ctx **out);
+int pvmvmd_bv_challenge(pvmvmd_bv_ctx *ctx, const pvmvmd_key *key, uint32_t *chal_dev, void *stream);
+int pvmvmd_bv_server_project(const pvmvmd_bv_ctx *ctx, const uint32_t *chal_dev, uint32_t *u_dev,
+                             void *stream);
+int pvmvmd_bv_check(pvmvmd_bv_ctx *ctx, const uint32_t *X_dev, const uint32_t *Y_dev,
+                    const uint32_t *chal_dev, const uint32_t *u_dev, const pvmvmd_key *key2,
+                    int32_t *accept_dev, void *stream);
+int pvmvmd_bv_info(const pvmvmd_bv_ctx *ctx, pvmvmd_bv_view *view);
+void pvmvmd_bv_destroy(pvmvmd_bv_ctx *ctx);
+
 /* Synchronise `stream`, then read and clear the library's device error word:
  * PVMVMD_E_DEVICE_TIMEOUT if any kernel gave up a bounded wait since the last
  * call, else PVMVMD_OK (or PVMVMD_E_CUDA if synchronisation failed). */

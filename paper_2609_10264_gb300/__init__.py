@@ -61,6 +61,16 @@ class pvmvmd_ctx_view(ctypes.Structure):
                 ("PT", ctypes.c_void_p), ("Q", ctypes.c_void_p)]
 
 
+class pvmvmd_bv_params(ctypes.Structure):
+    _fields_ = [("rate", ctypes.c_int), ("t", ctypes.c_int), ("ell", ctypes.c_int), ("t2", ctypes.c_int),
+                ("ell2", ctypes.c_int)]
+
+
+class pvmvmd_bv_view(ctypes.Structure):
+    _fields_ = [(f, ctypes.c_int) for f in ("B", "m", "n", "rate", "N", "N2", "t", "ell", "t2", "ell2")] + \
+               [("Qs", ctypes.c_void_p), ("QauxT", ctypes.c_void_p), ("chal2", ctypes.c_void_p)]
+
+
 class pvmvmd_mvm_job(ctypes.Structure):
     _fields_ = [("W_dev", ctypes.c_void_p), ("xhat_dev", ctypes.c_void_p), ("yhat_dev", ctypes.c_void_p),
                 ("m", ctypes.c_int), ("K", ctypes.c_int)]
@@ -82,6 +92,13 @@ SIGNATURES = {
     "pvmvmd_boost_encode": (_i, [_vp, _vp, _i, _i, _vp, _vp]),
     "pvmvmd_boost_decode_verify": (_i, [_vp, _vp, _vp, _vp, _i, ctypes.POINTER(pvmvmd_key), _vp, _vp,
                                         _vp]),
+    "pvmvmd_bv_preprocess": (_i, [_vp, _i, _i, _i, ctypes.POINTER(pvmvmd_bv_params), ctypes.POINTER(pvmvmd_key),
+                                  _vp, ctypes.POINTER(_vp)]),
+    "pvmvmd_bv_challenge": (_i, [_vp, ctypes.POINTER(pvmvmd_key), _vp, _vp]),
+    "pvmvmd_bv_server_project": (_i, [_vp, _vp, _vp, _vp]),
+    "pvmvmd_bv_check": (_i, [_vp, _vp, _vp, _vp, _vp, ctypes.POINTER(pvmvmd_key), _vp, _vp]),
+    "pvmvmd_bv_info": (_i, [_vp, ctypes.POINTER(pvmvmd_bv_view)]),
+    "pvmvmd_bv_destroy": (None, [_vp]),
     "pvmvmd_device_status": (_i, [_vp]),
     "pvmvmd_ctx_info": (_i, [_vp, ctypes.POINTER(pvmvmd_ctx_view)]),
     "pvmvmd_destroy": (None, [_vp]),
@@ -383,6 +400,78 @@ def pvmvmd_boost_decode_verify(ctx: Ctx, mask_out, Xhat, Yhat, challenge_key, Y=
                                            _dev_ptr(accept, "accept", (torch.int32,), B), _stream_ptr(stream)),
            "pvmvmd_boost_decode_verify")
     return Y, accept
+
+
+class BvCtx:
+    """A batch-verification (Protocol 2) context; released by destroy() or
+    garbage collection."""
+
+    def __init__(self, handle, view):
+        self.handle = handle
+        for f, _ in pvmvmd_bv_view._fields_:
+            setattr(self, f, getattr(view, f))
+
+    def destroy(self):
+        if self.handle:
+            _lib.pvmvmd_bv_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass
+
+
+def pvmvmd_bv_preprocess(Ws, key, params: pvmvmd_bv_params | None = None, stream=None) -> BvCtx:
+    """Ws: B x m x n int8 device tensor (the B matrices)."""
+    import torch
+    if Ws.dim() != 3:
+        raise ValueError("Ws must be B x m x n")
+    B, m, n = Ws.shape
+    h = ctypes.c_void_p()
+    _check(_lib.pvmvmd_bv_preprocess(_dev_ptr(Ws, "Ws", (torch.int8,)), B, m, n,
+                                     ctypes.byref(params) if params is not None else None,
+                                     ctypes.byref(make_key(key)), _stream_ptr(stream), ctypes.byref(h)),
+           "pvmvmd_bv_preprocess")
+    v = pvmvmd_bv_view()
+    _check(_lib.pvmvmd_bv_info(h, ctypes.byref(v)), "pvmvmd_bv_info")
+    return BvCtx(h, v)
+
+
+def pvmvmd_bv_challenge(ctx: BvCtx, key, chal=None, device=None, stream=None):
+    import torch
+    if chal is None:
+        chal = torch.empty((ctx.ell, 2 * ctx.t), dtype=torch.int32, device=device or "cuda")
+    _check(_lib.pvmvmd_bv_challenge(ctx.handle, ctypes.byref(make_key(key)),
+                                    _dev_ptr(chal, "chal", _u32_types(), ctx.ell * 2 * ctx.t), _stream_ptr(stream)),
+           "pvmvmd_bv_challenge")
+    return chal
+
+
+def pvmvmd_bv_server_project(ctx: BvCtx, chal, u=None, stream=None):
+    import torch
+    if u is None:
+        u = torch.empty((ctx.ell, ctx.B * ctx.n), dtype=torch.int32, device=chal.device)
+    _check(_lib.pvmvmd_bv_server_project(ctx.handle, _dev_ptr(chal, "chal", _u32_types(), ctx.ell * 2 * ctx.t),
+                                         _dev_ptr(u, "u", _u32_types(), ctx.ell * ctx.B * ctx.n), _stream_ptr(stream)),
+           "pvmvmd_bv_server_project")
+    return u
+
+
+def pvmvmd_bv_check(ctx: BvCtx, X, Y, chal, u, key2, accept=None, stream=None):
+    """-> int32 tensor of one element: 1 accept, 0 reject."""
+    import torch
+    if accept is None:
+        accept = torch.empty(1, dtype=torch.int32, device=X.device)
+    _check(_lib.pvmvmd_bv_check(ctx.handle, _dev_ptr(X, "X", _u32_types(), ctx.B * ctx.n),
+                                _dev_ptr(Y, "Y", _u32_types(), ctx.B * ctx.m),
+                                _dev_ptr(chal, "chal", _u32_types(), ctx.ell * 2 * ctx.t),
+                                _dev_ptr(u, "u", _u32_types(), ctx.ell * ctx.B * ctx.n),
+                                ctypes.byref(make_key(key2)), _dev_ptr(accept, "accept", (torch.int32,), 1),
+                                _stream_ptr(stream)),
+           "pvmvmd_bv_check")
+    return accept
 
 
 def pvmvmd_device_status(stream=None) -> int:

@@ -25,6 +25,8 @@ constexpr uint32_t kTagCodeX = 1;       // G_x: pi1 = 1, pi2 = 2, v1 = 3, v2 = 4
 constexpr uint32_t kTagCodeY = 5;       // G_y: pi1 = 5, pi2 = 6, v1 = 7, v2 = 8
 constexpr uint32_t kTagMask = 9;
 constexpr uint32_t kTagChallenge = 10;
+constexpr uint32_t kTagBvPrimary = 21;    // batch verification challenges
+constexpr uint32_t kTagBvSecondary = 22;
 // Encode batches of at least this many vectors as the lanes of N x B arrays
 // (launch_lane_syndrome) when the code needs a cluster per vector; smaller
 // batches and codes that fit one CTA use the fused kernel.
@@ -99,7 +101,9 @@ class KeyStream {
 
 void sample_code_host(const pvmvmd_key &key, int which, uint32_t N, uint32_t *pi1, uint32_t *pi2,
                       uint32_t *v1, uint32_t *v2) {
-    const uint32_t tag0 = which ? kTagCodeY : kTagCodeX;
+    // code `which` reads tags 4 which + 1 .. 4 which + 4 (G_x = 0, G_y = 1;
+    // the batch verification codes are 3 and 4)
+    const uint32_t tag0 = kTagCodeX + 4u * (uint32_t)which;
     uint32_t *perms[2] = {pi1, pi2};
     for (int p = 0; p < 2; ++p) {  // Fisher-Yates, last index first
         KeyStream ks(key, tag0 + p, 0);
@@ -184,18 +188,32 @@ struct pvmvmd_ctx {
     std::vector<void *> owned;
 };
 
+// Batch verification (Protocol 2) for B matrices of one shape m x n.
+struct pvmvmd_bv_ctx {
+    int device = 0;
+    int B = 0, m = 0, n = 0, rate = 0, N = 0, N2 = 0, t = 0, ell = 0, t2 = 0, ell2 = 0;
+    pv::CodeDev g, g2;       // primary code (dimension m), secondary code (dimension B n)
+    uint32_t *Qs = nullptr;    // N x B n: row i = (Q_1[i], ..., Q_B[i]) = Qt^T (public)
+    uint32_t *QauxT = nullptr; // N' x N: Qaux transposed
+    uint32_t *Yt = nullptr, *Z = nullptr;  // m x B, N x B
+    uint32_t *chal2 = nullptr, *R = nullptr, *F2 = nullptr;
+    uint32_t *eS = nullptr, *eagg = nullptr, *eincl = nullptr, *eflags = nullptr;  // encode scratch
+    unsigned long long *status = nullptr;
+    std::vector<void *> owned;
+};
+
 namespace pv {
 namespace {
 
-template <typename T>
-cudaError_t ctx_alloc(pvmvmd_ctx *c, T **p, size_t count) {
+template <typename Ctx, typename T>
+cudaError_t ctx_alloc(Ctx *c, T **p, size_t count) {
     cudaError_t e = dev_alloc(p, count);
     if (e == cudaSuccess) c->owned.push_back(*p);
     return e;
 }
 
-int upload_code(pvmvmd_ctx *c, CodeDev &d, const pvmvmd_key &key, int which, uint32_t N,
-                cudaStream_t s) {
+template <typename Ctx>
+int upload_code(Ctx *c, CodeDev &d, const pvmvmd_key &key, int which, uint32_t N, cudaStream_t s) {
     std::vector<uint32_t> pi1(N), pi2(N), v1(N), v2(N), pi1inv(N), pi2inv(N), v2p(N), v2m(N), v1pm(N);
     sample_code_host(key, which, N, pi1.data(), pi2.data(), v1.data(), v2.data());
     for (uint32_t j = 0; j < N; ++j) {
@@ -220,7 +238,25 @@ int upload_code(pvmvmd_ctx *c, CodeDev &d, const pvmvmd_key &key, int which, uin
 
 // Y (N x L lanes, row stride ldy) = G^T applied to the L lanes of X (n x L,
 // row stride ldx; row i holds message entry i of every lane), in lane chunks.
-int encode_lanes(const CodeDev &d, uint32_t n, uint32_t r, const int8_t *X, size_t ldx,
+// One chunk of lanes with caller-provided scratch (S: N x nl, agg / incl /
+// flags sized by encode_scan_*_words(N, nl)); no allocation, no sync.
+int encode_lanes_into(const CodeDev &d, uint32_t n, uint32_t r, const void *X, bool x_is_i8, size_t ldx,
+                      uint32_t nl, uint32_t *Y, size_t ldy, uint32_t *S, uint32_t *agg, uint32_t *incl,
+                      uint32_t *flags, uint32_t *err, cudaStream_t s) {
+    const uint32_t N = n * r;
+    cudaError_t e = cudaMemsetAsync(flags, 0, encode_scan_flag_words(N, nl) * 4, s);
+    if (e == cudaSuccess)  // S = A^T V1 Pi1^T R^T X
+        e = launch_encode_scan(X, x_is_i8, ldx, d.pi1, r, d.v1, N, nl, S, nl, agg, incl, flags, err, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(flags, 0, encode_scan_flag_words(N, nl) * 4, s);
+    if (e == cudaSuccess)  // Y = A^T V2 Pi2^T S
+        e = launch_encode_scan(S, false, nl, d.pi2, 1, d.v2, N, nl, Y, ldy, agg, incl, flags, err, s);
+    return e == cudaSuccess ? PVMVMD_OK : PVMVMD_E_CUDA;
+}
+
+// Y (N x L lanes, row stride ldy) = G^T applied to the L lanes of X (n x L,
+// row stride ldx; row i holds message entry i of every lane; int8 or
+// uint32), in lane chunks with scratch allocated here (preprocessing only).
+int encode_lanes(const CodeDev &d, uint32_t n, uint32_t r, const void *X, bool x_is_i8, size_t ldx,
                  uint32_t L, uint32_t *Y, size_t ldy, uint32_t *err, cudaStream_t s) {
     const uint32_t N = n * r;
     size_t lc = ((size_t)1 << 28) / N;  // lanes per chunk: about 1 GiB of scratch
@@ -237,15 +273,9 @@ int encode_lanes(const CodeDev &d, uint32_t n, uint32_t r, const int8_t *X, size
     }
     for (uint32_t l0 = 0; status == PVMVMD_OK && l0 < L; l0 += (uint32_t)lc) {
         const uint32_t nl = (uint32_t)((L - l0) < lc ? (L - l0) : lc);
-        cudaError_t e = cudaMemsetAsync(flags, 0, encode_scan_flag_words(N, nl) * 4, s);
-        if (e == cudaSuccess)  // S = A^T V1 Pi1^T R^T X
-            e = launch_encode_scan(X + l0, true, ldx, d.pi1, r, d.v1, N, nl, S, nl, agg, incl,
-                                   flags, err, s);
-        if (e == cudaSuccess) e = cudaMemsetAsync(flags, 0, encode_scan_flag_words(N, nl) * 4, s);
-        if (e == cudaSuccess)  // Y = A^T V2 Pi2^T S
-            e = launch_encode_scan(S, false, nl, d.pi2, 1, d.v2, N, nl, Y + l0, ldy, agg, incl,
-                                   flags, err, s);
-        if (e != cudaSuccess) status = PVMVMD_E_CUDA;
+        const void *Xl = x_is_i8 ? static_cast<const void *>(static_cast<const int8_t *>(X) + l0)
+                                 : static_cast<const void *>(static_cast<const uint32_t *>(X) + l0);
+        status = encode_lanes_into(d, n, r, Xl, x_is_i8, ldx, nl, Y + l0, ldy, S, agg, incl, flags, err, s);
     }
     if (cudaStreamSynchronize(s) != cudaSuccess) status = PVMVMD_E_CUDA;
     cudaFree(S);
@@ -399,11 +429,11 @@ int pvmvmd_preprocess(const int8_t *W_dev, int m, int K, const pvmvmd_params *pa
         cudaFree(MT);
         return fail(PVMVMD_E_CUDA);
     }
-    st = encode_lanes(c->gx, K, c->rate, MT, (size_t)m, m, c->PT, (size_t)m, err, s);
+    st = encode_lanes(c->gx, K, c->rate, MT, true, (size_t)m, m, c->PT, (size_t)m, err, s);
     cudaFree(MT);
     if (st) return fail(st);
     // Q = G_y^T M: the K columns of M are the lanes.
-    st = encode_lanes(c->gy, m, c->rate, W_dev, (size_t)K, K, c->Q, (size_t)K, err, s);
+    st = encode_lanes(c->gy, m, c->rate, W_dev, true, (size_t)K, K, c->Q, (size_t)K, err, s);
     if (st) return fail(st);
     if ((st = read_and_clear_error())) return fail(st);
     *out = c;
@@ -638,3 +668,149 @@ int pvmvmd_ctx_info(const pvmvmd_ctx *ctx, pvmvmd_ctx_view *v) {
 }
 
 }  // extern "C"
+
+
+// ---------------------------------------------------------------------------
+// Batch verification, Protocol 2
+// ---------------------------------------------------------------------------
+void pvmvmd_bv_destroy(pvmvmd_bv_ctx *ctx) {
+    if (!ctx) return;
+    int cur = 0;
+    cudaGetDevice(&cur);
+    cudaSetDevice(ctx->device);
+    for (void *p : ctx->owned) cudaFree(p);
+    cudaSetDevice(cur);
+    delete ctx;
+}
+
+int pvmvmd_bv_preprocess(const int8_t *W_dev, int B, int m, int n, const pvmvmd_bv_params *params,
+                         const pvmvmd_key *key, void *stream, pvmvmd_bv_ctx **out) {
+    using namespace pv;
+    if (!out) return PVMVMD_E_ARG;
+    *out = nullptr;
+    if (!W_dev || !key) return PVMVMD_E_ARG;
+    if (B < 1 || m < 1 || n < 1) return PVMVMD_E_SHAPE;
+    const int rate = params && params->rate ? params->rate : 8;
+    const long long N = (long long)rate * m, N2 = (long long)rate * B * n;
+    // the device sampler holds a bitmap of N bits in shared memory
+    if (rate < 2 || N > 8LL * PVMVMD_MAX_K || N2 > 8LL * PVMVMD_MAX_K) return PVMVMD_E_SHAPE;
+    const int t = params && params->t ? params->t : 31, ell = params && params->ell ? params->ell : 2;
+    const int t2 = params && params->t2 ? params->t2 : 31, ell2 = params && params->ell2 ? params->ell2 : 2;
+    if (t < 1 || ell < 1 || t2 < 1 || ell2 < 1 || t > N || t2 > N2) return PVMVMD_E_PARAM;
+    int st = check_device();
+    if (st) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    uint32_t *err = error_word();
+    if (!err) return PVMVMD_E_CUDA;
+    pvmvmd_bv_ctx *c = new (std::nothrow) pvmvmd_bv_ctx();
+    if (!c) return PVMVMD_E_NOMEM;
+    cudaGetDevice(&c->device);
+    c->B = B; c->m = m; c->n = n; c->rate = rate; c->N = (int)N; c->N2 = (int)N2;
+    c->t = t; c->ell = ell; c->t2 = t2; c->ell2 = ell2;
+    auto fail = [&](int code) {
+        pvmvmd_bv_destroy(c);
+        return code;
+    };
+    const uint32_t Bn = (uint32_t)B * n;
+    if ((st = upload_code(c, c->g, *key, 3, (uint32_t)N, s))) return fail(st);
+    if ((st = upload_code(c, c->g2, *key, 4, (uint32_t)N2, s))) return fail(st);
+    const size_t fw = encode_scan_flag_words((uint32_t)N, (uint32_t)B);
+    const size_t vw = encode_scan_value_words((uint32_t)N, (uint32_t)B);
+    if (ctx_alloc(c, &c->Qs, (size_t)N * Bn) != cudaSuccess ||
+        ctx_alloc(c, &c->QauxT, (size_t)N2 * N) != cudaSuccess ||
+        ctx_alloc(c, &c->Yt, (size_t)m * B) != cudaSuccess ||
+        ctx_alloc(c, &c->Z, (size_t)N * B) != cudaSuccess ||
+        ctx_alloc(c, &c->chal2, (size_t)ell2 * 2 * t2) != cudaSuccess ||
+        ctx_alloc(c, &c->R, (size_t)ell2 * Bn) != cudaSuccess ||
+        ctx_alloc(c, &c->F2, (size_t)ell2 * N2) != cudaSuccess ||
+        ctx_alloc(c, &c->eS, (size_t)N * B) != cudaSuccess || ctx_alloc(c, &c->eagg, vw) != cudaSuccess ||
+        ctx_alloc(c, &c->eincl, vw) != cudaSuccess || ctx_alloc(c, &c->eflags, fw) != cudaSuccess ||
+        ctx_alloc(c, &c->status, scan_status_words((uint32_t)N2, (uint32_t)ell2)) != cudaSuccess)
+        return fail(PVMVMD_E_NOMEM);
+    // Q_b = G^T M_b into the column block b n of Qs (the lanes are M_b's columns)
+    for (int b = 0; b < B; ++b) {
+        st = encode_lanes(c->g, (uint32_t)m, (uint32_t)rate, W_dev + (size_t)b * m * n, true, (size_t)n,
+                          (uint32_t)n, c->Qs + (size_t)b * n, (size_t)Bn, err, s);
+        if (st) return fail(st);
+    }
+    // Qaux = Qt^T G': row i is G'^T applied to row i of Qs; encode with the
+    // N rows of Qs as lanes, so Qs is transposed first (Qt, B n x N)
+    uint32_t *Qt = nullptr;
+    if (dev_alloc(&Qt, (size_t)Bn * N) != cudaSuccess) return fail(PVMVMD_E_NOMEM);
+    if (launch_transpose_u32(c->Qs, (int)N, (int)Bn, Qt, s) != cudaSuccess) {
+        cudaFree(Qt);
+        return fail(PVMVMD_E_CUDA);
+    }
+    st = encode_lanes(c->g2, Bn, (uint32_t)rate, Qt, false, (size_t)N, (uint32_t)N, c->QauxT, (size_t)N, err, s);
+    cudaFree(Qt);
+    if (st) return fail(st);
+    if ((st = read_and_clear_error())) return fail(st);
+    *out = c;
+    return PVMVMD_OK;
+}
+
+int pvmvmd_bv_challenge(pvmvmd_bv_ctx *ctx, const pvmvmd_key *key, uint32_t *chal_dev, void *stream) {
+    using namespace pv;
+    if (!ctx || !key || !chal_dev) return PVMVMD_E_ARG;
+    PV_CUDA(launch_sample_sparse(*key, kTagBvPrimary, 0, (uint32_t)ctx->N, (uint32_t)ctx->t,
+                                 (uint32_t)ctx->ell, chal_dev, nullptr, 0, static_cast<cudaStream_t>(stream)));
+    return PVMVMD_OK;
+}
+
+int pvmvmd_bv_server_project(const pvmvmd_bv_ctx *ctx, const uint32_t *chal_dev, uint32_t *u_dev,
+                             void *stream) {
+    using namespace pv;
+    if (!ctx || !chal_dev || !u_dev) return PVMVMD_E_ARG;
+    PV_CUDA(launch_verify_u(ctx->Qs, ctx->B * ctx->n, chal_dev, (uint32_t)ctx->t, (uint32_t)ctx->ell, u_dev,
+                            static_cast<cudaStream_t>(stream)));
+    return PVMVMD_OK;
+}
+
+int pvmvmd_bv_check(pvmvmd_bv_ctx *ctx, const uint32_t *X_dev, const uint32_t *Y_dev, const uint32_t *chal_dev,
+                    const uint32_t *u_dev, const pvmvmd_key *key2, int32_t *accept_dev, void *stream) {
+    using namespace pv;
+    if (!ctx || !X_dev || !Y_dev || !chal_dev || !u_dev || !key2 || !accept_dev) return PVMVMD_E_ARG;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    uint32_t *err = error_word();
+    if (!err) return PVMVMD_E_CUDA;
+    const uint32_t Bn = (uint32_t)ctx->B * ctx->n;
+    // z_b = G^T y_b (the B outputs as lanes)
+    PV_CUDA(launch_transpose_u32(Y_dev, ctx->B, ctx->m, ctx->Yt, s));
+    int st = encode_lanes_into(ctx->g, (uint32_t)ctx->m, (uint32_t)ctx->rate, ctx->Yt, false, (size_t)ctx->B,
+                               (uint32_t)ctx->B, ctx->Z, (size_t)ctx->B, ctx->eS, ctx->eagg, ctx->eincl,
+                               ctx->eflags, err, s);
+    if (st) return st;
+    // secondary challenges, drawn after the responses, and r^(j) = G' e'^(j)
+    const CodeDev &d = ctx->g2;
+    int C;
+    uint32_t slice;
+    size_t smem;
+    if (syndrome_fused_plan((uint32_t)ctx->N2, (uint32_t)ctx->t2, &C, &slice, &smem)) {
+        PV_CUDA(launch_syndrome_fused(*key2, kTagBvSecondary, 0, (uint32_t)ctx->N2, (uint32_t)ctx->t2,
+                                      (uint32_t)ctx->ell2, d.pi2inv, d.v2p, d.v1, d.pi1inv, d.pi2, d.v2m,
+                                      d.v1pm, Bn, (uint32_t)ctx->rate, ctx->chal2, nullptr, ctx->R, s));
+    } else {
+        PV_CUDA(launch_sample_sparse(*key2, kTagBvSecondary, 0, (uint32_t)ctx->N2, (uint32_t)ctx->t2,
+                                     (uint32_t)ctx->ell2, ctx->chal2, ctx->status,
+                                     scan_status_words((uint32_t)ctx->N2, (uint32_t)ctx->ell2), s));
+        PV_CUDA(launch_syndrome_scan(d.pi2inv, d.v2p, d.v1, (uint32_t)ctx->N2, ctx->chal2, (uint32_t)ctx->t2,
+                                     (uint32_t)ctx->ell2, ctx->F2, ctx->status, err, s));
+        PV_CUDA(launch_syndrome_gather(d.pi1inv, Bn, (uint32_t)ctx->rate, ctx->F2, (uint32_t)ctx->N2, nullptr,
+                                       ctx->R, (uint32_t)ctx->ell2, s));
+    }
+    PV_CUDA(launch_bv_checks(ctx->QauxT, ctx->N, (int)Bn, ctx->n, ctx->B, chal_dev, (uint32_t)ctx->t,
+                             (uint32_t)ctx->ell, ctx->chal2, (uint32_t)ctx->t2, (uint32_t)ctx->ell2, u_dev,
+                             ctx->R, X_dev, ctx->Z, accept_dev, s));
+    return PVMVMD_OK;
+}
+
+int pvmvmd_bv_info(const pvmvmd_bv_ctx *ctx, pvmvmd_bv_view *v) {
+    if (!ctx || !v) return PVMVMD_E_ARG;
+    v->B = ctx->B; v->m = ctx->m; v->n = ctx->n; v->rate = ctx->rate; v->N = ctx->N; v->N2 = ctx->N2;
+    v->t = ctx->t; v->ell = ctx->ell; v->t2 = ctx->t2; v->ell2 = ctx->ell2;
+    v->Qs = ctx->Qs;
+    v->QauxT = ctx->QauxT;
+    v->chal2 = ctx->chal2;
+    return PVMVMD_OK;
+}
+

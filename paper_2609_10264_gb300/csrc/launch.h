@@ -141,4 +141,16 @@ cudaError_t launch_field_add(const uint32_t *a, const uint32_t *b, size_t n, uin
 cudaError_t launch_output_mask(const uint32_t *PT, int m, const uint32_t *st, uint32_t t_x, int B,
                                uint32_t *out, cudaStream_t s);
 
+// out (C x R) = in (R x C) transposed, uint32.
+cudaError_t launch_transpose_u32(const uint32_t *in, int R, int C, uint32_t *out, cudaStream_t s);
+
+// Protocol 2's client checks; accept = 1 iff every check holds.  QauxT
+// [N'][N], chal [ell][2t] and chal2 [ell'][2t'] (ascending support, then
+// values), u [ell][Bn] the server's projections, R [ell'][Bn] = G' e',
+// X [B][n] the claims' inputs, Z [N][B] = G^T y_b.
+cudaError_t launch_bv_checks(const uint32_t *QauxT, int N, int Bn, int n, int B, const uint32_t *chal,
+                             uint32_t t, uint32_t ell, const uint32_t *chal2, uint32_t t2, uint32_t ell2,
+                             const uint32_t *u, const uint32_t *R, const uint32_t *X, const uint32_t *Z,
+                             int32_t *accept, cudaStream_t s);
+
 }  // namespace pv

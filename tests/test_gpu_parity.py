@@ -197,6 +197,51 @@ def test_boost_mode_matches_standard_mode(pv, wl, m, K, B):
     ctx.destroy()
 
 
+@pytest.mark.parametrize("B,m,n", [(3, 40, 30), (4, 96, 64), (2, 700, 600)])
+def test_batch_verification_protocol2(pv, wl, B, m, n):
+    """Protocol 2 on the GPU against the oracle: the preprocessed Qs and
+    Qaux, the server projection, the secondary challenges, and the verdicts
+    on honest claims, a wrong output and a wrong projection."""
+    import torch
+    rng = np.random.default_rng(B * 1000 + m + n)
+    Ws = rng.integers(-128, 128, size=(B, m, n), dtype=np.int8)
+    xs = rng.integers(0, Q, size=(B, n)).astype(np.uint32)
+    ys = np.stack([oracle.server_mvm(Ws[b], xs[b]) for b in range(B)])
+    ctx = pv.pvmvmd_bv_preprocess(to_dev(Ws), key=51)
+    bp = oracle.BatchParams(list(Ws), oracle.key_from_seed(51))
+    assert (ctx.N, ctx.N2, ctx.t, ctx.ell, ctx.t2, ctx.ell2) == (bp.N, bp.N2, bp.t, bp.ell, bp.t2, bp.ell2)
+    Qs = pv.as_u32(pv.device_view(ctx.Qs, ctx.N * B * n).view(ctx.N, B * n))
+    assert np.array_equal(Qs, bp.Qt.T)
+    cols = sample_rows(ctx.N2, 16, 3)
+    QauxT = pv.device_view(ctx.QauxT, ctx.N2 * ctx.N).view(ctx.N2, ctx.N)
+    assert np.array_equal(pv.as_u32(QauxT[torch.as_tensor(cols, device=QauxT.device)]), bp.Qaux[:, cols].T)
+    chal = pv.pvmvmd_bv_challenge(ctx, key=52)
+    ch_o = bp.challenges(oracle.key_from_seed(52))
+    ch_h = pv.as_u32(chal)
+    for q, (s_o, v_o) in enumerate(ch_o):
+        assert np.array_equal(ch_h[q], np.concatenate([s_o, v_o]))
+    u = pv.pvmvmd_bv_server_project(ctx, chal)
+    assert np.array_equal(pv.as_u32(u), bp.server_project(ch_o))
+    Xd, Yd = to_dev(xs), to_dev(ys)
+    acc = pv.pvmvmd_bv_check(ctx, Xd, Yd, chal, u, key2=53)
+    assert pv.as_u32(acc).tolist() == [1]
+    assert bp.check(list(xs), list(ys), ch_o, bp.server_project(ch_o), oracle.key_from_seed(53))
+    sec = pv.as_u32(pv.device_view(ctx.chal2, ctx.ell2 * 2 * ctx.t2).view(ctx.ell2, 2 * ctx.t2))
+    for j, (s_o, v_o) in enumerate(bp.secondary(oracle.key_from_seed(53))):
+        assert np.array_equal(sec[j], np.concatenate([s_o, v_o]))
+    # a wrong output, then a wrong projection: rejected by both
+    bad = ys.copy()
+    bad[B - 1, m // 3] = (int(bad[B - 1, m // 3]) + 9) % Q
+    assert pv.as_u32(pv.pvmvmd_bv_check(ctx, Xd, to_dev(bad), chal, u, key2=54)).tolist() == [0]
+    assert not bp.check(list(xs), list(bad), ch_o, bp.server_project(ch_o), oracle.key_from_seed(54))
+    ub = u.clone()
+    tamper(pv, ub, 0, (B * n) // 2, 3)
+    assert pv.as_u32(pv.pvmvmd_bv_check(ctx, Xd, Yd, chal, ub, key2=55)).tolist() == [0]
+    assert not bp.check(list(xs), list(ys), ch_o, pv.as_u32(ub), oracle.key_from_seed(55))
+    assert pv.pvmvmd_device_status() == 0
+    ctx.destroy()
+
+
 def test_server_mvm_extremes(pv):
     """Extreme weights and field values: -128, 127, x = 0, 1, (q-1)/2, (q+1)/2, q-1."""
     rng = np.random.default_rng(1)
