@@ -255,6 +255,25 @@ int pvmvmd_bv_check(pvmvmd_bv_ctx *ctx, const uint32_t *X_dev, const uint32_t *Y
 int pvmvmd_bv_info(const pvmvmd_bv_ctx *ctx, pvmvmd_bv_view *view);
 void pvmvmd_bv_destroy(pvmvmd_bv_ctx *ctx);
 
+/* 16-bit weights.  Sec. 7.2 quantises FP8 weights as round(2^8 W), which can
+ * exceed int8.  A 16-bit M (int16 m x K row-major, every entry in
+ * [-32768, 32639]; others give unspecified results) is split once into two
+ * int8 planes M = 256 M_hi + M_lo (M_lo the low byte read as signed), and
+ * the server's product runs on both planes:
+ *   pvmvmd_weights_split_i16   W -> Whi, Wlo (int8 m x K each);
+ *   pvmvmd_server_mvm_i16      Yhat = Mhi Xhat * 256 + Mlo Xhat over F_q,
+ *                              with Ytmp_dev (B x m) the caller's scratch;
+ *   pvmvmd_preprocess_i16      as pvmvmd_preprocess for the 16-bit M
+ *                              (encode, decode and verify then run
+ *                              unchanged on the returned context). */
+int pvmvmd_weights_split_i16(const int16_t *W_dev, int m, int K, int8_t *Whi_dev, int8_t *Wlo_dev,
+                             void *stream);
+int pvmvmd_server_mvm_i16(const int8_t *Whi_dev, const int8_t *Wlo_dev, int m, int K,
+                          const uint32_t *Xhat_dev, int B, uint32_t *Yhat_dev, uint32_t *Ytmp_dev,
+                          void *stream);
+int pvmvmd_preprocess_i16(const int16_t *W_dev, int m, int K, const pvmvmd_params *params,
+                          const pvmvmd_key *key, void *stream, pvmvmd_ctx **out);
+
 /* Synchronise `stream`, then read and clear the library's device error word:
  * PVMVMD_E_DEVICE_TIMEOUT if any kernel gave up a bounded wait since the last
  * call, else PVMVMD_OK (or PVMVMD_E_CUDA if synchronisation failed). */

@@ -99,6 +99,10 @@ SIGNATURES = {
     "pvmvmd_bv_check": (_i, [_vp, _vp, _vp, _vp, _vp, ctypes.POINTER(pvmvmd_key), _vp, _vp]),
     "pvmvmd_bv_info": (_i, [_vp, ctypes.POINTER(pvmvmd_bv_view)]),
     "pvmvmd_bv_destroy": (None, [_vp]),
+    "pvmvmd_weights_split_i16": (_i, [_vp, _i, _i, _vp, _vp, _vp]),
+    "pvmvmd_server_mvm_i16": (_i, [_vp, _vp, _i, _i, _vp, _i, _vp, _vp, _vp]),
+    "pvmvmd_preprocess_i16": (_i, [_vp, _i, _i, ctypes.POINTER(pvmvmd_params), ctypes.POINTER(pvmvmd_key), _vp,
+                                   ctypes.POINTER(_vp)]),
     "pvmvmd_device_status": (_i, [_vp]),
     "pvmvmd_ctx_info": (_i, [_vp, ctypes.POINTER(pvmvmd_ctx_view)]),
     "pvmvmd_destroy": (None, [_vp]),
@@ -238,6 +242,50 @@ def pvmvmd_preprocess(W, key, params: pvmvmd_params | None = None, stream=None) 
                                   ctypes.byref(k), _stream_ptr(stream), ctypes.byref(out)),
            "pvmvmd_preprocess")
     return Ctx(out.value, m, K)
+
+
+def pvmvmd_preprocess_i16(W, key, params: pvmvmd_params | None = None, stream=None) -> Ctx:
+    """As pvmvmd_preprocess for a 16-bit M (int16 m x K, entries in [-32768, 32639])."""
+    import torch
+    if W.dim() != 2:
+        raise ValueError("W must be m x K")
+    m, K = W.shape
+    out = ctypes.c_void_p()
+    _check(_lib.pvmvmd_preprocess_i16(_dev_ptr(W, "W", (torch.int16,)), m, K,
+                                      ctypes.byref(params) if params is not None else None,
+                                      ctypes.byref(make_key(key)), _stream_ptr(stream), ctypes.byref(out)),
+           "pvmvmd_preprocess_i16")
+    return Ctx(out.value, m, K)
+
+
+def pvmvmd_weights_split_i16(W, stream=None):
+    """16-bit M -> (M_hi, M_lo) int8 planes with M = 256 M_hi + M_lo."""
+    import torch
+    m, K = W.shape
+    hi = torch.empty((m, K), dtype=torch.int8, device=W.device)
+    lo = torch.empty((m, K), dtype=torch.int8, device=W.device)
+    _check(_lib.pvmvmd_weights_split_i16(_dev_ptr(W, "W", (torch.int16,)), m, K, _dev_ptr(hi, "hi", (torch.int8,)),
+                                         _dev_ptr(lo, "lo", (torch.int8,)), _stream_ptr(stream)),
+           "pvmvmd_weights_split_i16")
+    return hi, lo
+
+
+def pvmvmd_server_mvm_i16(Whi, Wlo, Xhat, Yhat=None, Ytmp=None, stream=None):
+    """Y_hat = (256 M_hi + M_lo) X_hat over F_q from the two int8 planes."""
+    import torch
+    m, K = Whi.shape
+    B = _batch(Xhat, K, "Xhat")
+    shape = (m,) if Xhat.dim() == 1 else (B, m)
+    if Yhat is None:
+        Yhat = _new_u32(shape, Xhat)
+    if Ytmp is None:
+        Ytmp = _new_u32(shape, Xhat)
+    _check(_lib.pvmvmd_server_mvm_i16(_dev_ptr(Whi, "Whi", (torch.int8,)), _dev_ptr(Wlo, "Wlo", (torch.int8,)), m, K,
+                                      _dev_ptr(Xhat, "Xhat", _u32_types()), B,
+                                      _dev_ptr(Yhat, "Yhat", _u32_types(), B * m),
+                                      _dev_ptr(Ytmp, "Ytmp", _u32_types(), B * m), _stream_ptr(stream)),
+           "pvmvmd_server_mvm_i16")
+    return Yhat
 
 
 def pvmvmd_ctx_info(ctx: Ctx) -> pvmvmd_ctx_view:

@@ -372,8 +372,27 @@ void pvmvmd_destroy(pvmvmd_ctx *ctx) {
     delete ctx;
 }
 
+namespace pv {
+namespace {
+int preprocess_impl(const void *W_dev, bool w16, int m, int K, const pvmvmd_params *params,
+                    const pvmvmd_key *key, void *stream, pvmvmd_ctx **out);
+}  // namespace
+}  // namespace pv
+
 int pvmvmd_preprocess(const int8_t *W_dev, int m, int K, const pvmvmd_params *params,
                       const pvmvmd_key *key, void *stream, pvmvmd_ctx **out) {
+    return pv::preprocess_impl(W_dev, false, m, K, params, key, stream, out);
+}
+
+int pvmvmd_preprocess_i16(const int16_t *W_dev, int m, int K, const pvmvmd_params *params,
+                          const pvmvmd_key *key, void *stream, pvmvmd_ctx **out) {
+    return pv::preprocess_impl(W_dev, true, m, K, params, key, stream, out);
+}
+
+namespace pv {
+namespace {
+int preprocess_impl(const void *W_dev, bool w16, int m, int K, const pvmvmd_params *params,
+                    const pvmvmd_key *key, void *stream, pvmvmd_ctx **out) {
     if (!out) return PVMVMD_E_ARG;
     *out = nullptr;
     if (!W_dev || !key) return PVMVMD_E_ARG;
@@ -422,10 +441,32 @@ int pvmvmd_preprocess(const int8_t *W_dev, int m, int K, const pvmvmd_params *pa
          ctx_alloc(c, &c->laux, lane_aux_words(c->Nx, c->sb)) != cudaSuccess))
         return fail(PVMVMD_E_NOMEM);
 
+    if (w16) {
+        // 16-bit M: lift it to F_q, then encode as uint32 lanes
+        uint32_t *M32 = nullptr, *MT32 = nullptr;
+        if (dev_alloc(&M32, (size_t)m * K) != cudaSuccess || dev_alloc(&MT32, (size_t)m * K) != cudaSuccess) {
+            cudaFree(M32);
+            return fail(PVMVMD_E_NOMEM);
+        }
+        if (launch_lift_i16(static_cast<const int16_t *>(W_dev), (size_t)m * K, M32, s) != cudaSuccess ||
+            launch_transpose_u32(M32, m, K, MT32, s) != cudaSuccess) {
+            cudaFree(M32);
+            cudaFree(MT32);
+            return fail(PVMVMD_E_CUDA);
+        }
+        st = encode_lanes(c->gx, K, c->rate, MT32, false, (size_t)m, m, c->PT, (size_t)m, err, s);
+        if (!st) st = encode_lanes(c->gy, m, c->rate, M32, false, (size_t)K, K, c->Q, (size_t)K, err, s);
+        cudaFree(M32);
+        cudaFree(MT32);
+        if (st) return fail(st);
+        if ((st = read_and_clear_error())) return fail(st);
+        *out = c;
+        return PVMVMD_OK;
+    }
     // P^T = G_x^T M^T: the m rows of M are the lanes, so transpose M first.
     int8_t *MT = nullptr;
     if (dev_alloc(&MT, (size_t)m * K) != cudaSuccess) return fail(PVMVMD_E_NOMEM);
-    if (launch_transpose_i8(W_dev, m, K, MT, s) != cudaSuccess) {
+    if (launch_transpose_i8(static_cast<const int8_t *>(W_dev), m, K, MT, s) != cudaSuccess) {
         cudaFree(MT);
         return fail(PVMVMD_E_CUDA);
     }
@@ -437,6 +478,29 @@ int pvmvmd_preprocess(const int8_t *W_dev, int m, int K, const pvmvmd_params *pa
     if (st) return fail(st);
     if ((st = read_and_clear_error())) return fail(st);
     *out = c;
+    return PVMVMD_OK;
+}
+}  // namespace
+}  // namespace pv
+
+int pvmvmd_weights_split_i16(const int16_t *W_dev, int m, int K, int8_t *Whi_dev, int8_t *Wlo_dev,
+                             void *stream) {
+    using namespace pv;
+    if (!W_dev || !Whi_dev || !Wlo_dev) return PVMVMD_E_ARG;
+    if (m < 1 || K < 1) return PVMVMD_E_SHAPE;
+    PV_CUDA(launch_split_i16(W_dev, (size_t)m * K, Whi_dev, Wlo_dev, static_cast<cudaStream_t>(stream)));
+    return PVMVMD_OK;
+}
+
+int pvmvmd_server_mvm_i16(const int8_t *Whi_dev, const int8_t *Wlo_dev, int m, int K, const uint32_t *Xhat_dev,
+                          int B, uint32_t *Yhat_dev, uint32_t *Ytmp_dev, void *stream) {
+    using namespace pv;
+    if (!Whi_dev || !Wlo_dev || !Ytmp_dev) return PVMVMD_E_ARG;
+    int st = pvmvmd_server_mvm(Whi_dev, m, K, Xhat_dev, B, Yhat_dev, stream);
+    if (st) return st;
+    st = pvmvmd_server_mvm(Wlo_dev, m, K, Xhat_dev, B, Ytmp_dev, stream);
+    if (st) return st;
+    PV_CUDA(launch_combine_256(Yhat_dev, Ytmp_dev, (size_t)B * m, static_cast<cudaStream_t>(stream)));
     return PVMVMD_OK;
 }
 

@@ -153,4 +153,10 @@ cudaError_t launch_bv_checks(const uint32_t *QauxT, int N, int Bn, int n, int B,
                              const uint32_t *u, const uint32_t *R, const uint32_t *X, const uint32_t *Z,
                              int32_t *accept, cudaStream_t s);
 
+// 16-bit weights: W = 256 hi + lo (int8 planes, w in [-32768, 32639]);
+// W lifted to F_q; y = 256 y + ylo over F_q.
+cudaError_t launch_split_i16(const int16_t *W, size_t n, int8_t *hi, int8_t *lo, cudaStream_t s);
+cudaError_t launch_lift_i16(const int16_t *W, size_t n, uint32_t *out, cudaStream_t s);
+cudaError_t launch_combine_256(uint32_t *y, const uint32_t *ylo, size_t n, cudaStream_t s);
+
 }  // namespace pv

@@ -242,6 +242,43 @@ def test_batch_verification_protocol2(pv, wl, B, m, n):
     ctx.destroy()
 
 
+@pytest.mark.parametrize("B", [1, 5, 40])
+def test_sixteen_bit_weights_round_trip(pv, wl, B):
+    """16-bit weights (Sec. 7.2 style, including both ends of the supported
+    range): the split planes recombine to M; P^T and Q equal 256 x the
+    tables of M_hi plus those of M_lo (linearity, each from the oracle); the
+    decrypted output equals the exact integer product W x for every vector."""
+    import torch
+    rng = np.random.default_rng(70 + B)
+    m, K = 300, 1000
+    W = rng.integers(-32768, 32640, size=(m, K)).astype(np.int16)
+    W[0, :5] = [-32768, 32639, -1, 0, 255]
+    x = rng.integers(-8, 9, size=(B, K)).astype(np.int64)       # |W x| < q / 2
+    Wd = torch.from_numpy(W).cuda()
+    hi, lo = pv.pvmvmd_weights_split_i16(Wd)
+    hi_h, lo_h = hi.cpu().numpy(), lo.cpu().numpy()
+    assert np.array_equal(256 * hi_h.astype(np.int64) + lo_h.astype(np.int64), W.astype(np.int64))
+    ctx = pv.pvmvmd_preprocess_i16(Wd, key=71)
+    v = pv.pvmvmd_ctx_info(ctx)
+    ph = oracle.PublicParams(hi_h, oracle.key_from_seed(71))
+    pl = oracle.PublicParams(lo_h, oracle.key_from_seed(71))
+    PT = pv.as_u32(pv.device_view(v.PT, v.N_x * m).view(v.N_x, m)).astype(np.int64)
+    Qm = pv.as_u32(pv.device_view(v.Q, v.N_y * K).view(v.N_y, K)).astype(np.int64)
+    assert np.array_equal(PT, (256 * ph.PT.astype(np.int64) + pl.PT) % Q)
+    assert np.array_equal(Qm, (256 * ph.Q.astype(np.int64) + pl.Q) % Q)
+    Xh, st = pv.pvmvmd_encode(ctx, to_dev(field(x)), key=72)
+    Yh = pv.pvmvmd_server_mvm_i16(hi, lo, Xh if B > 1 else Xh[0])
+    Yh2 = Yh.view(B, m)
+    Y, acc = pv.pvmvmd_decode_verify(ctx, st, Xh, Yh2, challenge_key=73)
+    assert pv.as_u32(acc).tolist() == [1] * B
+    assert np.array_equal(oracle.centered(pv.as_u32(Y)), x @ W.astype(np.int64).T)
+    tamper(pv, Yh2, 0, 7, 1)
+    _, acc2 = pv.pvmvmd_decode_verify(ctx, st, Xh, Yh2, challenge_key=74)
+    assert pv.as_u32(acc2).tolist() == [0] + [1] * (B - 1)
+    assert pv.pvmvmd_device_status() == 0
+    ctx.destroy()
+
+
 def test_server_mvm_extremes(pv):
     """Extreme weights and field values: -128, 127, x = 0, 1, (q-1)/2, (q+1)/2, q-1."""
     rng = np.random.default_rng(1)
