@@ -799,6 +799,54 @@ def run_bv(args):
     return 0
 
 
+def run_encode_shape(args):
+    """Encrypt alone for B vectors of length K (``--shape KxB``): x_hat =
+    x + G_x e_x with fresh sparse masks, timed over --steps calls.  The
+    matrix has 256 rows, so preprocessing and its tables stay small."""
+    import torch
+    rank, world, local = dist_env()
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    import paper_2609_10264_gb300 as pv
+    Q = pv.PVMVMD_Q
+    K, B = (int(v) for v in args.shape.lower().split("x"))
+    gen = torch.Generator(device=device)
+    gen.manual_seed(81)
+    W = torch.randint(-127, 128, (256, K), generator=gen, device=device, dtype=torch.int8)
+    X = torch.randint(0, Q, (B, K), generator=gen, device=device, dtype=torch.int64).to(torch.int32)
+    params = pv.pvmvmd_params()
+    params.scratch_batch = max(B, 1)
+    ctx = pv.pvmvmd_preprocess(W, key=82, params=params)
+    stream = torch.cuda.Stream(device)
+    Xh = torch.empty_like(X)
+    st = torch.empty((B, 2 * ctx.t_x), dtype=torch.int32, device=device)
+    with torch.cuda.stream(stream):
+        for s in range(args.warmup):
+            pv.pvmvmd_encode(ctx, X, 83 + s, Xhat=Xh, st=st, stream=stream)
+    stream.synchronize()
+    pv.pvmvmd_device_status(stream)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        t0.record(stream)
+        for s in range(args.steps):
+            pv.pvmvmd_encode(ctx, X, 1000 + s, Xhat=Xh, st=st, stream=stream)
+        t1.record(stream)
+    stream.synchronize()
+    pv.pvmvmd_device_status(stream)
+    ms = t0.elapsed_time(t1) / args.steps
+    N = ctx.N_x
+    if rank == 0:
+        print(json.dumps({
+            "metric": "encrypted vectors/s", "value": B / (ms / 1e3), "unit": "vectors/s", "n_gpus": 1,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "u32 (F_q exact)", "data": "synthetic",
+            "config": {"workload": "encode-shape", "K": K, "B": B, "N_x": N, "t_x": ctx.t_x},
+            "gpu_launches": None}), flush=True)
+    ctx.destroy()
+    return 0
+
+
 def run_server_shape(args):
     """The batched server product Y_hat = M X_hat alone on one m x K x B
     shape (``--shape MxKxB``), timed over --steps launches after --warmup.
@@ -873,9 +921,11 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-vectors", type=int, default=150)
     ap.add_argument("--server-mode", choices=["multi", "calls"], default="multi")
-    ap.add_argument("--workload", choices=["batch1-4096", "server-shape", "token8b-b1", "bv-b8-1024"] + sorted(BATCHED),
+    ap.add_argument("--workload", choices=["batch1-4096", "server-shape", "encode-shape", "token8b-b1", "bv-b8-1024"]
+                    + sorted(BATCHED),
                     default="batch1-4096")
-    ap.add_argument("--shape", default="4096x4096x64", help="m x K x B for --workload server-shape")
+    ap.add_argument("--shape", default="4096x4096x64",
+                    help="m x K x B for --workload server-shape, K x B for --workload encode-shape")
     ap.add_argument("--server-streams", type=int, default=2)
     ap.add_argument("--mode", choices=["standard", "boost", "pipelined"], default="standard",
                     help="client mode of the batch-1 workload (Sec. 7.2): standard (masks drawn during "
@@ -894,6 +944,8 @@ def main(argv=None):
         return run_token(args)
     if args.workload == "bv-b8-1024":
         return run_bv(args)
+    if args.workload == "encode-shape":
+        return run_encode_shape(args)
     return run_ours(args)
 
 

@@ -811,7 +811,7 @@ constexpr int kLaneCta = 256;      // threads per lane CTA
 constexpr int kLaneQuadsMax = 64;  // lane quads per CTA (256 lanes)
 constexpr int kExpandSpan = 32;    // positions per expand thread (a multiple of 4)
 constexpr int kGatherJ = 16;       // outputs per gather CTA
-constexpr int kCarryChunks = 128;  // tile chunks per lane quad in the carry kernel
+constexpr int kCarryThreads = 1024;  // tile chunks per lane quad in the carry kernel
 
 __host__ __device__ inline uint32_t lane_pad(uint32_t L) { return (L + 3) & ~3u; }
 __host__ __device__ inline uint32_t lane_cols(uint32_t L) {  // lane quads per CTA
@@ -958,34 +958,54 @@ __global__ void __launch_bounds__(kLaneCta) k_lane_tile_sum(const uint4 *__restr
     agg[(size_t)tau * Lq + g] = sum;
 }
 
-// carry[tau][b] = sum_{tau' > tau} agg[tau'][b]: a CTA takes 8 lane quads;
-// thread (chunk c, quad) sums its chunk of tiles, the chunk sums are
-// combined in shared memory, then each thread writes its chunk's carries
+// carry[tau][b] = sum_{tau' > tau} agg[tau'][b]: one CTA per lane quad;
+// thread c sums its chunk of consecutive tiles, a block-wide suffix scan of
+// the chunk sums (warp shuffles, then the 32 warp totals) gives each chunk
+// the sum of the tiles after it, and the thread writes its chunk's carries
 // walking down.
-__global__ void __launch_bounds__(8 * kCarryChunks) k_lane_carry(const uint4 *__restrict__ agg,
-                                                                uint32_t ntiles, uint32_t Lq,
-                                                                uint4 *__restrict__ carry) {
-    __shared__ uint4 part[kCarryChunks][8];
-    const uint32_t l = threadIdx.x & 7, c = threadIdx.x >> 3;
-    const uint32_t g = blockIdx.x * 8 + l;
-    const uint32_t per = (ntiles + kCarryChunks - 1) / kCarryChunks;
+__device__ __forceinline__ uint4 shfl_down4(uint4 v, int o) {
+    return make_uint4(__shfl_down_sync(kFull, v.x, o), __shfl_down_sync(kFull, v.y, o),
+                      __shfl_down_sync(kFull, v.z, o), __shfl_down_sync(kFull, v.w, o));
+}
+__device__ __forceinline__ uint4 fsub4(uint4 a, uint4 b) {
+    return make_uint4(fsub(a.x, b.x), fsub(a.y, b.y), fsub(a.z, b.z), fsub(a.w, b.w));
+}
+__global__ void __launch_bounds__(kCarryThreads) k_lane_carry(const uint4 *__restrict__ agg, uint32_t ntiles,
+                                                             uint32_t Lq, uint4 *__restrict__ carry) {
+    __shared__ uint4 wsum[kCarryThreads / 32];
+    const uint32_t g = blockIdx.x, c = threadIdx.x, lane = c & 31, warp = c >> 5;
+    const uint32_t per = (ntiles + kCarryThreads - 1) / kCarryThreads;
     const uint32_t t0 = min(ntiles, c * per), t1 = min(ntiles, t0 + per);
     uint4 sum = make_uint4(0u, 0u, 0u, 0u);
-    if (g < Lq) {
-        for (uint32_t tau = t0; tau < t1; tau += 8) {
-            uint4 v[8];
+    for (uint32_t tau = t0; tau < t1; tau += 8) {
+        uint4 v[8];
 #pragma unroll
-            for (int u = 0; u < 8; ++u)
-                v[u] = tau + u < t1 ? agg[(size_t)(tau + u) * Lq + g] : make_uint4(0u, 0u, 0u, 0u);
+        for (int u = 0; u < 8; ++u)
+            v[u] = tau + u < t1 ? agg[(size_t)(tau + u) * Lq + g] : make_uint4(0u, 0u, 0u, 0u);
 #pragma unroll
-            for (int u = 0; u < 8; ++u) sum = fadd4(sum, v[u]);
-        }
+        for (int u = 0; u < 8; ++u) sum = fadd4(sum, v[u]);
     }
-    part[c][l] = sum;
+    uint4 incl = sum;  // suffix within the warp: chunks lane .. 31
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const uint4 y = shfl_down4(incl, o);
+        if (lane + o < 32) incl = fadd4(incl, y);
+    }
+    if (lane == 0) wsum[warp] = incl;
     __syncthreads();
-    uint4 run = make_uint4(0u, 0u, 0u, 0u);  // sum over the chunks after this one
-    for (uint32_t cc = c + 1; cc < (uint32_t)kCarryChunks; ++cc) run = fadd4(run, part[cc][l]);
-    if (g >= Lq) return;
+    if (warp == 0) {  // suffix over the warp totals
+        const uint4 wv = wsum[lane];
+        uint4 wi = wv;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint4 y = shfl_down4(wi, o);
+            if (lane + o < 32) wi = fadd4(wi, y);
+        }
+        __syncwarp();
+        wsum[lane] = fsub4(wi, wv);  // totals of the warps after this one
+    }
+    __syncthreads();
+    uint4 run = fadd4(fsub4(incl, sum), wsum[warp]);  // sum over the chunks after this one
     for (uint32_t hi = t1; hi > t0;) {  // eight tiles at a time, loads first
         const uint32_t cnt = hi - t0 < 8u ? hi - t0 : 8u;
         uint4 v[8];
@@ -1238,8 +1258,8 @@ cudaError_t launch_lane_syndrome(const pvmvmd_key &key, uint32_t tag, uint64_t i
                                                                                  pi2, v2m, C4);
     k_lane_tile_sum<<<dim3((ntiles + per_cta - 1) / per_cta, gy), kLaneCta, 0, s>>>(
         C4, N, L, reinterpret_cast<uint4 *>(agg));
-    k_lane_carry<<<(Lp / 4 + 7) / 8, 8 * kCarryChunks, 0, s>>>(reinterpret_cast<const uint4 *>(agg), ntiles,
-                                                             Lp / 4, reinterpret_cast<uint4 *>(carry));
+    k_lane_carry<<<Lp / 4, kCarryThreads, 0, s>>>(reinterpret_cast<const uint4 *>(agg), ntiles, Lp / 4,
+                                                   reinterpret_cast<uint4 *>(carry));
     k_lane_scan<<<dim3((ntiles + per_cta - 1) / per_cta, gy), kLaneCta, 0, s>>>(
         C4, N, L, reinterpret_cast<const uint4 *>(carry), v1);
     k_lane_gather<<<dim3((n + kGatherJ - 1) / kGatherJ, gy), kLaneCta, 0, s>>>(C4, pi1inv, r, n, L,
