@@ -185,6 +185,10 @@ struct pvmvmd_ctx {
     unsigned long long *status = nullptr;
     // lane-parallel encode scratch (null when scratch_batch < kLaneMinBatch)
     uint32_t *S = nullptr, *laux = nullptr;
+    // decode: the challenge kernels run on `side`, forked from and joined
+    // back to the caller's stream, while the decrypt streams P^T
+    cudaStream_t side = nullptr;
+    cudaEvent_t fork = nullptr, join = nullptr;
     std::vector<void *> owned;
 };
 
@@ -368,6 +372,9 @@ void pvmvmd_destroy(pvmvmd_ctx *ctx) {
     cudaGetDevice(&cur);
     cudaSetDevice(ctx->device);
     for (void *p : ctx->owned) cudaFree(p);
+    if (ctx->fork) cudaEventDestroy(ctx->fork);
+    if (ctx->join) cudaEventDestroy(ctx->join);
+    if (ctx->side) cudaStreamDestroy(ctx->side);
     cudaSetDevice(cur);
     delete ctx;
 }
@@ -436,6 +443,10 @@ int preprocess_impl(const void *W_dev, bool w16, int m, int K, const pvmvmd_para
         ctx_alloc(c, &c->u, (size_t)c->ell * K) != cudaSuccess ||
         ctx_alloc(c, &c->status, statw) != cudaSuccess)
         return fail(PVMVMD_E_NOMEM);
+    if (cudaStreamCreateWithFlags(&c->side, cudaStreamNonBlocking) != cudaSuccess ||
+        cudaEventCreateWithFlags(&c->fork, cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&c->join, cudaEventDisableTiming) != cudaSuccess)
+        return fail(PVMVMD_E_CUDA);
     if (c->sb >= kLaneMinBatch &&
         (ctx_alloc(c, &c->S, (size_t)c->sb * (c->t_x + 1)) != cudaSuccess ||
          ctx_alloc(c, &c->laux, lane_aux_words(c->Nx, c->sb)) != cudaSuccess))
@@ -644,8 +655,12 @@ int pvmvmd_server_mvm_multi(const pvmvmd_mvm_job *jobs, int count, void *stream)
 
 namespace pv {
 namespace {
-// Challenges, u and g, then decrypt + verify: Y = Yhat - P e_x from st, or
-// Y = Yhat - mask_out when mask_out is given (boost mode).
+// Challenges (u and g), decrypt and verify: Y = Yhat - P e_x from st, or
+// Y = Yhat - mask_out when mask_out is given (boost mode).  The challenges
+// depend on the key alone, so they run on the context's side stream while
+// the decrypt streams P^T on the caller's stream; the check joins both.
+// When Y overwrites Yhat the check must read Yhat first, and the three
+// steps run in order on the caller's stream.
 int decode_verify_batch(pvmvmd_ctx *ctx, const void *st_dev, const uint32_t *mask_out_dev,
                         const uint32_t *Xhat_dev, const uint32_t *Yhat_dev, int B,
                         const pvmvmd_key *challenge_key, uint32_t *Y_dev, int32_t *accept_dev,
@@ -653,6 +668,14 @@ int decode_verify_batch(pvmvmd_ctx *ctx, const void *st_dev, const uint32_t *mas
     uint32_t *err = error_word();
     if (!err) return PVMVMD_E_CUDA;
     const CodeDev &d = ctx->gy;
+    const size_t ybytes = (size_t)B * ctx->m * sizeof(uint32_t);
+    const uintptr_t y0 = reinterpret_cast<uintptr_t>(Y_dev), h0 = reinterpret_cast<uintptr_t>(Yhat_dev);
+    const bool in_place = y0 < h0 + ybytes && h0 < y0 + ybytes;
+    const cudaStream_t cs = in_place ? s : ctx->side;
+    if (!in_place) {
+        PV_CUDA(cudaEventRecord(ctx->fork, s));
+        PV_CUDA(cudaStreamWaitEvent(ctx->side, ctx->fork, 0));
+    }
     // Challenges e_q <- E_{t_y}^{N_y}, shared by the B vectors; g_q = G_y e_q.
     int C;
     uint32_t slice;
@@ -660,20 +683,30 @@ int decode_verify_batch(pvmvmd_ctx *ctx, const void *st_dev, const uint32_t *mas
     if (syndrome_fused_plan(ctx->Ny, ctx->t_y, &C, &slice, &smem)) {
         PV_CUDA(launch_syndrome_fused(*challenge_key, kTagChallenge, 0, ctx->Ny, ctx->t_y,
                                       (uint32_t)ctx->ell, d.pi2inv, d.v2p, d.v1, d.pi1inv, d.pi2,
-                                      d.v2m, d.v1pm, ctx->m, ctx->rate, ctx->chal, nullptr, ctx->g, s));
+                                      d.v2m, d.v1pm, ctx->m, ctx->rate, ctx->chal, nullptr, ctx->g, cs));
     } else {
         PV_CUDA(launch_sample_sparse(*challenge_key, kTagChallenge, 0, ctx->Ny, ctx->t_y, ctx->ell,
-                                     ctx->chal, ctx->status, scan_status_words(ctx->Ny, ctx->ell), s));
+                                     ctx->chal, ctx->status, scan_status_words(ctx->Ny, ctx->ell), cs));
         PV_CUDA(launch_syndrome_scan(d.pi2inv, d.v2p, d.v1, ctx->Ny, ctx->chal, ctx->t_y, ctx->ell,
-                                     ctx->Fy, ctx->status, err, s));
+                                     ctx->Fy, ctx->status, err, cs));
         PV_CUDA(launch_syndrome_gather(d.pi1inv, ctx->m, ctx->rate, ctx->Fy, ctx->Ny, nullptr, ctx->g,
-                                       ctx->ell, s));
+                                       ctx->ell, cs));
     }
     // u_q = e_q^T Q.
-    PV_CUDA(launch_verify_u(ctx->Q, ctx->K, ctx->chal, ctx->t_y, ctx->ell, ctx->u, s));
-    PV_CUDA(launch_decode_verify(ctx->PT, ctx->m, ctx->K, static_cast<const uint32_t *>(st_dev),
-                                 ctx->t_x, Xhat_dev, Yhat_dev, ctx->g, ctx->u, ctx->ell, B, Y_dev,
-                                 accept_dev, s, mask_out_dev));
+    PV_CUDA(launch_verify_u(ctx->Q, ctx->K, ctx->chal, ctx->t_y, ctx->ell, ctx->u, cs));
+    if (in_place) {
+        PV_CUDA(launch_check(Xhat_dev, ctx->K, Yhat_dev, ctx->m, ctx->g, ctx->u, (uint32_t)ctx->ell, B,
+                             accept_dev, s));
+        PV_CUDA(launch_decrypt(ctx->PT, ctx->m, static_cast<const uint32_t *>(st_dev), ctx->t_x, Yhat_dev, B,
+                               Y_dev, s, mask_out_dev));
+        return PVMVMD_OK;
+    }
+    PV_CUDA(launch_decrypt(ctx->PT, ctx->m, static_cast<const uint32_t *>(st_dev), ctx->t_x, Yhat_dev, B,
+                           Y_dev, s, mask_out_dev));
+    PV_CUDA(cudaEventRecord(ctx->join, ctx->side));
+    PV_CUDA(cudaStreamWaitEvent(s, ctx->join, 0));
+    PV_CUDA(launch_check(Xhat_dev, ctx->K, Yhat_dev, ctx->m, ctx->g, ctx->u, (uint32_t)ctx->ell, B,
+                         accept_dev, s));
     return PVMVMD_OK;
 }
 }  // namespace

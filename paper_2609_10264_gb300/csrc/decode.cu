@@ -3,30 +3,23 @@
 //  * k_verify_u         u_q = e_q^T Q for the ell shared challenges
 //                       (sum of t_y rows of Q, cost (2t-1)n per repetition,
 //                       the e^T Q row of the cost table in Sec. 5.3).
-//  * k_decode_verify    one thread-block cluster per vector b:
-//                         Y_b = y_hat_b - P e_x,b   (t_x rows of P^T)
-//                         L_q = u_q . x_hat_b,  R_q = g_q . y_hat_b
-//                       where g_q = G_y e_q, so that
-//                       R_q = e_q^T (G_y^T y_hat_b) by transposition;
-//                       the CTAs of the cluster reduce their partial dot
-//                       products through distributed shared memory and
-//                       rank 0 writes accept_b = AND_q (L_q == R_q).
-//                       In boost mode (Sec. 7.2) P e_x,b was prepared ahead
-//                       and is read instead of the t_x rows of P^T.
+//  * k_decrypt          Y_b = y_hat_b - P e_x,b (t_x rows of P^T), many
+//                       short CTAs: 256 columns of one vector each, the
+//                       rows split over four groups; in boost mode
+//                       (Sec. 7.2) P e_x,b was prepared ahead and is read
+//                       instead of the t_x rows of P^T.
+//  * k_check            accept_b = AND_q (L_q == R_q), L_q = u_q . x_hat_b,
+//                       R_q = g_q . y_hat_b with g_q = G_y e_q, so that
+//                       R_q = e_q^T (G_y^T y_hat_b) by transposition.
 //  * k_output_mask      the output masks P e_x,b alone (boost mode's
 //                       offline step).
-#include <cooperative_groups.h>
-
 #include "common.cuh"
 #include "launch.h"
-
-namespace cg = cooperative_groups;
 
 namespace pv {
 namespace {
 
 constexpr int kDecThreads = 256;
-constexpr int kMaxEll = 16;
 
 __device__ __forceinline__ uint4 ldg4(const uint32_t *p) {
     return __ldg(reinterpret_cast<const uint4 *>(p));
@@ -133,117 +126,120 @@ __device__ __forceinline__ void pe_cols(const uint32_t *__restrict__ PT, int m, 
     pe[3] = fred(a3);
 }
 
-template <bool kBoost>
-__global__ void __launch_bounds__(kDecThreads) k_decode_verify(
-    const uint32_t *__restrict__ PT, int m, int K, const uint32_t *__restrict__ st, uint32_t t_x,
-    const uint32_t *__restrict__ Xhat, const uint32_t *Yhat, const uint32_t *__restrict__ g,
-    const uint32_t *__restrict__ u, uint32_t ell, uint32_t *Y, int32_t *__restrict__ accept,
-    bool vec, const uint32_t *__restrict__ mask) {
-    cg::cluster_group cluster = cg::this_cluster();
-    extern __shared__ uint32_t sm[];  // support[t_x], values[t_x]
-    __shared__ uint32_t s_part[2 * kMaxEll];
-    __shared__ uint32_t s_warp[kDecThreads / 32][2 * kMaxEll];
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const uint32_t rank = cluster.block_rank();
-    const uint32_t C = cluster.num_blocks();
-    const size_t b = blockIdx.y;
+// ---------------------------------------------------------------------------
+// Decrypt: Y_b = y_hat_b - P e_x,b.  A CTA owns 256 columns of one vector
+// (64 column threads x 4 columns) and splits the t_x rows of P^T over
+// kDecGroups row groups, so each thread streams about t_x / 4 row segments
+// (a few rounds of 8 loads in flight) and the grid holds many short CTAs
+// whatever m and B are.  The groups' partial sums meet in shared memory.
+// In boost mode (Sec. 7.2) P e_x,b was prepared ahead: Y_b = y_hat_b - mask_b.
+// ---------------------------------------------------------------------------
+constexpr int kDecGroups = 4;
+constexpr int kDecColThreads = kDecThreads / kDecGroups;  // 64
+constexpr int kDecCols = 4 * kDecColThreads;              // 256 columns per CTA
 
-    // Inputs of this kernel (P^T, st, x_hat, y_hat) were written before the
-    // challenge kernels that precede it in the stream; g and u come from
-    // those kernels, so they are read only after griddepcontrol.wait.
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+template <bool kBoost>
+__global__ void __launch_bounds__(kDecThreads) k_decrypt(const uint32_t *__restrict__ PT, int m,
+                                                        const uint32_t *__restrict__ st, uint32_t t_x,
+                                                        const uint32_t *Yhat, uint32_t *Y,
+                                                        const uint32_t *__restrict__ mask, bool vec) {
+    extern __shared__ uint32_t sm[];  // support[t_x], values[t_x]
+    __shared__ uint4 s_part[kDecGroups - 1][kDecColThreads];
+    const int tid = threadIdx.x;
+    const size_t b = blockIdx.y;
+    const int grp = tid / kDecColThreads, ct = tid % kDecColThreads;
+    // boost mode: no rows to split, every thread owns 4 of 1024 columns
+    const int i = kBoost ? ((int)blockIdx.x * kDecThreads + tid) * 4 : (int)blockIdx.x * kDecCols + ct * 4;
+    uint32_t pe[4] = {0u, 0u, 0u, 0u};
     if (!kBoost) {
         const uint32_t *stb = st + b * 2 * t_x;
         for (uint32_t j = tid; j < 2 * t_x; j += kDecThreads) sm[j] = stb[j];
-    }
-    uint32_t *ystage = sm + 2 * t_x;  // this CTA's y_hat columns (y may alias y_hat)
-    __syncthreads();
-    const uint32_t *supp = sm, *vals = sm + t_x;
-
-    uint64_t racc[kMaxEll], lacc[kMaxEll];
+        __syncthreads();
+        const uint32_t per = (t_x + kDecGroups - 1) / kDecGroups;
+        const uint32_t j0 = min(t_x, (uint32_t)grp * per), j1 = min(t_x, j0 + per);
+        if (i < m && j0 < j1) pe_cols(PT, m, sm + j0, sm + t_x + j0, j1 - j0, i, m, vec, pe);
+        if (grp > 0) s_part[grp - 1][ct] = make_uint4(pe[0], pe[1], pe[2], pe[3]);
+        __syncthreads();
+        if (grp > 0) return;
 #pragma unroll
-    for (int q = 0; q < kMaxEll; ++q) racc[q] = lacc[q] = 0;
-
-    // ---- decrypt and the y_hat side of the check over this CTA's columns
-    const int chunk = (((m + (int)C - 1) / (int)C) + 3) & ~3;
-    const int c0 = (int)rank * chunk;
-    const int c1 = min(m, c0 + chunk);
+        for (int g2 = 0; g2 < kDecGroups - 1; ++g2) {
+            const uint4 v = s_part[g2][ct];
+            pe[0] = fadd(pe[0], v.x);
+            pe[1] = fadd(pe[1], v.y);
+            pe[2] = fadd(pe[2], v.z);
+            pe[3] = fadd(pe[3], v.w);
+        }
+    }
+    if (i >= m) return;
     const uint32_t *yh = Yhat + b * m;
     uint32_t *yo = Y + b * m;
-    for (int i = c0 + tid * 4; i < c1; i += kDecThreads * 4) {
-        uint32_t pe[4];
-        if (kBoost) {
+    if (kBoost) {
+        const uint32_t *mk = mask + b * m;
 #pragma unroll
-            for (int q2 = 0; q2 < 4; ++q2) pe[q2] = i + q2 < c1 ? mask[b * m + i + q2] : 0u;
-        } else {
-            pe_cols(PT, m, supp, vals, t_x, i, c1, vec, pe);
-        }
-
+        for (int q2 = 0; q2 < 4; ++q2) pe[q2] = i + q2 < m ? mk[i + q2] : 0u;
+    }
+    if (vec) {
+        const uint4 y = *reinterpret_cast<const uint4 *>(yh + i);
+        *reinterpret_cast<uint4 *>(yo + i) =
+            make_uint4(fsub(y.x, pe[0]), fsub(y.y, pe[1]), fsub(y.z, pe[2]), fsub(y.w, pe[3]));
+    } else {
 #pragma unroll
-        for (int s = 0; s < 4; ++s) {
-            const int col = i + s;
-            if (col < c1) {
-                const uint32_t yv = yh[col];
-                ystage[col - c0] = yv;
-                yo[col] = fsub(yv, pe[s]);
-            }
-        }
+        for (int q2 = 0; q2 < 4; ++q2)
+            if (i + q2 < m) yo[i + q2] = fsub(yh[i + q2], pe[q2]);
     }
-    __syncthreads();
-    asm volatile("griddepcontrol.wait;" ::: "memory");  // g and u are complete from here on
-    int cnty = 0;
-    for (int col = c0 + tid; col < c1; col += kDecThreads) {
-        const uint64_t yv = ystage[col - c0];
-        for (uint32_t q = 0; q < ell; ++q) racc[q] += (uint64_t)g[(size_t)q * m + col] * yv;
-        if (++cnty == 4) {
-            cnty = 0;
-            for (uint32_t q = 0; q < ell; ++q) racc[q] = fred(racc[q]);
-        }
-    }
+}
 
-    // ---- the x_hat side over this CTA's slice of K
-    const int kc = (K + (int)C - 1) / (int)C;
-    const int k0 = (int)rank * kc, k1 = min(K, k0 + kc);
-    const uint32_t *xh = Xhat + b * K;
+// ---------------------------------------------------------------------------
+// Verify: accept_b = AND_q [ L_q == R_q ] with L_q = u_q . x_hat_b and
+// R_q = g_q . y_hat_b (= e_q^T (G_y^T y_hat_b) by transposition), u_q =
+// e_q^T Q and g_q = G_y e_q from the challenge kernels.  One CTA per vector;
+// the repetitions run one after the other over the (cached) vectors.
+// ---------------------------------------------------------------------------
+constexpr int kCheckThreads = 512;
+
+__device__ __forceinline__ uint32_t dot_mod(const uint32_t *__restrict__ a, const uint32_t *__restrict__ x,
+                                            int n, int tid) {
+    uint64_t acc = 0;
     int cnt = 0;
-    for (int k = k0 + tid; k < k1; k += kDecThreads) {
-        const uint64_t xv = xh[k];
-        for (uint32_t q = 0; q < ell; ++q) lacc[q] += (uint64_t)u[(size_t)q * K + k] * xv;
+    for (int k = tid; k < n; k += kCheckThreads) {
+        acc += (uint64_t)__ldg(a + k) * x[k];
         if (++cnt == 4) {
             cnt = 0;
-            for (uint32_t q = 0; q < ell; ++q) lacc[q] = fred(lacc[q]);
+            acc = fred(acc);
         }
     }
+    return warp_fsum(fred(acc));
+}
 
+__global__ void __launch_bounds__(kCheckThreads) k_check(const uint32_t *__restrict__ Xhat, int K,
+                                                        const uint32_t *__restrict__ Yhat, int m,
+                                                        const uint32_t *__restrict__ g,
+                                                        const uint32_t *__restrict__ u, uint32_t ell,
+                                                        int32_t *__restrict__ accept) {
+    __shared__ uint32_t s_l[kCheckThreads / 32], s_r[kCheckThreads / 32];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const size_t b = blockIdx.x;
+    const uint32_t *xh = Xhat + b * K, *yh = Yhat + b * m;
+    int ok = 1;
     for (uint32_t q = 0; q < ell; ++q) {
-        const uint32_t l = warp_fsum(fred(lacc[q]));
-        const uint32_t r = warp_fsum(fred(racc[q]));
+        const uint32_t l = dot_mod(u + (size_t)q * K, xh, K, tid);
+        const uint32_t r = dot_mod(g + (size_t)q * m, yh, m, tid);
         if (lane == 0) {
-            s_warp[warp][q] = l;
-            s_warp[warp][kMaxEll + q] = r;
+            s_l[warp] = l;
+            s_r[warp] = r;
         }
-    }
-    __syncthreads();
-    if (tid < 2 * kMaxEll) {
-        uint32_t s = 0;
-        for (int w = 0; w < kDecThreads / 32; ++w) s = fadd(s, s_warp[w][tid]);
-        s_part[tid] = s;
-    }
-    cluster.sync();
-    if (rank == 0 && tid == 0) {
-        int ok = 1;
-        for (uint32_t q = 0; q < ell; ++q) {
+        __syncthreads();
+        if (tid == 0) {
             uint32_t L = 0, R = 0;
-            for (uint32_t r = 0; r < C; ++r) {
-                const uint32_t *rp = cluster.map_shared_rank(s_part, r);
-                L = fadd(L, rp[q]);
-                R = fadd(R, rp[kMaxEll + q]);
+            for (int w = 0; w < kCheckThreads / 32; ++w) {
+                L = fadd(L, s_l[w]);
+                R = fadd(R, s_r[w]);
             }
             ok &= (L == R);
         }
-        accept[b] = ok;
+        __syncthreads();
     }
-    cluster.sync();
+    if (tid == 0) accept[b] = ok;
 }
 
 // out[b][col] = (P e_x,b)_col for the columns of this CTA (1024 per CTA).
@@ -320,48 +316,36 @@ cudaError_t launch_verify_u(const uint32_t *Qm, int K, const uint32_t *chal, uin
     return cudaLaunchKernelEx(&cfg, k_verify_u, Qm, K, chal, t_y, u);
 }
 
-cudaError_t launch_decode_verify(const uint32_t *PT, int m, int K, const uint32_t *st, uint32_t t_x,
-                                 const uint32_t *Xhat, const uint32_t *Yhat, const uint32_t *g,
-                                 const uint32_t *u, uint32_t ell, int B, uint32_t *Y,
-                                 int32_t *accept, cudaStream_t s, const uint32_t *mask) {
-    if (B <= 0) return cudaSuccess;
-    if (ell > (uint32_t)kMaxEll) return cudaErrorInvalidValue;
-    const bool vec = (m % 4 == 0) && ((reinterpret_cast<uintptr_t>(PT) & 15u) == 0);
-    int C = (m + 1023) / 1024;
-    C = C < 1 ? 1 : (C > 8 ? 8 : C);
-    const int chunk = (((m + C - 1) / C) + 3) & ~3;  // y_hat columns per CTA (staged in smem)
-    if ((2 * (size_t)t_x + (size_t)chunk) * sizeof(uint32_t) > 200 * 1024) return cudaErrorInvalidValue;
-    static const cudaError_t smem_attr = cudaFuncSetAttribute(
-        k_decode_verify<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
-    static const cudaError_t smem_attr2 = cudaFuncSetAttribute(
-        k_decode_verify<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
-    if (smem_attr != cudaSuccess) return smem_attr;
-    if (smem_attr2 != cudaSuccess) return smem_attr2;
+cudaError_t launch_decrypt(const uint32_t *PT, int m, const uint32_t *st, uint32_t t_x,
+                           const uint32_t *Yhat, int B, uint32_t *Y, cudaStream_t s, const uint32_t *mask) {
+    if (B <= 0 || m <= 0) return cudaSuccess;
+    const bool vec = (m % 4 == 0) &&
+                     ((reinterpret_cast<uintptr_t>(PT) | reinterpret_cast<uintptr_t>(Yhat) |
+                       reinterpret_cast<uintptr_t>(Y)) & 15u) == 0;
+    const size_t smem = mask ? 0 : 2 * (size_t)t_x * sizeof(uint32_t);
+    if (smem > 48 * 1024) return cudaErrorInvalidValue;
     for (int b0 = 0; b0 < B; b0 += 65535) {
         const int nb = B - b0 < 65535 ? B - b0 : 65535;
-        cudaLaunchConfig_t cfg = {};
-        cfg.gridDim = dim3(C, nb, 1);
-        cfg.blockDim = dim3(kDecThreads, 1, 1);
-        cfg.dynamicSmemBytes = (2 * (size_t)t_x + (size_t)chunk) * sizeof(uint32_t);
-        cfg.stream = s;
-        cudaLaunchAttribute attr[2];
-        attr[0].id = cudaLaunchAttributeClusterDimension;
-        attr[0].val.clusterDim.x = C;
-        attr[0].val.clusterDim.y = 1;
-        attr[0].val.clusterDim.z = 1;
-        attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-        attr[1].val.programmaticStreamSerializationAllowed = 1;
-        cfg.attrs = attr;
-        cfg.numAttrs = 2;
-        cudaError_t e = mask ? cudaLaunchKernelEx(&cfg, k_decode_verify<true>, PT, m, K, st, t_x,
-                                                  Xhat + (size_t)b0 * K, Yhat + (size_t)b0 * m, g, u,
-                                                  ell, Y + (size_t)b0 * m, accept + b0, vec,
-                                                  mask + (size_t)b0 * m)
-                             : cudaLaunchKernelEx(&cfg, k_decode_verify<false>, PT, m, K,
-                                                  st + (size_t)b0 * 2 * t_x, t_x, Xhat + (size_t)b0 * K,
-                                                  Yhat + (size_t)b0 * m, g, u, ell, Y + (size_t)b0 * m,
-                                                  accept + b0, vec, (const uint32_t *)nullptr);
-        if (e != cudaSuccess) return e;
+        const dim3 grid((m + kDecCols - 1) / kDecCols, nb);
+        const dim3 grid_mask((m + 4 * kDecThreads - 1) / (4 * kDecThreads), nb);
+        if (mask)
+            k_decrypt<true><<<grid_mask, kDecThreads, 0, s>>>(PT, m, nullptr, t_x, Yhat + (size_t)b0 * m,
+                                                         Y + (size_t)b0 * m, mask + (size_t)b0 * m, vec);
+        else
+            k_decrypt<false><<<grid, kDecThreads, smem, s>>>(PT, m, st + (size_t)b0 * 2 * t_x, t_x,
+                                                             Yhat + (size_t)b0 * m, Y + (size_t)b0 * m,
+                                                             nullptr, vec);
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_check(const uint32_t *Xhat, int K, const uint32_t *Yhat, int m, const uint32_t *g,
+                         const uint32_t *u, uint32_t ell, int B, int32_t *accept, cudaStream_t s) {
+    if (B <= 0) return cudaSuccess;
+    for (int b0 = 0; b0 < B; b0 += 0x7fffffff) {
+        const int nb = B - b0;
+        k_check<<<nb, kCheckThreads, 0, s>>>(Xhat + (size_t)b0 * K, K, Yhat + (size_t)b0 * m, m, g, u, ell,
+                                             accept + b0);
     }
     return cudaGetLastError();
 }

@@ -125,13 +125,16 @@ uint32_t *library_error_word();
 cudaError_t launch_verify_u(const uint32_t *Qm, int K, const uint32_t *chal, uint32_t t_y,
                             uint32_t ell, uint32_t *u, cudaStream_t s);
 
-// Fused decrypt and verify reduction for B vectors.  With mask non-null
-// (boost mode) Y = Y_hat - mask, mask [B][m] = P e_x per vector, and st is
-// not read.
-cudaError_t launch_decode_verify(const uint32_t *PT, int m, int K, const uint32_t *st, uint32_t t_x,
-                                 const uint32_t *Xhat, const uint32_t *Yhat, const uint32_t *g,
-                                 const uint32_t *u, uint32_t ell, int B, uint32_t *Y,
-                                 int32_t *accept, cudaStream_t s, const uint32_t *mask = nullptr);
+// Decrypt: Y[b] = Y_hat[b] - P e_x,b for B vectors (st [B][2t_x]); with
+// mask non-null (boost mode) Y = Y_hat - mask, mask [B][m] = P e_x per
+// vector, and st is not read.  Y may alias Y_hat.
+cudaError_t launch_decrypt(const uint32_t *PT, int m, const uint32_t *st, uint32_t t_x,
+                           const uint32_t *Yhat, int B, uint32_t *Y, cudaStream_t s,
+                           const uint32_t *mask = nullptr);
+// Verify: accept[b] = AND_q (u_q . Xhat[b] == g_q . Yhat[b]) for the ell
+// challenges' u (ell x K) and g (ell x m).
+cudaError_t launch_check(const uint32_t *Xhat, int K, const uint32_t *Yhat, int m, const uint32_t *g,
+                         const uint32_t *u, uint32_t ell, int B, int32_t *accept, cudaStream_t s);
 
 // out = a + b over F_q (n elements; out may alias a or b).
 cudaError_t launch_field_add(const uint32_t *a, const uint32_t *b, size_t n, uint32_t *out,

@@ -381,6 +381,15 @@ constexpr int kFusedBatch = 16;      // loads in flight per thread
 
 __device__ __forceinline__ uint32_t fpad(uint32_t i) { return i + (i >> 5); }  // bank padding
 
+// floor(x / d) as (x * ceil(2^40 / d)) >> 40 (division by an invariant
+// integer through a rounded-up reciprocal, Granlund and Montgomery 1994).
+// Exact when x * d < 2^40: the product is x / d + x * eps / 2^40 with
+// 0 <= eps < 1, and x / 2^40 < 1 / d never reaches the next integer.
+__host__ __device__ __forceinline__ uint64_t div_magic(uint32_t d) { return ((1ull << 40) + d - 1) / d; }
+__device__ __forceinline__ uint32_t div_by(uint32_t x, uint64_t magic) {
+    return (uint32_t)(((uint64_t)x * magic) >> 40);
+}
+
 __global__ void __launch_bounds__(kFusedThreads) k_syndrome_fused(
     pvmvmd_key key, uint32_t tag, uint64_t idx0, uint32_t N, uint32_t t, uint32_t slice,
     const uint32_t *__restrict__ pi2inv, const uint32_t *__restrict__ v2p,
@@ -567,6 +576,7 @@ __global__ void __launch_bounds__(kFusedThreads) k_syndrome_fused(
     // ---- c over this CTA's slice (coalesced positions, loads batched)
     const uint32_t base = rank * slice;
     const uint32_t items = slice / kFusedThreads;
+    const uint64_t items_magic = div_magic(items), slice_magic = div_magic(slice);
     for (uint32_t u0 = 0; u0 < items; u0 += kFusedBatch) {
         uint32_t kk[kFusedBatch], sc[kFusedBatch];
 #pragma unroll
@@ -635,7 +645,7 @@ __global__ void __launch_bounds__(kFusedThreads) k_syndrome_fused(
         for (int u = 0; u < kFusedBatch; ++u) {
             if (u0 + u < items) {
                 const uint32_t li = (u0 + u) * kFusedThreads + tid;
-                const uint32_t d = fadd(F[fpad(li)], fadd(s_texcl[li / items], after));
+                const uint32_t d = fadd(F[fpad(li)], fadd(s_texcl[div_by(li, items_magic)], after));
                 F[fpad(li)] = fmul(sc[u], d);
             }
         }
@@ -659,7 +669,7 @@ __global__ void __launch_bounds__(kFusedThreads) k_syndrome_fused(
             } else {
 #pragma unroll
                 for (int c = 0; c < 8; ++c) {
-                    const uint32_t owner = gi[c] / slice;
+                    const uint32_t owner = div_by(gi[c], slice_magic);
                     v[c] = cluster.map_shared_rank(F, owner)[fpad(gi[c] - owner * slice)];
                 }
             }
@@ -668,7 +678,7 @@ __global__ void __launch_bounds__(kFusedThreads) k_syndrome_fused(
         } else {
             for (uint32_t c = 0; c < r; ++c) {
                 const uint32_t gi = __ldg(p + c);
-                const uint32_t owner = gi / slice, off = gi - owner * slice;
+                const uint32_t owner = div_by(gi, slice_magic), off = gi - owner * slice;
                 acc = fadd(acc, C == 1 ? F[fpad(off)] : cluster.map_shared_rank(F, owner)[fpad(off)]);
             }
         }
@@ -1174,14 +1184,59 @@ cudaError_t launch_transpose_i8(const int8_t *in, int R, int C, int8_t *out, cud
 }
 
 
+namespace {
+uint32_t fused_slice(uint32_t N, int C) {
+    return (uint32_t)(((N + C - 1) / C + kFusedThreads - 1) / kFusedThreads) * kFusedThreads;
+}
+size_t fused_smem(uint32_t slice, uint32_t t) {
+    return ((size_t)slice + slice / 32 + 3 * (size_t)t + 1 + 1024) * sizeof(uint32_t);
+}
+constexpr size_t kFusedMaxSmem = 180 * 1024;
+
+// Largest cluster the fused kernel may use on this device: 16 CTAs where the
+// device schedules clusters of that (non-portable) size, else 8.
+int fused_max_cluster() {
+    static const int cmax = [] {
+        if (cudaFuncSetAttribute(k_syndrome_fused, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+            cudaSuccess) {
+            cudaGetLastError();
+            return 8;
+        }
+        if (cudaFuncSetAttribute(k_syndrome_fused, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)kFusedMaxSmem) != cudaSuccess) {
+            cudaGetLastError();
+            return 8;
+        }
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(16, 1, 1);
+        cfg.blockDim = dim3(kFusedThreads, 1, 1);
+        cfg.dynamicSmemBytes = kFusedMaxSmem / 2;
+        cudaLaunchAttribute a[1];
+        a[0].id = cudaLaunchAttributeClusterDimension;
+        a[0].val.clusterDim.x = 16;
+        a[0].val.clusterDim.y = 1;
+        a[0].val.clusterDim.z = 1;
+        cfg.attrs = a;
+        cfg.numAttrs = 1;
+        int n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, k_syndrome_fused, &cfg) != cudaSuccess) {
+            cudaGetLastError();
+            return 8;
+        }
+        return n > 0 ? 16 : 8;
+    }();
+    return cmax;
+}
+}  // namespace
+
 // Cluster size and slice for the fused syndrome; false if N is too long for
 // one cluster of at most 8 CTAs.
 bool syndrome_fused_plan(uint32_t N, uint32_t t, int *C_out, uint32_t *slice_out, size_t *smem_out) {
     // one CTA when the padded intermediate fits, else the smallest cluster
     for (int C = 1; C <= 8; C *= 2) {
-        const uint32_t slice = (uint32_t)(((N + C - 1) / C + kFusedThreads - 1) / kFusedThreads) * kFusedThreads;
-        const size_t smem = ((size_t)slice + slice / 32 + 3 * (size_t)t + 1 + 1024) * sizeof(uint32_t);
-        if (smem <= (size_t)180 * 1024) {
+        const uint32_t slice = fused_slice(N, C);
+        const size_t smem = fused_smem(slice, t);
+        if (smem <= kFusedMaxSmem) {
             *C_out = C;
             *slice_out = slice;
             *smem_out = smem;
@@ -1189,6 +1244,28 @@ bool syndrome_fused_plan(uint32_t N, uint32_t t, int *C_out, uint32_t *slice_out
         }
     }
     return false;
+}
+
+// The cluster size one launch of `count` vectors uses: the smallest that
+// holds the intermediate, and for a batch that leaves most SMs idle (at most
+// a quarter busy) doubled while count * C CTAs still fit the SMs and every
+// CTA keeps at least one position per thread.  A small batch (the ell
+// shared challenges, a few encodes) then spreads each vector's serial work
+// over up to 16 SMs instead of one; larger batches keep the cheaper
+// per-position work of the smallest cluster.
+static void syndrome_fused_launch_plan(uint32_t N, uint32_t t, uint32_t count, int *C, uint32_t *slice,
+                                       size_t *smem) {
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if ((uint64_t)count * (uint64_t)*C * 4 > (uint64_t)sms) return;
+    const int cmax = fused_max_cluster();
+    while (*C < cmax && (uint64_t)count * (uint64_t)(2 * *C) <= (uint64_t)sms &&
+           (uint64_t)(2 * *C) * kFusedThreads <= (uint64_t)N) {
+        *C *= 2;
+        *slice = fused_slice(N, *C);
+        *smem = fused_smem(*slice, t);
+    }
 }
 
 cudaError_t launch_syndrome_fused(const pvmvmd_key &key, uint32_t tag, uint64_t idx0, uint32_t N,
@@ -1203,8 +1280,9 @@ cudaError_t launch_syndrome_fused(const pvmvmd_key &key, uint32_t tag, uint64_t 
     size_t smem = 0;
     if (!syndrome_fused_plan(N, t, &C, &slice, &smem)) return cudaErrorNotSupported;
     static const cudaError_t attr = cudaFuncSetAttribute(
-        k_syndrome_fused, cudaFuncAttributeMaxDynamicSharedMemorySize, 180 * 1024);
+        k_syndrome_fused, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFusedMaxSmem);
     if (attr != cudaSuccess) return attr;
+    syndrome_fused_launch_plan(N, t, count < 65535 ? count : 65535, &C, &slice, &smem);
     for (uint32_t c0 = 0; c0 < count; c0 += 65535) {
         const uint32_t nb = count - c0 < 65535 ? count - c0 : 65535;
         cudaLaunchConfig_t cfg = {};

@@ -84,6 +84,14 @@ def _full_round_trip(pv, W, x_int, seeds=(11, 12, 13), params=None, oracle_kw=No
     assert pv.as_u32(acc_bad).tolist() == exp
     for b in range(0, B, 2):
         assert not pp.verify(Xh_h[b], bad_h[b], oracle.key_from_seed(seeds[2] + 1))
+    # in place: Y overwrites Y_hat, so the check reads Y_hat before the decrypt
+    Yip = YhB.clone()
+    _, acc_ip = pv.pvmvmd_decode_verify(ctx, st, Xh, Yip, challenge_key=seeds[2], Y=Yip)
+    assert np.array_equal(pv.as_u32(Yip), Y_h)
+    assert pv.as_u32(acc_ip).tolist() == [1] * B
+    bad_ip = bad.clone()
+    _, acc_bad_ip = pv.pvmvmd_decode_verify(ctx, st, Xh, bad_ip, challenge_key=seeds[2] + 1, Y=bad_ip)
+    assert pv.as_u32(acc_bad_ip).tolist() == exp
     assert pv.pvmvmd_device_status() == 0
     ctx.destroy()
 
