@@ -588,7 +588,7 @@ int encode_batch(pvmvmd_ctx *ctx, const uint32_t *X_dev, int B, const pvmvmd_key
         // sample, scan and gather in one launch per batch, no scratch
         PV_CUDA(launch_syndrome_fused(*key, kTagMask, 0, ctx->Nx, ctx->t_x, (uint32_t)B, d.pi2inv,
                                       d.v2p, d.v1, d.pi1inv, d.pi2, d.v2m, d.v1pm, ctx->K, ctx->rate,
-                                      stp, X_dev, Xhat_dev, s));
+                                      stp, X_dev, Xhat_dev, s, /*pdl=*/true));
         return PVMVMD_OK;
     }
     for (int b0 = 0; b0 < B; b0 += ctx->sb) {

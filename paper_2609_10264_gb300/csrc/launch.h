@@ -47,12 +47,17 @@ cudaError_t launch_syndrome_scan(const uint32_t *pi2inv, const uint32_t *v2p, co
 bool syndrome_fused_plan(uint32_t N, uint32_t t, int *C, uint32_t *slice, size_t *smem);
 // Tables: pi2inv, v2p = v2 o pi2^-1, v1 (cluster form); pi2, v2m = v2 R,
 // v1pm = (v1 o pi1^-1) R (single-CTA form, Montgomery-scaled, R = 2^32).
+// pdl: launch with programmatic stream serialisation.  The kernel reads
+// nothing but the key and the tables before griddepcontrol.wait, so its
+// sampling and scans overlap the kernel before it; st, out and addend are
+// touched only after the wait.
 cudaError_t launch_syndrome_fused(const pvmvmd_key &key, uint32_t tag, uint64_t idx0, uint32_t N,
                                   uint32_t t, uint32_t count, const uint32_t *pi2inv,
                                   const uint32_t *v2p, const uint32_t *v1, const uint32_t *pi1inv,
                                   const uint32_t *pi2, const uint32_t *v2m, const uint32_t *v1pm,
                                   uint32_t n, uint32_t r, uint32_t *sparse_out,
-                                  const uint32_t *addend, uint32_t *out, cudaStream_t s);
+                                  const uint32_t *addend, uint32_t *out, cudaStream_t s,
+                                  bool pdl = false);
 
 // Lane-parallel syndrome for L vectors (vector b uses index idx0 + b, as
 // launch_sample_sparse): sparse_out [L][2t] as there, S [L][t+1] suffix sums

@@ -390,6 +390,20 @@ __device__ __forceinline__ uint32_t div_by(uint32_t x, uint64_t magic) {
     return (uint32_t)(((uint64_t)x * magic) >> 40);
 }
 
+// Everything before this point reads only the key and the code tables; the
+// state st and the output are written after griddepcontrol.wait, so a launch
+// with programmatic serialisation may run its sampling and scans while the
+// kernel before it finishes.  Writes st = (support, e) with e_j recovered
+// from the suffix sums suf (suf[t] = 0).
+__device__ __forceinline__ void fused_publish(uint32_t *st, const uint32_t *supp, const uint32_t *suf,
+                                              uint32_t t, int tid) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    for (uint32_t j = tid; j < t; j += kFusedThreads) {
+        st[j] = supp[j];
+        st[t + j] = fsub(suf[j], suf[j + 1]);
+    }
+}
+
 __global__ void __launch_bounds__(kFusedThreads) k_syndrome_fused(
     pvmvmd_key key, uint32_t tag, uint64_t idx0, uint32_t N, uint32_t t, uint32_t slice,
     const uint32_t *__restrict__ pi2inv, const uint32_t *__restrict__ v2p,
@@ -432,14 +446,6 @@ __global__ void __launch_bounds__(kFusedThreads) k_syndrome_fused(
         uint32_t rk = 0;
         for (uint32_t j = 0; j < t; ++j) rk += list[j] < v;
         supp[rk] = v;
-    }
-    __syncthreads();
-    if (rank == 0) {
-        uint32_t *st = sparse_out + (size_t)vec * 2 * t;
-        for (uint32_t j = tid; j < t; j += kFusedThreads) {
-            st[j] = supp[j];
-            st[t + j] = suf[j];
-        }
     }
     __syncthreads();
     if (warp == 0) {  // suf[j] <- sum_{j' >= j} e_{j'}; suf[t] = 0
@@ -534,6 +540,7 @@ __global__ void __launch_bounds__(kFusedThreads) k_syndrome_fused(
             F[fpad(li)] = fadd(F[fpad(li)], add);
         }
         __syncthreads();
+        fused_publish(sparse_out + (size_t)vec * 2 * t, supp, suf, t, tid);
         // out_j = addend_j + sum_c v1[pi1^-1(r j + c)] d[pi1^-1(r j + c)]
         for (uint32_t jo = tid; jo < n; jo += kFusedThreads) {
             const uint32_t *p = pi1inv + (size_t)jo * r;
@@ -651,6 +658,8 @@ __global__ void __launch_bounds__(kFusedThreads) k_syndrome_fused(
         }
     }
     if (C > 1) cluster.sync(); else __syncthreads();
+    if (rank == 0) fused_publish(sparse_out + (size_t)vec * 2 * t, supp, suf, t, tid);
+    else asm volatile("griddepcontrol.wait;" ::: "memory");
 
     // ---- gather: out_j = addend_j + sum_c F[pi1^-1(r j + c)]
     const uint32_t nsl = (n + C - 1) / C;
@@ -1273,7 +1282,7 @@ cudaError_t launch_syndrome_fused(const pvmvmd_key &key, uint32_t tag, uint64_t 
                                   const uint32_t *v2p, const uint32_t *v1, const uint32_t *pi1inv,
                                   const uint32_t *pi2, const uint32_t *v2m, const uint32_t *v1pm,
                                   uint32_t n, uint32_t r, uint32_t *sparse_out,
-                                  const uint32_t *addend, uint32_t *out, cudaStream_t s) {
+                                  const uint32_t *addend, uint32_t *out, cudaStream_t s, bool pdl) {
     if (count == 0) return cudaSuccess;
     int C = 0;
     uint32_t slice = 0;
@@ -1290,13 +1299,15 @@ cudaError_t launch_syndrome_fused(const pvmvmd_key &key, uint32_t tag, uint64_t 
         cfg.blockDim = dim3(kFusedThreads, 1, 1);
         cfg.dynamicSmemBytes = smem;
         cfg.stream = s;
-        cudaLaunchAttribute attr1[1];
+        cudaLaunchAttribute attr1[2];
         attr1[0].id = cudaLaunchAttributeClusterDimension;
         attr1[0].val.clusterDim.x = C;
         attr1[0].val.clusterDim.y = 1;
         attr1[0].val.clusterDim.z = 1;
+        attr1[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr1[1].val.programmaticStreamSerializationAllowed = 1;
         cfg.attrs = attr1;
-        cfg.numAttrs = 1;
+        cfg.numAttrs = pdl ? 2 : 1;
         cudaError_t e = cudaLaunchKernelEx(&cfg, k_syndrome_fused, key, tag, idx0 + c0, N, t, slice,
                                            pi2inv, v2p, v1, pi1inv, n, r,
                                            sparse_out + (size_t)c0 * 2 * t,
