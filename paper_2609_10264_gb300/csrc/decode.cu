@@ -133,6 +133,9 @@ __device__ __forceinline__ void pe_cols(const uint32_t *__restrict__ PT, int m, 
 // (a few rounds of 8 loads in flight) and the grid holds many short CTAs
 // whatever m and B are.  The groups' partial sums meet in shared memory.
 // In boost mode (Sec. 7.2) P e_x,b was prepared ahead: Y_b = y_hat_b - mask_b.
+// The grid runs vectors fastest (blockIdx.x = b, blockIdx.y = column block),
+// so the CTAs in flight share a few column blocks and a row of P^T drawn by
+// several vectors' supports is read from HBM once and then from L2.
 // ---------------------------------------------------------------------------
 constexpr int kDecGroups = 4;
 constexpr int kDecColThreads = kDecThreads / kDecGroups;  // 64
@@ -146,10 +149,10 @@ __global__ void __launch_bounds__(kDecThreads) k_decrypt(const uint32_t *__restr
     extern __shared__ uint32_t sm[];  // support[t_x], values[t_x]
     __shared__ uint4 s_part[kDecGroups - 1][kDecColThreads];
     const int tid = threadIdx.x;
-    const size_t b = blockIdx.y;
+    const size_t b = blockIdx.x;
     const int grp = tid / kDecColThreads, ct = tid % kDecColThreads;
     // boost mode: no rows to split, every thread owns 4 of 1024 columns
-    const int i = kBoost ? ((int)blockIdx.x * kDecThreads + tid) * 4 : (int)blockIdx.x * kDecCols + ct * 4;
+    const int i = kBoost ? ((int)blockIdx.y * kDecThreads + tid) * 4 : (int)blockIdx.y * kDecCols + ct * 4;
     uint32_t pe[4] = {0u, 0u, 0u, 0u};
     if (!kBoost) {
         const uint32_t *stb = st + b * 2 * t_x;
@@ -324,29 +327,20 @@ cudaError_t launch_decrypt(const uint32_t *PT, int m, const uint32_t *st, uint32
                        reinterpret_cast<uintptr_t>(Y)) & 15u) == 0;
     const size_t smem = mask ? 0 : 2 * (size_t)t_x * sizeof(uint32_t);
     if (smem > 48 * 1024) return cudaErrorInvalidValue;
-    for (int b0 = 0; b0 < B; b0 += 65535) {
-        const int nb = B - b0 < 65535 ? B - b0 : 65535;
-        const dim3 grid((m + kDecCols - 1) / kDecCols, nb);
-        const dim3 grid_mask((m + 4 * kDecThreads - 1) / (4 * kDecThreads), nb);
-        if (mask)
-            k_decrypt<true><<<grid_mask, kDecThreads, 0, s>>>(PT, m, nullptr, t_x, Yhat + (size_t)b0 * m,
-                                                         Y + (size_t)b0 * m, mask + (size_t)b0 * m, vec);
-        else
-            k_decrypt<false><<<grid, kDecThreads, smem, s>>>(PT, m, st + (size_t)b0 * 2 * t_x, t_x,
-                                                             Yhat + (size_t)b0 * m, Y + (size_t)b0 * m,
-                                                             nullptr, vec);
-    }
+    if ((m + kDecCols - 1) / kDecCols > 65535) return cudaErrorInvalidValue;
+    const dim3 grid((unsigned)B, (m + kDecCols - 1) / kDecCols);
+    const dim3 grid_mask((unsigned)B, (m + 4 * kDecThreads - 1) / (4 * kDecThreads));
+    if (mask)
+        k_decrypt<true><<<grid_mask, kDecThreads, 0, s>>>(PT, m, nullptr, t_x, Yhat, Y, mask, vec);
+    else
+        k_decrypt<false><<<grid, kDecThreads, smem, s>>>(PT, m, st, t_x, Yhat, Y, nullptr, vec);
     return cudaGetLastError();
 }
 
 cudaError_t launch_check(const uint32_t *Xhat, int K, const uint32_t *Yhat, int m, const uint32_t *g,
                          const uint32_t *u, uint32_t ell, int B, int32_t *accept, cudaStream_t s) {
     if (B <= 0) return cudaSuccess;
-    for (int b0 = 0; b0 < B; b0 += 0x7fffffff) {
-        const int nb = B - b0;
-        k_check<<<nb, kCheckThreads, 0, s>>>(Xhat + (size_t)b0 * K, K, Yhat + (size_t)b0 * m, m, g, u, ell,
-                                             accept + b0);
-    }
+    k_check<<<(unsigned)B, kCheckThreads, 0, s>>>(Xhat, K, Yhat, m, g, u, ell, accept);
     return cudaGetLastError();
 }
 
