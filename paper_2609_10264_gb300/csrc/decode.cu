@@ -198,21 +198,8 @@ __global__ void __launch_bounds__(kDecThreads) k_decrypt(const uint32_t *__restr
 // e_q^T Q and g_q = G_y e_q from the challenge kernels.  One CTA per vector;
 // the repetitions run one after the other over the (cached) vectors.
 // ---------------------------------------------------------------------------
-constexpr int kCheckThreads = 512;
-
-__device__ __forceinline__ uint32_t dot_mod(const uint32_t *__restrict__ a, const uint32_t *__restrict__ x,
-                                            int n, int tid) {
-    uint64_t acc = 0;
-    int cnt = 0;
-    for (int k = tid; k < n; k += kCheckThreads) {
-        acc += (uint64_t)__ldg(a + k) * x[k];
-        if (++cnt == 4) {
-            cnt = 0;
-            acc = fred(acc);
-        }
-    }
-    return warp_fsum(fred(acc));
-}
+constexpr int kCheckThreads = 1024;
+constexpr int kCheckBatch = 4;  // loads in flight per operand and thread
 
 __global__ void __launch_bounds__(kCheckThreads) k_check(const uint32_t *__restrict__ Xhat, int K,
                                                         const uint32_t *__restrict__ Yhat, int m,
@@ -223,10 +210,35 @@ __global__ void __launch_bounds__(kCheckThreads) k_check(const uint32_t *__restr
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const size_t b = blockIdx.x;
     const uint32_t *xh = Xhat + b * K, *yh = Yhat + b * m;
+    // the kernel after this one (the next call's encode) may start its
+    // key-only work now
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    const int n = K > m ? K : m;
     int ok = 1;
     for (uint32_t q = 0; q < ell; ++q) {
-        const uint32_t l = dot_mod(u + (size_t)q * K, xh, K, tid);
-        const uint32_t r = dot_mod(g + (size_t)q * m, yh, m, tid);
+        const uint32_t *uq = u + (size_t)q * K, *gq = g + (size_t)q * m;
+        uint64_t la = 0, ra = 0;
+        for (int k0 = tid; k0 < n; k0 += kCheckBatch * kCheckThreads) {
+            uint32_t a[kCheckBatch], x[kCheckBatch], c[kCheckBatch], y[kCheckBatch];
+#pragma unroll
+            for (int v = 0; v < kCheckBatch; ++v) {
+                const int k = k0 + v * kCheckThreads;
+                a[v] = k < K ? __ldg(uq + k) : 0u;
+                x[v] = k < K ? xh[k] : 0u;
+                c[v] = k < m ? __ldg(gq + k) : 0u;
+                y[v] = k < m ? yh[k] : 0u;
+            }
+            // four products of values below q stay below 2^64 with the
+            // reduced running sum
+#pragma unroll
+            for (int v = 0; v < kCheckBatch; ++v) {
+                la += (uint64_t)a[v] * x[v];
+                ra += (uint64_t)c[v] * y[v];
+            }
+            la = fred(la);
+            ra = fred(ra);
+        }
+        const uint32_t l = warp_fsum((uint32_t)la), r = warp_fsum((uint32_t)ra);
         if (lane == 0) {
             s_l[warp] = l;
             s_r[warp] = r;
