@@ -823,7 +823,12 @@ __global__ void k_transpose_i8(const int8_t *__restrict__ in, int R, int C, int8
 //                                                   (k_lane_gather)
 // A thread owns four consecutive lanes (16-byte accesses) of one tile or
 // span; a CTA of 256 threads covers `cols` lane quads (Lp/4 rounded up to 32,
-// at most 64) of 256 / cols tiles or spans.
+// at most 64) of 256 / cols tiles or spans.  The six kernels launch with
+// programmatic serialisation and wait (griddepcontrol.wait) before touching
+// their predecessor's output.  Only the sampler, whose work needs the key
+// alone, lets its successor launch early; the others let it launch at their
+// completion.  Early launches of the large grids held SM slots with waiting
+// CTAs and were slower (K = 28672, B = 256: 341 against 307 us).
 // -----------------------------------------------------------------------------
 constexpr int kLaneTile = 32;      // positions per tile (one thread walks them)
 constexpr int kLaneCta = 256;      // threads per lane CTA
@@ -843,7 +848,9 @@ __device__ __forceinline__ uint4 fadd4(uint4 a, uint4 b) {
 
 // e_b for vector idx0 + blockIdx.x as in k_sample_sparse (warp 0 the
 // support, warp 1 the values), written as st[b] = (ascending support,
-// values), and S[b][j] = sum_{j' >= j} values[j'], S[b][t] = 0.
+// values), and S[b][j] = sum_{j' >= j} values[j'], S[b][t] = 0.  Everything
+// is computed in shared memory from the key alone; st and S are written
+// after griddepcontrol.wait (a kernel before this one may still read them).
 __global__ void __launch_bounds__(128) k_lane_sample(pvmvmd_key key, uint32_t tag, uint64_t idx0,
                                                     uint32_t N, uint32_t t, uint32_t *__restrict__ st,
                                                     uint32_t *__restrict__ S) {
@@ -854,9 +861,11 @@ __global__ void __launch_bounds__(128) k_lane_sample(pvmvmd_key key, uint32_t ta
     uint32_t *words2 = words + 512;  // 512 keystream words (values)
     uint32_t *list = words2 + 512;   // t, in the order accepted
     uint32_t *vals = list + t;       // t
+    uint32_t *sorted = vals + t;     // t
+    uint32_t *suf = sorted + t;      // t + 1
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const uint64_t idx = idx0 + blockIdx.x;
-    uint32_t *supp = st + (size_t)blockIdx.x * 2 * t;
     for (uint32_t w = tid; w < nbw; w += 128) bitmap[w] = 0u;
     __syncthreads();
     if (warp == 0) warp_sample_support_list(key, tag, 2 * idx, N, t, bitmap, words, list, lane);
@@ -866,28 +875,36 @@ __global__ void __launch_bounds__(128) k_lane_sample(pvmvmd_key key, uint32_t ta
         const uint32_t v = list[i];
         uint32_t rk = 0;
         for (uint32_t j = 0; j < t; ++j) rk += list[j] < v;
-        supp[rk] = v;
-        supp[t + i] = vals[i];
+        sorted[rk] = v;
     }
-    if (warp != 0) return;
-    uint32_t *Sb = S + (size_t)blockIdx.x * (t + 1);
-    // suffix sums: lane owns a contiguous chunk, chunks combined by shuffles
-    const uint32_t per = (t + 31) / 32;
-    const uint32_t lo = min(t, lane * per), hi = min(t, lo + per);
-    uint32_t sum = 0;
-    for (uint32_t j = hi; j-- > lo;) sum = fadd(sum, vals[j]);
-    uint32_t incl = sum;
+    if (warp == 0) {
+        // suffix sums: lane owns a contiguous chunk, chunks combined by shuffles
+        const uint32_t per = (t + 31) / 32;
+        const uint32_t lo = min(t, lane * per), hi = min(t, lo + per);
+        uint32_t sum = 0;
+        for (uint32_t j = hi; j-- > lo;) sum = fadd(sum, vals[j]);
+        uint32_t incl = sum;
 #pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        const uint32_t y = __shfl_down_sync(kFull, incl, o);
-        if (lane + o < 32) incl = fadd(incl, y);
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t y = __shfl_down_sync(kFull, incl, o);
+            if (lane + o < 32) incl = fadd(incl, y);
+        }
+        uint32_t run = fsub(incl, sum);  // sum over the chunks after this lane's
+        for (uint32_t j = hi; j-- > lo;) {
+            run = fadd(run, vals[j]);
+            suf[j] = run;
+        }
+        if (lane == 0) suf[t] = 0u;
     }
-    uint32_t run = fsub(incl, sum);  // sum over the chunks after this lane's
-    for (uint32_t j = hi; j-- > lo;) {
-        run = fadd(run, vals[j]);
-        Sb[j] = run;
+    __syncthreads();
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    uint32_t *stb = st + (size_t)blockIdx.x * 2 * t;
+    uint32_t *Sb = S + (size_t)blockIdx.x * (t + 1);
+    for (uint32_t j = tid; j < t; j += 128) {
+        stb[j] = sorted[j];
+        stb[t + j] = vals[j];
     }
-    if (lane == 0) Sb[t] = 0u;
+    for (uint32_t j = tid; j <= t; j += 128) Sb[j] = suf[j];
 }
 
 // C[pi2(k)][b] = v2_k (A e_b)_k: a thread walks kExpandSpan positions k of
@@ -899,6 +916,7 @@ __global__ void __launch_bounds__(kLaneCta) k_lane_expand(const uint32_t *__rest
                                                          const uint32_t *__restrict__ pi2,
                                                          const uint32_t *__restrict__ v2m,
                                                          uint4 *__restrict__ C) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");  // inputs come from the kernel before
     const uint32_t cols = lane_cols(L), Lq = lane_pad(L) / 4;
     const uint32_t g = blockIdx.y * cols + threadIdx.x % cols;
     const uint32_t k0 = (blockIdx.x * (kLaneCta / cols) + threadIdx.x / cols) * kExpandSpan;
@@ -960,6 +978,7 @@ __global__ void __launch_bounds__(kLaneCta) k_lane_expand(const uint32_t *__rest
 // agg[tau][b] = sum over the tile's positions of C[i][b].
 __global__ void __launch_bounds__(kLaneCta) k_lane_tile_sum(const uint4 *__restrict__ C, uint32_t N,
                                                            uint32_t L, uint4 *__restrict__ agg) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");  // inputs come from the kernel before
     const uint32_t cols = lane_cols(L), Lq = lane_pad(L) / 4, ntiles = (N + kLaneTile - 1) / kLaneTile;
     const uint32_t g = blockIdx.y * cols + threadIdx.x % cols;
     const uint32_t tau = blockIdx.x * (kLaneCta / cols) + threadIdx.x / cols;
@@ -991,6 +1010,7 @@ __device__ __forceinline__ uint4 fsub4(uint4 a, uint4 b) {
 }
 __global__ void __launch_bounds__(kCarryThreads) k_lane_carry(const uint4 *__restrict__ agg, uint32_t ntiles,
                                                              uint32_t Lq, uint4 *__restrict__ carry) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");  // inputs come from the kernel before
     __shared__ uint4 wsum[kCarryThreads / 32];
     const uint32_t g = blockIdx.x, c = threadIdx.x, lane = c & 31, warp = c >> 5;
     const uint32_t per = (ntiles + kCarryThreads - 1) / kCarryThreads;
@@ -1046,6 +1066,7 @@ __global__ void __launch_bounds__(kCarryThreads) k_lane_carry(const uint4 *__res
 __global__ void __launch_bounds__(kLaneCta) k_lane_scan(uint4 *__restrict__ C, uint32_t N, uint32_t L,
                                                        const uint4 *__restrict__ carry,
                                                        const uint32_t *__restrict__ v1) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");  // inputs come from the kernel before
     const uint32_t cols = lane_cols(L), Lq = lane_pad(L) / 4, ntiles = (N + kLaneTile - 1) / kLaneTile;
     const uint32_t g = blockIdx.y * cols + threadIdx.x % cols;
     const uint32_t tau = blockIdx.x * (kLaneCta / cols) + threadIdx.x / cols;
@@ -1077,6 +1098,7 @@ __global__ void __launch_bounds__(kLaneCta) k_lane_gather(const uint4 *__restric
                                                          const uint32_t *__restrict__ pi1inv,
                                                          uint32_t r, uint32_t n, uint32_t L,
                                                          const uint32_t *addend, uint32_t *out) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");  // inputs come from the kernel before
     __shared__ uint32_t tile[kGatherJ][4 * kLaneQuadsMax + 1];
     const uint32_t cols = lane_cols(L), subs = kLaneCta / cols, Lq = lane_pad(L) / 4;
     const uint32_t tid = threadIdx.x, gl = tid % cols, sub = tid / cols;
@@ -1318,6 +1340,22 @@ cudaError_t launch_syndrome_fused(const pvmvmd_key &key, uint32_t tag, uint64_t 
     return cudaSuccess;
 }
 
+namespace {
+cudaError_t launch_pdl(const void *fn, dim3 grid, dim3 block, size_t smem, cudaStream_t s, void **args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute a[1];
+    a[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    a[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = a;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelExC(&cfg, fn, args);
+}
+}  // namespace
+
 size_t lane_aux_words(uint32_t N, uint32_t L) {
     return 2 * (size_t)((N + kLaneTile - 1) / kLaneTile) * lane_pad(L);
 }
@@ -1328,7 +1366,7 @@ cudaError_t launch_lane_syndrome(const pvmvmd_key &key, uint32_t tag, uint64_t i
                                  uint32_t *sparse_out, uint32_t *S, uint32_t *C, uint32_t *aux,
                                  const uint32_t *addend, uint32_t *out, cudaStream_t s) {
     if (L == 0) return cudaSuccess;
-    const size_t smem = ((size_t)(N + 31) / 32 + 1024 + 2 * (size_t)t) * sizeof(uint32_t);
+    const size_t smem = ((size_t)(N + 31) / 32 + 1024 + 4 * (size_t)t + 1) * sizeof(uint32_t);
     if (smem > kSampleMaxSmem) return cudaErrorInvalidValue;
     static const cudaError_t a1 = cudaFuncSetAttribute(
         k_lane_sample, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSampleMaxSmem);
@@ -1340,19 +1378,32 @@ cudaError_t launch_lane_syndrome(const pvmvmd_key &key, uint32_t tag, uint64_t i
     const uint32_t ntiles = (N + kLaneTile - 1) / kLaneTile;
     const uint32_t nspans = (N + kExpandSpan - 1) / kExpandSpan;
     if (gy > 65535u || L > 0x7fffffffu) return cudaErrorInvalidValue;
-    uint32_t *agg = aux, *carry = aux + (size_t)ntiles * Lp;
+    uint4 *agg = reinterpret_cast<uint4 *>(aux), *carry = reinterpret_cast<uint4 *>(aux + (size_t)ntiles * Lp);
     uint4 *C4 = reinterpret_cast<uint4 *>(C);
-    k_lane_sample<<<L, 128, smem, s>>>(key, tag, idx0, N, t, sparse_out, S);
-    k_lane_expand<<<dim3((nspans + per_cta - 1) / per_cta, gy), kLaneCta, 0, s>>>(sparse_out, S, t, N, L,
-                                                                                 pi2, v2m, C4);
-    k_lane_tile_sum<<<dim3((ntiles + per_cta - 1) / per_cta, gy), kLaneCta, 0, s>>>(
-        C4, N, L, reinterpret_cast<uint4 *>(agg));
-    k_lane_carry<<<Lp / 4, kCarryThreads, 0, s>>>(reinterpret_cast<const uint4 *>(agg), ntiles, Lp / 4,
-                                                   reinterpret_cast<uint4 *>(carry));
-    k_lane_scan<<<dim3((ntiles + per_cta - 1) / per_cta, gy), kLaneCta, 0, s>>>(
-        C4, N, L, reinterpret_cast<const uint4 *>(carry), v1);
-    k_lane_gather<<<dim3((n + kGatherJ - 1) / kGatherJ, gy), kLaneCta, 0, s>>>(C4, pi1inv, r, n, L,
-                                                                              addend, out);
+    const uint4 *C4c = C4, *aggc = agg, *carryc = carry;
+    const uint32_t Lq = Lp / 4;
+    const uint32_t *stc = sparse_out, *Sc = S;
+    cudaError_t e;
+    void *a0[] = {(void *)&key, &tag, &idx0, &N, &t, &sparse_out, &S};
+    if ((e = launch_pdl((const void *)k_lane_sample, dim3(L), dim3(128), smem, s, a0)) != cudaSuccess) return e;
+    void *a1x[] = {&stc, &Sc, &t, &N, &L, (void *)&pi2, (void *)&v2m, &C4};
+    if ((e = launch_pdl((const void *)k_lane_expand, dim3((nspans + per_cta - 1) / per_cta, gy), dim3(kLaneCta), 0, s,
+                        a1x)) != cudaSuccess)
+        return e;
+    void *a2[] = {&C4c, &N, &L, &agg};
+    if ((e = launch_pdl((const void *)k_lane_tile_sum, dim3((ntiles + per_cta - 1) / per_cta, gy), dim3(kLaneCta), 0,
+                        s, a2)) != cudaSuccess)
+        return e;
+    void *a3[] = {&aggc, (void *)&ntiles, (void *)&Lq, &carry};
+    if ((e = launch_pdl((const void *)k_lane_carry, dim3(Lq), dim3(kCarryThreads), 0, s, a3)) != cudaSuccess) return e;
+    void *a4[] = {&C4, &N, &L, &carryc, (void *)&v1};
+    if ((e = launch_pdl((const void *)k_lane_scan, dim3((ntiles + per_cta - 1) / per_cta, gy), dim3(kLaneCta), 0, s,
+                        a4)) != cudaSuccess)
+        return e;
+    void *a5[] = {&C4c, (void *)&pi1inv, &r, &n, &L, (void *)&addend, &out};
+    if ((e = launch_pdl((const void *)k_lane_gather, dim3((n + kGatherJ - 1) / kGatherJ, gy), dim3(kLaneCta), 0, s,
+                        a5)) != cudaSuccess)
+        return e;
     return cudaGetLastError();
 }
 
