@@ -154,6 +154,10 @@ __global__ void __launch_bounds__(kDecThreads) k_decrypt(const uint32_t *__restr
     // boost mode: no rows to split, every thread owns 4 of 1024 columns
     const int i = kBoost ? ((int)blockIdx.y * kDecThreads + tid) * 4 : (int)blockIdx.y * kDecCols + ct * 4;
     uint32_t pe[4] = {0u, 0u, 0u, 0u};
+    // y_hat of the output columns, loaded now so that its latency overlaps
+    // the row streaming (vector path; the scalar path reads it at the end)
+    uint4 yv = make_uint4(0u, 0u, 0u, 0u);
+    if (vec && (kBoost || grp == 0) && i < m) yv = *reinterpret_cast<const uint4 *>(Yhat + b * m + i);
     if (!kBoost) {
         const uint32_t *stb = st + b * 2 * t_x;
         for (uint32_t j = tid; j < 2 * t_x; j += kDecThreads) sm[j] = stb[j];
@@ -182,9 +186,8 @@ __global__ void __launch_bounds__(kDecThreads) k_decrypt(const uint32_t *__restr
         for (int q2 = 0; q2 < 4; ++q2) pe[q2] = i + q2 < m ? mk[i + q2] : 0u;
     }
     if (vec) {
-        const uint4 y = *reinterpret_cast<const uint4 *>(yh + i);
         *reinterpret_cast<uint4 *>(yo + i) =
-            make_uint4(fsub(y.x, pe[0]), fsub(y.y, pe[1]), fsub(y.z, pe[2]), fsub(y.w, pe[3]));
+            make_uint4(fsub(yv.x, pe[0]), fsub(yv.y, pe[1]), fsub(yv.z, pe[2]), fsub(yv.w, pe[3]));
     } else {
 #pragma unroll
         for (int q2 = 0; q2 < 4; ++q2)
@@ -206,7 +209,7 @@ __global__ void __launch_bounds__(kCheckThreads) k_check(const uint32_t *__restr
                                                         const uint32_t *__restrict__ g,
                                                         const uint32_t *__restrict__ u, uint32_t ell,
                                                         int32_t *__restrict__ accept) {
-    __shared__ uint32_t s_l[kCheckThreads / 32], s_r[kCheckThreads / 32];
+    __shared__ uint32_t s_part[4][kCheckThreads / 32];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const size_t b = blockIdx.x;
     const uint32_t *xh = Xhat + b * K, *yh = Yhat + b * m;
@@ -215,42 +218,59 @@ __global__ void __launch_bounds__(kCheckThreads) k_check(const uint32_t *__restr
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const int n = K > m ? K : m;
     int ok = 1;
-    for (uint32_t q = 0; q < ell; ++q) {
-        const uint32_t *uq = u + (size_t)q * K, *gq = g + (size_t)q * m;
-        uint64_t la = 0, ra = 0;
+    // two repetitions per pass: x_hat and y_hat are read once per pair
+    for (uint32_t q = 0; q < ell; q += 2) {
+        const bool two = q + 1 < ell;
+        const uint32_t *u0 = u + (size_t)q * K, *g0 = g + (size_t)q * m;
+        const uint32_t *u1 = two ? u0 + K : u0, *g1 = two ? g0 + m : g0;
+        uint64_t l0 = 0, l1 = 0, r0 = 0, r1 = 0;
         for (int k0 = tid; k0 < n; k0 += kCheckBatch * kCheckThreads) {
-            uint32_t a[kCheckBatch], x[kCheckBatch], c[kCheckBatch], y[kCheckBatch];
+            uint32_t x[kCheckBatch], y[kCheckBatch], a0[kCheckBatch], a1[kCheckBatch], c0[kCheckBatch],
+                c1[kCheckBatch];
 #pragma unroll
             for (int v = 0; v < kCheckBatch; ++v) {
                 const int k = k0 + v * kCheckThreads;
-                a[v] = k < K ? __ldg(uq + k) : 0u;
-                x[v] = k < K ? xh[k] : 0u;
-                c[v] = k < m ? __ldg(gq + k) : 0u;
-                y[v] = k < m ? yh[k] : 0u;
+                const bool kx = k < K, ky = k < m;
+                x[v] = kx ? xh[k] : 0u;
+                a0[v] = kx ? __ldg(u0 + k) : 0u;
+                a1[v] = kx ? __ldg(u1 + k) : 0u;
+                y[v] = ky ? yh[k] : 0u;
+                c0[v] = ky ? __ldg(g0 + k) : 0u;
+                c1[v] = ky ? __ldg(g1 + k) : 0u;
             }
             // four products of values below q stay below 2^64 with the
             // reduced running sum
 #pragma unroll
             for (int v = 0; v < kCheckBatch; ++v) {
-                la += (uint64_t)a[v] * x[v];
-                ra += (uint64_t)c[v] * y[v];
+                l0 += (uint64_t)a0[v] * x[v];
+                l1 += (uint64_t)a1[v] * x[v];
+                r0 += (uint64_t)c0[v] * y[v];
+                r1 += (uint64_t)c1[v] * y[v];
             }
-            la = fred(la);
-            ra = fred(ra);
+            l0 = fred(l0);
+            l1 = fred(l1);
+            r0 = fred(r0);
+            r1 = fred(r1);
         }
-        const uint32_t l = warp_fsum((uint32_t)la), r = warp_fsum((uint32_t)ra);
+        const uint32_t w0 = warp_fsum((uint32_t)l0), w1 = warp_fsum((uint32_t)l1);
+        const uint32_t w2 = warp_fsum((uint32_t)r0), w3 = warp_fsum((uint32_t)r1);
         if (lane == 0) {
-            s_l[warp] = l;
-            s_r[warp] = r;
+            s_part[0][warp] = w0;
+            s_part[1][warp] = w1;
+            s_part[2][warp] = w2;
+            s_part[3][warp] = w3;
         }
         __syncthreads();
         if (tid == 0) {
-            uint32_t L = 0, R = 0;
+            uint32_t L0 = 0, L1 = 0, R0 = 0, R1 = 0;
             for (int w = 0; w < kCheckThreads / 32; ++w) {
-                L = fadd(L, s_l[w]);
-                R = fadd(R, s_r[w]);
+                L0 = fadd(L0, s_part[0][w]);
+                L1 = fadd(L1, s_part[1][w]);
+                R0 = fadd(R0, s_part[2][w]);
+                R1 = fadd(R1, s_part[3][w]);
             }
-            ok &= (L == R);
+            ok &= (L0 == R0);
+            if (two) ok &= (L1 == R1);
         }
         __syncthreads();
     }

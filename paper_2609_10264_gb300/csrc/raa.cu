@@ -368,7 +368,8 @@ __global__ void __launch_bounds__(256) k_syndrome_gather(const uint32_t *__restr
 // a slice (CTA `rank` owns positions [rank*slice, (rank+1)*slice)) and read
 // each other's through DSMEM.  Steps (App. B, syndrome direction):
 //   sample e (warp 0: support; warp 1: values; every CTA of a cluster draws
-//     the same keystream, rank 0 writes the state), sort the support by rank;
+//     the same keystream, rank 0 writes the state), the ascending support
+//     read off the sampling bitmap by a block-wide scan;
 //   c_i = v2[pi2^-1(i)] * (A e)_{pi2^-1(i)}, the step function (A e)_k found
 //     through a bucket index over the sorted support;
 //   d = A c: a block suffix scan plus the aggregates of later CTAs;
@@ -441,11 +442,42 @@ __global__ void __launch_bounds__(kFusedThreads) k_syndrome_fused(
     else if (warp == 1)
         warp_sample_values(key, tag, 2 * idx + 1, t, words1, suf, lane);
     __syncthreads();
-    for (uint32_t i = tid; i < t; i += kFusedThreads) {  // ascending support by rank
-        const uint32_t v = list[i];
-        uint32_t rk = 0;
-        for (uint32_t j = 0; j < t; ++j) rk += list[j] < v;
-        supp[rk] = v;
+    {
+        // ascending support: the set bits of the sampling bitmap, compacted
+        // with a block-wide exclusive scan of the per-thread bit counts
+        const uint32_t per = (nbw + kFusedThreads - 1) / kFusedThreads;
+        const uint32_t w0 = min(nbw, tid * per), w1 = min(nbw, w0 + per);
+        uint32_t cnt = 0;
+        for (uint32_t w = w0; w < w1; ++w) cnt += __popc(F[w]);
+        uint32_t incl = cnt;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t y = __shfl_up_sync(kFull, incl, o);
+            if (lane >= o) incl += y;
+        }
+        if (lane == 31) s_wsum[warp] = incl;
+        __syncthreads();
+        if (warp == 0) {
+            constexpr int nw = kFusedThreads / 32;
+            const uint32_t wv = lane < nw ? s_wsum[lane] : 0u;
+            uint32_t wi = wv;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const uint32_t y = __shfl_up_sync(kFull, wi, o);
+                if (lane >= o) wi += y;
+            }
+            __syncwarp();
+            if (lane < nw) s_wsum[lane] = wi - wv;
+        }
+        __syncthreads();
+        uint32_t pos = s_wsum[warp] + incl - cnt;
+        for (uint32_t w = w0; w < w1; ++w) {
+            uint32_t bits = F[w];
+            while (bits) {
+                supp[pos++] = w * 32 + (uint32_t)(__ffs(bits) - 1);
+                bits &= bits - 1;
+            }
+        }
     }
     __syncthreads();
     if (warp == 0) {  // suf[j] <- sum_{j' >= j} e_{j'}; suf[t] = 0
