@@ -657,10 +657,11 @@ namespace pv {
 namespace {
 // Challenges (u and g), decrypt and verify: Y = Yhat - P e_x from st, or
 // Y = Yhat - mask_out when mask_out is given (boost mode).  The challenges
-// depend on the key alone, so they run on the context's side stream while
-// the decrypt streams P^T on the caller's stream; the check joins both.
-// When Y overwrites Yhat the check must read Yhat first, and the three
-// steps run in order on the caller's stream.
+// depend on the key alone and the check does not read Y, so both run on the
+// context's side stream while the decrypt streams P^T on the caller's
+// stream; the caller's stream then waits for the side stream.  When Y
+// overwrites Yhat the check must read Yhat first, and the steps run in order
+// on the caller's stream.
 int decode_verify_batch(pvmvmd_ctx *ctx, const void *st_dev, const uint32_t *mask_out_dev,
                         const uint32_t *Xhat_dev, const uint32_t *Yhat_dev, int B,
                         const pvmvmd_key *challenge_key, uint32_t *Y_dev, int32_t *accept_dev,
@@ -701,12 +702,14 @@ int decode_verify_batch(pvmvmd_ctx *ctx, const void *st_dev, const uint32_t *mas
                                Y_dev, s, mask_out_dev));
         return PVMVMD_OK;
     }
+    // the check reads x_hat, y_hat, u and g but not Y, so it follows the
+    // challenges on the side stream, beside the decrypt
+    PV_CUDA(launch_check(Xhat_dev, ctx->K, Yhat_dev, ctx->m, ctx->g, ctx->u, (uint32_t)ctx->ell, B,
+                         accept_dev, ctx->side));
     PV_CUDA(launch_decrypt(ctx->PT, ctx->m, static_cast<const uint32_t *>(st_dev), ctx->t_x, Yhat_dev, B,
                            Y_dev, s, mask_out_dev));
     PV_CUDA(cudaEventRecord(ctx->join, ctx->side));
     PV_CUDA(cudaStreamWaitEvent(s, ctx->join, 0));
-    PV_CUDA(launch_check(Xhat_dev, ctx->K, Yhat_dev, ctx->m, ctx->g, ctx->u, (uint32_t)ctx->ell, B,
-                         accept_dev, s));
     return PVMVMD_OK;
 }
 }  // namespace

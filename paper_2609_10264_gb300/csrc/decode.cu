@@ -154,10 +154,6 @@ __global__ void __launch_bounds__(kDecThreads) k_decrypt(const uint32_t *__restr
     // boost mode: no rows to split, every thread owns 4 of 1024 columns
     const int i = kBoost ? ((int)blockIdx.y * kDecThreads + tid) * 4 : (int)blockIdx.y * kDecCols + ct * 4;
     uint32_t pe[4] = {0u, 0u, 0u, 0u};
-    // y_hat of the output columns, loaded now so that its latency overlaps
-    // the row streaming (vector path; the scalar path reads it at the end)
-    uint4 yv = make_uint4(0u, 0u, 0u, 0u);
-    if (vec && (kBoost || grp == 0) && i < m) yv = *reinterpret_cast<const uint4 *>(Yhat + b * m + i);
     if (!kBoost) {
         const uint32_t *stb = st + b * 2 * t_x;
         for (uint32_t j = tid; j < 2 * t_x; j += kDecThreads) sm[j] = stb[j];
@@ -186,6 +182,10 @@ __global__ void __launch_bounds__(kDecThreads) k_decrypt(const uint32_t *__restr
         for (int q2 = 0; q2 < 4; ++q2) pe[q2] = i + q2 < m ? mk[i + q2] : 0u;
     }
     if (vec) {
+        // y_hat is read here rather than prefetched before the row loop: a
+        // live uint4 across the loop raises the kernel to 70 registers and
+        // four CTAs per SM to three
+        const uint4 yv = *reinterpret_cast<const uint4 *>(yh + i);
         *reinterpret_cast<uint4 *>(yo + i) =
             make_uint4(fsub(yv.x, pe[0]), fsub(yv.y, pe[1]), fsub(yv.z, pe[2]), fsub(yv.w, pe[3]));
     } else {
