@@ -448,7 +448,7 @@ int preprocess_impl(const void *W_dev, bool w16, int m, int K, const pvmvmd_para
         cudaEventCreateWithFlags(&c->join, cudaEventDisableTiming) != cudaSuccess)
         return fail(PVMVMD_E_CUDA);
     if (c->sb >= kLaneMinBatch &&
-        (ctx_alloc(c, &c->S, (size_t)c->sb * (c->t_x + 1)) != cudaSuccess ||
+        (ctx_alloc(c, &c->S, lane_state_words(c->t_x, c->sb)) != cudaSuccess ||
          ctx_alloc(c, &c->laux, lane_aux_words(c->Nx, c->sb)) != cudaSuccess))
         return fail(PVMVMD_E_NOMEM);
 

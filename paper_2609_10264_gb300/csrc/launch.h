@@ -60,11 +60,13 @@ cudaError_t launch_syndrome_fused(const pvmvmd_key &key, uint32_t tag, uint64_t 
                                   bool pdl = false);
 
 // Lane-parallel syndrome for L vectors (vector b uses index idx0 + b, as
-// launch_sample_sparse): sparse_out [L][2t] as there, S [L][t+1] suffix sums
-// of the values, C [N][L rounded up to 4] the intermediate (16-byte
+// launch_sample_sparse): sparse_out [L][2t] as there, S lane_state_words(t,
+// L) words (suffix sums of the values, then a bucket index into the sorted
+// supports), C [N][L rounded up to 4] the intermediate (16-byte
 // aligned), aux lane_aux_words(N, L) words (16-byte aligned); out = addend +
 // G e with out, addend [L][n] (addend may be null or alias out).  Tables:
 // pi2, v2m = v2 R (Montgomery, R = 2^32), v1, pi1inv.
+size_t lane_state_words(uint32_t t, uint32_t L);
 size_t lane_aux_words(uint32_t N, uint32_t L);
 cudaError_t launch_lane_syndrome(const pvmvmd_key &key, uint32_t tag, uint64_t idx0, uint32_t N,
                                  uint32_t t, uint32_t L, const uint32_t *pi2, const uint32_t *v2m,

@@ -865,7 +865,8 @@ __global__ void k_transpose_i8(const int8_t *__restrict__ in, int R, int C, int8
 constexpr int kLaneTile = 32;      // positions per tile (one thread walks them)
 constexpr int kLaneCta = 256;      // threads per lane CTA
 constexpr int kLaneQuadsMax = 64;  // lane quads per CTA (256 lanes)
-constexpr int kExpandSpan = 32;    // positions per expand thread (a multiple of 4)
+constexpr int kExpandSpan = 16;    // positions per expand thread (a multiple of 4)
+constexpr int kLaneBuckets = 256;  // bucket index into each lane's sorted support
 constexpr int kGatherJ = 16;       // outputs per gather CTA
 constexpr int kCarryThreads = 1024;  // tile chunks per lane quad in the carry kernel
 
@@ -878,14 +879,23 @@ __device__ __forceinline__ uint4 fadd4(uint4 a, uint4 b) {
     return make_uint4(fadd(a.x, b.x), fadd(a.y, b.y), fadd(a.z, b.z), fadd(a.w, b.w));
 }
 
+// Positions q << lane_bshift(N), q < kLaneBuckets, cover [0, N).
+__host__ __device__ inline uint32_t lane_bshift(uint32_t N) {
+    uint32_t b = 0;
+    while (b < 31 && ((N - 1) >> b) >= (uint32_t)kLaneBuckets) ++b;
+    return N > 1 ? b : 0u;
+}
+
 // e_b for vector idx0 + blockIdx.x as in k_sample_sparse (warp 0 the
 // support, warp 1 the values), written as st[b] = (ascending support,
-// values), and S[b][j] = sum_{j' >= j} values[j'], S[b][t] = 0.  Everything
-// is computed in shared memory from the key alone; st and S are written
-// after griddepcontrol.wait (a kernel before this one may still read them).
+// values), S[b][j] = sum_{j' >= j} values[j'], S[b][t] = 0, and the bucket
+// index first[b][q] = the first support index at or above position
+// q << lane_bshift(N).  Everything is computed in shared memory from the key
+// alone; st, S and first are written after griddepcontrol.wait (a kernel
+// before this one may still read them).
 __global__ void __launch_bounds__(128) k_lane_sample(pvmvmd_key key, uint32_t tag, uint64_t idx0,
                                                     uint32_t N, uint32_t t, uint32_t *__restrict__ st,
-                                                    uint32_t *__restrict__ S) {
+                                                    uint32_t *__restrict__ S, uint16_t *__restrict__ first) {
     extern __shared__ uint32_t sm[];
     const uint32_t nbw = (N + 31) / 32;
     uint32_t *bitmap = sm;
@@ -929,6 +939,18 @@ __global__ void __launch_bounds__(128) k_lane_sample(pvmvmd_key key, uint32_t ta
         if (lane == 0) suf[t] = 0u;
     }
     __syncthreads();
+    const uint32_t bshift = lane_bshift(N);
+    uint16_t fq[kLaneBuckets / 128];
+#pragma unroll
+    for (int h = 0; h < kLaneBuckets / 128; ++h) {
+        const uint32_t pos = (uint32_t)(tid + 128 * h) << bshift;
+        uint32_t lo = 0, hi = t;
+        while (lo < hi) {
+            const uint32_t mid = (lo + hi) >> 1;
+            if (sorted[mid] < pos) lo = mid + 1; else hi = mid;
+        }
+        fq[h] = (uint16_t)lo;
+    }
     asm volatile("griddepcontrol.wait;" ::: "memory");
     uint32_t *stb = st + (size_t)blockIdx.x * 2 * t;
     uint32_t *Sb = S + (size_t)blockIdx.x * (t + 1);
@@ -937,13 +959,17 @@ __global__ void __launch_bounds__(128) k_lane_sample(pvmvmd_key key, uint32_t ta
         stb[t + j] = vals[j];
     }
     for (uint32_t j = tid; j <= t; j += 128) Sb[j] = suf[j];
+#pragma unroll
+    for (int h = 0; h < kLaneBuckets / 128; ++h)
+        first[(size_t)blockIdx.x * kLaneBuckets + tid + 128 * h] = fq[h];
 }
 
 // C[pi2(k)][b] = v2_k (A e_b)_k: a thread walks kExpandSpan positions k of
 // four lanes in order with a pointer per lane into the sorted support, and
 // writes the four lanes of row pi2(k) with one 16-byte store.
 __global__ void __launch_bounds__(kLaneCta) k_lane_expand(const uint32_t *__restrict__ st,
-                                                         const uint32_t *__restrict__ S, uint32_t t,
+                                                         const uint32_t *__restrict__ S,
+                                                         const uint16_t *__restrict__ first, uint32_t t,
                                                          uint32_t N, uint32_t L,
                                                          const uint32_t *__restrict__ pi2,
                                                          const uint32_t *__restrict__ v2m,
@@ -962,14 +988,17 @@ __global__ void __launch_bounds__(kLaneCta) k_lane_expand(const uint32_t *__rest
         cur[q] = 0u;
         j[q] = 0u;
         if (b < L) {
+            // first support index with s_j >= k0: from the bucket of k0, then
+            // past the few supports between the bucket's start and k0
             const uint32_t *supp = st + (size_t)b * 2 * t;
-            uint32_t lo = 0, hi = t;  // first support index with s_j >= k0
-            while (lo < hi) {
-                const uint32_t mid = (lo + hi) >> 1;
-                if (__ldg(supp + mid) < k0) lo = mid + 1; else hi = mid;
+            uint32_t lo = __ldg(first + (size_t)b * kLaneBuckets + (k0 >> lane_bshift(N)));
+            uint32_t nx = lo < t ? __ldg(supp + lo) : 0xffffffffu;
+            while (nx < k0) {
+                ++lo;
+                nx = lo < t ? __ldg(supp + lo) : 0xffffffffu;
             }
             j[q] = lo;
-            next[q] = lo < t ? __ldg(supp + lo) : 0xffffffffu;
+            next[q] = nx;
             cur[q] = __ldg(S + (size_t)b * (t + 1) + lo);
         }
     }
@@ -1388,6 +1417,10 @@ cudaError_t launch_pdl(const void *fn, dim3 grid, dim3 block, size_t smem, cudaS
 }
 }  // namespace
 
+size_t lane_state_words(uint32_t t, uint32_t L) {
+    return (size_t)L * (t + 1) + (size_t)L * kLaneBuckets / 2;
+}
+
 size_t lane_aux_words(uint32_t N, uint32_t L) {
     return 2 * (size_t)((N + kLaneTile - 1) / kLaneTile) * lane_pad(L);
 }
@@ -1415,10 +1448,13 @@ cudaError_t launch_lane_syndrome(const pvmvmd_key &key, uint32_t tag, uint64_t i
     const uint4 *C4c = C4, *aggc = agg, *carryc = carry;
     const uint32_t Lq = Lp / 4;
     const uint32_t *stc = sparse_out, *Sc = S;
+    // S holds the suffix sums [L][t+1], then the bucket index [L][kLaneBuckets] (uint16)
+    uint16_t *first = reinterpret_cast<uint16_t *>(S + (size_t)L * (t + 1));
+    const uint16_t *fc = first;
     cudaError_t e;
-    void *a0[] = {(void *)&key, &tag, &idx0, &N, &t, &sparse_out, &S};
+    void *a0[] = {(void *)&key, &tag, &idx0, &N, &t, &sparse_out, &S, &first};
     if ((e = launch_pdl((const void *)k_lane_sample, dim3(L), dim3(128), smem, s, a0)) != cudaSuccess) return e;
-    void *a1x[] = {&stc, &Sc, &t, &N, &L, (void *)&pi2, (void *)&v2m, &C4};
+    void *a1x[] = {&stc, &Sc, &fc, &t, &N, &L, (void *)&pi2, (void *)&v2m, &C4};
     if ((e = launch_pdl((const void *)k_lane_expand, dim3((nspans + per_cta - 1) / per_cta, gy), dim3(kLaneCta), 0, s,
                         a1x)) != cudaSuccess)
         return e;
