@@ -170,6 +170,7 @@ struct CodeDev {
     uint32_t *pi1 = nullptr, *pi2 = nullptr, *v1 = nullptr, *v2 = nullptr;
     uint32_t *pi1inv = nullptr, *pi2inv = nullptr, *v2p = nullptr;
     uint32_t *v2m = nullptr, *v1pm = nullptr;  // Montgomery-scaled v2 and v1 o pi1^-1
+    uint32_t *v1m = nullptr;                   // Montgomery-scaled v1
 };
 
 }  // namespace
@@ -218,7 +219,7 @@ cudaError_t ctx_alloc(Ctx *c, T **p, size_t count) {
 
 template <typename Ctx>
 int upload_code(Ctx *c, CodeDev &d, const pvmvmd_key &key, int which, uint32_t N, cudaStream_t s) {
-    std::vector<uint32_t> pi1(N), pi2(N), v1(N), v2(N), pi1inv(N), pi2inv(N), v2p(N), v2m(N), v1pm(N);
+    std::vector<uint32_t> pi1(N), pi2(N), v1(N), v2(N), pi1inv(N), pi2inv(N), v2p(N), v2m(N), v1pm(N), v1m(N);
     sample_code_host(key, which, N, pi1.data(), pi2.data(), v1.data(), v2.data());
     for (uint32_t j = 0; j < N; ++j) {
         pi1inv[pi1[j]] = j;
@@ -228,10 +229,11 @@ int upload_code(Ctx *c, CodeDev &d, const pvmvmd_key &key, int which, uint32_t N
         v2p[i] = v2[pi2inv[i]];
         v2m[i] = to_mont(v2[i]);
         v1pm[i] = to_mont(v1[pi1inv[i]]);
+        v1m[i] = to_mont(v1[i]);
     }
-    uint32_t **dst[9] = {&d.pi1, &d.pi2, &d.v1, &d.v2, &d.pi1inv, &d.pi2inv, &d.v2p, &d.v2m, &d.v1pm};
-    const std::vector<uint32_t> *src[9] = {&pi1, &pi2, &v1, &v2, &pi1inv, &pi2inv, &v2p, &v2m, &v1pm};
-    for (int i = 0; i < 9; ++i) {
+    uint32_t **dst[10] = {&d.pi1, &d.pi2, &d.v1, &d.v2, &d.pi1inv, &d.pi2inv, &d.v2p, &d.v2m, &d.v1pm, &d.v1m};
+    const std::vector<uint32_t> *src[10] = {&pi1, &pi2, &v1, &v2, &pi1inv, &pi2inv, &v2p, &v2m, &v1pm, &v1m};
+    for (int i = 0; i < 10; ++i) {
         PV_CUDA(ctx_alloc(c, dst[i], N));
         PV_CUDA(cudaMemcpyAsync(*dst[i], src[i]->data(), (size_t)N * 4, cudaMemcpyHostToDevice, s));
     }
@@ -577,7 +579,7 @@ int encode_batch(pvmvmd_ctx *ctx, const uint32_t *X_dev, int B, const pvmvmd_key
         for (int b0 = 0; b0 < B; b0 += ctx->sb) {
             const uint32_t L = (uint32_t)(B - b0 < ctx->sb ? B - b0 : ctx->sb);
             PV_CUDA(launch_lane_syndrome(*key, kTagMask, (uint64_t)b0, ctx->Nx, ctx->t_x, L, d.pi2,
-                                         d.v2m, d.v1, d.pi1inv, ctx->K, ctx->rate,
+                                         d.v2m, d.v1m, d.pi1inv, ctx->K, ctx->rate,
                                          stp + (size_t)b0 * 2 * ctx->t_x, ctx->S, ctx->F, ctx->laux,
                                          X_dev ? X_dev + (size_t)b0 * ctx->K : nullptr,
                                          Xhat_dev + (size_t)b0 * ctx->K, s));

@@ -65,12 +65,12 @@ cudaError_t launch_syndrome_fused(const pvmvmd_key &key, uint32_t tag, uint64_t 
 // supports), C [N][L rounded up to 4] the intermediate (16-byte
 // aligned), aux lane_aux_words(N, L) words (16-byte aligned); out = addend +
 // G e with out, addend [L][n] (addend may be null or alias out).  Tables:
-// pi2, v2m = v2 R (Montgomery, R = 2^32), v1, pi1inv.
+// pi2, v2m = v2 R and v1m = v1 R (Montgomery, R = 2^32), pi1inv.
 size_t lane_state_words(uint32_t t, uint32_t L);
 size_t lane_aux_words(uint32_t N, uint32_t L);
 cudaError_t launch_lane_syndrome(const pvmvmd_key &key, uint32_t tag, uint64_t idx0, uint32_t N,
                                  uint32_t t, uint32_t L, const uint32_t *pi2, const uint32_t *v2m,
-                                 const uint32_t *v1, const uint32_t *pi1inv, uint32_t n, uint32_t r,
+                                 const uint32_t *v1m, const uint32_t *pi1inv, uint32_t n, uint32_t r,
                                  uint32_t *sparse_out, uint32_t *S, uint32_t *C, uint32_t *aux,
                                  const uint32_t *addend, uint32_t *out, cudaStream_t s);
 

@@ -862,7 +862,8 @@ __global__ void k_transpose_i8(const int8_t *__restrict__ in, int R, int C, int8
 // completion.  Early launches of the large grids held SM slots with waiting
 // CTAs and were slower (K = 28672, B = 256: 341 against 307 us).
 // -----------------------------------------------------------------------------
-constexpr int kLaneTile = 32;      // positions per tile (one thread walks them)
+constexpr int kLaneTileMin = 32;   // positions per tile (one thread walks them):
+constexpr int kLaneTileMax = 128;  // the launch picks 32, 64 or 128
 constexpr int kLaneCta = 256;      // threads per lane CTA
 constexpr int kLaneQuadsMax = 64;  // lane quads per CTA (256 lanes)
 constexpr int kExpandSpan = 16;    // positions per expand thread (a multiple of 4)
@@ -1037,14 +1038,14 @@ __global__ void __launch_bounds__(kLaneCta) k_lane_expand(const uint32_t *__rest
 }
 
 // agg[tau][b] = sum over the tile's positions of C[i][b].
-__global__ void __launch_bounds__(kLaneCta) k_lane_tile_sum(const uint4 *__restrict__ C, uint32_t N,
+__global__ void __launch_bounds__(kLaneCta) k_lane_tile_sum(const uint4 *__restrict__ C, uint32_t N, uint32_t tile,
                                                            uint32_t L, uint4 *__restrict__ agg) {
     asm volatile("griddepcontrol.wait;" ::: "memory");  // inputs come from the kernel before
-    const uint32_t cols = lane_cols(L), Lq = lane_pad(L) / 4, ntiles = (N + kLaneTile - 1) / kLaneTile;
+    const uint32_t cols = lane_cols(L), Lq = lane_pad(L) / 4, ntiles = (N + tile - 1) / tile;
     const uint32_t g = blockIdx.y * cols + threadIdx.x % cols;
     const uint32_t tau = blockIdx.x * (kLaneCta / cols) + threadIdx.x / cols;
     if (g >= Lq || tau >= ntiles) return;
-    const uint32_t i0 = tau * kLaneTile, i1 = min(N, i0 + kLaneTile);
+    const uint32_t i0 = tau * tile, i1 = min(N, i0 + tile);
     uint4 sum = make_uint4(0u, 0u, 0u, 0u);
     for (uint32_t i = i0; i < i1; i += 8) {
         uint4 v[8];
@@ -1123,16 +1124,17 @@ __global__ void __launch_bounds__(kCarryThreads) k_lane_carry(const uint4 *__res
     }
 }
 
-// In place: C[i][b] <- v1_i (carry[tau][b] + sum_{i' >= i in tile tau} C[i'][b]).
-__global__ void __launch_bounds__(kLaneCta) k_lane_scan(uint4 *__restrict__ C, uint32_t N, uint32_t L,
+// In place: C[i][b] <- v1_i (carry[tau][b] + sum_{i' >= i in tile tau} C[i'][b]),
+// with v1m = v1 R (Montgomery, R = 2^32) so that each product is one REDC.
+__global__ void __launch_bounds__(kLaneCta) k_lane_scan(uint4 *__restrict__ C, uint32_t N, uint32_t tile, uint32_t L,
                                                        const uint4 *__restrict__ carry,
-                                                       const uint32_t *__restrict__ v1) {
+                                                       const uint32_t *__restrict__ v1m) {
     asm volatile("griddepcontrol.wait;" ::: "memory");  // inputs come from the kernel before
-    const uint32_t cols = lane_cols(L), Lq = lane_pad(L) / 4, ntiles = (N + kLaneTile - 1) / kLaneTile;
+    const uint32_t cols = lane_cols(L), Lq = lane_pad(L) / 4, ntiles = (N + tile - 1) / tile;
     const uint32_t g = blockIdx.y * cols + threadIdx.x % cols;
     const uint32_t tau = blockIdx.x * (kLaneCta / cols) + threadIdx.x / cols;
     if (g >= Lq || tau >= ntiles) return;
-    const uint32_t i0 = tau * kLaneTile, i1 = min(N, i0 + kLaneTile);
+    const uint32_t i0 = tau * tile, i1 = min(N, i0 + tile);
     uint4 run = carry[(size_t)tau * Lq + g];
     for (uint32_t hi = i1; hi > i0;) {
         const uint32_t cnt = hi - i0 < 8u ? hi - i0 : 8u;  // positions hi-1 .. hi-cnt
@@ -1143,9 +1145,10 @@ __global__ void __launch_bounds__(kLaneCta) k_lane_scan(uint4 *__restrict__ C, u
 #pragma unroll
         for (int u = 0; u < 8; ++u) {
             if ((uint32_t)u < cnt) {
-                const uint32_t i = hi - 1 - u, w = __ldg(v1 + i);
+                const uint32_t i = hi - 1 - u, w = __ldg(v1m + i);
                 run = fadd4(run, v[u]);
-                C[(size_t)i * Lq + g] = make_uint4(fmul(w, run.x), fmul(w, run.y), fmul(w, run.z), fmul(w, run.w));
+                C[(size_t)i * Lq + g] = make_uint4(fmul_mont(run.x, w), fmul_mont(run.y, w), fmul_mont(run.z, w),
+                                                   fmul_mont(run.w, w));
             }
         }
         hi -= cnt;
@@ -1422,12 +1425,12 @@ size_t lane_state_words(uint32_t t, uint32_t L) {
 }
 
 size_t lane_aux_words(uint32_t N, uint32_t L) {
-    return 2 * (size_t)((N + kLaneTile - 1) / kLaneTile) * lane_pad(L);
+    return 2 * (size_t)((N + kLaneTileMin - 1) / kLaneTileMin) * lane_pad(L);
 }
 
 cudaError_t launch_lane_syndrome(const pvmvmd_key &key, uint32_t tag, uint64_t idx0, uint32_t N,
                                  uint32_t t, uint32_t L, const uint32_t *pi2, const uint32_t *v2m,
-                                 const uint32_t *v1, const uint32_t *pi1inv, uint32_t n, uint32_t r,
+                                 const uint32_t *v1m, const uint32_t *pi1inv, uint32_t n, uint32_t r,
                                  uint32_t *sparse_out, uint32_t *S, uint32_t *C, uint32_t *aux,
                                  const uint32_t *addend, uint32_t *out, cudaStream_t s) {
     if (L == 0) return cudaSuccess;
@@ -1440,7 +1443,16 @@ cudaError_t launch_lane_syndrome(const pvmvmd_key &key, uint32_t tag, uint64_t i
         return cudaErrorInvalidValue;
     const uint32_t Lp = lane_pad(L), cols = lane_cols(L), per_cta = kLaneCta / cols;
     const unsigned gy = (Lp / 4 + cols - 1) / cols;
-    const uint32_t ntiles = (N + kLaneTile - 1) / kLaneTile;
+    // tiles of 32 positions, or 64 / 128 when the tile-sum and scan grids
+    // still hold two CTAs of threads per SM: longer tiles shorten the carry
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    uint32_t tile = kLaneTileMin;
+    while (tile < (uint32_t)kLaneTileMax &&
+           (uint64_t)((N + 2 * tile - 1) / (2 * tile)) * (lane_pad(L) / 4) >= (uint64_t)2 * sms * kLaneCta)
+        tile *= 2;
+    const uint32_t ntiles = (N + tile - 1) / tile;
     const uint32_t nspans = (N + kExpandSpan - 1) / kExpandSpan;
     if (gy > 65535u || L > 0x7fffffffu) return cudaErrorInvalidValue;
     uint4 *agg = reinterpret_cast<uint4 *>(aux), *carry = reinterpret_cast<uint4 *>(aux + (size_t)ntiles * Lp);
@@ -1458,13 +1470,13 @@ cudaError_t launch_lane_syndrome(const pvmvmd_key &key, uint32_t tag, uint64_t i
     if ((e = launch_pdl((const void *)k_lane_expand, dim3((nspans + per_cta - 1) / per_cta, gy), dim3(kLaneCta), 0, s,
                         a1x)) != cudaSuccess)
         return e;
-    void *a2[] = {&C4c, &N, &L, &agg};
+    void *a2[] = {&C4c, &N, &tile, &L, &agg};
     if ((e = launch_pdl((const void *)k_lane_tile_sum, dim3((ntiles + per_cta - 1) / per_cta, gy), dim3(kLaneCta), 0,
                         s, a2)) != cudaSuccess)
         return e;
     void *a3[] = {&aggc, (void *)&ntiles, (void *)&Lq, &carry};
     if ((e = launch_pdl((const void *)k_lane_carry, dim3(Lq), dim3(kCarryThreads), 0, s, a3)) != cudaSuccess) return e;
-    void *a4[] = {&C4, &N, &L, &carryc, (void *)&v1};
+    void *a4[] = {&C4, &N, &tile, &L, &carryc, (void *)&v1m};
     if ((e = launch_pdl((const void *)k_lane_scan, dim3((ntiles + per_cta - 1) / per_cta, gy), dim3(kLaneCta), 0, s,
                         a4)) != cudaSuccess)
         return e;
