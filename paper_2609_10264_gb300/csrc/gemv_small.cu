@@ -58,16 +58,47 @@ constexpr int kNbMaxJobs = 32;
 
 struct NbJob {
     const int8_t *W;
-    const uint32_t *xhat;  // vector v at xhat + v * ldx
-    uint32_t *y;           // vector v at y + v * ldy
+    const uint32_t *planes;  // row (p, v) of the segment at planes + (p * kNbVec + v) * ldp
+    uint32_t *y;             // vector v at y + v * ldy
     int m, K, nb, accumulate;
-    size_t ldw, ldx, ldy;
+    size_t ldw, ldp, ldy;    // ldp in 32-bit words
 };
 struct NbArgs {
     int count;
     long long base[kNbMaxJobs + 1];
     NbJob job[kNbMaxJobs];
 };
+
+// Digit planes of the batch, once per call: planes[j][p][v][k] (int8) is
+// digit p of centred x_hat[4j + v][k]; vectors past B are zero.  One thread
+// per four consecutive K-elements of one vector.
+__global__ void __launch_bounds__(256) k_nb_planes(const uint32_t *__restrict__ Xhat, int B, int K, int Bp,
+                                                  uint32_t *__restrict__ planes) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");  // x_hat comes from the kernel before
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    const size_t gid = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const size_t per_vec = (size_t)K / 4;
+    if (gid >= (size_t)Bp * per_vec) return;
+    const int b = (int)(gid / per_vec), q4 = (int)(gid % per_vec);
+    uint32_t p[4] = {0u, 0u, 0u, 0u};
+    if (b < B) {
+        const uint4 xv = __ldg(reinterpret_cast<const uint4 *>(Xhat + (size_t)b * K) + q4);
+        const uint32_t xs[4] = {xv.x, xv.y, xv.z, xv.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            int d0, d1, d2, d3;
+            limb_split(xs[e], d0, d1, d2, d3);
+            p[0] |= (uint32_t)(d0 & 0xff) << (8 * e);
+            p[1] |= (uint32_t)(d1 & 0xff) << (8 * e);
+            p[2] |= (uint32_t)(d2 & 0xff) << (8 * e);
+            p[3] |= (uint32_t)(d3 & 0xff) << (8 * e);
+        }
+    }
+    const int j = b / kNbVec, v = b % kNbVec;
+    uint32_t *dst = planes + (size_t)j * 4 * kNbVec * per_vec;
+#pragma unroll
+    for (int d = 0; d < 4; ++d) dst[((size_t)d * kNbVec + v) * per_vec + q4] = p[d];
+}
 
 template <int ROWS, int UNROLL>
 __global__ void __launch_bounds__(kMultiThreads, 2) k_gemv_nb(const __grid_constant__ NbArgs args) {
@@ -108,29 +139,26 @@ __global__ void __launch_bounds__(kMultiThreads, 2) k_gemv_nb(const __grid_const
         if (g < ngroups) issue(g, lane);
 
         __syncthreads();  // the previous job's planes are no longer read
-        // planes: [plane p][vector v][K/4 words]; vectors past nb are zero
+        // planes: [plane p][vector v][K/4 words], copied from the planes the
+        // call built once; rows of vectors past nb are zero there
         uint32_t *planes = reinterpret_cast<uint32_t *>(s_planes);
-        const int pstride = K / 4;
-        for (int idx = tid; idx < kNbVec * pstride; idx += kMultiThreads) {
-            const int v = idx / pstride, q4 = idx % pstride;
-            uint32_t p0 = 0, p1 = 0, p2 = 0, p3 = 0;
-            if (v < job.nb) {
-                const uint4 xv = __ldg(reinterpret_cast<const uint4 *>(job.xhat + (size_t)v * job.ldx) + q4);
-                const uint32_t xs[4] = {xv.x, xv.y, xv.z, xv.w};
+        const int pstride = K / 4, q16 = K / 16;  // words and 16-byte chunks per row
+        for (int idx0 = tid; idx0 < 4 * kNbVec * q16; idx0 += 4 * kMultiThreads) {
+            uint4 c[4];
 #pragma unroll
-                for (int b = 0; b < 4; ++b) {
-                    int d0, d1, d2, d3;
-                    limb_split(xs[b], d0, d1, d2, d3);
-                    p0 |= (uint32_t)(d0 & 0xff) << (8 * b);
-                    p1 |= (uint32_t)(d1 & 0xff) << (8 * b);
-                    p2 |= (uint32_t)(d2 & 0xff) << (8 * b);
-                    p3 |= (uint32_t)(d3 & 0xff) << (8 * b);
-                }
+            for (int u = 0; u < 4; ++u) {
+                const int idx = idx0 + u * kMultiThreads;
+                const int row = idx / q16, c4 = idx % q16;
+                c[u] = idx < 4 * kNbVec * q16
+                           ? __ldg(reinterpret_cast<const uint4 *>(job.planes + (size_t)row * job.ldp) + c4)
+                           : make_uint4(0u, 0u, 0u, 0u);
             }
-            planes[(0 * kNbVec + v) * pstride + q4] = p0;
-            planes[(1 * kNbVec + v) * pstride + q4] = p1;
-            planes[(2 * kNbVec + v) * pstride + q4] = p2;
-            planes[(3 * kNbVec + v) * pstride + q4] = p3;
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int idx = idx0 + u * kMultiThreads;
+                if (idx < 4 * kNbVec * q16)
+                    reinterpret_cast<uint4 *>(planes)[(idx / q16) * (pstride / 4) + idx % q16] = c[u];
+            }
         }
         __syncthreads();
 
@@ -236,11 +264,59 @@ cudaError_t run_gemv_nb(const NbJob *jobs, int count, cudaStream_t s) {
     return cudaLaunchKernelEx(&cfg, k_gemv_nb<2, 2>, args);
 }
 
+// Per-device buffer for the digit planes (grown when a call needs more;
+// growing waits for the device, since the old buffer may still be read).
+cudaError_t planes_scratch(size_t need, uint32_t **out) {
+    struct Scratch {
+        uint32_t *ptr = nullptr;
+        size_t bytes = 0;
+    };
+    static Scratch per_dev[64];
+    static std::mutex mu;
+    std::lock_guard<std::mutex> lock(mu);
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    Scratch &sc = per_dev[dev];
+    if (sc.bytes < need) {
+        if (sc.ptr) {
+            if ((e = cudaDeviceSynchronize()) != cudaSuccess) return e;
+            cudaFree(sc.ptr);
+            sc.ptr = nullptr;
+            sc.bytes = 0;
+        }
+        if ((e = cudaMalloc(&sc.ptr, need)) != cudaSuccess) return e;
+        sc.bytes = need;
+    }
+    *out = sc.ptr;
+    return cudaSuccess;
+}
+
 }  // namespace
 
 cudaError_t launch_gemv_small_batch(const int8_t *W, int m, int K, const uint32_t *Xhat, int B,
                                     uint32_t *Yhat, cudaStream_t s) {
     if (m <= 0 || K <= 0 || B <= 0) return cudaSuccess;
+    // digit planes of all vectors once: [job][plane][vector][K] bytes
+    const int Bp = (B + kNbVec - 1) / kNbVec * kNbVec;
+    const size_t row_words = (size_t)K / 4, job_words = 4 * kNbVec * row_words;
+    uint32_t *planes = nullptr;
+    cudaError_t e = planes_scratch((size_t)Bp / kNbVec * job_words * sizeof(uint32_t), &planes);
+    if (e != cudaSuccess) return e;
+    {
+        const size_t threads = (size_t)Bp * row_words;
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3((unsigned)((threads + 255) / 256), 1, 1);
+        cfg.blockDim = dim3(256, 1, 1);
+        cfg.stream = s;
+        cudaLaunchAttribute attrs[1];
+        attrs[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attrs[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attrs;
+        cfg.numAttrs = 1;
+        if ((e = cudaLaunchKernelEx(&cfg, k_nb_planes, Xhat, B, K, Bp, planes)) != cudaSuccess) return e;
+    }
     // groups of four vectors; K in segments whose planes fit shared memory,
     // later segments accumulating
     std::vector<NbJob> jobs;
@@ -250,20 +326,20 @@ cudaError_t launch_gemv_small_batch(const int8_t *W, int m, int K, const uint32_
         for (int b0 = 0; b0 < B; b0 += kNbVec) {
             NbJob j;
             j.W = W + k0;
-            j.xhat = Xhat + (size_t)b0 * K + k0;
+            j.planes = planes + (size_t)(b0 / kNbVec) * job_words + (size_t)k0 / 4;
             j.y = Yhat + (size_t)b0 * m;
             j.m = m;
             j.K = kl;
             j.nb = B - b0 < kNbVec ? B - b0 : kNbVec;
             j.accumulate = k0 > 0;
             j.ldw = (size_t)K;
-            j.ldx = (size_t)K;
+            j.ldp = row_words;
             j.ldy = (size_t)m;
             jobs.push_back(j);
         }
         for (size_t a = 0; a < jobs.size(); a += kNbMaxJobs) {
             const int n = (int)std::min(jobs.size() - a, (size_t)kNbMaxJobs);
-            cudaError_t e = run_gemv_nb(jobs.data() + a, n, s);
+            e = run_gemv_nb(jobs.data() + a, n, s);
             if (e != cudaSuccess) return e;
         }
     }
