@@ -379,6 +379,7 @@ __global__ void __launch_bounds__(256) k_syndrome_gather(const uint32_t *__restr
 constexpr int kFusedThreads = 1024;
 constexpr int kFusedBuckets = 512;   // index over the sorted support
 constexpr int kFusedBatch = 16;      // loads in flight per thread
+constexpr int kFusedBatch1 = 8;      // the same in the single-CTA scatter
 
 __device__ __forceinline__ uint32_t fpad(uint32_t i) { return i + (i >> 5); }  // bank padding
 
@@ -499,40 +500,41 @@ __global__ void __launch_bounds__(kFusedThreads) k_syndrome_fused(
         if (lane == 0) suf[t] = 0;
     }
     if (C == 1) {
-        // ---- the whole vector in this CTA.  Thread tid walks positions k of
-        // its own range in order, so (A e)_k is a running pointer into the
-        // sorted support, and scatters c_{pi2(k)} = v2_k (A e)_k.
+        // ---- the whole vector in this CTA: c_{pi2(k)} = v2_k (A e)_k,
+        // scattered into the slice.  Positions are interleaved over the
+        // threads (k = u * 1024 + tid), so the table loads are coalesced and
+        // kFusedBatch1 of them are in flight per thread; (A e)_k is found
+        // from a bucket index into the sorted support.
+        int bshift = 0;
+        while ((N >> bshift) > (uint32_t)kFusedBuckets - 1) ++bshift;
+        const uint32_t nbk = (N >> bshift) + 1;
+        for (uint32_t b = tid; b < nbk; b += kFusedThreads) {
+            const uint32_t start = b << bshift;
+            uint32_t lo = 0, hi = t;
+            while (lo < hi) {
+                const uint32_t mid = (lo + hi) >> 1;
+                if (supp[mid] < start) lo = mid + 1; else hi = mid;
+            }
+            s_first[b] = lo;
+        }
         __syncthreads();
         const uint32_t items = slice / kFusedThreads;
         for (uint32_t i = N + tid; i < slice; i += kFusedThreads) F[fpad(i)] = 0u;  // padding
-        const uint32_t k0 = tid * items, k1 = min(N, k0 + items);
-        uint32_t j = 0;
-        if (k0 < k1) {
-            uint32_t lo = 0, hi = t;  // first support index >= k0
-            while (lo < hi) {
-                const uint32_t mid = (lo + hi) >> 1;
-                if (supp[mid] < k0) lo = mid + 1; else hi = mid;
-            }
-            j = lo;
-        }
-        for (uint32_t k = k0; k < k1; k += 4) {
-            uint32_t pk[4], vk[4];
-            if (k + 4 <= k1 && (k & 3) == 0) {
-                const uint4 a = __ldg(reinterpret_cast<const uint4 *>(pi2 + k));
-                const uint4 b = __ldg(reinterpret_cast<const uint4 *>(v2m + k));
-                pk[0] = a.x; pk[1] = a.y; pk[2] = a.z; pk[3] = a.w;
-                vk[0] = b.x; vk[1] = b.y; vk[2] = b.z; vk[3] = b.w;
-            } else {
+        for (uint32_t u0 = 0; u0 < items; u0 += kFusedBatch1) {
+            uint32_t pk[kFusedBatch1], vk[kFusedBatch1];
 #pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                    pk[u] = k + u < k1 ? __ldg(pi2 + k + u) : 0u;
-                    vk[u] = k + u < k1 ? __ldg(v2m + k + u) : 0u;
-                }
+            for (int u = 0; u < kFusedBatch1; ++u) {
+                const uint32_t k = (u0 + u) * kFusedThreads + tid;
+                const bool ok = u0 + u < items && k < N;
+                pk[u] = ok ? __ldg(pi2 + k) : 0u;
+                vk[u] = ok ? __ldg(v2m + k) : 0u;
             }
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                if (k + u < k1) {
-                    while (j < t && supp[j] < k + u) ++j;
+            for (int u = 0; u < kFusedBatch1; ++u) {
+                const uint32_t k = (u0 + u) * kFusedThreads + tid;
+                if (u0 + u < items && k < N) {
+                    uint32_t j = s_first[k >> bshift];
+                    while (j < t && supp[j] < k) ++j;
                     F[fpad(pk[u])] = fmul_mont(suf[j], vk[u]);
                 }
             }

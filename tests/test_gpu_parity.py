@@ -434,6 +434,27 @@ def test_config5_70b(pv, wl, name):
     _batched_pipeline_sampled(pv, W, 256, seed=500 + len(name), n_rows=12, n_verify=1)
 
 
+@pytest.mark.parametrize("L", [256, 128])
+def test_lane_encode_long_tiles(pv, wl, L):
+    """The lane encode on a long code (K = 28672, N_x = 229376) with every
+    vector in one lane group: on a 152-SM GB300, 256 lanes run the tile sums
+    and the scan over tiles of 128 positions, 128 lanes over tiles of 64;
+    every x_hat and state equals the oracle."""
+    W = wl.weights_uniform(24, 28672, 31)
+    x = wl.int8_vectors(L, 28672, 32)
+    X = field(x)
+    ctx = pv.pvmvmd_preprocess(to_dev(W), key=33, params=_params(pv, scratch_batch=L))
+    pp = oracle.PublicParams(W, oracle.key_from_seed(33), with_tables=False)
+    Xh, st = pv.pvmvmd_encode(ctx, to_dev(X), key=34)
+    Xh_h, st_h = pv.as_u32(Xh), pv.as_u32(st)
+    for b in range(L):
+        xh_o, s_o, v_o = pp.encrypt(X[b], oracle.key_from_seed(34), b)
+        assert np.array_equal(Xh_h[b], xh_o), b
+        assert np.array_equal(st_h[b], np.concatenate([s_o, v_o])), b
+    assert pv.pvmvmd_device_status() == 0
+    ctx.destroy()
+
+
 @pytest.mark.parametrize("m,K,B", [(4096, 2560, 8), (37, 6144 + 96, 5), (300, 16, 2), (2560, 9728, 16),
                                    (1000, 4096, 3)])
 def test_small_batch_server_product(pv, wl, m, K, B):
