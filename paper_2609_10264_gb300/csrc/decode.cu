@@ -127,19 +127,21 @@ __device__ __forceinline__ void pe_cols(const uint32_t *__restrict__ PT, int m, 
 }
 
 // ---------------------------------------------------------------------------
-// Decrypt: Y_b = y_hat_b - P e_x,b.  A CTA owns 256 columns of one vector
-// (64 column threads x 4 columns) and splits the t_x rows of P^T over
-// kDecGroups row groups, so each thread streams about t_x / 4 row segments
-// (a few rounds of 8 loads in flight) and the grid holds many short CTAs
-// whatever m and B are.  The groups' partial sums meet in shared memory.
+// Decrypt: Y_b = y_hat_b - P e_x,b.  A CTA owns 512 columns of one vector
+// (128 column threads x 4 columns, so each row of P^T is read in 2 KiB
+// segments) and splits the t_x rows over kDecGroups = 2 row groups, so each
+// thread streams about t_x / 2 row segments (rounds of 8 loads in flight)
+// and the grid holds many short CTAs whatever m and B are.  The groups'
+// partial sums meet in shared memory.  (256 columns and 4 groups, or 1024
+// columns and 1 group, were 6 and 13 % slower at m = K = 8192, B = 256.)
 // In boost mode (Sec. 7.2) P e_x,b was prepared ahead: Y_b = y_hat_b - mask_b.
 // The grid runs vectors fastest (blockIdx.x = b, blockIdx.y = column block),
 // so the CTAs in flight share a few column blocks and a row of P^T drawn by
 // several vectors' supports is read from HBM once and then from L2.
 // ---------------------------------------------------------------------------
-constexpr int kDecGroups = 4;
-constexpr int kDecColThreads = kDecThreads / kDecGroups;  // 64
-constexpr int kDecCols = 4 * kDecColThreads;              // 256 columns per CTA
+constexpr int kDecGroups = 2;
+constexpr int kDecColThreads = kDecThreads / kDecGroups;  // 128
+constexpr int kDecCols = 4 * kDecColThreads;              // 512 columns per CTA
 
 template <bool kBoost>
 __global__ void __launch_bounds__(kDecThreads) k_decrypt(const uint32_t *__restrict__ PT, int m,
@@ -147,7 +149,7 @@ __global__ void __launch_bounds__(kDecThreads) k_decrypt(const uint32_t *__restr
                                                         const uint32_t *Yhat, uint32_t *Y,
                                                         const uint32_t *__restrict__ mask, bool vec) {
     extern __shared__ uint32_t sm[];  // support[t_x], values[t_x]
-    __shared__ uint4 s_part[kDecGroups - 1][kDecColThreads];
+    __shared__ uint4 s_part[kDecGroups > 1 ? kDecGroups - 1 : 1][kDecColThreads];
     const int tid = threadIdx.x;
     const size_t b = blockIdx.x;
     const int grp = tid / kDecColThreads, ct = tid % kDecColThreads;
