@@ -856,8 +856,8 @@ __global__ void k_transpose_i8(const int8_t *__restrict__ in, int R, int C, int8
 //   out[b][j] = addend[b][j] + sum_{c<r} C[pi1^-1(r j + c)][b]
 //                                                   (k_lane_gather)
 // A thread owns four consecutive lanes (16-byte accesses) of one tile or
-// span; a CTA of 256 threads covers `cols` lane quads (Lp/4 rounded up to 32,
-// at most 64) of 256 / cols tiles or spans.  The six kernels launch with
+// span; a CTA of 256 threads covers `cols` lane quads (Lp/4 rounded up to a
+// power of two, at most 64) of 256 / cols tiles or spans.  The six kernels launch with
 // programmatic serialisation and wait (griddepcontrol.wait) before touching
 // their predecessor's output.  Only the sampler, whose work needs the key
 // alone, lets its successor launch early; the others let it launch at their
@@ -874,9 +874,13 @@ constexpr int kGatherJ = 16;       // outputs per gather CTA
 constexpr int kCarryThreads = 1024;  // tile chunks per lane quad in the carry kernel
 
 __host__ __device__ inline uint32_t lane_pad(uint32_t L) { return (L + 3) & ~3u; }
-__host__ __device__ inline uint32_t lane_cols(uint32_t L) {  // lane quads per CTA
-    const uint32_t q = lane_pad(L) / 4, q32 = (q + 31) / 32 * 32;
-    return q32 < (uint32_t)kLaneQuadsMax ? q32 : (uint32_t)kLaneQuadsMax;
+// Lane quads per CTA: Lp/4 rounded up to a power of two, at most 64 (a CTA
+// then holds 256 / cols tiles or spans, and no thread idles for Lp/4 = 16).
+__host__ __device__ inline uint32_t lane_cols(uint32_t L) {
+    const uint32_t q = lane_pad(L) / 4;
+    uint32_t c = 1;
+    while (c < q && c < (uint32_t)kLaneQuadsMax) c *= 2;
+    return c;
 }
 __device__ __forceinline__ uint4 fadd4(uint4 a, uint4 b) {
     return make_uint4(fadd(a.x, b.x), fadd(a.y, b.y), fadd(a.z, b.z), fadd(a.w, b.w));
