@@ -657,29 +657,14 @@ int pvmvmd_server_mvm_multi(const pvmvmd_mvm_job *jobs, int count, void *stream)
 
 namespace pv {
 namespace {
-// Challenges (u and g), decrypt and verify: Y = Yhat - P e_x from st, or
-// Y = Yhat - mask_out when mask_out is given (boost mode).  The challenges
-// depend on the key alone and the check does not read Y, so both run on the
-// context's side stream while the decrypt streams P^T on the caller's
-// stream; the caller's stream then waits for the side stream.  When Y
-// overwrites Yhat the check must read Yhat first, and the steps run in order
-// on the caller's stream.
-int decode_verify_batch(pvmvmd_ctx *ctx, const void *st_dev, const uint32_t *mask_out_dev,
-                        const uint32_t *Xhat_dev, const uint32_t *Yhat_dev, int B,
-                        const pvmvmd_key *challenge_key, uint32_t *Y_dev, int32_t *accept_dev,
-                        cudaStream_t s) {
+// The verification of a call: challenges e_q <- E_{t_y}^{N_y} shared by the
+// B vectors, g_q = G_y e_q, u_q = e_q^T Q, and accept_b from x_hat_b and
+// y_hat_b, all on stream cs.
+int verify_chain(pvmvmd_ctx *ctx, const pvmvmd_key *challenge_key, const uint32_t *Xhat_dev,
+                 const uint32_t *Yhat_dev, int B, int32_t *accept_dev, cudaStream_t cs) {
     uint32_t *err = error_word();
     if (!err) return PVMVMD_E_CUDA;
     const CodeDev &d = ctx->gy;
-    const size_t ybytes = (size_t)B * ctx->m * sizeof(uint32_t);
-    const uintptr_t y0 = reinterpret_cast<uintptr_t>(Y_dev), h0 = reinterpret_cast<uintptr_t>(Yhat_dev);
-    const bool in_place = y0 < h0 + ybytes && h0 < y0 + ybytes;
-    const cudaStream_t cs = in_place ? s : ctx->side;
-    if (!in_place) {
-        PV_CUDA(cudaEventRecord(ctx->fork, s));
-        PV_CUDA(cudaStreamWaitEvent(ctx->side, ctx->fork, 0));
-    }
-    // Challenges e_q <- E_{t_y}^{N_y}, shared by the B vectors; g_q = G_y e_q.
     int C;
     uint32_t slice;
     size_t smem;
@@ -695,23 +680,41 @@ int decode_verify_batch(pvmvmd_ctx *ctx, const void *st_dev, const uint32_t *mas
         PV_CUDA(launch_syndrome_gather(d.pi1inv, ctx->m, ctx->rate, ctx->Fy, ctx->Ny, nullptr, ctx->g,
                                        ctx->ell, cs));
     }
-    // u_q = e_q^T Q.
     PV_CUDA(launch_verify_u(ctx->Q, ctx->K, ctx->chal, ctx->t_y, ctx->ell, ctx->u, cs));
-    if (in_place) {
-        PV_CUDA(launch_check(Xhat_dev, ctx->K, Yhat_dev, ctx->m, ctx->g, ctx->u, (uint32_t)ctx->ell, B,
-                             accept_dev, s));
-        PV_CUDA(launch_decrypt(ctx->PT, ctx->m, static_cast<const uint32_t *>(st_dev), ctx->t_x, Yhat_dev, B,
-                               Y_dev, s, mask_out_dev));
-        return PVMVMD_OK;
-    }
-    // the check reads x_hat, y_hat, u and g but not Y, so it follows the
-    // challenges on the side stream, beside the decrypt
     PV_CUDA(launch_check(Xhat_dev, ctx->K, Yhat_dev, ctx->m, ctx->g, ctx->u, (uint32_t)ctx->ell, B,
-                         accept_dev, ctx->side));
+                         accept_dev, cs));
+    return PVMVMD_OK;
+}
+
+bool overlaps(const void *a, const void *b, size_t bytes) {
+    const uintptr_t x = reinterpret_cast<uintptr_t>(a), y = reinterpret_cast<uintptr_t>(b);
+    return x < y + bytes && y < x + bytes;
+}
+
+// Verify and decrypt: Y = Yhat - P e_x from st, or Y = Yhat - mask_out when
+// mask_out is given (boost mode).  The verification depends on the key,
+// x_hat and y_hat but not on Y, so it runs on the context's side stream
+// while the decrypt streams P^T on the caller's stream; the caller's stream
+// then waits for the side stream.  When Y overwrites Yhat the verification
+// must read Yhat first, and both run in order on the caller's stream.
+int decode_verify_batch(pvmvmd_ctx *ctx, const void *st_dev, const uint32_t *mask_out_dev,
+                        const uint32_t *Xhat_dev, const uint32_t *Yhat_dev, int B,
+                        const pvmvmd_key *challenge_key, uint32_t *Y_dev, int32_t *accept_dev,
+                        cudaStream_t s) {
+    const bool in_place = overlaps(Y_dev, Yhat_dev, (size_t)B * ctx->m * sizeof(uint32_t));
+    const cudaStream_t cs = in_place ? s : ctx->side;
+    if (!in_place) {
+        PV_CUDA(cudaEventRecord(ctx->fork, s));
+        PV_CUDA(cudaStreamWaitEvent(ctx->side, ctx->fork, 0));
+    }
+    int st = verify_chain(ctx, challenge_key, Xhat_dev, Yhat_dev, B, accept_dev, cs);
+    if (st) return st;
     PV_CUDA(launch_decrypt(ctx->PT, ctx->m, static_cast<const uint32_t *>(st_dev), ctx->t_x, Yhat_dev, B,
                            Y_dev, s, mask_out_dev));
-    PV_CUDA(cudaEventRecord(ctx->join, ctx->side));
-    PV_CUDA(cudaStreamWaitEvent(s, ctx->join, 0));
+    if (!in_place) {
+        PV_CUDA(cudaEventRecord(ctx->join, ctx->side));
+        PV_CUDA(cudaStreamWaitEvent(s, ctx->join, 0));
+    }
     return PVMVMD_OK;
 }
 }  // namespace

@@ -25,33 +25,50 @@ __device__ __forceinline__ uint4 ldg4(const uint32_t *p) {
     return __ldg(reinterpret_cast<const uint4 *>(p));
 }
 
-__global__ void __launch_bounds__(256) k_verify_u(const uint32_t *__restrict__ Qm, int K,
-                                                 const uint32_t *__restrict__ chal, uint32_t t,
-                                                 uint32_t *__restrict__ u) {
+// u[q][k] = sum_j chal_val[q][j] Q[chal_supp[q][j]][k]: a CTA covers 64
+// columns with the t rows split over four row groups (so a thread streams
+// about t/4 rows, one round of loads for t = 31), the groups' sums meeting
+// in shared memory.
+constexpr int kVuCols = 64, kVuGroups = 4;
+__global__ void __launch_bounds__(kVuCols * kVuGroups) k_verify_u(const uint32_t *__restrict__ Qm, int K,
+                                                                 const uint32_t *__restrict__ chal, uint32_t t,
+                                                                 uint32_t *__restrict__ u) {
     extern __shared__ uint32_t sm[];
+    __shared__ uint32_t s_part[kVuGroups - 1][kVuCols];
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     asm volatile("griddepcontrol.wait;" ::: "memory");  // the challenges come from the kernel before
     const uint32_t q = blockIdx.y;
-    const uint32_t *c = chal + (size_t)q * 2 * t;
-    for (uint32_t j = threadIdx.x; j < 2 * t; j += blockDim.x) sm[j] = c[j];
+    const int tid = threadIdx.x, grp = tid / kVuCols, c = tid % kVuCols;
+    const uint32_t *ch = chal + (size_t)q * 2 * t;
+    for (uint32_t j = tid; j < 2 * t; j += kVuCols * kVuGroups) sm[j] = ch[j];
     __syncthreads();
-    const int k = blockIdx.x * blockDim.x + threadIdx.x;
-    if (k >= K) return;
+    const int k = blockIdx.x * kVuCols + c;
+    const uint32_t per = (t + kVuGroups - 1) / kVuGroups;
+    const uint32_t j0 = min(t, (uint32_t)grp * per), j1 = min(t, j0 + per);
     uint64_t acc = 0;
-    uint32_t j = 0;
-    for (; j + 8 <= t; j += 8) {
-        uint32_t v[8];
+    if (k < K) {
+        uint32_t j = j0;
+        for (; j + 8 <= j1; j += 8) {
+            uint32_t v[8];
 #pragma unroll
-        for (int s2 = 0; s2 < 8; ++s2) v[s2] = __ldg(Qm + (size_t)sm[j + s2] * K + k);
+            for (int s2 = 0; s2 < 8; ++s2) v[s2] = __ldg(Qm + (size_t)sm[j + s2] * K + k);
 #pragma unroll
-        for (int s2 = 0; s2 < 4; ++s2) acc += (uint64_t)sm[t + j + s2] * v[s2];
-        acc = fred(acc);
+            for (int s2 = 0; s2 < 4; ++s2) acc += (uint64_t)sm[t + j + s2] * v[s2];
+            acc = fred(acc);
 #pragma unroll
-        for (int s2 = 4; s2 < 8; ++s2) acc += (uint64_t)sm[t + j + s2] * v[s2];
-        acc = fred(acc);
+            for (int s2 = 4; s2 < 8; ++s2) acc += (uint64_t)sm[t + j + s2] * v[s2];
+            acc = fred(acc);
+        }
+        for (; j < j1; ++j) acc = fred(acc + (uint64_t)sm[t + j] * __ldg(Qm + (size_t)sm[j] * K + k));
     }
-    for (; j < t; ++j) acc = fred(acc + (uint64_t)sm[t + j] * __ldg(Qm + (size_t)sm[j] * K + k));
-    u[(size_t)q * K + k] = (uint32_t)acc;
+    if (grp > 0) s_part[grp - 1][c] = (uint32_t)acc;
+    __syncthreads();
+    if (grp == 0 && k < K) {
+        uint32_t sum = (uint32_t)acc;
+#pragma unroll
+        for (int g2 = 0; g2 < kVuGroups - 1; ++g2) sum = fadd(sum, s_part[g2][c]);
+        u[(size_t)q * K + k] = sum;
+    }
 }
 
 __device__ __forceinline__ uint32_t warp_fsum(uint32_t v) {
@@ -341,8 +358,8 @@ cudaError_t launch_verify_u(const uint32_t *Qm, int K, const uint32_t *chal, uin
                             uint32_t ell, uint32_t *u, cudaStream_t s) {
     if (K <= 0 || ell == 0) return cudaSuccess;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((K + 255) / 256, ell, 1);
-    cfg.blockDim = dim3(256, 1, 1);
+    cfg.gridDim = dim3((K + kVuCols - 1) / kVuCols, ell, 1);
+    cfg.blockDim = dim3(kVuCols * kVuGroups, 1, 1);
     cfg.dynamicSmemBytes = 2 * (size_t)t_y * sizeof(uint32_t);
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
