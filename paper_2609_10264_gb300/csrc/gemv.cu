@@ -224,8 +224,12 @@ __global__ void __launch_bounds__(kMultiThreads, 2) k_gemv_multi(const __grid_co
     const long long lo = total * blockIdx.x / gridDim.x;
     const long long hi = total * (blockIdx.x + 1) / gridDim.x;
 
-    asm volatile("griddepcontrol.wait;" ::: "memory");
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    // The first loads of M go out before griddepcontrol.wait, so they overlap
+    // the end of the kernel before this one: M is the server's weight
+    // matrix, never written by a kernel that signals its dependents early.
+    // Everything else (x_hat, y_hat) is touched only after the wait.
+    bool waited = false;
 
     for (int j = 0; j < args.count; ++j) {
         const long long b0 = args.base[j], b1 = args.base[j + 1];
@@ -252,6 +256,10 @@ __global__ void __launch_bounds__(kMultiThreads, 2) k_gemv_multi(const __grid_co
         };
         int g = warp;
         if (g < ngroups) issue(g, lane);
+        if (!waited) {
+            asm volatile("griddepcontrol.wait;" ::: "memory");
+            waited = true;
+        }
 
         __syncthreads();  // the previous job's planes are no longer read
         uint32_t *planes = reinterpret_cast<uint32_t *>(s_planes);
@@ -341,6 +349,7 @@ __global__ void __launch_bounds__(kMultiThreads, 2) k_gemv_multi(const __grid_co
             }
         }
     }
+    if (!waited) asm volatile("griddepcontrol.wait;" ::: "memory");
 }
 
 cudaError_t run_gemv_multi(const MvmJob *jobs, int count, cudaStream_t s) {
