@@ -595,9 +595,23 @@ def run_batched(args):
     def enc():
         for p in projs:
             pv.pvmvmd_encode(p["ctx"], p["X"], 21, Xhat=p["Xh"], st=p["st"], stream=stream)
+    # the layer's independent server products, spread over a few streams so
+    # that a small projection's product can use the SMs a larger one leaves
+    srv_streams = [torch.cuda.Stream(device) for _ in range(max(1, args.server_streams))]
+
     def srv():
-        for p in projs:
-            pv.pvmvmd_server_mvm(p["W"], p["Xh"], Yhat=p["Yh"], stream=stream)
+        fork = torch.cuda.Event()
+        fork.record(stream)
+        for ss in srv_streams:
+            ss.wait_event(fork)
+        for j, p in enumerate(projs):
+            ss = srv_streams[j % len(srv_streams)]
+            pv.pvmvmd_server_mvm(p["W"], p["Xh"], Yhat=p["Yh"], stream=ss)
+        for ss in srv_streams:
+            join = torch.cuda.Event()
+            join.record(ss)
+            stream.wait_event(join)
+
     def dec():
         for p in projs:
             pv.pvmvmd_decode_verify(p["ctx"], p["st"], p["Xh"], p["Yh"], 22, Y=p["Y"], accept=p["acc"], stream=stream)
@@ -983,7 +997,7 @@ def main(argv=None):
                     default="batch1-4096")
     ap.add_argument("--shape", default="4096x4096x64",
                     help="m x K x B for --workload server-shape, K x B for --workload encode-shape")
-    ap.add_argument("--server-streams", type=int, default=2)
+    ap.add_argument("--server-streams", type=int, default=3)
     ap.add_argument("--mode", choices=["standard", "boost", "pipelined"], default="standard",
                     help="client mode of the batch-1 workload (Sec. 7.2): standard (masks drawn during "
                          "the step), boost (masks prepared ahead, untimed) or pipelined (standard mode "

@@ -132,7 +132,11 @@ int pvmvmd_encode(pvmvmd_ctx *ctx, const uint32_t *X_dev, int B, const pvmvmd_ke
  * kernel before it on the stream finishes, when that kernel signals its
  * dependents early (programmatic dependent launch); such a kernel must not
  * write M.  Kernels that do not use programmatic dependent launch, and all
- * of this library's kernels, are safe. */
+ * of this library's kernels, are safe.  The B > 1 paths keep their digit
+ * operand in library scratch held per stream: calls on different streams
+ * may run concurrently, and a buffer grows (with a synchronisation of the
+ * stream) only when a call needs more than any earlier call on that stream,
+ * which must not happen while the stream is being captured. */
 int pvmvmd_server_mvm(const int8_t *W_dev, int m, int K, const uint32_t *Xhat_dev, int B,
                       uint32_t *Yhat_dev, void *stream);
 

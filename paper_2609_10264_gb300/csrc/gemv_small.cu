@@ -264,35 +264,6 @@ cudaError_t run_gemv_nb(const NbJob *jobs, int count, cudaStream_t s) {
     return cudaLaunchKernelEx(&cfg, k_gemv_nb<2, 2>, args);
 }
 
-// Per-device buffer for the digit planes (grown when a call needs more;
-// growing waits for the device, since the old buffer may still be read).
-cudaError_t planes_scratch(size_t need, uint32_t **out) {
-    struct Scratch {
-        uint32_t *ptr = nullptr;
-        size_t bytes = 0;
-    };
-    static Scratch per_dev[64];
-    static std::mutex mu;
-    std::lock_guard<std::mutex> lock(mu);
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return e;
-    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-    Scratch &sc = per_dev[dev];
-    if (sc.bytes < need) {
-        if (sc.ptr) {
-            if ((e = cudaDeviceSynchronize()) != cudaSuccess) return e;
-            cudaFree(sc.ptr);
-            sc.ptr = nullptr;
-            sc.bytes = 0;
-        }
-        if ((e = cudaMalloc(&sc.ptr, need)) != cudaSuccess) return e;
-        sc.bytes = need;
-    }
-    *out = sc.ptr;
-    return cudaSuccess;
-}
-
 }  // namespace
 
 cudaError_t launch_gemv_small_batch(const int8_t *W, int m, int K, const uint32_t *Xhat, int B,
@@ -301,9 +272,10 @@ cudaError_t launch_gemv_small_batch(const int8_t *W, int m, int K, const uint32_
     // digit planes of all vectors once: [job][plane][vector][K] bytes
     const int Bp = (B + kNbVec - 1) / kNbVec * kNbVec;
     const size_t row_words = (size_t)K / 4, job_words = 4 * kNbVec * row_words;
-    uint32_t *planes = nullptr;
-    cudaError_t e = planes_scratch((size_t)Bp / kNbVec * job_words * sizeof(uint32_t), &planes);
+    void *pbuf = nullptr;
+    cudaError_t e = stream_scratch(kScratchDigitPlanes, (size_t)Bp / kNbVec * job_words * sizeof(uint32_t), s, &pbuf);
     if (e != cudaSuccess) return e;
+    uint32_t *planes = static_cast<uint32_t *>(pbuf);
     {
         const size_t threads = (size_t)Bp * row_words;
         cudaLaunchConfig_t cfg = {};

@@ -125,6 +125,11 @@ cudaError_t launch_gemv(const int8_t *W, int m, int K, const uint32_t *xhat, uin
 cudaError_t launch_batched(const int8_t *W, int m, int K, const uint32_t *Xhat, int B,
                            uint32_t *Yhat, uint32_t *err, cudaStream_t s);
 
+// Grow-only scratch of at least `need` bytes for `purpose` on the current
+// device, one buffer per stream (see scratch.cu).
+enum ScratchPurpose { kScratchDigitTiles = 0, kScratchDigitPlanes = 1 };
+cudaError_t stream_scratch(int purpose, size_t need, cudaStream_t s, void **out);
+
 // The library's device error word on the current device (null on failure).
 uint32_t *library_error_word();
 

@@ -689,35 +689,6 @@ cudaError_t batched_launch(const int8_t *W, int m, int K, const uint32_t *Xhat, 
     return cudaLaunchKernelEx(&cfg, kern, tmap, W, m, K, (const uint8_t *)D, nkb, B, Yhat, err);
 }
 
-// ---------------------------------------------------------------- scratch for the digit operand
-struct Scratch {
-    uint8_t *ptr = nullptr;
-    size_t bytes = 0;
-};
-
-cudaError_t digit_scratch(size_t need, uint8_t **out) {
-    static Scratch per_dev[64];
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return e;
-    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-    Scratch &s = per_dev[dev];
-    if (s.bytes < need) {
-        if (s.ptr) {
-            e = cudaDeviceSynchronize();  // the old buffer may still be in use
-            if (e != cudaSuccess) return e;
-            cudaFree(s.ptr);
-            s.ptr = nullptr;
-            s.bytes = 0;
-        }
-        e = cudaMalloc(&s.ptr, need);
-        if (e != cudaSuccess) return e;
-        s.bytes = need;
-    }
-    *out = s.ptr;
-    return cudaSuccess;
-}
-
 }  // namespace
 
 cudaError_t launch_batched(const int8_t *W, int m, int K, const uint32_t *Xhat, int B,
@@ -725,10 +696,10 @@ cudaError_t launch_batched(const int8_t *W, int m, int K, const uint32_t *Xhat, 
     if (m <= 0 || K <= 0 || B <= 0) return cudaSuccess;
     const int nkb = (K + kBK - 1) / kBK;
     const int nvt = (B + kBV - 1) / kBV;
-    uint8_t *D = nullptr;
-    cudaError_t e = digit_scratch((size_t)nvt * nkb * kBTile, &D);
+    void *D = nullptr;
+    cudaError_t e = stream_scratch(kScratchDigitTiles, (size_t)nvt * nkb * kBTile, s, &D);
     if (e != cudaSuccess) return e;
-    return batched_launch(W, m, K, Xhat, B, Yhat, err, D, s);
+    return batched_launch(W, m, K, Xhat, B, Yhat, err, static_cast<uint8_t *>(D), s);
 }
 
 }  // namespace pv
