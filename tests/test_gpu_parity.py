@@ -434,6 +434,34 @@ def test_config5_70b(pv, wl, name):
     _batched_pipeline_sampled(pv, W, 256, seed=500 + len(name), n_rows=12, n_verify=1)
 
 
+def test_server_mvm_concurrent_streams(pv, wl):
+    """Batched and small-batch products issued on two streams at once keep
+    their digit operands apart: every output equals the oracle's."""
+    import torch
+    cases = [(512, 3072, 64), (384, 2048, 96), (700, 1024, 8), (256, 4096, 12)]
+    streams = [torch.cuda.Stream(), torch.cuda.Stream()]
+    ins, outs = [], []
+    for j, (m, K, B) in enumerate(cases):
+        W = wl.weights_uniform(m, K, (51, j))
+        X = np.random.default_rng(52 + j).integers(0, Q, size=(B, K), dtype=np.int64).astype(np.uint32)
+        ins.append((W, X, to_dev(W), to_dev(X)))
+    torch.cuda.synchronize()
+    for rep in range(3):
+        outs = []
+        for j, (W, X, Wd, Xd) in enumerate(ins):
+            s = streams[j % 2]
+            with torch.cuda.stream(s):
+                outs.append(pv.pvmvmd_server_mvm(Wd, Xd, stream=s))
+        torch.cuda.synchronize()
+    for (W, X, _, _), Yh in zip(ins, outs):
+        m = W.shape[0]
+        rows = sample_rows(m, 16, 53)
+        Yh_h = pv.as_u32(Yh)
+        for b in range(X.shape[0]):
+            assert np.array_equal(Yh_h[b, rows], oracle.server_mvm_rows(W, X[b], rows)), b
+    assert pv.pvmvmd_device_status() == 0
+
+
 @pytest.mark.parametrize("L", [256, 128])
 def test_lane_encode_long_tiles(pv, wl, L):
     """The lane encode on a long code (K = 28672, N_x = 229376) with every
