@@ -1027,8 +1027,8 @@ def main(argv=None):
                     default="batch1-4096")
     ap.add_argument("--shape", default="4096x4096x64",
                     help="m x K x B for --workload server-shape, K x B for --workload encode-shape")
-    ap.add_argument("--server-streams", type=int, default=3)
-    ap.add_argument("--schedule", choices=["phases", "projections"], default="phases",
+    ap.add_argument("--server-streams", type=int, default=4)
+    ap.add_argument("--schedule", choices=["phases", "projections"], default="projections",
                     help="batched workloads: all encodes, then all products, then all decodes "
                          "(phases), or each projection's three calls in order on one of "
                          "--server-streams streams (projections)")
