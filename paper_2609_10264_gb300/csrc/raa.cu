@@ -1132,7 +1132,7 @@ __global__ void __launch_bounds__(kCarryThreads) k_lane_carry(const uint4 *__res
 
 // In place: C[i][b] <- v1_i (carry[tau][b] + sum_{i' >= i in tile tau} C[i'][b]),
 // with v1m = v1 R (Montgomery, R = 2^32) so that each product is one REDC.
-__global__ void __launch_bounds__(kLaneCta) k_lane_scan(uint4 *__restrict__ C, uint32_t N, uint32_t tile, uint32_t L,
+__global__ void __launch_bounds__(kLaneCta, 4) k_lane_scan(uint4 *__restrict__ C, uint32_t N, uint32_t tile, uint32_t L,
                                                        const uint4 *__restrict__ carry,
                                                        const uint32_t *__restrict__ v1m) {
     asm volatile("griddepcontrol.wait;" ::: "memory");  // inputs come from the kernel before
@@ -1164,7 +1164,7 @@ __global__ void __launch_bounds__(kLaneCta) k_lane_scan(uint4 *__restrict__ C, u
 // out[b][j] = addend[b][j] + sum_{c<r} C[pi1^-1(r j + c)][b] for kGatherJ
 // outputs and the CTA's lanes, transposed through shared memory so that out
 // rows are written 128 bytes at a time.  addend may be null or alias out.
-__global__ void __launch_bounds__(kLaneCta) k_lane_gather(const uint4 *__restrict__ C,
+__global__ void __launch_bounds__(kLaneCta, 4) k_lane_gather(const uint4 *__restrict__ C,
                                                          const uint32_t *__restrict__ pi1inv,
                                                          uint32_t r, uint32_t n, uint32_t L,
                                                          const uint32_t *addend, uint32_t *out) {
