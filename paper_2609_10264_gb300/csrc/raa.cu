@@ -670,8 +670,12 @@ __global__ void __launch_bounds__(kFusedThreads) k_syndrome_fused(
     uint32_t after = 0;  // sum over the positions owned by later CTAs
     if (C > 1) {
         cluster.sync();
-        for (uint32_t rr = rank + 1; rr < C; ++rr)
-            after = fadd(after, *cluster.map_shared_rank(&s_agg, rr));
+        // every warp reads the later ranks' totals at once (one DSMEM load
+        // per lane) and sums them with shuffles
+        const uint32_t rr = rank + 1 + (uint32_t)lane;
+        after = rr < C ? *cluster.map_shared_rank(&s_agg, rr) : 0u;
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1) after = fadd(after, __shfl_xor_sync(kFull, after, o));
     } else {
         __syncthreads();
     }
