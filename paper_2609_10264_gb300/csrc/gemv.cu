@@ -367,8 +367,8 @@ cudaError_t run_gemv_multi(const MvmJob *jobs, int count, cudaStream_t s) {
     long long rows = 0;
     for (int j = 0; j < count; ++j) rows += jobs[j].m;
     if (rows == 0) return cudaSuccess;
-    static const cudaError_t attr = cudaFuncSetAttribute(
-        k_gemv_multi<2, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, 4 * kMultiMaxK);
+    const cudaError_t attr = func_attr((const void *)k_gemv_multi<2, 4>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, 4 * kMultiMaxK);
     if (attr != cudaSuccess) return attr;
     int dev = 0, sms = 0;
     cudaGetDevice(&dev);
@@ -395,8 +395,8 @@ cudaError_t run_gemv(const int8_t *W, size_t ldw, int m, int K, const uint32_t *
     const size_t smem = (size_t)nchunks * 16 * 4;
     auto kern = k_gemv<ROWS, UNROLL, kVec>;
     // set once (outside any stream capture that a later call might be part of)
-    static const cudaError_t attr = cudaFuncSetAttribute(
-        kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kGemvMaxK * 4);
+    const cudaError_t attr = func_attr((const void *)kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       kGemvMaxK * 4);
     if (attr != cudaSuccess) return attr;
     int dev = 0, sms = 0;
     cudaGetDevice(&dev);

@@ -243,8 +243,8 @@ cudaError_t run_gemv_nb(const NbJob *jobs, int count, cudaStream_t s) {
         rows += jobs[j].m;
     }
     if (rows == 0) return cudaSuccess;
-    static const cudaError_t attr = cudaFuncSetAttribute(
-        k_gemv_nb<2, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, 4 * kNbVec * kNbMaxK);
+    const cudaError_t attr = func_attr((const void *)k_gemv_nb<2, 2>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, 4 * kNbVec * kNbMaxK);
     if (attr != cudaSuccess) return attr;
     int dev = 0, sms = 0;
     cudaGetDevice(&dev);

@@ -130,6 +130,11 @@ cudaError_t launch_batched(const int8_t *W, int m, int K, const uint32_t *Xhat, 
 enum ScratchPurpose { kScratchDigitTiles = 0, kScratchDigitPlanes = 1 };
 cudaError_t stream_scratch(int purpose, size_t need, cudaStream_t s, void **out);
 
+// cudaFuncSetAttribute for the current device, done once per (kernel,
+// attribute, device): function attributes belong to each device's instance
+// of the kernel.
+cudaError_t func_attr(const void *fn, cudaFuncAttribute attr, int value);
+
 // The library's device error word on the current device (null on failure).
 uint32_t *library_error_word();
 

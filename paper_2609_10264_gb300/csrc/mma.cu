@@ -43,7 +43,9 @@
 #include <cuda_fp16.h>
 
 #include <cstring>
+#include <map>
 #include <mutex>
+#include <tuple>
 
 #include "common.cuh"
 #include "launch.h"
@@ -571,12 +573,15 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // Resident clusters of (2, 1, split) CTAs of the kernel, from the occupancy
-// calculator (a cluster must fit in one GPC), cached per split.
+// calculator (a cluster must fit in one GPC), cached per (kernel, split,
+// device).
 int resident_clusters(const void *kern, int split) {
-    static int cache[8] = {0};
+    static std::map<std::tuple<const void *, int, int>, int> cache;
     static std::mutex mu;
+    int cur = 0;
+    cudaGetDevice(&cur);
     std::lock_guard<std::mutex> lock(mu);
-    int &c = cache[split];
+    int &c = cache[std::make_tuple(kern, split, cur)];
     if (c == 0) {
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(2, 1, split);
@@ -663,10 +668,10 @@ cudaError_t batched_launch(const int8_t *W, int m, int K, const uint32_t *Xhat, 
             return cudaErrorInvalidValue;
     }
     auto kern = vec ? k_batched<true> : k_batched<false>;
-    static const cudaError_t a1 =
-        cudaFuncSetAttribute(k_batched<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
-    static const cudaError_t a2 =
-        cudaFuncSetAttribute(k_batched<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
+    const cudaError_t a1 =
+        func_attr((const void *)k_batched<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
+    const cudaError_t a2 =
+        func_attr((const void *)k_batched<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
     if (a1 != cudaSuccess) return a1;
     if (a2 != cudaSuccess) return a2;
     const int split = choose_split((const void *)kern, mp * nvt, nkb);

@@ -10,6 +10,8 @@
 //                         lanes (preprocessing of P^T and Q, Sec. 6.3).
 //  * k_lane_*             the syndrome for a batch of vectors held as the lanes
 //                         of an N x B array (sample, step function, scan, gather).
+#include <map>
+#include <mutex>
 #include <cooperative_groups.h>
 
 #include "common.cuh"
@@ -1229,8 +1231,8 @@ cudaError_t launch_sample_sparse(const pvmvmd_key &key, uint32_t tag, uint64_t i
     if (count == 0) return cudaSuccess;
     const size_t smem = ((size_t)(N + 31) / 32 + 512) * sizeof(uint32_t);
     if (smem > kSampleMaxSmem) return cudaErrorInvalidValue;
-    static const cudaError_t attr = cudaFuncSetAttribute(
-        k_sample_sparse, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSampleMaxSmem);
+    const cudaError_t attr = func_attr((const void *)k_sample_sparse, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)kSampleMaxSmem);
     if (attr != cudaSuccess) return attr;
     k_sample_sparse<<<count, 32, smem, s>>>(key, tag, idx0, N, t, out, clear, clear_words);
     return cudaGetLastError();
@@ -1301,17 +1303,21 @@ constexpr size_t kFusedMaxSmem = 180 * 1024;
 // Largest cluster the fused kernel may use on this device: 16 CTAs where the
 // device schedules clusters of that (non-portable) size, else 8.
 int fused_max_cluster() {
-    static const int cmax = [] {
-        if (cudaFuncSetAttribute(k_syndrome_fused, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
-            cudaSuccess) {
-            cudaGetLastError();
-            return 8;
-        }
-        if (cudaFuncSetAttribute(k_syndrome_fused, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)kFusedMaxSmem) != cudaSuccess) {
-            cudaGetLastError();
-            return 8;
-        }
+    static std::mutex mu;
+    static std::map<int, int> cache;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        cudaGetLastError();
+        return 8;
+    }
+    std::lock_guard<std::mutex> lock(mu);
+    auto it = cache.find(dev);
+    if (it != cache.end()) return it->second;
+    int cmax = 8;
+    if (func_attr((const void *)k_syndrome_fused, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) ==
+            cudaSuccess &&
+        func_attr((const void *)k_syndrome_fused, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                  (int)kFusedMaxSmem) == cudaSuccess) {
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(16, 1, 1);
         cfg.blockDim = dim3(kFusedThreads, 1, 1);
@@ -1324,12 +1330,10 @@ int fused_max_cluster() {
         cfg.attrs = a;
         cfg.numAttrs = 1;
         int n = 0;
-        if (cudaOccupancyMaxActiveClusters(&n, k_syndrome_fused, &cfg) != cudaSuccess) {
-            cudaGetLastError();
-            return 8;
-        }
-        return n > 0 ? 16 : 8;
-    }();
+        if (cudaOccupancyMaxActiveClusters(&n, k_syndrome_fused, &cfg) == cudaSuccess && n > 0) cmax = 16;
+    }
+    cudaGetLastError();
+    cache[dev] = cmax;
     return cmax;
 }
 }  // namespace
@@ -1384,8 +1388,8 @@ cudaError_t launch_syndrome_fused(const pvmvmd_key &key, uint32_t tag, uint64_t 
     uint32_t slice = 0;
     size_t smem = 0;
     if (!syndrome_fused_plan(N, t, &C, &slice, &smem)) return cudaErrorNotSupported;
-    static const cudaError_t attr = cudaFuncSetAttribute(
-        k_syndrome_fused, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFusedMaxSmem);
+    const cudaError_t attr = func_attr((const void *)k_syndrome_fused, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)kFusedMaxSmem);
     if (attr != cudaSuccess) return attr;
     syndrome_fused_launch_plan(N, t, count < 65535 ? count : 65535, &C, &slice, &smem);
     for (uint32_t c0 = 0; c0 < count; c0 += 65535) {
@@ -1446,8 +1450,8 @@ cudaError_t launch_lane_syndrome(const pvmvmd_key &key, uint32_t tag, uint64_t i
     if (L == 0) return cudaSuccess;
     const size_t smem = ((size_t)(N + 31) / 32 + 1024 + 4 * (size_t)t + 1) * sizeof(uint32_t);
     if (smem > kSampleMaxSmem) return cudaErrorInvalidValue;
-    static const cudaError_t a1 = cudaFuncSetAttribute(
-        k_lane_sample, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSampleMaxSmem);
+    const cudaError_t a1 = func_attr((const void *)k_lane_sample, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)kSampleMaxSmem);
     if (a1 != cudaSuccess) return a1;
     if ((reinterpret_cast<uintptr_t>(C) | reinterpret_cast<uintptr_t>(aux)) & 15u)
         return cudaErrorInvalidValue;

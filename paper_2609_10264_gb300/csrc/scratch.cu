@@ -1,3 +1,5 @@
+// Host-side state kept per device.
+//
 // Grow-only device scratch held per (purpose, device, stream).
 //
 // The batched product's digit tiles and the small-batch product's digit
@@ -39,6 +41,21 @@ cudaError_t stream_scratch(int purpose, size_t need, cudaStream_t s, void **out)
     }
     *out = b.ptr;
     return cudaSuccess;
+}
+
+cudaError_t func_attr(const void *fn, cudaFuncAttribute attr, int value) {
+    static std::mutex mu;
+    static std::map<std::tuple<const void *, int, int>, std::pair<int, cudaError_t>> done;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lock(mu);
+    auto key = std::make_tuple(fn, (int)attr, dev);
+    auto it = done.find(key);
+    if (it != done.end() && it->second.first == value) return it->second.second;
+    e = cudaFuncSetAttribute(fn, attr, value);
+    done[key] = std::make_pair(value, e);
+    return e;
 }
 
 }  // namespace pv
