@@ -128,8 +128,9 @@ int pvmvmd_encode(pvmvmd_ctx *ctx, const uint32_t *X_dev, int B, const pvmvmd_ke
  * Needs no context and no secret.  B == 1 runs the bandwidth-bound GEMV;
  * 2 <= B <= 16 (K a multiple of 16, 16-byte aligned W and Xhat) a GEMV that
  * reads M once per four vectors; larger B the byte-limb tensor-core product.
- * 1 <= K <= PVMVMD_MAX_K.  The batch-1 GEMV may start reading M while the
- * kernel before it on the stream finishes, when that kernel signals its
+ * 1 <= K <= PVMVMD_MAX_K.  The batch-1 GEMV and the 2 <= B <= 16 GEMV may
+ * start reading M while the kernel before it on the stream finishes, when
+ * that kernel signals its
  * dependents early (programmatic dependent launch); such a kernel must not
  * write M.  Kernels that do not use programmatic dependent launch, and all
  * of this library's kernels, are safe.  The B > 1 paths keep their digit

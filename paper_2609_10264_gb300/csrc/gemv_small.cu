@@ -55,6 +55,11 @@ __device__ __forceinline__ int transposed_reduce(int (&v)[V], int lane) {
 constexpr int kNbVec = 4;          // vectors per pass
 constexpr int kNbMaxK = 6144;      // K per pass (4 planes x 4 vectors x K bytes)
 constexpr int kNbMaxJobs = 32;
+// Each of the 16 plane rows in shared memory is kNbMaxK bytes apart whatever
+// K is, so the 16 row offsets of the inner loop are compile-time constants
+// (immediate offsets of one address per chunk).
+constexpr int kNbStride = kNbMaxK / 16;  // 16-byte chunks per plane row
+constexpr int kNbSmem = 4 * kNbVec * kNbMaxK;
 
 struct NbJob {
     const int8_t *W;
@@ -110,8 +115,11 @@ __global__ void __launch_bounds__(kMultiThreads, 2) k_gemv_nb(const __grid_const
     const long long lo = total * blockIdx.x / gridDim.x;
     const long long hi = total * (blockIdx.x + 1) / gridDim.x;
 
-    asm volatile("griddepcontrol.wait;" ::: "memory");
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    // The first loads of M go out before griddepcontrol.wait (M is the
+    // server's weight matrix, never written by a kernel of the chain); the
+    // planes and y_hat are touched only after it.
+    bool waited = false;
 
     for (int j = 0; j < args.count; ++j) {
         const long long b0 = args.base[j], b1 = args.base[j + 1];
@@ -137,27 +145,23 @@ __global__ void __launch_bounds__(kMultiThreads, 2) k_gemv_nb(const __grid_const
         };
         int g = warp;
         if (g < ngroups) issue(g, lane);
+        if (!waited) {
+            asm volatile("griddepcontrol.wait;" ::: "memory");
+            waited = true;
+        }
 
         __syncthreads();  // the previous job's planes are no longer read
-        // planes: [plane p][vector v][K/4 words], copied from the planes the
-        // call built once; rows of vectors past nb are zero there
-        uint32_t *planes = reinterpret_cast<uint32_t *>(s_planes);
-        const int pstride = K / 4, q16 = K / 16;  // words and 16-byte chunks per row
-        for (int idx0 = tid; idx0 < 4 * kNbVec * q16; idx0 += 4 * kMultiThreads) {
-            uint4 c[4];
+        // planes: row p * kNbVec + v holds plane p of vector v, copied from
+        // the planes the call built once; rows of vectors past nb are zero
+        for (int c = tid; c < nchunks; c += kMultiThreads) {
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int idx = idx0 + u * kMultiThreads;
-                const int row = idx / q16, c4 = idx % q16;
-                c[u] = idx < 4 * kNbVec * q16
-                           ? __ldg(reinterpret_cast<const uint4 *>(job.planes + (size_t)row * job.ldp) + c4)
-                           : make_uint4(0u, 0u, 0u, 0u);
-            }
+            for (int h = 0; h < 2; ++h) {
+                uint4 t[8];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int idx = idx0 + u * kMultiThreads;
-                if (idx < 4 * kNbVec * q16)
-                    reinterpret_cast<uint4 *>(planes)[(idx / q16) * (pstride / 4) + idx % q16] = c[u];
+                for (int r = 0; r < 8; ++r)
+                    t[r] = __ldg(reinterpret_cast<const uint4 *>(job.planes + (size_t)(8 * h + r) * job.ldp) + c);
+#pragma unroll
+                for (int r = 0; r < 8; ++r) s_planes[(8 * h + r) * kNbStride + c] = t[r];
             }
         }
         __syncthreads();
@@ -185,7 +189,7 @@ __global__ void __launch_bounds__(kMultiThreads, 2) k_gemv_nb(const __grid_const
                         for (int v = 0; v < kNbVec; ++v) {
                             uint4 l[4];
 #pragma unroll
-                            for (int p = 0; p < 4; ++p) l[p] = s_planes[(size_t)(p * kNbVec + v) * nchunks + cc];
+                            for (int p = 0; p < 4; ++p) l[p] = s_planes[(p * kNbVec + v) * kNbStride + cc];
 #pragma unroll
                             for (int r = 0; r < ROWS; ++r) {
                                 const uint4 w = cur[u][r];
@@ -226,6 +230,9 @@ __global__ void __launch_bounds__(kMultiThreads, 2) k_gemv_nb(const __grid_const
             }
         }
     }
+    // a CTA with no rows still waits, so that the kernel completes only
+    // after the one before it (dependents rely on that order)
+    if (!waited) asm volatile("griddepcontrol.wait;" ::: "memory");
 }
 
 cudaError_t run_gemv_nb(const NbJob *jobs, int count, cudaStream_t s) {
@@ -234,17 +241,15 @@ cudaError_t run_gemv_nb(const NbJob *jobs, int count, cudaStream_t s) {
     std::lock_guard<std::mutex> lock(mu);
     args.count = count;
     args.base[0] = 0;
-    int kmax = 16;
     long long rows = 0;
     for (int j = 0; j < count; ++j) {
         args.job[j] = jobs[j];
         args.base[j + 1] = args.base[j] + (long long)jobs[j].m * jobs[j].K;
-        if (jobs[j].K > kmax) kmax = jobs[j].K;
         rows += jobs[j].m;
     }
     if (rows == 0) return cudaSuccess;
-    const cudaError_t attr = func_attr((const void *)k_gemv_nb<2, 2>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, 4 * kNbVec * kNbMaxK);
+    const cudaError_t attr =
+        func_attr((const void *)k_gemv_nb<2, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, kNbSmem);
     if (attr != cudaSuccess) return attr;
     int dev = 0, sms = 0;
     cudaGetDevice(&dev);
@@ -254,7 +259,7 @@ cudaError_t run_gemv_nb(const NbJob *jobs, int count, cudaStream_t s) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)grid, 1, 1);
     cfg.blockDim = dim3(kMultiThreads, 1, 1);
-    cfg.dynamicSmemBytes = (size_t)4 * kNbVec * kmax;
+    cfg.dynamicSmemBytes = kNbSmem;
     cfg.stream = s;
     cudaLaunchAttribute attrs[1];
     attrs[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
