@@ -266,8 +266,15 @@ def run_ours(args):
     params.scratch_batch = VECTORS                        # one encode chunk per step
     ctx = pv.pvmvmd_preprocess(Wd, key=20, params=params)
     stream = torch.cuda.Stream(device)
-    Xh = torch.empty_like(Xd)
-    st = torch.empty((VECTORS, 2 * ctx.t_x), dtype=torch.int32, device=device)
+    # "overlap" (standard mode): the next batch's encode runs on enc_stream
+    # beside this batch's decode (an encode and a decode of one context share
+    # no scratch), so x_hat and st alternate between two sets
+    overlap = args.mode == "standard" and args.step_schedule == "overlap"
+    enc_stream = torch.cuda.Stream(device)
+    Xh_sets = [torch.empty_like(Xd) for _ in range(2 if overlap else 1)]
+    st_sets = [torch.empty((VECTORS, 2 * ctx.t_x), dtype=torch.int32, device=device)
+               for _ in range(2 if overlap else 1)]
+    Xh, st = Xh_sets[0], st_sets[0]
     Yh = torch.empty((VECTORS, M), dtype=torch.int32, device=device)
     Y = torch.empty_like(Yh)
     acc = torch.empty(VECTORS, dtype=torch.int32, device=device)
@@ -298,7 +305,8 @@ def run_ours(args):
         pv.pvmvmd_encode(ctx, Xd, 21 + rank, Xhat=Xh, st=st, stream=stream)
 
     side = [torch.cuda.Stream(device) for _ in range(args.server_streams)]
-    jobs = pv.mvm_jobs([(Wv[b], Xh[b], Yh[b]) for b in range(VECTORS)])
+    jobs_sets = [pv.mvm_jobs([(Wv[b], xs[b], Yh[b]) for b in range(VECTORS)]) for xs in Xh_sets]
+    jobs = jobs_sets[0]
 
     def server():
         if args.server_mode == "multi":
@@ -374,7 +382,37 @@ def run_ours(args):
             join.record(prep_stream)
             stream.wait_event(join)
 
-    g_steps = [capture(lambda k=k: whole_step(k), stream) for k in range(nsets)]
+    def overlapped_step(k, x_in=None, host_in=None, host_out=None):
+        # this batch (set k): server, then decode on `stream`; the next batch
+        # (set 1 - k): encode on enc_stream, forked after the server call.
+        # (Forked at the start of the step instead, beside the server call,
+        # it saved nothing: 338 against 330 us per step.)
+        pv.pvmvmd_server_mvm_multi(jobs_sets[k], stream=stream)
+        fork = torch.cuda.Event()
+        fork.record(stream)
+        enc_stream.wait_event(fork)
+        with torch.cuda.stream(enc_stream):
+            src = Xd
+            if host_in is not None:
+                x_in[1 - k].copy_(host_in, non_blocking=True)
+                src = x_in[1 - k]
+            pv.pvmvmd_encode(ctx, src, 21 + rank, Xhat=Xh_sets[1 - k], st=st_sets[1 - k], stream=enc_stream)
+        pv.pvmvmd_decode_verify(ctx, st_sets[k], Xh_sets[k], Yh, 22 + rank, Y=Y, accept=acc, stream=stream)
+        if host_out is not None:
+            host_out[0].copy_(Y, non_blocking=True)
+            host_out[1].copy_(acc, non_blocking=True)
+        join = torch.cuda.Event()
+        join.record(enc_stream)
+        stream.wait_event(join)
+
+    if overlap:
+        # set 0 holds an encoded batch before the first step
+        with torch.cuda.stream(stream):
+            pv.pvmvmd_encode(ctx, Xd, 21 + rank, Xhat=Xh_sets[0], st=st_sets[0], stream=stream)
+        stream.synchronize()
+        g_steps = [capture(lambda k=k: overlapped_step(k), stream) for k in range(2)]
+    else:
+        g_steps = [capture(lambda k=k: whole_step(k), stream) for k in range(nsets)]
     cur[0] = 0
     # encode: the fused syndrome kernel (standard), or k_field_add with masks
     # prepared ahead (boost; pipelined adds the preparation: fused syndrome +
@@ -416,9 +454,10 @@ def run_ours(args):
     stream.synchronize()
 
     # ---- timed region: whole steps, one graph per step
+    nsteps_sets = len(g_steps)
     with torch.cuda.stream(stream):
         for w in range(args.warmup):
-            g_steps[w % nsets].replay()
+            g_steps[w % nsteps_sets].replay()
     stream.synchronize()
     clocks = ClockSampler(device.index)
     barrier(device)
@@ -429,7 +468,7 @@ def run_ours(args):
     with torch.cuda.stream(stream):
         t_start.record(stream)
         for s in range(args.steps):
-            g_steps[s % nsets].replay()
+            g_steps[s % nsteps_sets].replay()
         t_stop.record(stream)
     stream.synchronize()
     torch.cuda.synchronize(device)
@@ -479,22 +518,30 @@ def run_ours(args):
         Yhost.copy_(Y, non_blocking=True)
         Ahost.copy_(acc, non_blocking=True)
 
+    if overlap:
+        # the same pipeline through the public calls: the next batch's host
+        # copy and encode beside this batch's decode and copy back
+        Xins = [torch.empty_like(Xd) for _ in range(2)]
+        with torch.cuda.stream(stream):
+            Xins[0].copy_(Xhost, non_blocking=True)
+            pv.pvmvmd_encode(ctx, Xins[0], 21 + rank, Xhat=Xh_sets[0], st=st_sets[0], stream=stream)
+        stream.synchronize()
+        ges = [capture(lambda k=k: overlapped_step(k, Xins, Xhost, (Yhost, Ahost)), stream) for k in range(2)]
+    else:
+        with torch.cuda.stream(stream):
+            e2e_step()
+        stream.synchronize()
+        ges = [capture(e2e_step, stream)]
+    e2e_steps = max(2, args.steps // 2)
     with torch.cuda.stream(stream):
-        e2e_step()
-    stream.synchronize()
-    ge = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(ge, stream=stream):
-        e2e_step()
-    e2e_steps = max(1, args.steps // 2)
-    with torch.cuda.stream(stream):
-        for _ in range(args.warmup):
-            ge.replay()
+        for w in range(args.warmup):
+            ges[w % len(ges)].replay()
     stream.synchronize()
     barrier(device)
     t0 = time.perf_counter()
     with torch.cuda.stream(stream):
-        for _ in range(e2e_steps):
-            ge.replay()
+        for s_ in range(e2e_steps):
+            ges[s_ % len(ges)].replay()
     stream.synchronize()
     e2e_s = max_over_ranks(time.perf_counter() - t0, device)
     assert int(Ahost.sum()) == VECTORS
@@ -515,6 +562,10 @@ def run_ours(args):
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "u32 (F_q exact; int8 weights, dp4a digits)",
             "data": "synthetic", "config": dict(workload_config(), mode=args.mode,
+                                                step_schedule=("overlap: each step's server call, then its "
+                                                               "decode beside the next batch's encode on a "
+                                                               "second stream" if overlap else
+                                                               "serial: encode, server, decode"),
                                                 **({"masks": "prepared ahead and reused across the timed steps "
                                                              "(the same work as fresh masks)"} if args.mode == "boost"
                                                    else {})),
@@ -530,6 +581,7 @@ def run_ours(args):
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(Xhost.numel() * 4),
                     "d2h_bytes_per_step": int(Yhost.numel() * 4 + Ahost.numel() * 4),
                     "how": "CUDA graph of the public calls with pinned host copies inside, replayed"
+                           + ("; the next batch's copy-in and encode beside this batch's decode" if overlap else "")
                            + ("" if args.mode == "standard" else "; masks prepared ahead (boost encode and decode)")},
             "gpu_launches": launches_per_step * args.steps,
             "clocks": clk,
@@ -1043,6 +1095,9 @@ def main(argv=None):
                     help="batched workloads: all encodes, then all products, then all decodes "
                          "(phases), or each projection's three calls in order on one of "
                          "--server-streams streams (projections)")
+    ap.add_argument("--step-schedule", choices=["overlap", "serial"], default="overlap",
+                    help="batch1-4096 standard mode: overlap the next batch's encode with this batch's "
+                         "decode on a second stream, or run encode, server and decode in order")
     ap.add_argument("--mode", choices=["standard", "boost", "pipelined"], default="standard",
                     help="client mode of the batch-1 workload (Sec. 7.2): standard (masks drawn during "
                          "the step), boost (masks prepared ahead, untimed) or pipelined (standard mode "

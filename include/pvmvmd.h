@@ -23,8 +23,12 @@
  *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default
  *    stream).  Every call only enqueues work on that stream and returns;
  *    results are valid once the stream has been synchronised.  Calls that use
- *    one context must be ordered on one stream: a context's internal scratch
- *    is shared by its calls.
+ *    one context must be ordered on one stream (a context's internal scratch
+ *    is shared by its calls), with one exception: an encode
+ *    (pvmvmd_encode, pvmvmd_boost_prepare) and a decode
+ *    (pvmvmd_decode_verify, pvmvmd_boost_decode_verify) share no scratch, so
+ *    the encode of one batch may run on another stream while an earlier
+ *    batch is decoded.
  *  - Return value: PVMVMD_OK (0) or a negative PVMVMD_E_* status.  Nothing
  *    throws across the ABI.  A device-side bounded wait that expires is
  *    reported later by pvmvmd_device_status.

@@ -183,7 +183,9 @@ struct pvmvmd_ctx {
     pv::CodeDev gx, gy;
     uint32_t *PT = nullptr, *Q = nullptr;
     uint32_t *F = nullptr, *Fy = nullptr, *chal = nullptr, *g = nullptr, *u = nullptr;
-    unsigned long long *status = nullptr;
+    // scan status words of the encode (status) and of the challenges
+    // (status_y): an encode and a decode share no scratch
+    unsigned long long *status = nullptr, *status_y = nullptr;
     // lane-parallel encode scratch (null when scratch_batch < kLaneMinBatch)
     uint32_t *S = nullptr, *laux = nullptr;
     // decode: the challenge kernels run on `side`, forked from and joined
@@ -435,7 +437,6 @@ int preprocess_impl(const void *W_dev, bool w16, int m, int K, const pvmvmd_para
     };
     if ((st = upload_code(c, c->gx, *key, 0, c->Nx, s))) return fail(st);
     if ((st = upload_code(c, c->gy, *key, 1, c->Ny, s))) return fail(st);
-    const size_t statw = std::max(scan_status_words(c->Nx, c->sb), scan_status_words(c->Ny, c->ell));
     if (ctx_alloc(c, &c->PT, (size_t)c->Nx * m) != cudaSuccess ||
         ctx_alloc(c, &c->Q, (size_t)c->Ny * K) != cudaSuccess ||
         ctx_alloc(c, &c->F, (size_t)((c->sb + 3) & ~3) * c->Nx) != cudaSuccess ||  // lanes padded to 4
@@ -443,7 +444,8 @@ int preprocess_impl(const void *W_dev, bool w16, int m, int K, const pvmvmd_para
         ctx_alloc(c, &c->chal, (size_t)c->ell * 2 * c->t_y) != cudaSuccess ||
         ctx_alloc(c, &c->g, (size_t)c->ell * m) != cudaSuccess ||
         ctx_alloc(c, &c->u, (size_t)c->ell * K) != cudaSuccess ||
-        ctx_alloc(c, &c->status, statw) != cudaSuccess)
+        ctx_alloc(c, &c->status, scan_status_words(c->Nx, c->sb)) != cudaSuccess ||
+        ctx_alloc(c, &c->status_y, scan_status_words(c->Ny, c->ell)) != cudaSuccess)
         return fail(PVMVMD_E_NOMEM);
     if (cudaStreamCreateWithFlags(&c->side, cudaStreamNonBlocking) != cudaSuccess ||
         cudaEventCreateWithFlags(&c->fork, cudaEventDisableTiming) != cudaSuccess ||
@@ -674,9 +676,9 @@ int verify_chain(pvmvmd_ctx *ctx, const pvmvmd_key *challenge_key, const uint32_
                                       d.v2m, d.v1pm, ctx->m, ctx->rate, ctx->chal, nullptr, ctx->g, cs));
     } else {
         PV_CUDA(launch_sample_sparse(*challenge_key, kTagChallenge, 0, ctx->Ny, ctx->t_y, ctx->ell,
-                                     ctx->chal, ctx->status, scan_status_words(ctx->Ny, ctx->ell), cs));
+                                     ctx->chal, ctx->status_y, scan_status_words(ctx->Ny, ctx->ell), cs));
         PV_CUDA(launch_syndrome_scan(d.pi2inv, d.v2p, d.v1, ctx->Ny, ctx->chal, ctx->t_y, ctx->ell,
-                                     ctx->Fy, ctx->status, err, cs));
+                                     ctx->Fy, ctx->status_y, err, cs));
         PV_CUDA(launch_syndrome_gather(d.pi1inv, ctx->m, ctx->rate, ctx->Fy, ctx->Ny, nullptr, ctx->g,
                                        ctx->ell, cs));
     }

@@ -305,6 +305,30 @@ def test_server_mvm_extremes(pv):
         assert np.array_equal(pv.as_u32(pv.pvmvmd_server_mvm(Wd, Xd[0])), exp[0])
 
 
+@pytest.mark.parametrize("B", [1, 8, 64])
+@pytest.mark.parametrize("K", [131071, 131056])
+def test_server_mvm_max_k(pv, K, B):
+    """The largest K the ABI accepts (and the largest multiple of 16 below
+    it) on each server path, at the digit sums' extreme: M = -128 against
+    x_hat centred at -128 (1 + 2^8 + 2^16), whose three low signed base-256
+    digits are all -128, so each of those exact digit sums is 16384 K, just
+    below 2^31."""
+    assert K <= pv.PVMVMD_MAX_K and 16384 * pv.PVMVMD_MAX_K < 2**31
+    rng = np.random.default_rng(K + B)
+    W = rng.integers(-128, 128, size=(5, K), dtype=np.int8)
+    W[0] = -128
+    W[1] = 127
+    low = 128 * (1 + 256 + 65536)
+    X = rng.integers(0, Q, size=(B, K)).astype(np.uint32)
+    X[0] = Q - low                 # centred -low: digits (-128, -128, -128, 0)
+    if B > 1:
+        X[1] = (1 << 24) - low     # digits (-128, -128, -128, 1)
+    got = pv.as_u32(pv.pvmvmd_server_mvm(to_dev(W), to_dev(X if B > 1 else X[0])))
+    exp = np.stack([oracle.server_mvm(W, X[b]) for b in range(B)])
+    assert np.array_equal(got.reshape(B, 5), exp)
+    assert pv.pvmvmd_device_status() == 0
+
+
 def test_server_mvm_long_k_segments(pv):
     """K beyond one shared-memory segment of digit planes (60000 > 49152)."""
     rng = np.random.default_rng(2)
@@ -541,6 +565,52 @@ def test_server_mvm_multi_mixed_jobs(pv, wl):
     Xs_h = pv.as_u32(Xs)
     assert np.array_equal(pv.as_u32(Ys), np.stack([oracle.server_mvm(W[4], Xs_h[b]) for b in range(300)]))
     assert pv.pvmvmd_device_status() == 0
+
+
+@pytest.mark.parametrize("m,K,B,sb", [(4096, 4096, 8, 0),      # fused encode and challenges
+                                       (16, 50000, 3, 0),       # sample / scan / gather encode
+                                       (1024, 8192, 40, 40)])   # lane-parallel encode
+def test_encode_overlaps_decode(pv, wl, m, K, B, sb):
+    """An encode may run on another stream while an earlier batch of the
+    same context is decoded: both give exactly what they give in order."""
+    import torch
+    W = wl.weights_uniform(m, K, 70 + B)
+    x1, x2 = wl.int8_vectors(B, K, 71), wl.int8_vectors(B, K, 72)
+    params = _params(pv, scratch_batch=sb) if sb else None
+    Wd = to_dev(W)
+    ctx = pv.pvmvmd_preprocess(Wd, key=73, params=params)
+    X1, X2 = to_dev(field(x1)), to_dev(field(x2))
+    Xh1, st1 = pv.pvmvmd_encode(ctx, X1, key=74)
+    Yh1 = pv.pvmvmd_server_mvm(Wd, Xh1)
+    # in order
+    Xh2_ref, st2_ref = pv.pvmvmd_encode(ctx, X2, key=75)
+    Y1_ref, acc_ref = pv.pvmvmd_decode_verify(ctx, st1, Xh1, Yh1, challenge_key=76)
+    torch.cuda.synchronize()
+    assert pv.as_u32(acc_ref).tolist() == [1] * B
+    assert np.array_equal(oracle.centered(pv.as_u32(Y1_ref)), x1.astype(np.int64) @ W.astype(np.int64).T)
+    # overlapped: the decode on one stream, the next batch's encode on another
+    sa, sb_ = torch.cuda.Stream(), torch.cuda.Stream()
+    Xh2, st2 = torch.empty_like(Xh2_ref), torch.empty_like(st2_ref)
+    Y1, acc = torch.empty_like(Y1_ref), torch.empty_like(acc_ref)
+    for _ in range(3):
+        ev = torch.cuda.Event()
+        ev.record(torch.cuda.current_stream())
+        sa.wait_event(ev)
+        sb_.wait_event(ev)
+        Xh2.zero_(); st2.zero_(); Y1.zero_(); acc.zero_()
+        ev2 = torch.cuda.Event()
+        ev2.record(torch.cuda.current_stream())
+        sa.wait_event(ev2)
+        sb_.wait_event(ev2)
+        pv.pvmvmd_decode_verify(ctx, st1, Xh1, Yh1, challenge_key=76, Y=Y1, accept=acc, stream=sa)
+        pv.pvmvmd_encode(ctx, X2, key=75, Xhat=Xh2, st=st2, stream=sb_)
+        torch.cuda.synchronize()
+        assert np.array_equal(pv.as_u32(Xh2), pv.as_u32(Xh2_ref))
+        assert np.array_equal(pv.as_u32(st2), pv.as_u32(st2_ref))
+        assert np.array_equal(pv.as_u32(Y1), pv.as_u32(Y1_ref))
+        assert pv.as_u32(acc).tolist() == [1] * B
+    assert pv.pvmvmd_device_status() == 0
+    ctx.destroy()
 
 
 def test_long_code_uses_three_kernel_path(pv, wl):
