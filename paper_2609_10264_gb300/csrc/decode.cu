@@ -4,8 +4,8 @@
 //                       (sum of t_y rows of Q, cost (2t-1)n per repetition,
 //                       the e^T Q row of the cost table in Sec. 5.3).
 //  * k_decrypt          Y_b = y_hat_b - P e_x,b (t_x rows of P^T), many
-//                       short CTAs: 256 columns of one vector each, the
-//                       rows split over four groups; in boost mode
+//                       short CTAs: 512 columns of one vector each, the
+//                       rows split over two groups; in boost mode
 //                       (Sec. 7.2) P e_x,b was prepared ahead and is read
 //                       instead of the t_x rows of P^T.
 //  * k_check            accept_b = AND_q (L_q == R_q), L_q = u_q . x_hat_b,
@@ -150,7 +150,10 @@ __device__ __forceinline__ void pe_cols(const uint32_t *__restrict__ PT, int m, 
 // thread streams about t_x / 2 row segments (rounds of 8 loads in flight)
 // and the grid holds many short CTAs whatever m and B are.  The groups'
 // partial sums meet in shared memory.  (256 columns and 4 groups, or 1024
-// columns and 1 group, were 6 and 13 % slower at m = K = 8192, B = 256.)
+// columns and 1 group, were 6 and 13 % slower at m = K = 8192, B = 256.
+// At m = K = 4096, B = 100, where 800 CTAs are 1.3 waves of the 608
+// resident ones, 256 columns left the decode call at 54.6 us: its check
+// waits for the challenge kernels that run beside the decrypt.)
 // In boost mode (Sec. 7.2) P e_x,b was prepared ahead: Y_b = y_hat_b - mask_b.
 // The grid runs vectors fastest (blockIdx.x = b, blockIdx.y = column block),
 // so the CTAs in flight share a few column blocks and a row of P^T drawn by
