@@ -1001,6 +1001,68 @@ def run_encode_shape(args):
     return 0
 
 
+def run_encoder_shape(args):
+    """The RAA encoder G^T alone (App. B; the operation preprocessing runs):
+    ``--shape mxK`` encodes the m rows of an m x K matrix with G_x, i.e. L = m
+    lanes of length n = K into N_x = 8K positions, as pvmvmd_preprocess does
+    for P^T.  Each call is two gather / scale / decoupled-look-back
+    prefix-scan launches over the N_x x m array.  Inputs are uniform in F_q;
+    the arrays (a 4096 x 4096 shape moves 1.7 GB per call) exceed L2."""
+    import torch
+    rank, world, local = dist_env()
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    import paper_2609_10264_gb300 as pv
+    Q = pv.PVMVMD_Q
+    m, K = (int(v) for v in args.shape.lower().split("x")[:2])
+    gen = torch.Generator(device=device)
+    gen.manual_seed(85)
+    W = torch.randint(-127, 128, (16, K), generator=gen, device=device, dtype=torch.int8)
+    ctx = pv.pvmvmd_preprocess(W, key=86)
+    X = torch.randint(0, Q, (K, m), generator=gen, device=device, dtype=torch.int64).to(torch.int32)
+    N = ctx.N_x
+    Y = torch.empty((N, m), dtype=torch.int32, device=device)
+    scratch = torch.empty(pv.pvmvmd_code_encode_scratch(ctx, 0, m), dtype=torch.uint8, device=device)
+    stream = torch.cuda.Stream(device)
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            pv.pvmvmd_code_encode_lanes(ctx, 0, X, Y=Y, scratch=scratch, stream=stream)
+    stream.synchronize()
+    assert pv.pvmvmd_device_status(stream) == 0
+    clocks = ClockSampler(device.index)
+    clocks.start()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        t0.record(stream)
+        for _ in range(args.steps):
+            pv.pvmvmd_code_encode_lanes(ctx, 0, X, Y=Y, scratch=scratch, stream=stream)
+        t1.record(stream)
+    stream.synchronize()
+    clk = clocks.stop()
+    assert pv.pvmvmd_device_status(stream) == 0
+    ms = t0.elapsed_time(t1) / args.steps
+    # one read of X, the intermediate written and read once, Y written once
+    nbytes = 4 * m * (K + 3 * N)
+    peaks, kind = measured_peaks()
+    achieved = nbytes / (ms / 1e3) / 1e9
+    if rank == 0:
+        print(json.dumps({
+            "metric": "encoded field elements/s", "value": N * m / (ms / 1e3), "unit": "elements/s",
+            "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u32 (F_q exact)",
+            "data": "synthetic",
+            "config": {"workload": "encoder-shape", "lanes": m, "n": K, "N": N,
+                       "l2": "arrays larger than L2"},
+            "roofline": {"bound": "hbm", "kernel": "k_encode_scan (two launches per call)",
+                         "achieved": achieved, "peak": peaks.get("hbm_gbs", 0.0), "unit": "GB/s",
+                         "frac": achieved / peaks["hbm_gbs"] if peaks.get("hbm_gbs") else None,
+                         "peak_kind": f"{kind} hbm_gbs", "algorithmic_bytes_per_call": nbytes},
+            "gpu_launches": 2 * args.steps, "clocks": clk}), flush=True)
+    ctx.destroy()
+    return 0
+
+
 def run_server_shape(args):
     """The batched server product Y_hat = M X_hat alone on one m x K x B
     shape (``--shape MxKxB``), timed over --steps launches after --warmup.
@@ -1085,7 +1147,8 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-vectors", type=int, default=150)
     ap.add_argument("--server-mode", choices=["multi", "calls"], default="multi")
-    ap.add_argument("--workload", choices=["batch1-4096", "server-shape", "encode-shape", "token8b-b1", "bv-b8-1024"]
+    ap.add_argument("--workload", choices=["batch1-4096", "server-shape", "encode-shape", "encoder-shape",
+                                           "token8b-b1", "bv-b8-1024"]
                     + sorted(BATCHED),
                     default="batch1-4096")
     ap.add_argument("--shape", default="4096x4096x64",
@@ -1115,6 +1178,8 @@ def main(argv=None):
         return run_token(args)
     if args.workload == "bv-b8-1024":
         return run_bv(args)
+    if args.workload == "encoder-shape":
+        return run_encoder_shape(args)
     if args.workload == "encode-shape":
         return run_encode_shape(args)
     return run_ours(args)

@@ -287,6 +287,25 @@ int pvmvmd_server_mvm_i16(const int8_t *Whi_dev, const int8_t *Wlo_dev, int m, i
 int pvmvmd_preprocess_i16(const int16_t *W_dev, int m, int K, const pvmvmd_params *params,
                           const pvmvmd_key *key, void *stream, pvmvmd_ctx **out);
 
+/* The encoding Y = G^T X of one of a context's codes applied to L message
+ * vectors held as lanes (App. B, encoding direction: G^T = A^T V2 Pi2^T A^T
+ * V1 Pi1^T R^T, i.e. repeat r times, gather by pi1, scale by v1, prefix-sum,
+ * gather by pi2, scale by v2, prefix-sum, all mod q).  This is the operation
+ * pvmvmd_preprocess runs on the rows of M (P^T, which = 0) and its columns
+ * (Q, which = 1).  which = 0 selects G_x (n = K), 1 selects G_y (n = m);
+ * N = rate * n.  X_dev: n x L uint32 row-major (row i holds entry i of every
+ * lane), canonical; Y_dev: N x L uint32 row-major.  scratch_dev: caller-owned
+ * device memory of pvmvmd_code_encode_scratch bytes, 16-byte aligned, not
+ * overlapping X_dev or Y_dev; its contents need no initialisation.  The call
+ * allocates nothing and does not synchronise; it reads only the context's
+ * code tables, so it may run beside any other call on the context.
+ * Errors: PVMVMD_E_ARG for a null pointer or which outside {0, 1},
+ * PVMVMD_E_SHAPE for L < 1; a look-back wait that expires is reported by
+ * pvmvmd_device_status. */
+int pvmvmd_code_encode_scratch(const pvmvmd_ctx *ctx, int which, int L, size_t *bytes);
+int pvmvmd_code_encode_lanes(const pvmvmd_ctx *ctx, int which, const uint32_t *X_dev, int L,
+                             uint32_t *Y_dev, void *scratch_dev, void *stream);
+
 /* Synchronise `stream`, then read and clear the library's device error word:
  * PVMVMD_E_DEVICE_TIMEOUT if any kernel gave up a bounded wait since the last
  * call, else PVMVMD_OK (or PVMVMD_E_CUDA if synchronisation failed). */

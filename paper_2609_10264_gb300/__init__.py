@@ -103,6 +103,8 @@ SIGNATURES = {
     "pvmvmd_server_mvm_i16": (_i, [_vp, _vp, _i, _i, _vp, _i, _vp, _vp, _vp]),
     "pvmvmd_preprocess_i16": (_i, [_vp, _i, _i, ctypes.POINTER(pvmvmd_params), ctypes.POINTER(pvmvmd_key), _vp,
                                    ctypes.POINTER(_vp)]),
+    "pvmvmd_code_encode_scratch": (_i, [_vp, _i, _i, ctypes.POINTER(_sz)]),
+    "pvmvmd_code_encode_lanes": (_i, [_vp, _i, _vp, _i, _vp, _vp, _vp]),
     "pvmvmd_device_status": (_i, [_vp]),
     "pvmvmd_ctx_info": (_i, [_vp, ctypes.POINTER(pvmvmd_ctx_view)]),
     "pvmvmd_destroy": (None, [_vp]),
@@ -323,6 +325,33 @@ def pvmvmd_encode(ctx: Ctx, X, key, Xhat=None, st=None, stream=None):
                               _dev_ptr(st, "st", _u32_types(), B * 2 * ctx.t_x), _stream_ptr(stream)),
            "pvmvmd_encode")
     return Xhat, st
+
+
+def pvmvmd_code_encode_scratch(ctx: Ctx, which: int, L: int) -> int:
+    """Bytes of scratch pvmvmd_code_encode_lanes needs for L lanes."""
+    n = _sz()
+    _check(_lib.pvmvmd_code_encode_scratch(ctx.handle, which, L, ctypes.byref(n)), "pvmvmd_code_encode_scratch")
+    return n.value
+
+
+def pvmvmd_code_encode_lanes(ctx: Ctx, which: int, X, Y=None, scratch=None, stream=None):
+    """Y = G^T X for the context's code G_x (which = 0) or G_y (which = 1):
+    X is n x L (row i holds entry i of every lane), Y is N x L."""
+    import torch
+    n = ctx.K if which == 0 else ctx.m
+    N = n * ctx.rate
+    if X.dim() != 2 or X.shape[0] != n:
+        raise ValueError(f"X must be {n} x L")
+    L = X.shape[1]
+    if Y is None:
+        Y = _new_u32((N, L), X)
+    if scratch is None:
+        scratch = torch.empty(pvmvmd_code_encode_scratch(ctx, which, L), dtype=torch.uint8, device=X.device)
+    _check(_lib.pvmvmd_code_encode_lanes(ctx.handle, which, _dev_ptr(X, "X", _u32_types()), L,
+                                         _dev_ptr(Y, "Y", _u32_types(), N * L),
+                                         _dev_ptr(scratch, "scratch", (torch.uint8,)), _stream_ptr(stream)),
+           "pvmvmd_code_encode_lanes")
+    return Y
 
 
 def pvmvmd_server_mvm(W, Xhat, Yhat=None, stream=None):

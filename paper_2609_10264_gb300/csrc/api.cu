@@ -254,10 +254,10 @@ int encode_lanes_into(const CodeDev &d, uint32_t n, uint32_t r, const void *X, b
     const uint32_t N = n * r;
     cudaError_t e = cudaMemsetAsync(flags, 0, encode_scan_flag_words(N, nl) * 4, s);
     if (e == cudaSuccess)  // S = A^T V1 Pi1^T R^T X
-        e = launch_encode_scan(X, x_is_i8, ldx, d.pi1, r, d.v1, N, nl, S, nl, agg, incl, flags, err, s);
+        e = launch_encode_scan(X, x_is_i8, ldx, d.pi1, r, d.v1m, N, nl, S, nl, agg, incl, flags, err, s);
     if (e == cudaSuccess) e = cudaMemsetAsync(flags, 0, encode_scan_flag_words(N, nl) * 4, s);
     if (e == cudaSuccess)  // Y = A^T V2 Pi2^T S
-        e = launch_encode_scan(S, false, nl, d.pi2, 1, d.v2, N, nl, Y, ldy, agg, incl, flags, err, s);
+        e = launch_encode_scan(S, false, nl, d.pi2, 1, d.v2m, N, nl, Y, ldy, agg, incl, flags, err, s);
     return e == cudaSuccess ? PVMVMD_OK : PVMVMD_E_CUDA;
 }
 
@@ -741,6 +741,53 @@ int pvmvmd_boost_decode_verify(pvmvmd_ctx *ctx, const uint32_t *mask_out_dev,
     if (B < 1) return PVMVMD_E_SHAPE;
     return pv::decode_verify_batch(ctx, nullptr, mask_out_dev, Xhat_dev, Yhat_dev, B, challenge_key,
                                    Y_dev, accept_dev, static_cast<cudaStream_t>(stream));
+}
+
+namespace pv {
+namespace {
+// Scratch of pvmvmd_code_encode_lanes: S (N x L), agg, incl (value words),
+// flags, each at a 16-byte aligned offset.
+struct EncodeScratch {
+    size_t s_off, agg_off, incl_off, flag_off, bytes;
+};
+EncodeScratch encode_scratch_layout(uint32_t N, uint32_t L) {
+    auto up = [](size_t b) { return (b + 15) & ~(size_t)15; };
+    EncodeScratch e;
+    e.s_off = 0;
+    e.agg_off = up((size_t)N * L * 4);
+    e.incl_off = e.agg_off + up(encode_scan_value_words(N, L) * 4);
+    e.flag_off = e.incl_off + up(encode_scan_value_words(N, L) * 4);
+    e.bytes = e.flag_off + up(encode_scan_flag_words(N, L) * 4);
+    return e;
+}
+}  // namespace
+}  // namespace pv
+
+int pvmvmd_code_encode_scratch(const pvmvmd_ctx *ctx, int which, int L, size_t *bytes) {
+    if (!ctx || !bytes || (which != 0 && which != 1)) return PVMVMD_E_ARG;
+    if (L < 1) return PVMVMD_E_SHAPE;
+    const uint32_t N = which == 0 ? ctx->Nx : ctx->Ny;
+    *bytes = pv::encode_scratch_layout(N, (uint32_t)L).bytes;
+    return PVMVMD_OK;
+}
+
+int pvmvmd_code_encode_lanes(const pvmvmd_ctx *ctx, int which, const uint32_t *X_dev, int L,
+                             uint32_t *Y_dev, void *scratch_dev, void *stream) {
+    using namespace pv;
+    if (!ctx || !X_dev || !Y_dev || !scratch_dev || (which != 0 && which != 1)) return PVMVMD_E_ARG;
+    if (L < 1) return PVMVMD_E_SHAPE;
+    uint32_t *err = error_word();
+    if (!err) return PVMVMD_E_CUDA;
+    const CodeDev &d = which == 0 ? ctx->gx : ctx->gy;
+    const uint32_t n = which == 0 ? (uint32_t)ctx->K : (uint32_t)ctx->m;
+    const EncodeScratch lay = encode_scratch_layout(n * (uint32_t)ctx->rate, (uint32_t)L);
+    uint8_t *base = static_cast<uint8_t *>(scratch_dev);
+    return encode_lanes_into(d, n, (uint32_t)ctx->rate, X_dev, false, (size_t)L, (uint32_t)L, Y_dev, (size_t)L,
+                             reinterpret_cast<uint32_t *>(base + lay.s_off),
+                             reinterpret_cast<uint32_t *>(base + lay.agg_off),
+                             reinterpret_cast<uint32_t *>(base + lay.incl_off),
+                             reinterpret_cast<uint32_t *>(base + lay.flag_off), err,
+                             static_cast<cudaStream_t>(stream));
 }
 
 int pvmvmd_device_status(void *stream) {

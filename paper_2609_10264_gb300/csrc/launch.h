@@ -82,13 +82,14 @@ cudaError_t launch_syndrome_gather(const uint32_t *pi1inv, uint32_t n, uint32_t 
 
 // One accumulate stage of the encoding G^T w over L lanes (App. B, encoding
 // direction): Y[j][l] = sum_{j' <= j} vscale[j'] * X[perm[j'] / div][l] for
-// j < N.  X is int8 (lifted to F_q) when x_is_i8, else uint32.  The scratch
+// j < N, with vscale_m = vscale R mod q (Montgomery form, R = 2^32).  X is
+// int8 (lifted to F_q) when x_is_i8, else uint32.  The scratch
 // `flags` holds ceil(L/256) * ceil(N/kEncTile) + 1 words and must be zero.
 constexpr int kEncTile = 32;
 size_t encode_scan_flag_words(uint32_t N, uint32_t L);
 size_t encode_scan_value_words(uint32_t N, uint32_t L);
 cudaError_t launch_encode_scan(const void *X, bool x_is_i8, size_t ldx, const uint32_t *perm,
-                               uint32_t div, const uint32_t *vscale, uint32_t N, uint32_t L,
+                               uint32_t div, const uint32_t *vscale_m, uint32_t N, uint32_t L,
                                uint32_t *Y, size_t ldy, uint32_t *agg, uint32_t *incl,
                                uint32_t *flags, uint32_t *err, cudaStream_t s);
 

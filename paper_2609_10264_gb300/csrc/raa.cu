@@ -741,18 +741,23 @@ __global__ void __launch_bounds__(kFusedThreads) k_syndrome_fused(
 // One accumulate stage of G^T w (App. B, encoding direction) over L lanes:
 //   Y[j][l] = sum_{j' <= j} vscale[j'] * X[perm[j'] / div][l]
 // With (perm, div, vscale) = (pi1, r, v1) this is A^T V1 Pi1^T R^T; with
-// (pi2, 1, v2) it is A^T V2 Pi2^T.  A CTA owns 256 lanes and kEncTile
-// positions; tiles of one lane block are chained by a decoupled look-back
-// over per-lane aggregates (flags: 1 = aggregate, 2 = inclusive prefix).
+// (pi2, 1, v2) it is A^T V2 Pi2^T.  vscale_m holds vscale in Montgomery form
+// (v R mod q).  A CTA owns 256 lanes and kEncTile positions: the source row
+// and scale of each position are looked up once per CTA (in shared memory),
+// every thread then issues all kEncTile row loads of its lane before the
+// arithmetic, and tiles of one lane block are chained by a decoupled
+// look-back over per-lane aggregates (flags: 1 = aggregate, 2 = inclusive
+// prefix).
 // -----------------------------------------------------------------------------
 template <bool kI8>
 __global__ void __launch_bounds__(256) k_encode_scan(const void *__restrict__ Xv, size_t ldx,
                                                     const uint32_t *__restrict__ perm, uint32_t div,
-                                                    const uint32_t *__restrict__ vscale, uint32_t N,
+                                                    const uint32_t *__restrict__ vscale_m, uint32_t N,
                                                     uint32_t L, uint32_t *__restrict__ Y, size_t ldy,
                                                     uint32_t *agg, uint32_t *incl, uint32_t *flags,
                                                     uint32_t *__restrict__ err) {
-    __shared__ uint32_t s_ticket, s_flag;
+    __shared__ uint32_t s_ticket, s_nagg, s_state;
+    __shared__ uint32_t s_src[kEncTile], s_vs[kEncTile];
     const int tid = threadIdx.x;
     const uint32_t nlb = (L + 255) / 256;
     const uint32_t ntiles = (N + kEncTile - 1) / kEncTile;
@@ -767,22 +772,27 @@ __global__ void __launch_bounds__(256) k_encode_scan(const void *__restrict__ Xv
     const uint32_t l = lb * 256 + tid;
     const bool lane_ok = l < L;
     const uint32_t j0 = tile * kEncTile;
+    if (tid < kEncTile) {
+        const uint32_t j = j0 + tid;
+        s_src[tid] = j < N ? __ldg(perm + j) / div : 0u;
+        s_vs[tid] = j < N ? __ldg(vscale_m + j) : 0u;  // 0 past N: adds nothing
+    }
+    __syncthreads();
 
     uint32_t v[kEncTile];
+#pragma unroll
+    for (int u = 0; u < kEncTile; ++u) {
+        const bool ok = lane_ok && j0 + u < N;
+        const size_t src = (size_t)s_src[u] * ldx + l;
+        if (kI8)
+            v[u] = ok ? flift_i8(static_cast<const int8_t *>(Xv)[src]) : 0u;
+        else
+            v[u] = ok ? static_cast<const uint32_t *>(Xv)[src] : 0u;
+    }
     uint32_t run = 0;
 #pragma unroll
     for (int u = 0; u < kEncTile; ++u) {
-        const uint32_t j = j0 + u;
-        uint32_t x = 0;
-        if (j < N && lane_ok) {
-            const size_t src = __ldg(perm + j) / div;
-            if (kI8)
-                x = flift_i8(static_cast<const int8_t *>(Xv)[src * ldx + l]);
-            else
-                x = static_cast<const uint32_t *>(Xv)[src * ldx + l];
-            x = fmul(__ldg(vscale + j), x);
-        }
-        run = fadd(run, x);
+        run = fadd(run, fmul_mont(v[u], s_vs[u]));
         v[u] = run;
     }
 
@@ -799,26 +809,51 @@ __global__ void __launch_bounds__(256) k_encode_scan(const void *__restrict__ Xv
         __threadfence();
         __syncthreads();
         if (tid == 0) st_release_u32(fl + slot, 1u);
-        for (uint32_t j = tile - 1;; --j) {
-            const size_t ps = (size_t)lb * ntiles + j;
-            if (tid == 0) {
-                uint32_t f, spins = 0;
-                while ((f = ld_acquire_u32(fl + ps)) == 0u) {
+        // Look back over windows of 32 predecessors at once: warp 0 reads
+        // their flags (lane i: tile hi - i) until every tile newer than the
+        // nearest inclusive one has published its aggregate, then all
+        // threads add those aggregates and that inclusive prefix for their
+        // lanes with independent loads.  Tile 0 is always inclusive, so the
+        // walk ends there at the latest.
+        const size_t base = (size_t)lb * ntiles;
+        int32_t hi = (int32_t)tile - 1;  // newest predecessor not yet added
+        for (;;) {
+            if (tid < 32) {
+                const int32_t j = hi - tid;
+                uint32_t spins = 0, nagg = 32, state = 0;  // 0: go on, 1: inclusive found, 2: gave up
+                for (;;) {
+                    const uint32_t f = j >= 0 ? ld_acquire_u32(fl + base + j) : 2u;
+                    const unsigned incl_mask = __ballot_sync(kFull, f == 2u);
+                    const unsigned zero_mask = __ballot_sync(kFull, f == 0u);
+                    nagg = incl_mask ? (uint32_t)(__ffs(incl_mask) - 1) : 32u;
+                    const unsigned need = nagg >= 32u ? kFull : ((1u << nagg) - 1u);
+                    if ((zero_mask & need) == 0u) {
+                        state = incl_mask ? 1u : 0u;
+                        break;
+                    }
                     if (++spins > kSpinLimit) {
-                        record_error(err, kErrScanTimeout);
-                        f = 2u;
+                        if (tid == 0) record_error(err, kErrScanTimeout);
+                        nagg = 0;
+                        state = 2;
                         break;
                     }
                     __nanosleep(32);
                 }
-                s_flag = f;
+                if (tid == 0) {
+                    s_nagg = nagg;
+                    s_state = state;
+                }
             }
             __syncthreads();
-            const uint32_t f = s_flag;
-            prefix = fadd(prefix, f == 2u ? ld_cg_u32(incl + ps * 256 + tid)
-                                          : ld_cg_u32(agg + ps * 256 + tid));
-            __syncthreads();
-            if (f == 2u || j == 0) break;
+            const int nagg = (int)s_nagg;
+            const uint32_t state = s_state;
+            __syncthreads();  // s_nagg / s_state are rewritten for the next window
+#pragma unroll 8
+            for (int c = 0; c < nagg; ++c) prefix = fadd(prefix, ld_cg_u32(agg + (base + hi - c) * 256 + tid));
+            if (state == 1u && hi - nagg >= 0)
+                prefix = fadd(prefix, ld_cg_u32(incl + (base + hi - nagg) * 256 + tid));
+            if (state != 0u) break;
+            hi -= 32;
         }
         incl[slot * 256 + tid] = fadd(run, prefix);
         __threadfence();
@@ -1267,17 +1302,17 @@ size_t encode_scan_value_words(uint32_t N, uint32_t L) {
 }
 
 cudaError_t launch_encode_scan(const void *X, bool x_is_i8, size_t ldx, const uint32_t *perm,
-                               uint32_t div, const uint32_t *vscale, uint32_t N, uint32_t L,
+                               uint32_t div, const uint32_t *vscale_m, uint32_t N, uint32_t L,
                                uint32_t *Y, size_t ldy, uint32_t *agg, uint32_t *incl,
                                uint32_t *flags, uint32_t *err, cudaStream_t s) {
     const size_t ctas = encode_scan_flag_words(N, L) - 1;
     if (ctas == 0) return cudaSuccess;
     if (ctas > 0x7fffffffu) return cudaErrorInvalidValue;
     if (x_is_i8)
-        k_encode_scan<true><<<(unsigned)ctas, 256, 0, s>>>(X, ldx, perm, div, vscale, N, L, Y, ldy,
+        k_encode_scan<true><<<(unsigned)ctas, 256, 0, s>>>(X, ldx, perm, div, vscale_m, N, L, Y, ldy,
                                                            agg, incl, flags, err);
     else
-        k_encode_scan<false><<<(unsigned)ctas, 256, 0, s>>>(X, ldx, perm, div, vscale, N, L, Y, ldy,
+        k_encode_scan<false><<<(unsigned)ctas, 256, 0, s>>>(X, ldx, perm, div, vscale_m, N, L, Y, ldy,
                                                             agg, incl, flags, err);
     return cudaGetLastError();
 }

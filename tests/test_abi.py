@@ -94,6 +94,11 @@ def test_bad_arguments_rejected_before_device_use(pv):
     assert lib.pvmvmd_encode(None, one, 1, None, one, one, None) == pv.PVMVMD_E_ARG
     assert lib.pvmvmd_decode_verify(None, one, one, one, 1, None, one, one, None) == pv.PVMVMD_E_ARG
     assert lib.pvmvmd_ctx_info(None, None) == pv.PVMVMD_E_ARG
+    nbytes = ctypes.c_size_t()
+    assert lib.pvmvmd_code_encode_scratch(None, 0, 4, ctypes.byref(nbytes)) == pv.PVMVMD_E_ARG
+    assert lib.pvmvmd_code_encode_scratch(one, 2, 4, ctypes.byref(nbytes)) == pv.PVMVMD_E_ARG
+    assert lib.pvmvmd_code_encode_lanes(one, 0, one, 4, None, one, None) == pv.PVMVMD_E_ARG
+    assert lib.pvmvmd_code_encode_lanes(one, -1, one, 4, one, one, None) == pv.PVMVMD_E_ARG
     lib.pvmvmd_destroy(None)
 
 

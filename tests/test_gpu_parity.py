@@ -613,6 +613,33 @@ def test_encode_overlaps_decode(pv, wl, m, K, B, sb):
     ctx.destroy()
 
 
+@pytest.mark.parametrize("m,K,which,L", [(64, 300, 0, 300), (300, 64, 1, 257), (4096, 4096, 0, 4096)])
+def test_code_encode_lanes(pv, wl, m, K, which, L):
+    """G^T over lanes (the encoder of App. B that preprocessing runs) equals
+    the oracle's encoding lane by lane, with ragged lane blocks; with the
+    rows of M as lanes it reproduces the context's P^T."""
+    W = wl.weights_uniform(m, K, 90)
+    ctx = pv.pvmvmd_preprocess(to_dev(W), key=91)
+    pp = oracle.PublicParams(W, oracle.key_from_seed(91), with_tables=False)
+    code = pp.Gx if which == 0 else pp.Gy
+    n = K if which == 0 else m
+    rng = np.random.default_rng(92)
+    X = rng.integers(0, Q, size=(n, L)).astype(np.uint32)
+    X[:, 0] = Q - 1
+    X[:, -1] = 0
+    Y = pv.as_u32(pv.pvmvmd_code_encode_lanes(ctx, which, to_dev(X)))
+    assert Y.shape == (n * ctx.rate, L)
+    for l in sorted({0, 1, L // 2, L - 1, *rng.integers(0, L, 8).tolist()}):
+        assert np.array_equal(Y[:, l], code.encode(X[:, l])), l
+    if which == 0 and L == m:
+        v, _ = ctx_tables(pv, ctx)
+        PT = pv.as_u32(pv.device_view(v.PT, v.N_x * m).view(v.N_x, m))
+        got = pv.as_u32(pv.pvmvmd_code_encode_lanes(ctx, 0, to_dev(field(W.T.copy()))))
+        assert np.array_equal(got, PT)
+    assert pv.pvmvmd_device_status() == 0
+    ctx.destroy()
+
+
 def test_long_code_uses_three_kernel_path(pv, wl):
     """K = 50000 gives N_x = 400000, too long for one cluster's shared memory,
     so encode takes the sample / look-back scan / gather kernels; the result
