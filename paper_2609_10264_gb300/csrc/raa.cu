@@ -747,10 +747,12 @@ __global__ void __launch_bounds__(kFusedThreads) k_syndrome_fused(
 // every thread then issues all kEncTile row loads of its lane before the
 // arithmetic, and tiles of one lane block are chained by a decoupled
 // look-back over per-lane aggregates (flags: 1 = aggregate, 2 = inclusive
-// prefix).
+// prefix).  At 32 positions per tile the kernel is held to 64 registers, four
+// CTAs per SM: 0.755 against 0.823 ms per 4096 x 4096 encoding at three CTAs
+// (80 registers); 16-position tiles, twice as many per chain, took 1.16 ms.
 // -----------------------------------------------------------------------------
 template <bool kI8>
-__global__ void __launch_bounds__(256) k_encode_scan(const void *__restrict__ Xv, size_t ldx,
+__global__ void __launch_bounds__(256, 4) k_encode_scan(const void *__restrict__ Xv, size_t ldx,
                                                     const uint32_t *__restrict__ perm, uint32_t div,
                                                     const uint32_t *__restrict__ vscale_m, uint32_t N,
                                                     uint32_t L, uint32_t *__restrict__ Y, size_t ldy,
