@@ -3,9 +3,12 @@
 A step is one pass of the whole online path over one batch of synthetic
 inputs (the 4096 x 4096 single-projection workload, batch 1):
     pvmvmd_encode        (100 vectors)
-    pvmvmd_server_mvm    100 times at batch 1 (one GEMV per vector)
+    pvmvmd_server_mvm    100 times at batch 1 (one grouped call)
     pvmvmd_decode_verify (100 vectors)
-Preprocessing (P^T and Q) happens once, before timing.  The 100 GEMVs rotate
+By default (--step-schedule overlap) the next batch's encode runs on a second
+stream beside this batch's decode; every step still encodes, multiplies and
+decodes 100 vectors.  Preprocessing (P^T and Q) happens once, before timing.
+The 100 GEMVs rotate
 over 64 copies of the weights (1 GiB in all), so every timed GEMV streams its
 matrix from HBM rather than from the 126 MB L2.
 
@@ -35,6 +38,57 @@ M = K = 4096
 VECTORS = 100
 REPLICAS = 64
 SEED_W, SEED_X = 2, 3
+
+
+# --------------------------------------------------------------------------- host CPU and the oracle on all cores
+
+def host_cpu() -> dict:
+    """The host's logical CPU count and model (from /proc/cpuinfo)."""
+    import platform
+    model = ""
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                key, _, val = line.partition(":")
+                key, val = key.strip().lower(), val.strip()
+                if key == "model name" and val:
+                    model = val
+                    break
+                if key == "cpu part" and val and not model:
+                    model = "CPU part " + val
+    except OSError:
+        pass
+    return {"cpu_count": os.cpu_count(), "model": model or platform.machine()}
+
+
+_ORACLE_W = None
+
+
+def _oracle_rows_init(W):
+    global _ORACLE_W
+    _ORACLE_W = W
+
+
+def _oracle_rows(job):
+    import oracle
+    x, r0, r1 = job
+    return oracle.server_mvm(_ORACLE_W[r0:r1], x)
+
+
+def oracle_rows_parallel(W, X, procs: int):
+    """The oracle's server MVM (unchanged) of every vector of X with the rows
+    of W split over `procs` spawned processes.  Returns (field MACs, seconds,
+    the product of the last vector)."""
+    import multiprocessing as mp
+    m = W.shape[0]
+    bounds = [(m * i // procs, m * (i + 1) // procs) for i in range(procs)]
+    with mp.get_context("spawn").Pool(procs, initializer=_oracle_rows_init, initargs=(W,)) as pool:
+        pool.map(_oracle_rows, [(X[0], r0, r1) for r0, r1 in bounds])  # every worker has loaded the oracle
+        t0 = time.perf_counter()
+        for x in X:
+            parts = pool.map(_oracle_rows, [(x, r0, r1) for r0, r1 in bounds])
+        dt = time.perf_counter() - t0
+    return len(X) * W.size, dt, np.concatenate(parts)
 
 
 # --------------------------------------------------------------------------- distributed helpers
@@ -547,14 +601,25 @@ def run_ours(args):
     assert int(Ahost.sum()) == VECTORS
     e2e_value = world * macs_per_step * e2e_steps / e2e_s
 
-    cpu = None
+    cpu = cpu_all = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         n = args.cpu_vectors
-        macs, dt = OracleWorkload().full_vectors(n)
+        ow = OracleWorkload()
+        macs, dt = ow.full_vectors(n)
+        host = host_cpu()
         cpu = {"value": macs / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
                "sample": f"{n} vector round trips (encrypt, server MVM, verify, decrypt) cycling over "
                          f"the workload's {VECTORS} vectors; single-threaded C oracle on the host; "
-                         "its preprocessing untimed"}
+                         "its preprocessing untimed", "host": host}
+        # the oracle's server MVM on every core: rows of W split over processes
+        procs = max(1, host["cpu_count"] or 1)
+        Xo = np.stack([ow.x[b % VECTORS] for b in range(8 * procs)])
+        macs_p, dt_p, y_last = oracle_rows_parallel(ow.W, Xo, procs)
+        assert np.array_equal(y_last, ow.o.server_mvm(ow.W, Xo[-1]))
+        cpu_all = {"value": macs_p / dt_p, "unit": UNIT, "cores": procs, "kind": "oracle",
+                   "sample": f"server MVM only (the bulk of a round trip) of {len(Xo)} vectors, the rows "
+                             f"of W split over {procs} spawned processes running the unchanged C oracle",
+                   "host": host}
 
     if rank == 0:
         line = {
@@ -578,6 +643,7 @@ def run_ours(args):
                          "algorithmic_bytes_per_launch": gemv_bytes * (VECTORS if args.server_mode == "multi" else 1),
                          "launch_ms": srv_ms if args.server_mode == "multi" else srv_ms / VECTORS},
             "cpu_baseline": cpu,
+            "cpu_baseline_all_cores": cpu_all,
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(Xhost.numel() * 4),
                     "d2h_bytes_per_step": int(Yhost.numel() * 4 + Ahost.numel() * 4),
                     "how": "CUDA graph of the public calls with pinned host copies inside, replayed"

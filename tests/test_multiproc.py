@@ -56,3 +56,20 @@ def test_bench_rejects_short_warmup(argv):
     import bench
     with pytest.raises(SystemExit):
         bench.main(argv)
+
+
+def test_oracle_rows_parallel_matches_oracle():
+    """The all-cores CPU baseline: the oracle's server MVM with the rows of W
+    split over spawned processes gives the single-process oracle's result."""
+    import numpy as np
+
+    import bench
+    import oracle
+    rng = np.random.default_rng(5)
+    W = rng.integers(-128, 128, size=(37, 96), dtype=np.int8)
+    X = rng.integers(0, oracle.Q, size=(3, 96)).astype(np.uint32)
+    macs, dt, y = bench.oracle_rows_parallel(W, X, 2)
+    assert macs == 3 * 37 * 96 and dt > 0
+    assert np.array_equal(y, oracle.server_mvm(W, X[-1]))
+    info = bench.host_cpu()
+    assert info["cpu_count"] >= 1 and info["model"]
