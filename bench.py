@@ -1129,6 +1129,45 @@ def run_encoder_shape(args):
     return 0
 
 
+def run_preprocess_shape(args):
+    """pvmvmd_preprocess alone for an m x K int8 matrix (``--shape mxK``):
+    both codes sampled on the host, P^T = G_x^T M^T and Q = G_y^T M encoded
+    on the device, wall-clock per call (allocation included).  The paper's
+    single-threaded CPU figures for the same step are 6.03 s at n = 2^12 and
+    135.8 s at n = 2^14 (context, another machine)."""
+    import torch
+    rank, world, local = dist_env()
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    import paper_2609_10264_gb300 as pv
+    m, K = (int(v) for v in args.shape.lower().split("x")[:2])
+    gen = torch.Generator(device=device)
+    gen.manual_seed(87)
+    W = torch.randint(-127, 128, (m, K), generator=gen, device=device, dtype=torch.int8)
+    stream = torch.cuda.Stream(device)
+    for w in range(args.warmup):
+        pv.pvmvmd_preprocess(W, key=88 + w, stream=stream).destroy()
+    torch.cuda.synchronize(device)
+    times = []
+    for s_ in range(args.steps):
+        t0 = time.perf_counter()
+        ctx = pv.pvmvmd_preprocess(W, key=200 + s_, stream=stream)
+        stream.synchronize()
+        times.append(time.perf_counter() - t0)
+        assert pv.pvmvmd_device_status(stream) == 0
+        ctx.destroy()
+    sec = statistics.median(times)
+    if rank == 0:
+        print(json.dumps({
+            "metric": "preprocessing time", "value": sec, "unit": "s", "n_gpus": 1, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": sec * 1e3, "higher_is_better": False, "scaling": "weak",
+            "vs_baseline": None, "dtype": "u32 (F_q exact)", "data": "synthetic",
+            "config": {"workload": "preprocess-shape", "m": m, "K": K, "N_x": 8 * K, "N_y": 8 * m,
+                       "tables_bytes": 4 * 8 * 2 * m * K, "timing": "wall clock per call, median"},
+            "gpu_launches": None}), flush=True)
+    return 0
+
+
 def run_server_shape(args):
     """The batched server product Y_hat = M X_hat alone on one m x K x B
     shape (``--shape MxKxB``), timed over --steps launches after --warmup.
@@ -1214,7 +1253,7 @@ def main(argv=None):
     ap.add_argument("--cpu-vectors", type=int, default=150)
     ap.add_argument("--server-mode", choices=["multi", "calls"], default="multi")
     ap.add_argument("--workload", choices=["batch1-4096", "server-shape", "encode-shape", "encoder-shape",
-                                           "token8b-b1", "bv-b8-1024"]
+                                           "preprocess-shape", "token8b-b1", "bv-b8-1024"]
                     + sorted(BATCHED),
                     default="batch1-4096")
     ap.add_argument("--shape", default="4096x4096x64",
@@ -1246,6 +1285,8 @@ def main(argv=None):
         return run_bv(args)
     if args.workload == "encoder-shape":
         return run_encoder_shape(args)
+    if args.workload == "preprocess-shape":
+        return run_preprocess_shape(args)
     if args.workload == "encode-shape":
         return run_encode_shape(args)
     return run_ours(args)
