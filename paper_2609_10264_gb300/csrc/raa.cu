@@ -749,7 +749,9 @@ __global__ void __launch_bounds__(kFusedThreads) k_syndrome_fused(
 // look-back over per-lane aggregates (flags: 1 = aggregate, 2 = inclusive
 // prefix).  At 32 positions per tile the kernel is held to 64 registers, four
 // CTAs per SM: 0.755 against 0.823 ms per 4096 x 4096 encoding at three CTAs
-// (80 registers); 16-position tiles, twice as many per chain, took 1.16 ms.
+// (80 registers); 16-position tiles, twice as many per chain, took 1.16 ms,
+// and 64-position tiles (two halves of 32, the first half's sums in shared
+// memory) 0.864 ms at 80 registers and 1.49 ms held to 64.
 // -----------------------------------------------------------------------------
 template <bool kI8>
 __global__ void __launch_bounds__(256, 4) k_encode_scan(const void *__restrict__ Xv, size_t ldx,
