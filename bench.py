@@ -440,7 +440,8 @@ def run_ours(args):
         # this batch (set k): server, then decode on `stream`; the next batch
         # (set 1 - k): encode on enc_stream, forked after the server call.
         # (Forked at the start of the step instead, beside the server call,
-        # it saved nothing: 338 against 330 us per step.)
+        # it saved nothing: 338 against 330 us per step; enqueueing the
+        # decode before the encode changed nothing either.)
         pv.pvmvmd_server_mvm_multi(jobs_sets[k], stream=stream)
         fork = torch.cuda.Event()
         fork.record(stream)
