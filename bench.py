@@ -121,7 +121,12 @@ def barrier(device=None):
 # --------------------------------------------------------------------------- clocks
 
 class ClockSampler:
-    """Samples nvidia-smi SM clocks and throttle reasons while running."""
+    """Samples nvidia-smi SM clocks and throttle reasons while running.
+
+    start() returns once the first sample has arrived, so the sampler is live
+    before the timed region begins; region_started() marks the start of the
+    region, and stop() summarises the samples taken from that mark on (the
+    timed region and the load queued after it, see clock_tail)."""
     FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
               "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
               "clocks_event_reasons.sw_power_cap")
@@ -130,8 +135,9 @@ class ClockSampler:
         self.index = index
         self.proc = None
         self.lines = []
+        self.t_mark = None
 
-    def start(self):
+    def start(self, wait_s: float = 3.0):
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
@@ -141,14 +147,21 @@ class ClockSampler:
             self.thread.start()
         except (OSError, ValueError):
             self.proc = None
+            return
+        t_end = time.monotonic() + wait_s
+        while not self.lines and time.monotonic() < t_end and self.proc.poll() is None:
+            time.sleep(0.01)
+
+    def region_started(self):
+        self.t_mark = time.monotonic()
 
     def _read(self):
         for line in self.proc.stdout:
-            self.lines.append(line.strip())
+            self.lines.append((time.monotonic(), line.strip()))
 
     def stop(self):
         if self.proc is None:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
         self.proc.terminate()
         try:
             self.proc.wait(timeout=5)
@@ -157,7 +170,8 @@ class ClockSampler:
         self.thread.join(timeout=2)
         sm, smax, reasons = [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for line in self.lines:
+        lines = [ln for ts, ln in self.lines if self.t_mark is None or ts >= self.t_mark]
+        for line in lines:
             parts = [p.strip() for p in line.split(",")]
             if len(parts) < 7:
                 continue
@@ -172,7 +186,19 @@ class ClockSampler:
         if not sm:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
-                "samples": len(sm)}
+                "samples": len(sm), "window": "from the start of the timed region to the end of the "
+                                              "same steps queued after it (clock tail)"}
+
+
+def clock_tail(replay, ms_per_call: float, seconds: float = 0.5) -> int:
+    """Queue untimed calls of `replay` after the timed region's stop event, so
+    that the clock sampler (100 ms period) sees the GPU under the same load
+    for `seconds` even when the timed region itself is only milliseconds
+    long.  Returns the number of calls queued."""
+    n = max(1, int(seconds * 1e3 / max(ms_per_call, 1e-3)))
+    for i in range(n):
+        replay(i)
+    return n
 
 
 # --------------------------------------------------------------------------- roofline inputs
@@ -273,7 +299,7 @@ def run_reference(args):
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total_s / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u32 (F_q, exact)",
-        "data": "synthetic", "config": workload_config(),
+        "data": "synthetic", "config": arm_config(args),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                          "sample": f"per step: server MVM of one vector on {R} sampled rows; every "
                                    f"{every} steps one full vector (encrypt, MVM, verify, decrypt); "
@@ -294,6 +320,17 @@ def workload_config():
             "parallelism": "replicas (one independent workload per GPU)",
             "server": "100 independent batch-1 products (one weight copy each) in one "
                       "pvmvmd_server_mvm_multi call"}
+
+
+def arm_config(args) -> dict:
+    """The `config` of the default workload's line, identical for both arms."""
+    overlap = args.mode == "standard" and args.step_schedule == "overlap"
+    cfg = dict(workload_config(), mode=args.mode,
+               step_schedule=("overlap: each step's server call, then its decode beside the next batch's "
+                              "encode on a second stream" if overlap else "serial: encode, server, decode"))
+    if args.mode == "boost":
+        cfg["masks"] = "prepared ahead and reused across the timed steps (the same work as fresh masks)"
+    return cfg
 
 
 # --------------------------------------------------------------------------- our arm
@@ -510,21 +547,28 @@ def run_ours(args):
 
     # ---- timed region: whole steps, one graph per step
     nsteps_sets = len(g_steps)
+    w0, w1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with torch.cuda.stream(stream):
+        w0.record(stream)
         for w in range(args.warmup):
             g_steps[w % nsteps_sets].replay()
+        w1.record(stream)
     stream.synchronize()
+    ms_est = w0.elapsed_time(w1) / args.warmup
     clocks = ClockSampler(device.index)
+    clocks.start()
     barrier(device)
     torch.cuda.synchronize(device)
-    clocks.start()
     t_start = torch.cuda.Event(enable_timing=True)
     t_stop = torch.cuda.Event(enable_timing=True)
+    clocks.region_started()
     with torch.cuda.stream(stream):
         t_start.record(stream)
         for s in range(args.steps):
             g_steps[s % nsteps_sets].replay()
         t_stop.record(stream)
+        # untimed: the same steps, so that the clock samples see this load
+        clock_tail(lambda i: g_steps[(args.steps + i) % nsteps_sets].replay(), ms_est)
     stream.synchronize()
     torch.cuda.synchronize(device)
     clk = clocks.stop()
@@ -622,19 +666,11 @@ def run_ours(args):
                              f"of W split over {procs} spawned processes running the unchanged C oracle",
                    "host": host}
 
-    if rank == 0:
-        line = {
+    line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "u32 (F_q exact; int8 weights, dp4a digits)",
-            "data": "synthetic", "config": dict(workload_config(), mode=args.mode,
-                                                step_schedule=("overlap: each step's server call, then its "
-                                                               "decode beside the next batch's encode on a "
-                                                               "second stream" if overlap else
-                                                               "serial: encode, server, decode"),
-                                                **({"masks": "prepared ahead and reused across the timed steps "
-                                                             "(the same work as fresh masks)"} if args.mode == "boost"
-                                                   else {})),
+            "data": "synthetic", "config": arm_config(args),
             "hbm_gbs_gemv": achieved,
             "phases_ms": {"encode": enc_ms, "server_100_gemv": srv_ms, "decode_verify": dec_ms},
             "roofline": {"bound": "hbm", "kernel": "k_gemv_multi (batch-1 field GEMV, 100 requests per launch)",
@@ -653,8 +689,21 @@ def run_ours(args):
             "gpu_launches": launches_per_step * args.steps,
             "clocks": clk,
         }
-        print(json.dumps(line), flush=True)
     ctx.destroy()
+    del Wrep, Wd, jobs_sets, jobs, g_steps, ges, g_encs, g_decs, g_preps, g_srv
+    torch.cuda.synchronize(device)
+    torch.cuda.empty_cache()
+    if world == 1 and not args.no_extra_configs:
+        # the other configurations the metric is quoted on, as sub-records of
+        # this line: the 70B-class batched pipeline (the tensor-core half of
+        # the metric) and one 8B-class token at batch 1
+        line["configs"] = {
+            "layer70b-b256": measure_batched(args, "layer70b-b256", device, rank, world,
+                                             with_cpu=not args.no_cpu_baseline),
+            "token8b-b1": measure_token(args, device, rank),
+        }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
@@ -678,22 +727,16 @@ BATCHED = {
 }
 
 
-def run_batched(args):
+def measure_batched(args, workload, device, rank=0, world=1, with_cpu=True, with_e2e=True):
     """Step = for every projection of the layer: encode B vectors, the
     batched server product, decode+verify.  The server phase (tcgen05 digit
     GEMM) is reported against the 16-bit tensor peak: it executes
-    2 * m * K * 4 * B fp16 flops (four digit planes per field MAC)."""
+    2 * m * K * 4 * B fp16 flops (four digit planes per field MAC).  Returns
+    the record (a dict); run_batched prints it as the bench line."""
     import torch
-    rank, world, local = dist_env()
-    if world > 1:
-        import torch.distributed as dist
-        torch.cuda.set_device(local)
-        dist.init_process_group("nccl")
-    device = torch.device("cuda", local)
-    torch.cuda.set_device(device)
     import paper_2609_10264_gb300 as pv
     from paper_2609_10264_gb300 import workloads as wl
-    spec = BATCHED[args.workload]
+    spec = BATCHED[workload]
     B = spec["B"]
     stream = torch.cuda.Stream(device)
     projs = []
@@ -711,6 +754,7 @@ def run_batched(args):
                           Yh=torch.empty((B, m), dtype=torch.int32, device=device),
                           Y=torch.empty((B, m), dtype=torch.int32, device=device),
                           acc=torch.empty(B, dtype=torch.int32, device=device)))
+
     def enc():
         for p in projs:
             pv.pvmvmd_encode(p["ctx"], p["X"], 21, Xhat=p["Xh"], st=p["st"], stream=stream)
@@ -741,21 +785,34 @@ def run_batched(args):
     # independent projections)
     proj_streams = [torch.cuda.Stream(device) for _ in range(max(1, args.server_streams))]
 
-    def pipelined():
+    def pipelined(host=None):
         fork = torch.cuda.Event()
         fork.record(stream)
         for ss in proj_streams:
             ss.wait_event(fork)
         for j, p in enumerate(projs):
             ss = proj_streams[j % len(proj_streams)]
-            pv.pvmvmd_encode(p["ctx"], p["X"], 21, Xhat=p["Xh"], st=p["st"], stream=ss)
-            pv.pvmvmd_server_mvm(p["W"], p["Xh"], Yhat=p["Yh"], stream=ss)
-            pv.pvmvmd_decode_verify(p["ctx"], p["st"], p["Xh"], p["Yh"], 22, Y=p["Y"], accept=p["acc"], stream=ss)
+            with torch.cuda.stream(ss):
+                src = p["X"]
+                if host is not None:      # end to end: the inputs arrive from pinned host memory
+                    p["Xin"].copy_(p["Xhost"], non_blocking=True)
+                    src = p["Xin"]
+                pv.pvmvmd_encode(p["ctx"], src, 21, Xhat=p["Xh"], st=p["st"], stream=ss)
+                pv.pvmvmd_server_mvm(p["W"], p["Xh"], Yhat=p["Yh"], stream=ss)
+                pv.pvmvmd_decode_verify(p["ctx"], p["st"], p["Xh"], p["Yh"], 22, Y=p["Y"], accept=p["acc"],
+                                        stream=ss)
+                if host is not None:
+                    p["Yhost"].copy_(p["Y"], non_blocking=True)
+                    p["Ahost"].copy_(p["acc"], non_blocking=True)
         for ss in proj_streams:
             join = torch.cuda.Event()
             join.record(ss)
             stream.wait_event(join)
 
+    def phases():
+        enc(); srv(); dec()
+
+    step_fn = pipelined if args.schedule == "projections" else phases
     # eager runs of every schedule that is captured below (the first call on
     # a stream sizes its scratch, which a capture may not do)
     with torch.cuda.stream(stream):
@@ -763,7 +820,7 @@ def run_batched(args):
         if args.schedule == "projections":
             pipelined()
     stream.synchronize()
-    pv.pvmvmd_device_status(stream)
+    assert pv.pvmvmd_device_status(stream) == 0
     for p in projs:
         assert int(p["acc"].sum()) == B
         rows = [0, p["m"] // 2, p["m"] - 1]
@@ -780,29 +837,34 @@ def run_batched(args):
     # give the phase split
     g_step = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g_step, stream=stream):
-        if args.schedule == "projections":
-            pipelined()
-        else:
-            enc(); srv(); dec()
+        step_fn()
+    w0, w1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with torch.cuda.stream(stream):
+        for g in graphs:
+            g.replay()
+        w0.record(stream)
         for _ in range(args.warmup):
             g_step.replay()
-            for g in graphs:
-                g.replay()
+        w1.record(stream)
     stream.synchronize()
+    ms_est = w0.elapsed_time(w1) / args.warmup
     clocks = ClockSampler(device.index)
+    clocks.start()
     barrier(device)
     torch.cuda.synchronize(device)
-    clocks.start()
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
+    clocks.region_started()
     with torch.cuda.stream(stream):
         t0.record(stream)
         for s in range(args.steps):
             g_step.replay()
         t1.record(stream)
+        clock_tail(lambda i: g_step.replay(), ms_est)
     stream.synchronize()
+    torch.cuda.synchronize(device)
     clk = clocks.stop()
+    barrier(device)
     ms = max_over_ranks(t0.elapsed_time(t1), device)
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
     with torch.cuda.stream(stream):
@@ -816,49 +878,157 @@ def run_batched(args):
     macs = sum(p["m"] * p["K"] for p in projs) * B
     flops = 2 * 4 * macs
     peaks, kind = measured_peaks()
+
+    # the dominant projection's product alone, by CUDA events on its stream
+    big = max(projs, key=lambda p: p["m"] * p["K"])
+    with torch.cuda.stream(stream):   # sizes this stream's scratch before the capture
+        pv.pvmvmd_server_mvm(big["W"], big["Xh"], Yhat=big["Yh"], stream=stream)
+    stream.synchronize()
+    g_big = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_big, stream=stream):
+        pv.pvmvmd_server_mvm(big["W"], big["Xh"], Yhat=big["Yh"], stream=stream)
+    k0, k1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    reps = max(args.steps, 5)
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            g_big.replay()
+        k0.record(stream)
+        for _ in range(reps):
+            g_big.replay()
+        k1.record(stream)
+    stream.synchronize()
+    big_ms = k0.elapsed_time(k1) / reps
+
     if B <= 16 and all(p["K"] % 16 == 0 for p in projs):
         # a few vectors run the dp4a GEMV over four vectors' digit planes: one
         # pass over M per four vectors, x_hat read and y_hat written once
         nbytes = sum(p["m"] * p["K"] * ((B + 3) // 4) + 4 * B * (p["K"] + p["m"]) for p in projs)
-        roof = {"bound": "hbm", "kernel": "k_gemv_nb (dp4a, four vectors per pass over M)",
+        roof = {"bound": "hbm", "kernel": "k_gemv_nb (dp4a, four vectors per pass over M), server phase",
                 "achieved": nbytes / (ph[1] / 1e3) / 1e9, "peak": peaks.get("hbm_gbs", 0.0), "unit": "GB/s",
-                "peak_kind": f"{kind} hbm_gbs", "bytes_per_step": nbytes}
+                "peak_kind": f"{kind} hbm_gbs", "bytes_per_step": nbytes, "traffic": None}
         dtype = "u32 (F_q exact; int8 weights, dp4a digits)"
     else:
         peak = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"])
-        roof = {"bound": "tensor", "kernel": "k_batched (tcgen05 kind::f16 digit GEMM)",
-                "achieved": flops / (ph[1] / 1e3) / 1e12, "peak": peak, "unit": "TFLOP/s",
-                "peak_kind": f"{kind} bf16_tflops_sustained", "flops_per_step": flops}
+        big_flops = 2 * 4 * big["m"] * big["K"] * B
+        roof = {"bound": "tensor",
+                "kernel": f"k_batched (tcgen05 kind::f16 digit GEMM) on {big['name']} "
+                          f"{big['m']}x{big['K']}x{B}, one pvmvmd_server_mvm call (k_digit_tiles + k_batched) "
+                          "timed alone by CUDA events",
+                "achieved": big_flops / (big_ms / 1e3) / 1e12, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                "peak_kind": f"{kind} bf16_tflops (burst; the kernel timed alone)", "traffic": None,
+                "flops_per_launch": big_flops, "launch_ms": big_ms,
+                "server_phase": {"achieved": flops / (ph[1] / 1e3) / 1e12, "peak": peak, "unit": "TFLOP/s",
+                                 "frac": flops / (ph[1] / 1e3) / 1e12 / peak,
+                                 "peak_kind": f"{kind} bf16_tflops_sustained (inside the step)",
+                                 "flops_per_step": flops}}
         dtype = "u32 (F_q exact; fp16 digit MMAs, fp32 TMEM accumulation)"
     roof["frac"] = roof["achieved"] / roof["peak"] if roof["peak"] else None
     roof["field_macs_per_step"] = macs
     roof["field_mac_per_s_server"] = macs / (ph[1] / 1e3)
-    if rank == 0:
-        print(json.dumps({
-            "metric": METRIC, "value": world * macs * args.steps / (ms / 1e3), "unit": UNIT, "n_gpus": world,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-            "dtype": dtype, "data": "synthetic",
-            "config": {"workload": args.workload, "B": B, "projections": [[p["name"], p["m"], p["K"]] for p in projs],
-                       "schedule": args.schedule, "streams": args.server_streams},
-            "phases_ms": {"encode": ph[0], "server_batched": ph[2 - 1], "decode_verify": ph[2]},
-            "roofline": roof,
-            "gpu_launches": None, "clocks": clk}), flush=True)
+
+    e2e = None
+    if with_e2e:
+        for p in projs:
+            p["Xhost"] = pv_host_copy(p["X"])
+            p["Xin"] = torch.empty_like(p["X"])
+            p["Yhost"] = torch.empty((B, p["m"]), dtype=torch.int32).pin_memory()
+            p["Ahost"] = torch.empty(B, dtype=torch.int32).pin_memory()
+        with torch.cuda.stream(stream):
+            pipelined(host=True)
+        stream.synchronize()
+        g_e2e = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g_e2e, stream=stream):
+            pipelined(host=True)
+        with torch.cuda.stream(stream):
+            for _ in range(args.warmup):
+                g_e2e.replay()
+        stream.synchronize()
+        barrier(device)
+        n_e2e = max(2, args.steps)
+        te = time.perf_counter()
+        with torch.cuda.stream(stream):
+            for _ in range(n_e2e):
+                g_e2e.replay()
+        stream.synchronize()
+        e2e_s = max_over_ranks(time.perf_counter() - te, device)
+        for p in projs:
+            assert int(p["Ahost"].sum()) == B
+        e2e = {"value": world * macs * n_e2e / e2e_s, "unit": UNIT,
+               "h2d_bytes_per_step": int(sum(p["Xhost"].numel() * 4 for p in projs)),
+               "d2h_bytes_per_step": int(sum(p["Yhost"].numel() * 4 + p["Ahost"].numel() * 4 for p in projs)),
+               "how": "CUDA graph of the public calls (each projection's encode, product, decode on one of "
+                      f"{len(proj_streams)} streams) with pinned host copies of X in and Y, accept out, "
+                      "replayed; wall clock"}
+
+    cpu = None
+    if with_cpu and rank == 0:
+        # the oracle's server MVM (the per-MAC C loop, unchanged) on every host
+        # core, on a row sample of the dominant projection
+        host = host_cpu()
+        procs = max(1, host["cpu_count"] or 1)
+        rows = min(big["m"], 2048)
+        Xo = pv.as_u32(big["Xh"])[: min(B, 4 * procs)]
+        macs_p, dt_p, y_last = oracle_rows_parallel(np.ascontiguousarray(big["Wh"][:rows]), Xo, procs)
+        assert np.array_equal(y_last, pv.as_u32(big["Yh"])[len(Xo) - 1, :rows]), "oracle and GPU products differ"
+        cpu = {"value": macs_p / dt_p, "unit": UNIT, "cores": procs, "kind": "oracle",
+               "sample": f"server MVM only, {len(Xo)} masked vectors of the {big['name']} projection on its first "
+                         f"{rows} rows (K = {big['K']}), the rows split over {procs} spawned processes running "
+                         "the unchanged C oracle; its last product equals the GPU's",
+               "host": host}
+    rec = {
+        "metric": METRIC, "value": world * macs * args.steps / (ms / 1e3), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": dtype, "data": "synthetic",
+        "config": {"workload": workload, "B": B, "projections": [[p["name"], p["m"], p["K"]] for p in projs],
+                   "schedule": args.schedule, "streams": args.server_streams,
+                   "l2": "weights, P^T and Q of the layer exceed L2"},
+        "phases_ms": {"encode": ph[0], "server_batched": ph[1], "decode_verify": ph[2]},
+        "roofline": roof, "e2e": e2e, "cpu_baseline": cpu,
+        "gpu_launches": None, "clocks": clk}
     for p in projs:
         p["ctx"].destroy()
+    projs.clear()
+    torch.cuda.synchronize(device)
+    torch.cuda.empty_cache()
+    return rec
+
+
+def pv_host_copy(t):
+    """A pinned host copy of a device tensor."""
+    return t.cpu().pin_memory()
+
+
+def run_batched(args):
+    import torch
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    rec = measure_batched(args, args.workload, device, rank, world, with_cpu=not args.no_cpu_baseline)
+    if rank == 0:
+        print(json.dumps(rec), flush=True)
     return 0
 
 
-def run_token(args):
+TOKEN_GROUPS = (("q", "k", "v"), ("o",), ("gate", "up"), ("down",))
+
+
+def measure_token(args, device, rank=0):
     """One token of 32 independent 8B-class layers at batch 1 (the server's
-    side): the 7 projections of each layer as one grouped product call,
-    32 calls per token in one CUDA graph.  Weights are seeded int8 (Gaussian,
-    sigma 32, rounded and clipped), 6.98 GB per token, so every token streams
-    them from HBM; x_hat is uniform in F_q."""
+    side).  Within a layer the products depend on one another as in a
+    decoder: q, k and v read the layer input; o reads the attention output;
+    gate and up read the attention block's output; down reads the MLP's
+    hidden state.  So a token is 4 dependent grouped calls per layer,
+    {q,k,v} -> o -> {gate,up} -> down, 128 calls in order on one stream (one
+    CUDA graph).  Weights are seeded int8 (Gaussian, sigma 32, rounded and
+    clipped), 6.98 GB per token, so every token streams them from HBM; x_hat
+    is uniform in F_q.  The relaxed schedules (one grouped call per layer,
+    one per token) are reported beside it as context."""
     import torch
-    rank, world, local = dist_env()
-    device = torch.device("cuda", local)
-    torch.cuda.set_device(device)
     import paper_2609_10264_gb300 as pv
     from paper_2609_10264_gb300 import workloads as wl
     Q = pv.PVMVMD_Q
@@ -866,84 +1036,120 @@ def run_token(args):
     gen = torch.Generator(device=device)
     layers = []
     for l in range(nlayers):
-        trip = []
+        trip = {}
         for j, (name, (m, K)) in enumerate(wl.LAYER_8B.items()):
             gen.manual_seed(1000 + 7 * l + j)
             W = (torch.randn((m, K), generator=gen, device=device) * 32.0).round_().clamp_(-127, 127).to(torch.int8)
             xh = torch.randint(0, Q, (K,), generator=gen, device=device, dtype=torch.int64).to(torch.int32)
-            trip.append((W, xh, torch.empty(m, dtype=torch.int32, device=device)))
+            trip[name] = (W, xh, torch.empty(m, dtype=torch.int32, device=device))
         layers.append(trip)
-    jobs = [pv.mvm_jobs(t) for t in layers]
+    dep_jobs = [[pv.mvm_jobs([t[n] for n in grp]) for grp in TOKEN_GROUPS] for t in layers]
+    layer_jobs = [pv.mvm_jobs(list(t.values())) for t in layers]
+    all_jobs = pv.mvm_jobs([v for t in layers for v in t.values()])
     stream = torch.cuda.Stream(device)
 
-    def token():
+    def token_dep():
         for l in range(nlayers):
-            pv.pvmvmd_server_mvm_multi(jobs[l], stream=stream)
+            for jobs in dep_jobs[l]:
+                pv.pvmvmd_server_mvm_multi(jobs, stream=stream)
+
+    def token_layer():
+        for l in range(nlayers):
+            pv.pvmvmd_server_mvm_multi(layer_jobs[l], stream=stream)
+
+    def token_one():
+        pv.pvmvmd_server_mvm_multi(all_jobs, stream=stream)
 
     with torch.cuda.stream(stream):
-        token()
+        token_dep()
     stream.synchronize()
-    pv.pvmvmd_device_status(stream)
-    # exact check of sampled rows of one projection per layer (int64 numpy)
+    assert pv.pvmvmd_device_status(stream) == 0
+    # exact check of sampled rows of every projection of two layers (int64 numpy)
     for l in (0, nlayers - 1):
-        W, xh, yh = layers[l][6]
-        rows = [0, 1, W.shape[0] // 2, W.shape[0] - 1]
-        Wr = W[rows].cpu().numpy().astype(np.int64)
-        x = pv.as_u32(xh).astype(np.int64)
-        assert np.array_equal(pv.as_u32(yh)[rows].astype(np.int64), (Wr @ x) % Q), f"layer {l}"
-    g = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(g, stream=stream):
-        token()
+        for name, (W, xh, yh) in layers[l].items():
+            rows = [0, 1, W.shape[0] // 2, W.shape[0] - 1]
+            Wr = W[rows].cpu().numpy().astype(np.int64)
+            x = pv.as_u32(xh).astype(np.int64)
+            assert np.array_equal(pv.as_u32(yh)[rows].astype(np.int64), (Wr @ x) % Q), f"layer {l} {name}"
+    graphs = {}
+    for key, fn in (("dep", token_dep), ("layer", token_layer), ("one", token_one)):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            fn()
+        graphs[key] = g
+    w0, w1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with torch.cuda.stream(stream):
+        w0.record(stream)
         for _ in range(args.warmup):
-            g.replay()
+            graphs["dep"].replay()
+        w1.record(stream)
     stream.synchronize()
+    ms_est = w0.elapsed_time(w1) / args.warmup
     clocks = ClockSampler(device.index)
     clocks.start()
+    torch.cuda.synchronize(device)
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
+    clocks.region_started()
     with torch.cuda.stream(stream):
         t0.record(stream)
         for _ in range(args.steps):
-            g.replay()
+            graphs["dep"].replay()
         t1.record(stream)
+        clock_tail(lambda i: graphs["dep"].replay(), ms_est)
     stream.synchronize()
     clk = clocks.stop()
-    pv.pvmvmd_device_status(stream)
+    assert pv.pvmvmd_device_status(stream) == 0
     ms = t0.elapsed_time(t1) / args.steps
-    # the same 224 requests as one grouped call (the server's view when the
-    # layers' inputs are all known, e.g. when it replays a finished token)
-    all_jobs = pv.mvm_jobs([t for trip in layers for t in trip])
-    g1 = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(g1, stream=stream):
-        pv.pvmvmd_server_mvm_multi(all_jobs, stream=stream)
-    with torch.cuda.stream(stream):
-        for _ in range(args.warmup):
-            g1.replay()
-        t0.record(stream)
-        for _ in range(args.steps):
-            g1.replay()
-        t1.record(stream)
-    stream.synchronize()
-    ms_one = t0.elapsed_time(t1) / args.steps
+    relaxed = {}
+    for key in ("layer", "one"):
+        with torch.cuda.stream(stream):
+            for _ in range(args.warmup):
+                graphs[key].replay()
+            t0.record(stream)
+            for _ in range(args.steps):
+                graphs[key].replay()
+            t1.record(stream)
+        stream.synchronize()
+        relaxed[key] = t0.elapsed_time(t1) / args.steps
     macs = nlayers * sum(m * K for (m, K) in wl.LAYER_8B.values())
     nbytes = nlayers * sum(m * K + 4 * K + 4 * m for (m, K) in wl.LAYER_8B.values())
     peaks, kind = measured_peaks()
     achieved = nbytes / (ms / 1e3) / 1e9
+    del graphs, layers
+    torch.cuda.synchronize(device)
+    torch.cuda.empty_cache()
+    return {
+        "metric": METRIC, "value": macs / (ms / 1e3), "unit": UNIT, "n_gpus": 1, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "ms_per_token": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "u32 (F_q exact; int8 weights, dp4a digits)",
+        "data": "synthetic",
+        "config": {"workload": "token8b-b1", "layers": nlayers, "projections": list(wl.LAYER_8B),
+                   "schedule": "per layer {q,k,v} -> o -> {gate,up} -> down: 4 dependent grouped "
+                               "pvmvmd_server_mvm_multi calls, 128 per token, in order on one stream",
+                   "weight_bytes_per_token": nbytes,
+                   "l2": "6.98 GB of distinct weights per token (larger than L2)"},
+        "relaxed_schedules": {
+            "one_call_per_layer": {"ms": relaxed["layer"], "hbm_gbs": nbytes / (relaxed["layer"] / 1e3) / 1e9,
+                                   "note": "the 7 products of a layer in one call, ignoring o's and "
+                                           "down's dependence on q/k/v and gate/up"},
+            "one_call_per_token": {"ms": relaxed["one"], "hbm_gbs": nbytes / (relaxed["one"] / 1e3) / 1e9,
+                                   "note": "all 224 products in one call (a replay of a finished token)"}},
+        "roofline": {"bound": "hbm", "kernel": "k_gemv_multi (1-3 requests per launch, 128 dependent launches)",
+                     "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                     "frac": achieved / peaks["hbm_gbs"], "peak_kind": f"{kind} hbm_gbs", "traffic": None,
+                     "algorithmic_bytes_per_token": nbytes},
+        "gpu_launches": 4 * nlayers * args.steps, "clocks": clk}
+
+
+def run_token(args):
+    import torch
+    rank, world, local = dist_env()
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    rec = measure_token(args, device, rank)
     if rank == 0:
-        print(json.dumps({
-            "metric": METRIC, "value": macs / (ms / 1e3), "unit": UNIT, "n_gpus": 1, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "u32 (F_q exact; int8 weights, dp4a digits)", "data": "synthetic",
-            "config": {"workload": "token8b-b1", "layers": nlayers, "projections": list(wl.LAYER_8B),
-                       "calls_per_token": nlayers, "weight_bytes_per_token": nbytes,
-                       "l2": "6.98 GB of distinct weights per token (larger than L2)"},
-            "one_call_per_token": {"ms": ms_one, "hbm_gbs": nbytes / (ms_one / 1e3) / 1e9,
-                                   "value": macs / (ms_one / 1e3)},
-            "roofline": {"bound": "hbm", "kernel": "k_gemv_multi (7 requests per launch)", "achieved": achieved,
-                         "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],
-                         "peak_kind": f"{kind} hbm_gbs", "traffic": None},
-            "gpu_launches": nlayers * args.steps, "clocks": clk}), flush=True)
+        print(json.dumps(rec), flush=True)
     return 0
 
 
@@ -1251,6 +1457,8 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extra-configs", action="store_true",
+                    help="default workload: skip the 70B-class batched and 8B-class token sub-records")
     ap.add_argument("--cpu-vectors", type=int, default=150)
     ap.add_argument("--server-mode", choices=["multi", "calls"], default="multi")
     ap.add_argument("--workload", choices=["batch1-4096", "server-shape", "encode-shape", "encoder-shape",

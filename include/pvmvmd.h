@@ -175,17 +175,21 @@ int pvmvmd_server_mvm_multi(const pvmvmd_mvm_job *jobs, int count, void *stream)
  * latency-critical loop that cannot afford the regular call's first-use
  * allocation, or the device-wide synchronisation of replacing an outgrown
  * buffer.  It always runs the tensor-core digit product (also for B = 1),
- * whose bf16 digit tiles then live in one file-scope __device__ array of
+ * whose fp16 digit tiles then live in one file-scope __device__ array of
  * PVMVMD_NOALLOC_SCRATCH_BYTES (16 MiB) that every GPU which loads the
  * library holds until the process exits.  The tiles take
  * ceil(B/64) * ceil(K/64) * 32 KiB, so for example B <= 64 allows
  * K <= 32768 and B <= 256 allows K <= 8192; a larger problem returns
  * PVMVMD_E_SHAPE and does nothing.  The first call on each device looks up
  * the array's device address (cudaGetSymbolAddress) with that device
- * current; make that first call before any stream capture.  All calls share
- * the one array, so calls that overlap on the GPU (e.g. on two streams) race
- * and give wrong results; order them on one stream.  Arguments and results
- * are those of pvmvmd_server_mvm. */
+ * current.  With CUDA's lazy module loading (the default) that lookup is
+ * also when the device reserves the array, so make the first call on each
+ * device before the caller reserves the rest of its device memory, and
+ * before any stream capture; if the device cannot reserve the array then,
+ * the call returns PVMVMD_E_NOMEM.  All calls share the one array, so calls
+ * that overlap on the GPU (e.g. on two streams) race and give wrong
+ * results; order them on one stream.  Arguments and results are those of
+ * pvmvmd_server_mvm. */
 int pvmvmd_server_mvm_noalloc(const int8_t *W_dev, int m, int K, const uint32_t *Xhat_dev, int B,
                               uint32_t *Yhat_dev, void *stream);
 
@@ -310,6 +314,33 @@ int pvmvmd_code_encode_lanes(const pvmvmd_ctx *ctx, int which, const uint32_t *X
  * PVMVMD_E_DEVICE_TIMEOUT if any kernel gave up a bounded wait since the last
  * call, else PVMVMD_OK (or PVMVMD_E_CUDA if synchronisation failed). */
 int pvmvmd_device_status(void *stream);
+
+/* Test hook for the failure path of the bounded device waits (no paper
+ * counterpart; off by default).  Every wait of the library's kernels on
+ * another CTA or on the asynchronous units is bounded: when it expires the
+ * kernel records PVMVMD_E_DEVICE_TIMEOUT in the device error word and
+ * finishes (its results are then unspecified), instead of waiting forever.
+ * This call lets a test make one such wait expire on purpose, with a short
+ * limit, so that the expiry path itself runs:
+ *   PVMVMD_DEBUG_WAIT_SCAN     the single-pass look-back scan of the syndrome
+ *                              (encode of codes too long for a thread-block
+ *                              cluster): tile `index` of every vector
+ *                              publishes no status word, and look-back spins
+ *                              give up after `limit` polls;
+ *   PVMVMD_DEBUG_WAIT_PRODUCT  the tensor-core batched product: the second
+ *                              CTA of every pair withholds its report for
+ *                              K-block `index`, and pipeline waits give up
+ *                              after `limit` nanoseconds;
+ *   PVMVMD_DEBUG_WAIT_OFF      restore the normal behaviour (index and limit
+ *                              ignored).
+ * The setting is process-wide and is read when a kernel is launched (a
+ * captured graph keeps the value it was captured with).  Returns
+ * PVMVMD_E_ARG for an unknown site or a zero limit.  Not for production
+ * use: every affected call gives wrong results. */
+#define PVMVMD_DEBUG_WAIT_OFF 0
+#define PVMVMD_DEBUG_WAIT_SCAN 1
+#define PVMVMD_DEBUG_WAIT_PRODUCT 2
+int pvmvmd_debug_expire_wait(int site, uint32_t index, uint64_t limit);
 
 /* Fill *view with the context's public parameters. */
 int pvmvmd_ctx_info(const pvmvmd_ctx *ctx, pvmvmd_ctx_view *view);

@@ -16,6 +16,8 @@ Parity status of each function (what pins it is listed in the tests):
                                       build's own reading; see the design notes)
   raa_encode / raa_syndrome ........ pinned (dense App. B matrices, adjoint)
   server_mvm ....................... pinned (Python big-int brute force)
+  server_mvm_batch ................. pinned (big-int brute force, server_mvm
+                                      at extremes and at K = 131071)
   encrypt / decrypt / verify ....... pinned (completeness, Lemma 5.1 rate)
   BatchParams (Protocol 2) ......... pinned (dense Q~^T G' product, the
                                       bilinear identity, completeness,
@@ -230,6 +232,34 @@ def server_mvm(W: np.ndarray, xhat) -> np.ndarray:
     m, K = W.shape
     out = np.zeros(m, np.uint32)
     _load().orc_server_mvm(W, m, K, _u32a(xhat), out)
+    return out
+
+
+def server_mvm_batch(W: np.ndarray, Xhat, row_block: int = 4096) -> np.ndarray:
+    """The server's product for a batch (Sec. 6.1, y_hat = M x_hat for every
+    masked vector): Y[b] = (M Xhat[b]) mod q, B x m uint32.
+
+    The exact integer product of the int8 matrix with the canonical
+    representatives, then one reduction mod q.  A library matrix product
+    serves as the step: each x_hat entry (< 2^31) is written 2^16 h + l with
+    h < 2^15 and l < 2^16, and M h and M l are float64 products.  Every
+    product |w| l <= 2^7 * 2^16 is an integer, and every partial sum is below
+    2^7 * 2^16 * K < 2^40 for K < 2^17, so the float64 sums are exact in any
+    summation order.  Then Y = (2^16 (M h mod q) + (M l mod q)) mod q in int64.
+    Rows of M are taken in blocks of `row_block` to bound host memory."""
+    W = np.asarray(W, dtype=np.int8)
+    m, K = W.shape
+    if K >= 1 << 17:
+        raise ValueError("exact float64 sums need K < 2^17")
+    X = np.asarray(Xhat, dtype=np.uint32).reshape(-1, K)
+    hi = (X >> 16).astype(np.float64).T.copy()          # K x B
+    lo = (X & 0xFFFF).astype(np.float64).T.copy()
+    out = np.empty((X.shape[0], m), np.uint32)
+    for r0 in range(0, m, row_block):
+        Wf = W[r0:r0 + row_block].astype(np.float64)
+        ph = np.mod((Wf @ hi).astype(np.int64), Q)      # exact integers < 2^40
+        pl = np.mod((Wf @ lo).astype(np.int64), Q)
+        out[:, r0:r0 + row_block] = ((ph * 65536 + pl) % Q).T.astype(np.uint32)
     return out
 
 

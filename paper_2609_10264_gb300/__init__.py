@@ -6,7 +6,9 @@ torch.uint32; both are passed as raw 32-bit words).  Streams default to
 torch's current stream.  Errors raise PvmvmdError with the library's message.
 
 The library must be built (``python -m paper_2609_10264_gb300.build`` or
-``__graft_entry__.build()``); importing this package without it fails loudly.
+``__graft_entry__.build()``).  It is opened on the first call (or by
+``load_library()``), which fails loudly when it is missing: there is no
+fallback path.
 """
 from __future__ import annotations
 
@@ -106,6 +108,7 @@ SIGNATURES = {
     "pvmvmd_code_encode_scratch": (_i, [_vp, _i, _i, ctypes.POINTER(_sz)]),
     "pvmvmd_code_encode_lanes": (_i, [_vp, _i, _vp, _i, _vp, _vp, _vp]),
     "pvmvmd_device_status": (_i, [_vp]),
+    "pvmvmd_debug_expire_wait": (_i, [_i, ctypes.c_uint32, ctypes.c_uint64]),
     "pvmvmd_ctx_info": (_i, [_vp, ctypes.POINTER(pvmvmd_ctx_view)]),
     "pvmvmd_destroy": (None, [_vp]),
     "pvmvmd_strerror": (ctypes.c_char_p, [_i]),
@@ -127,7 +130,26 @@ def _load():
     return lib
 
 
-_lib = _load()
+class _Library:
+    """libpvmvmd.so, opened on first use.  Importing the package (for example
+    only its input generators) maps no CUDA library; the first call of any
+    entry point opens it and raises ImportError if it is not built."""
+    _handle = None
+
+    def __getattr__(self, name):
+        if _Library._handle is None:
+            _Library._handle = _load()
+        return getattr(_Library._handle, name)
+
+
+_lib = _Library()
+
+
+def load_library():
+    """Open libpvmvmd.so now (ImportError if it is missing) and return it."""
+    if _Library._handle is None:
+        _Library._handle = _load()
+    return _Library._handle
 
 
 def _check(status: int, where: str) -> None:
@@ -549,6 +571,16 @@ def pvmvmd_bv_check(ctx: BvCtx, X, Y, chal, u, key2, accept=None, stream=None):
                                 _stream_ptr(stream)),
            "pvmvmd_bv_check")
     return accept
+
+
+PVMVMD_DEBUG_WAIT_OFF = 0
+PVMVMD_DEBUG_WAIT_SCAN = 1
+PVMVMD_DEBUG_WAIT_PRODUCT = 2
+
+
+def pvmvmd_debug_expire_wait(site: int, index: int = 0, limit: int = 0) -> None:
+    """Test hook: make one bounded device wait expire (see the header)."""
+    _check(_lib.pvmvmd_debug_expire_wait(int(site), int(index), int(limit)), "pvmvmd_debug_expire_wait")
 
 
 def pvmvmd_device_status(stream=None) -> int:

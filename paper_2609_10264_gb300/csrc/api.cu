@@ -310,6 +310,16 @@ int read_and_clear_error() {
 
 uint32_t *library_error_word() { return error_word(); }
 
+namespace {
+std::mutex g_debug_mu;
+DebugWait g_debug;
+}  // namespace
+
+DebugWait debug_wait() {
+    std::lock_guard<std::mutex> lock(g_debug_mu);
+    return g_debug;
+}
+
 }  // namespace pv
 
 using namespace pv;
@@ -788,6 +798,17 @@ int pvmvmd_code_encode_lanes(const pvmvmd_ctx *ctx, int which, const uint32_t *X
                              reinterpret_cast<uint32_t *>(base + lay.incl_off),
                              reinterpret_cast<uint32_t *>(base + lay.flag_off), err,
                              static_cast<cudaStream_t>(stream));
+}
+
+int pvmvmd_debug_expire_wait(int site, uint32_t index, uint64_t limit) {
+    if (site != PVMVMD_DEBUG_WAIT_OFF && site != PVMVMD_DEBUG_WAIT_SCAN && site != PVMVMD_DEBUG_WAIT_PRODUCT)
+        return PVMVMD_E_ARG;
+    if (site != PVMVMD_DEBUG_WAIT_OFF && limit == 0) return PVMVMD_E_ARG;
+    std::lock_guard<std::mutex> lock(g_debug_mu);
+    g_debug.site = site;
+    g_debug.index = site == PVMVMD_DEBUG_WAIT_OFF ? 0u : index;
+    g_debug.limit = site == PVMVMD_DEBUG_WAIT_OFF ? 0u : limit;
+    return PVMVMD_OK;
 }
 
 int pvmvmd_device_status(void *stream) {

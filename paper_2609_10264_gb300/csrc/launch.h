@@ -139,6 +139,15 @@ cudaError_t func_attr(const void *fn, cudaFuncAttribute attr, int value);
 // The library's device error word on the current device (null on failure).
 uint32_t *library_error_word();
 
+// The failure-path test hook (pvmvmd_debug_expire_wait): which bounded wait
+// to make expire, where, and the shortened limit.  site 0 = off.
+struct DebugWait {
+    int site = 0;
+    uint32_t index = 0;
+    uint64_t limit = 0;
+};
+DebugWait debug_wait();
+
 // Verify part 1: u[q][k] = sum_j e_{q,j} Q[supp_{q,j}][k] (e_q^T Q).
 cudaError_t launch_verify_u(const uint32_t *Qm, int K, const uint32_t *chal, uint32_t t_y,
                             uint32_t ell, uint32_t *u, cudaStream_t s);

@@ -24,7 +24,7 @@
 // are added through distributed shared memory, each rank finishing a slice
 // of the vectors.
 //
-// Warp roles (576 threads per CTA):
+// Warp roles (608 threads per CTA, 19 warps):
 //   warps 0-7    convert the int8 M tile to fp16 in the 128-byte-swizzled
 //                K-major layout the MMA reads: warps 0-3 take the even
 //                K-blocks, warps 4-7 the odd ones (four threads per row);
@@ -58,7 +58,7 @@ namespace {
 constexpr int kBM = 128;            // rows of M per CTA
 constexpr int kBV = 64;             // vectors per CTA
 constexpr int kBN = 4 * kBV;        // MMA N (digit rows)
-constexpr int kBK = 64;             // K-elements per stage (128 bytes of bf16)
+constexpr int kBK = 64;             // K-elements per stage (128 bytes of fp16)
 constexpr int kStages = 5;
 constexpr int kRaw = 8;                 // raw int8 tiles of M in flight
 constexpr int kChunkBlocks = 16;    // 16 x 64 = 1024 K-elements per exact chunk
@@ -111,14 +111,15 @@ __device__ __forceinline__ uint64_t global_ns() {
     return t;
 }
 // Bounded wait for the phase of parity `parity`: false (and an error bit)
-// after kWaitNs nanoseconds or kWaitLimit attempts, whichever comes first.
+// after wait_ns nanoseconds (kWaitNs unless a test shortens it) or kWaitLimit
+// attempts, whichever comes first.
 constexpr uint64_t kWaitNs = 1000000000ull;
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, uint32_t *err) {
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, uint32_t *err, uint64_t wait_ns) {
     if (mbar_try(bar, parity)) return true;
     const uint64_t t0 = global_ns();
     for (uint32_t i = 0; i < kWaitLimit; ++i) {
         if (mbar_try(bar, parity)) return true;
-        if (global_ns() - t0 > kWaitNs) break;
+        if (global_ns() - t0 > wait_ns) break;
     }
     record_error(err, kErrMmaTimeout);
     return false;
@@ -127,8 +128,8 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, uint32
 // The same wait taken by a whole warp: every lane polls, and the warp goes on
 // only if every lane saw the phase, so the lanes stay converged for the
 // .sync.aligned tcgen05 instructions and the warp-level arrivals that follow.
-__device__ __forceinline__ bool mbar_wait_warp(uint64_t *bar, uint32_t parity, uint32_t *err) {
-    return __all_sync(kFull, mbar_wait(bar, parity, err));
+__device__ __forceinline__ bool mbar_wait_warp(uint64_t *bar, uint32_t parity, uint32_t *err, uint64_t wait_ns) {
+    return __all_sync(kFull, mbar_wait(bar, parity, err, wait_ns));
 }
 
 // Arrival on a barrier of any CTA of the cluster (address from mapa).
@@ -305,7 +306,7 @@ template <bool kVec>
 __global__ void __launch_bounds__(kThreads, 1)
     k_batched(const __grid_constant__ CUtensorMap tmap_w, const int8_t *__restrict__ W, int m, int K,
               const uint8_t *__restrict__ D, int nkb, int B, uint32_t *__restrict__ Yhat,
-              uint32_t *__restrict__ err) {
+              uint32_t *__restrict__ err, int skip_report, uint64_t wait_ns) {
     cg::cluster_group cluster = cg::this_cluster();
     extern __shared__ uint8_t smem_raw[];
     // full: this CTA's stage is complete -- the converter group's warps have
@@ -396,7 +397,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int i = grp; i < nblk; i += 2) {
                 const int s = i % kStages, rs = i % kRaw;
                 const uint32_t ph = (uint32_t)(i / kStages) & 1u, rph = (uint32_t)(i / kRaw) & 1u;
-                if (!mbar_wait_warp(&raw_full[rs], rph, err) || !mbar_wait_warp(&empty_bar[s], ph ^ 1u, err))
+                if (!mbar_wait_warp(&raw_full[rs], rph, err, wait_ns) || !mbar_wait_warp(&empty_bar[s], ph ^ 1u, err, wait_ns))
                     break;
                 const uint8_t *raw = smem + kRawOff + rs * kRawTile;
                 uint4 v[4];
@@ -427,7 +428,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                             w[e >> 2] |= (uint32_t)(uint8_t)W[(size_t)grow * K + k0 + e] << (8 * (e & 3));
                     v[j] = make_uint4(w[0], w[1], w[2], w[3]);
                 }
-                if (!mbar_wait_warp(&empty_bar[s], ph ^ 1u, err)) break;
+                if (!mbar_wait_warp(&empty_bar[s], ph ^ 1u, err, wait_ns)) break;
                 convert_store(smem + s * kStageBytes, v);
                 fence_async_smem();
                 __syncwarp();
@@ -441,7 +442,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t acc_empty_leader = cluster_addr(&acc_empty[0], leader);
         for (int c = 0; c < nchunks; ++c) {
             const int bsel = c & 1;
-            if (!mbar_wait_warp(&acc_full[bsel], (uint32_t)(c >> 1) & 1u, err)) break;
+            if (!mbar_wait_warp(&acc_full[bsel], (uint32_t)(c >> 1) & 1u, err, wait_ns)) break;
             tc_fence_after();
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
@@ -470,7 +471,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int i = 0; i < nblk; ++i) {
                 const int s = i % kStages;
                 const uint32_t ph = (uint32_t)(i / kStages) & 1u;
-                if (!mbar_wait(&empty_bar[s], ph ^ 1u, err)) break;
+                if (!mbar_wait(&empty_bar[s], ph ^ 1u, err, wait_ns)) break;
                 uint8_t *b = smem + s * kStageBytes + kATile;
                 mbar_arrive_tx(&full[s], kBHalf);
                 bulk_g2s(b, src + (size_t)i * kBTile, kBHalf, &full[s]);
@@ -478,7 +479,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             // copies in flight complete before the CTA may exit
             for (int i = max(0, issued - kStages); i < issued; ++i)
-                mbar_wait(&full[i % kStages], (uint32_t)(i / kStages) & 1u, err);
+                mbar_wait(&full[i % kStages], (uint32_t)(i / kStages) & 1u, err, wait_ns);
         }
     } else if (warp == kWarpWLoad) {
         // ------------------------------------------------ raw int8 tiles of M by TMA
@@ -487,14 +488,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int i = 0; i < nblk; ++i) {
                 const int rs = i % kRaw;
                 const uint32_t rph = (uint32_t)(i / kRaw) & 1u;
-                if (!mbar_wait(&raw_empty[rs], rph ^ 1u, err)) break;
+                if (!mbar_wait(&raw_empty[rs], rph ^ 1u, err, wait_ns)) break;
                 mbar_arrive_tx(&raw_full[rs], kRawTile);
                 tma_load_2d(smem + kRawOff + rs * kRawTile, &tmap_w, (kb0 + i) * kBK, m0, &raw_full[rs]);
                 issued = i + 1;
             }
             // copies in flight complete before the CTA may exit
             for (int i = max(0, issued - kRaw); i < issued; ++i)
-                mbar_wait(&raw_full[i % kRaw], (uint32_t)(i / kRaw) & 1u, err);
+                mbar_wait(&raw_full[i % kRaw], (uint32_t)(i / kRaw) & 1u, err, wait_ns);
         }
     } else if (half == 0) {
         // ------------------------------------------------ MMA issuer (even CTA)
@@ -502,14 +503,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             bool ok = true;
             for (int c = 0; c < nchunks && ok; ++c) {
                 const int bsel = c & 1;
-                if (!mbar_wait(&acc_empty[bsel], ((uint32_t)(c >> 1) & 1u) ^ 1u, err)) break;
+                if (!mbar_wait(&acc_empty[bsel], ((uint32_t)(c >> 1) & 1u) ^ 1u, err, wait_ns)) break;
                 tc_fence_after();
                 const uint32_t dcol = tmem + (uint32_t)(bsel * kBN);
                 const int i_end = min(nblk, (c + 1) * kChunkBlocks);
                 for (int i = c * kChunkBlocks; i < i_end; ++i) {
                     const int s = i % kStages;
                     const uint32_t ph = (uint32_t)(i / kStages) & 1u;
-                    if (!mbar_wait(&full[s], ph, err)) {
+                    if (!mbar_wait(&full[s], ph, err, wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -527,7 +528,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             // all issued MMAs have finished before TMEM is released
             mma_commit_pair(&mma_done, (uint16_t)(1u << leader));
-            mbar_wait(&mma_done, 0, err);
+            mbar_wait(&mma_done, 0, err, wait_ns);
         }
     } else {
         // ------------------------------------------------ stage relay (odd CTA)
@@ -536,7 +537,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int i = 0; i < nblk; ++i) {
                 const int s = i % kStages;
                 const uint32_t ph = (uint32_t)(i / kStages) & 1u;
-                if (!mbar_wait(&full[s], ph, err)) break;
+                if (!mbar_wait(&full[s], ph, err, wait_ns)) break;
+                // a failure-path test withholds one report, so that the even
+                // CTA's wait for this stage expires (off: skip_report < 0)
+                if (i == skip_report) continue;
                 mbar_arrive_cluster(full_leader + 8u * (uint32_t)s);
             }
         }
@@ -691,7 +695,11 @@ cudaError_t batched_launch(const int8_t *W, int m, int K, const uint32_t *Xhat, 
     attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    return cudaLaunchKernelEx(&cfg, kern, tmap, W, m, K, (const uint8_t *)D, nkb, B, Yhat, err);
+    const DebugWait dbg = debug_wait();
+    const int skip_report = dbg.site == PVMVMD_DEBUG_WAIT_PRODUCT ? (int)dbg.index : -1;
+    const uint64_t wait_ns = dbg.site == PVMVMD_DEBUG_WAIT_PRODUCT ? dbg.limit : kWaitNs;
+    return cudaLaunchKernelEx(&cfg, kern, tmap, W, m, K, (const uint8_t *)D, nkb, B, Yhat, err, skip_report,
+                              wait_ns);
 }
 
 }  // namespace
@@ -721,7 +729,9 @@ static __device__ __align__(256) uint8_t g_noalloc_tiles[kNoAllocBytes];
 
 // Device address of g_noalloc_tiles on the current device.  Host code may
 // not use the symbol itself (its host-side name is only a stand-in), so it is
-// looked up once per device, with that device current.
+// looked up once per device, with that device current.  Under lazy module
+// loading the lookup loads this file's module on the device, which is when
+// the device reserves the array.
 cudaError_t noalloc_tiles(uint8_t **out) {
     static std::mutex mu;
     static uint8_t *addr[64] = {nullptr};
@@ -753,7 +763,12 @@ extern "C" int pvmvmd_server_mvm_noalloc(const int8_t *W_dev, int m, int K, cons
     const size_t need = (size_t)nvt * nkb * kBTile;
     if (need > kNoAllocBytes) return PVMVMD_E_SHAPE;  // beyond the fixed buffer
     uint8_t *D = nullptr;
-    if (noalloc_tiles(&D) != cudaSuccess) return PVMVMD_E_CUDA;
+    const cudaError_t lookup = noalloc_tiles(&D);
+    if (lookup != cudaSuccess) {
+        (void)cudaGetLastError();
+        // under lazy module loading the lookup is when the array is reserved
+        return lookup == cudaErrorMemoryAllocation ? PVMVMD_E_NOMEM : PVMVMD_E_CUDA;
+    }
     uint32_t *err = library_error_word();
     if (!err) return PVMVMD_E_CUDA;
     cudaStream_t s = static_cast<cudaStream_t>(stream);

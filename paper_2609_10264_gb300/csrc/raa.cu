@@ -197,7 +197,7 @@ __global__ void __launch_bounds__(kScanThreads) k_syndrome_scan(
     const uint32_t *__restrict__ pi2inv, const uint32_t *__restrict__ v2p,
     const uint32_t *__restrict__ v1, uint32_t N, const uint32_t *__restrict__ sparse, uint32_t t,
     uint32_t count, uint32_t *__restrict__ F, unsigned long long *__restrict__ status,
-    uint32_t *__restrict__ err) {
+    uint32_t *__restrict__ err, uint32_t skip_tile, uint32_t spin_limit) {
     extern __shared__ uint32_t sm[];
     uint32_t *s_supp = sm;     // t
     uint32_t *s_suf = sm + t;  // t + 1
@@ -305,17 +305,20 @@ __global__ void __launch_bounds__(kScanThreads) k_syndrome_scan(
 
     if (tid == 0) {
         const uint32_t agg = s_agg;
+        // a failure-path test withholds this tile's status words, so that the
+        // look-back of the tile before it expires (off: skip_tile >= ntiles)
+        const bool publish = tile != skip_tile;
         uint32_t prefix = 0;
         if (tile == ntiles - 1) {
-            st_release_u64(st + tile, (2ull << 32) | agg);
+            if (publish) st_release_u64(st + tile, (2ull << 32) | agg);
         } else {
-            st_release_u64(st + tile, (1ull << 32) | agg);
+            if (publish) st_release_u64(st + tile, (1ull << 32) | agg);
             uint32_t j = tile + 1, spins = 0;
             for (;;) {
                 const unsigned long long w = ld_acquire_u64(st + j);
                 const uint32_t flag = (uint32_t)(w >> 32);
                 if (flag == 0u) {
-                    if (++spins > kSpinLimit) {
+                    if (++spins > spin_limit) {
                         record_error(err, kErrScanTimeout);
                         break;
                     }
@@ -326,7 +329,7 @@ __global__ void __launch_bounds__(kScanThreads) k_syndrome_scan(
                 if (flag == 2u || j + 1 >= ntiles) break;
                 ++j;
             }
-            st_release_u64(st + tile, (2ull << 32) | fadd(agg, prefix));
+            if (publish) st_release_u64(st + tile, (2ull << 32) | fadd(agg, prefix));
         }
         s_prefix = prefix;
     }
@@ -1284,8 +1287,11 @@ cudaError_t launch_syndrome_scan(const uint32_t *pi2inv, const uint32_t *v2p, co
     if (count == 0) return cudaSuccess;
     const size_t smem = (2 * (size_t)t + 1) * sizeof(uint32_t);
     const unsigned grid = count * scan_tiles(N);
+    const DebugWait dbg = debug_wait();
+    const bool inject = dbg.site == PVMVMD_DEBUG_WAIT_SCAN;
     k_syndrome_scan<<<grid, kScanThreads, smem, s>>>(pi2inv, v2p, v1, N, sparse, t, count, F, status,
-                                                     err);
+                                                     err, inject ? dbg.index : 0xFFFFFFFFu,
+                                                     inject ? (uint32_t)dbg.limit : kSpinLimit);
     return cudaGetLastError();
 }
 

@@ -55,6 +55,24 @@ def exact_product_rows(W: np.ndarray, x_int: np.ndarray, rows) -> np.ndarray:
     return W[rows].astype(np.int64) @ x_int.astype(np.int64)
 
 
+def exact_product(W: np.ndarray, x_int: np.ndarray) -> np.ndarray:
+    """Integer (not field) x_b . W for every vector, B x m int64: a float64
+    matrix product, exact while every partial sum stays below 2^53 (int8
+    weights and vectors: |sum| <= 2^14 K)."""
+    K = W.shape[1]
+    assert np.abs(x_int).max(initial=0) * 128 * K < 2**53
+    return (np.asarray(x_int, dtype=np.float64) @ W.astype(np.float64).T).astype(np.int64)
+
+
+def assert_equal_report(got: np.ndarray, exp: np.ndarray, what: str) -> None:
+    """Element-by-element equality; on failure name the count and the first
+    differing (vector, row) pairs."""
+    got, exp = np.asarray(got), np.asarray(exp)
+    assert got.shape == exp.shape, (what, got.shape, exp.shape)
+    bad = np.argwhere(got != exp)
+    assert bad.size == 0, f"{what}: {len(bad)} of {got.size} elements differ, first at {bad[:8].tolist()}"
+
+
 def sample_rows(m: int, k: int, seed: int) -> np.ndarray:
     rng = np.random.default_rng(seed)
     r = set(rng.choice(m, size=min(k, m), replace=False).tolist())

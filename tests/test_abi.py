@@ -116,3 +116,31 @@ def test_key_conventions_agree(pv):
     k = pv.make_key(s)
     assert list(k.k) == oracle.key_from_seed(s).tolist()
     assert list(pv.make_key(bytes(range(32))).k) == list(np.frombuffer(bytes(range(32)), "<u4"))
+
+
+def test_input_generators_map_no_cuda_library():
+    """The seeded input generators (which the oracle arm of the bench and the
+    oracle tests use) load without opening libpvmvmd.so: the package opens it
+    only on its first call."""
+    import subprocess
+    import sys
+    code = ("import sys; sys.path.insert(0, %r)\n"
+            "from paper_2609_10264_gb300 import workloads\n"
+            "workloads.weights_gaussian(4, 8, 0)\n"
+            "maps = open('/proc/self/maps').read()\n"
+            "assert 'libpvmvmd' not in maps, 'library mapped at import'\n"
+            "import paper_2609_10264_gb300 as pv\n"
+            "assert pv.pvmvmd_strerror(0) == 'success'\n"
+            "assert 'libpvmvmd' in open('/proc/self/maps').read()\n") % ROOT
+    r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+
+
+def test_debug_wait_hook_arguments(pv):
+    """The failure-path test hook is host-only state: it rejects unknown sites
+    and zero limits, and switches off cleanly."""
+    lib = pv._lib
+    assert lib.pvmvmd_debug_expire_wait(7, 0, 1) == pv.PVMVMD_E_ARG
+    assert lib.pvmvmd_debug_expire_wait(pv.PVMVMD_DEBUG_WAIT_SCAN, 0, 0) == pv.PVMVMD_E_ARG
+    assert lib.pvmvmd_debug_expire_wait(pv.PVMVMD_DEBUG_WAIT_PRODUCT, 3, 1000) == pv.PVMVMD_OK
+    assert lib.pvmvmd_debug_expire_wait(pv.PVMVMD_DEBUG_WAIT_OFF, 0, 0) == pv.PVMVMD_OK

@@ -4,7 +4,8 @@ import numpy as np
 import pytest
 
 import oracle
-from gpu_util import (Q, ctx_tables, field, pt_columns, q_columns, sample_rows, tamper,
+from gpu_util import (Q, assert_equal_report, ctx_tables, exact_product, field, pt_columns, q_columns,
+                      sample_rows, tamper,
                       to_dev)
 
 pytestmark = pytest.mark.gpu
@@ -386,21 +387,21 @@ def test_config2_round_trip(pv, wl):
 
 
 @pytest.mark.parametrize("layer", [0, 31])
-def test_config3_layer_gemv_sampled(pv, wl, layer):
-    """One 8B-class decoder layer at batch 1 (7 projections), sampled rows."""
+def test_config3_layer_gemv(pv, wl, layer):
+    """One 8B-class decoder layer at batch 1 (7 projections), every output."""
     for j, (name, (m, K)) in enumerate(wl.LAYER_8B.items()):
         W = wl.weights_gaussian(m, K, (3, layer, j))
         x = wl.field_vectors(1, K, (3, layer, j, 1))[0]
         got = pv.as_u32(pv.pvmvmd_server_mvm(to_dev(W), to_dev(x)))
-        rows = sample_rows(m, 48, layer * 10 + j)
-        assert np.array_equal(got[rows], oracle.server_mvm_rows(W, x, rows)), name
+        assert_equal_report(got, oracle.server_mvm_batch(W, x)[0], name)
 
 
-def _batched_pipeline_sampled(pv, W, B, seed, n_rows=24, n_verify=2):
-    """Preprocess/encode/server/decode_verify at a large shape; checks: P^T and
-    Q columns, every x_hat and mask, server outputs on sampled rows for all
-    vectors, decoded rows equal the exact integer product, all accepted, and
-    the oracle's verdict for a few vectors."""
+def _batched_pipeline(pv, W, B, seed, n_rows=24, n_verify=2):
+    """Preprocess/encode/server/decode_verify at a large shape.  Checks: P^T
+    and Q columns, every x_hat and mask, every element of the server's output
+    against the oracle, every decoded element against the exact integer
+    product (completeness), all accepted, and the oracle's verdict and
+    decryption for a few vectors."""
     m, K = W.shape
     x = np.random.default_rng(seed).integers(-127, 128, size=(B, K), dtype=np.int64)
     X = field(x)
@@ -423,12 +424,12 @@ def _batched_pipeline_sampled(pv, W, B, seed, n_rows=24, n_verify=2):
         assert np.array_equal(st_h[b], np.concatenate([s_o, v_o])), b
     Yh = pv.pvmvmd_server_mvm(Wd, Xh)
     Yh_h = pv.as_u32(Yh)
-    for b in range(B):
-        assert np.array_equal(Yh_h[b, rows], oracle.server_mvm_rows(W, Xh_h[b], rows)), b
+    # every output element, bit for bit
+    assert_equal_report(Yh_h, oracle.server_mvm_batch(W, Xh_h), "server product")
     Y, acc = pv.pvmvmd_decode_verify(ctx, st, Xh, Yh, challenge_key=seed + 2)
     Y_h = pv.as_u32(Y)
-    exact = (x @ W[rows].astype(np.int64).T)
-    assert np.array_equal(oracle.centered(Y_h[:, rows]), exact)
+    # completeness on every element: y = W x exactly (|W x| < q / 2)
+    assert_equal_report(oracle.centered(Y_h), exact_product(W, x), "decrypted output")
     assert pv.as_u32(acc).tolist() == [1] * B
     for b in range(n_verify):
         assert pp.verify(Xh_h[b], Yh_h[b], oracle.key_from_seed(seed + 2))
@@ -447,7 +448,7 @@ def test_config4_batched_8b(pv, wl, name):
     """8B-class layer shapes with 64 vectors per call (the batched product)."""
     m, K = wl.LAYER_8B[name]
     W = wl.weights_gaussian(m, K, (4, list(wl.LAYER_8B).index(name)))
-    _batched_pipeline_sampled(pv, W, 64, seed=400 + len(name))
+    _batched_pipeline(pv, W, 64, seed=400 + len(name))
 
 
 @pytest.mark.parametrize("name", ["q", "kv", "gate_up", "down"])
@@ -455,7 +456,32 @@ def test_config5_70b(pv, wl, name):
     """70B-class shapes with 256 vectors per call; the largest K is 28672."""
     m, K = wl.LAYER_70B[name]
     W = wl.weights_gaussian(m, K, (5, list(wl.LAYER_70B).index(name)))
-    _batched_pipeline_sampled(pv, W, 256, seed=500 + len(name), n_rows=12, n_verify=1)
+    _batched_pipeline(pv, W, 256, seed=500 + len(name), n_rows=12, n_verify=1)
+
+
+@pytest.mark.parametrize("m,K,B", [
+    (600, 1000, 70),      # K % 16 != 0: byte-load path; two vector tiles, the second ragged
+    (513, 4144, 130),     # TMA path; m crosses a CTA pair by one row; K % 64 = 48; three vector tiles
+    (1030, 16384, 257),   # five row pairs (the last ragged), five vector tiles (one vector in the last)
+    (257, 4100, 65),      # byte-load path, ragged in every dimension
+    (4096, 4096, 64),     # an 8B-class projection with 64 vectors (K split over the cluster)
+    (128, 8192, 512),     # one CTA pair on half-used rows, eight vector tiles, long K
+])
+def test_batched_product_full_multi_tile(pv, m, K, B):
+    """The tensor-core product on shapes that span several CTA pairs, vector
+    tiles and K-split ranks with ragged edges in m, K and B: every output
+    element equals the oracle's, with extreme weights and x_hat in some rows
+    and vectors."""
+    rng = np.random.default_rng(m * 7 + K * 3 + B)
+    W = rng.integers(-128, 128, size=(m, K), dtype=np.int8)
+    W[0] = -128
+    W[m - 1] = 127
+    X = rng.integers(0, Q, size=(B, K)).astype(np.uint32)
+    X[0] = (Q + 1) // 2
+    X[B - 1] = Q - 1
+    Y = pv.as_u32(pv.pvmvmd_server_mvm(to_dev(W), to_dev(X)))
+    assert_equal_report(Y, oracle.server_mvm_batch(W, X), f"{m}x{K}x{B}")
+    assert pv.pvmvmd_device_status() == 0
 
 
 def test_server_mvm_concurrent_streams(pv, wl):
@@ -478,11 +504,7 @@ def test_server_mvm_concurrent_streams(pv, wl):
                 outs.append(pv.pvmvmd_server_mvm(Wd, Xd, stream=s))
         torch.cuda.synchronize()
     for (W, X, _, _), Yh in zip(ins, outs):
-        m = W.shape[0]
-        rows = sample_rows(m, 16, 53)
-        Yh_h = pv.as_u32(Yh)
-        for b in range(X.shape[0]):
-            assert np.array_equal(Yh_h[b, rows], oracle.server_mvm_rows(W, X[b], rows)), b
+        assert_equal_report(pv.as_u32(Yh), oracle.server_mvm_batch(W, X), str(W.shape))
     assert pv.pvmvmd_device_status() == 0
 
 
@@ -512,7 +534,7 @@ def test_lane_encode_long_tiles(pv, wl, L):
 def test_small_batch_server_product(pv, wl, m, K, B):
     """2 <= B <= 16 runs the small-batch GEMV (one pass over M per four
     vectors, K in segments of 6144): equal to the per-vector GEMV and to the
-    oracle on sampled rows, with full-range x_hat and extreme weights."""
+    oracle on every output, with full-range x_hat and extreme weights."""
     import torch
     rng = np.random.default_rng(m + K + B)
     W = rng.integers(-128, 128, size=(m, K), dtype=np.int8)
@@ -523,9 +545,7 @@ def test_small_batch_server_product(pv, wl, m, K, B):
     Y = pv.as_u32(pv.pvmvmd_server_mvm(Wd, Xd))
     Y1 = np.stack([pv.as_u32(pv.pvmvmd_server_mvm(Wd, Xd[b])) for b in range(B)])
     assert np.array_equal(Y, Y1)
-    rows = sample_rows(m, 24, B)
-    for b in range(B):
-        assert np.array_equal(Y[b, rows], oracle.server_mvm_rows(W, X[b], rows)), b
+    assert_equal_report(Y, oracle.server_mvm_batch(W, X), "small-batch product")
     assert pv.pvmvmd_device_status() == 0
 
 
@@ -535,7 +555,7 @@ def test_qwen3_4b_block_8_tokens(pv, wl, name):
     eight-token batch, synthetic weights."""
     m, K = wl.LAYER_QWEN3_4B[name]
     W = wl.weights_gaussian(m, K, (6, list(wl.LAYER_QWEN3_4B).index(name)))
-    _batched_pipeline_sampled(pv, W, 8, seed=600 + len(name))
+    _batched_pipeline(pv, W, 8, seed=600 + len(name))
 
 
 def test_server_mvm_multi_mixed_jobs(pv, wl):
@@ -555,8 +575,7 @@ def test_server_mvm_multi_mixed_jobs(pv, wl):
         single = pv.as_u32(pv.pvmvmd_server_mvm(Wd[i], Xd[i]))
         got = pv.as_u32(Yd[i])
         assert np.array_equal(got, single), s
-        rows = sample_rows(s[0], 32, i)
-        assert np.array_equal(got[rows], oracle.server_mvm_rows(W[i], X[i], rows)), s
+        assert_equal_report(got, oracle.server_mvm_batch(W[i], X[i])[0], str(s))
     # many jobs (more than one launch's worth) on replicas of one matrix
     Wr = Wd[4]
     Xs = to_dev(rng.integers(0, Q, size=(300, 16)).astype(np.uint32))

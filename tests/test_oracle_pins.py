@@ -230,6 +230,39 @@ def test_server_mvm_bruteforce(shape):
     assert oracle.server_mvm_rows(W, x, rows).tolist() == [ref[i] for i in rows]
 
 
+@pytest.mark.parametrize("shape", [(4, 4, 1), (5, 7, 3), (33, 64, 5), (9, 300, 2)])
+def test_server_mvm_batch_bruteforce(shape):
+    """The batched oracle product against Python big integers, with the
+    extremes of both operands in every vector."""
+    m, K, B = shape
+    rng = np.random.default_rng(m * 1000 + K + B)
+    W = rng.integers(-128, 128, (m, K)).astype(np.int8)
+    W[0] = -128
+    X = rng.integers(0, Q, (B, K)).astype(np.uint32)
+    X[:, 0] = Q - 1
+    X[0] = (Q + 1) // 2
+    ref = [[sum(int(W[i, k]) * int(X[b, k]) for k in range(K)) % Q for i in range(m)] for b in range(B)]
+    assert oracle.server_mvm_batch(W, X).tolist() == ref
+
+
+@pytest.mark.parametrize("m,K,B,block", [(70, 1000, 6, 4096), (300, 2048, 4, 64), (5, 131071, 2, 4096)])
+def test_server_mvm_batch_matches_per_mac_loop(m, K, B, block):
+    """The batched product equals the per-MAC C loop (itself pinned by brute
+    force), up to the largest K the library accepts, over row blocks, with
+    every weight at -128 or 127 and every x_hat at q - 1 or (q + 1) / 2 in
+    some rows and vectors (the largest float64 partial sums)."""
+    rng = np.random.default_rng(m + K + B)
+    W = rng.integers(-128, 128, (m, K)).astype(np.int8)
+    W[0] = -128
+    W[1] = 127
+    X = rng.integers(0, Q, (B, K)).astype(np.uint32)
+    X[0] = Q - 1
+    X[1] = (Q + 1) // 2
+    got = oracle.server_mvm_batch(W, X, row_block=block)
+    for b in range(B):
+        assert np.array_equal(got[b], oracle.server_mvm(W, X[b])), b
+
+
 def test_server_mvm_extremes_and_special_cases():
     K = 300
     W = np.full((3, K), -128, np.int8)

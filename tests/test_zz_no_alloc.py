@@ -3,34 +3,46 @@
 Some callers cannot let the library call cudaMalloc: a server whose device
 memory is reserved up front by its own allocator, or a latency-critical loop
 that must not pay a first-use allocation.  For them the batched product can
-run on a fixed device buffer that the library holds.  This checks, through
-the C-ABI, that it gives exactly what the allocating call gives, on two calls
-in a row (the second must not see anything left over by the first), and that
-a problem too large for the buffer is refused.  The file is named to be
-collected last.
+run on a fixed device buffer that the library holds.  Through the C-ABI, each
+case below runs twice in a row, larger problems before smaller ones (so a
+call that read a leftover of the call before it would show), and every
+output is compared with the oracle and with the allocating call; a problem
+too large for the buffer is refused.  The file is named to be collected
+last.
 """
 import numpy as np
 import pytest
 
-from gpu_util import Q, to_dev
+import oracle
+from gpu_util import Q, assert_equal_report, to_dev
 
 pytestmark = pytest.mark.gpu
 
+# (m, K, B): an 8B-class projection with 64 vectors, then a ragged small
+# problem, then batch 1 (which this entry point also runs on the tensor cores)
+CASES = ((4096, 4096, 64), (300, 1000, 5), (1000, 4096, 1))
 
-def test_noalloc_matches_allocating_call_twice():
+
+def test_noalloc_matches_oracle_twice_larger_first():
     import torch
     import paper_2609_10264_gb300 as pv
     rng = np.random.default_rng(2024)
-    for m, K, B in ((300, 1000, 5), (4096, 4096, 64)):
+    for m, K, B in CASES:
         W = rng.integers(-128, 128, size=(m, K), dtype=np.int8)
+        W[0] = -128
         X = rng.integers(0, Q, size=(B, K)).astype(np.uint32)
+        X[0] = (Q + 1) // 2
+        exp = oracle.server_mvm_batch(W, X)
         Wd, Xd = to_dev(W), to_dev(X)
-        ref = pv.pvmvmd_server_mvm(Wd, Xd)
-        out = torch.zeros_like(ref)
-        pv.pvmvmd_server_mvm_noalloc(Wd, Xd, out)
-        torch.cuda.synchronize()
-        # integer (field) results: bit-exact, the tolerance of every parity test here
-        assert np.array_equal(pv.as_u32(out), pv.as_u32(ref)), (m, K, B)
+        ref = pv.as_u32(pv.pvmvmd_server_mvm(Wd, Xd if B > 1 else Xd[0])).reshape(B, m)
+        for call in range(2):
+            out = torch.full((B, m), -1, dtype=torch.int32, device="cuda")
+            pv.pvmvmd_server_mvm_noalloc(Wd, Xd, out)
+            torch.cuda.synchronize()
+            # integer (field) results: bit-exact, the tolerance of every parity test here
+            got = pv.as_u32(out)
+            assert_equal_report(got, exp, f"no-alloc call {call} at {m}x{K}x{B} vs the oracle")
+            assert_equal_report(got, ref, f"no-alloc call {call} at {m}x{K}x{B} vs pvmvmd_server_mvm")
     assert pv.pvmvmd_device_status() == 0
 
 
