@@ -356,6 +356,7 @@ def run_ours(args):
     params = pv.pvmvmd_params()
     params.scratch_batch = VECTORS                        # one encode chunk per step
     ctx = pv.pvmvmd_preprocess(Wd, key=20, params=params)
+    torch.cuda.synchronize(device)   # the inputs, made on torch's stream, are ready for `stream`
     stream = torch.cuda.Stream(device)
     # "overlap" (standard mode): the next batch's encode runs on enc_stream
     # beside this batch's decode (an encode and a decode of one context share
@@ -738,6 +739,7 @@ def measure_batched(args, workload, device, rank=0, world=1, with_cpu=True, with
     from paper_2609_10264_gb300 import workloads as wl
     spec = BATCHED[workload]
     B = spec["B"]
+    torch.cuda.synchronize(device)
     stream = torch.cuda.Stream(device)
     projs = []
     for j, (name, m, K) in enumerate(spec["shapes"]):
@@ -754,6 +756,7 @@ def measure_batched(args, workload, device, rank=0, world=1, with_cpu=True, with
                           Yh=torch.empty((B, m), dtype=torch.int32, device=device),
                           Y=torch.empty((B, m), dtype=torch.int32, device=device),
                           acc=torch.empty(B, dtype=torch.int32, device=device)))
+    torch.cuda.synchronize(device)   # the inputs, made on torch's stream, are ready for the others
 
     def enc():
         for p in projs:
@@ -1043,9 +1046,11 @@ def measure_token(args, device, rank=0):
             xh = torch.randint(0, Q, (K,), generator=gen, device=device, dtype=torch.int64).to(torch.int32)
             trip[name] = (W, xh, torch.empty(m, dtype=torch.int32, device=device))
         layers.append(trip)
+    torch.cuda.synchronize(device)   # the inputs, made on torch's stream, are ready for `stream`
     dep_jobs = [[pv.mvm_jobs([t[n] for n in grp]) for grp in TOKEN_GROUPS] for t in layers]
     layer_jobs = [pv.mvm_jobs(list(t.values())) for t in layers]
     all_jobs = pv.mvm_jobs([v for t in layers for v in t.values()])
+    torch.cuda.synchronize(device)
     stream = torch.cuda.Stream(device)
 
     def token_dep():
@@ -1176,6 +1181,7 @@ def run_bv(args):
     ctx = pv.pvmvmd_bv_preprocess(Ws, key=61)
     torch.cuda.synchronize(device)
     prep_s = time.perf_counter() - t0
+    torch.cuda.synchronize(device)
     stream = torch.cuda.Stream(device)
     chal = torch.empty((ctx.ell, 2 * ctx.t), dtype=torch.int32, device=device)
     u = torch.empty((ctx.ell, B * n), dtype=torch.int32, device=device)
@@ -1244,6 +1250,7 @@ def run_encode_shape(args):
     params = pv.pvmvmd_params()
     params.scratch_batch = max(B, 1)
     ctx = pv.pvmvmd_preprocess(W, key=82, params=params)
+    torch.cuda.synchronize(device)
     stream = torch.cuda.Stream(device)
     Xh = torch.empty_like(X)
     st = torch.empty((B, 2 * ctx.t_x), dtype=torch.int32, device=device)
@@ -1296,6 +1303,7 @@ def run_encoder_shape(args):
     N = ctx.N_x
     Y = torch.empty((N, m), dtype=torch.int32, device=device)
     scratch = torch.empty(pv.pvmvmd_code_encode_scratch(ctx, 0, m), dtype=torch.uint8, device=device)
+    torch.cuda.synchronize(device)
     stream = torch.cuda.Stream(device)
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
@@ -1351,6 +1359,7 @@ def run_preprocess_shape(args):
     gen = torch.Generator(device=device)
     gen.manual_seed(87)
     W = torch.randint(-127, 128, (m, K), generator=gen, device=device, dtype=torch.int8)
+    torch.cuda.synchronize(device)
     stream = torch.cuda.Stream(device)
     for w in range(args.warmup):
         pv.pvmvmd_preprocess(W, key=88 + w, stream=stream).destroy()
@@ -1394,6 +1403,7 @@ def run_server_shape(args):
     x = wl.int8_vectors(B, K, (10, 0))
     Xd = torch.from_numpy(np.mod(x, pv.PVMVMD_Q).astype(np.uint32).view(np.int32)).to(device)
     Y = torch.empty((B, m), dtype=torch.int32, device=device)
+    torch.cuda.synchronize(device)
     stream = torch.cuda.Stream(device)
     with torch.cuda.stream(stream):
         pv.pvmvmd_server_mvm(W0, Xd, Yhat=Y, stream=stream)
