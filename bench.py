@@ -765,7 +765,13 @@ def measure_batched(args, workload, device, rank=0, world=1, with_cpu=True, with
     # that a small projection's product can use the SMs a larger one leaves
     srv_streams = [torch.cuda.Stream(device) for _ in range(max(1, args.server_streams))]
 
+    grouped_jobs = pv.batch_jobs([(p["W"], p["Xh"], p["Yh"]) for p in projs])
+
     def srv():
+        if args.server_call == "grouped":
+            # the layer's products in one call: one persistent launch
+            pv.pvmvmd_server_mvm_grouped(grouped_jobs, stream=stream)
+            return
         fork = torch.cuda.Event()
         fork.record(stream)
         for ss in srv_streams:
@@ -815,13 +821,46 @@ def measure_batched(args, workload, device, rank=0, world=1, with_cpu=True, with
     def phases():
         enc(); srv(); dec()
 
-    step_fn = pipelined if args.schedule == "projections" else phases
+    def forked(per_proj):
+        # per_proj(p, on) for every projection on one of the side streams
+        fork = torch.cuda.Event()
+        fork.record(stream)
+        for ss in proj_streams:
+            ss.wait_event(fork)
+        for j, p in enumerate(projs):
+            ss = proj_streams[j % len(proj_streams)]
+            with torch.cuda.stream(ss):
+                per_proj(p, ss)
+        for ss in proj_streams:
+            join = torch.cuda.Event()
+            join.record(ss)
+            stream.wait_event(join)
+
+    def grouped(host=None):
+        # --schedule grouped: the encodes side by side on the side streams,
+        # the layer's products in one grouped call, the decodes side by side
+        def e(p, on):
+            src = p["X"]
+            if host is not None:
+                p["Xin"].copy_(p["Xhost"], non_blocking=True)
+                src = p["Xin"]
+            pv.pvmvmd_encode(p["ctx"], src, 21, Xhat=p["Xh"], st=p["st"], stream=on)
+
+        def d(p, on):
+            pv.pvmvmd_decode_verify(p["ctx"], p["st"], p["Xh"], p["Yh"], 22, Y=p["Y"], accept=p["acc"], stream=on)
+            if host is not None:
+                p["Yhost"].copy_(p["Y"], non_blocking=True)
+                p["Ahost"].copy_(p["acc"], non_blocking=True)
+        forked(e)
+        pv.pvmvmd_server_mvm_grouped(grouped_jobs, stream=stream)
+        forked(d)
+
+    step_fn = {"projections": pipelined, "phases": phases, "grouped": grouped}[args.schedule]
     # eager runs of every schedule that is captured below (the first call on
     # a stream sizes its scratch, which a capture may not do)
     with torch.cuda.stream(stream):
         enc(); srv(); dec()
-        if args.schedule == "projections":
-            pipelined()
+        step_fn()
     stream.synchronize()
     assert pv.pvmvmd_device_status(stream) == 0
     for p in projs:
@@ -936,12 +975,13 @@ def measure_batched(args, workload, device, rank=0, world=1, with_cpu=True, with
             p["Xin"] = torch.empty_like(p["X"])
             p["Yhost"] = torch.empty((B, p["m"]), dtype=torch.int32).pin_memory()
             p["Ahost"] = torch.empty(B, dtype=torch.int32).pin_memory()
+        e2e_fn = grouped if args.schedule == "grouped" else pipelined
         with torch.cuda.stream(stream):
-            pipelined(host=True)
+            e2e_fn(host=True)
         stream.synchronize()
         g_e2e = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g_e2e, stream=stream):
-            pipelined(host=True)
+            e2e_fn(host=True)
         with torch.cuda.stream(stream):
             for _ in range(args.warmup):
                 g_e2e.replay()
@@ -959,8 +999,11 @@ def measure_batched(args, workload, device, rank=0, world=1, with_cpu=True, with
         e2e = {"value": world * macs * n_e2e / e2e_s, "unit": UNIT,
                "h2d_bytes_per_step": int(sum(p["Xhost"].numel() * 4 for p in projs)),
                "d2h_bytes_per_step": int(sum(p["Yhost"].numel() * 4 + p["Ahost"].numel() * 4 for p in projs)),
-               "how": "CUDA graph of the public calls (each projection's encode, product, decode on one of "
-                      f"{len(proj_streams)} streams) with pinned host copies of X in and Y, accept out, "
+               "how": ("CUDA graph of the public calls (the encodes side by side on "
+                       f"{len(proj_streams)} streams, one grouped product call, the decodes side by side)"
+                       if args.schedule == "grouped" else
+                       "CUDA graph of the public calls (each projection's encode, product, decode on one of "
+                       f"{len(proj_streams)} streams)") + " with pinned host copies of X in and Y, accept out, "
                       "replayed; wall clock"}
 
     cpu = None
@@ -984,7 +1027,7 @@ def measure_batched(args, workload, device, rank=0, world=1, with_cpu=True, with
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": dtype, "data": "synthetic",
         "config": {"workload": workload, "B": B, "projections": [[p["name"], p["m"], p["K"]] for p in projs],
-                   "schedule": args.schedule, "streams": args.server_streams,
+                   "schedule": args.schedule, "server_call": args.server_call, "streams": args.server_streams,
                    "l2": "weights, P^T and Q of the layer exceed L2"},
         "phases_ms": {"encode": ph[0], "server_batched": ph[1], "decode_verify": ph[2]},
         "roofline": roof, "e2e": e2e, "cpu_baseline": cpu,
@@ -1413,23 +1456,32 @@ def run_server_shape(args):
     got = pv.as_u32(Y)[:, rows].astype(np.int64)
     got = np.where(got > (pv.PVMVMD_Q - 1) // 2, got - pv.PVMVMD_Q, got)
     assert np.array_equal(got, x @ Wh[rows].astype(np.int64).T), "server product mismatch"
+    # one CUDA graph of one call per weight copy, so that host-side call
+    # overhead is not timed
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for c in range(copies):
+            pv.pvmvmd_server_mvm(W[c], Xd, Yhat=Y, stream=stream)
+    reps = max(1, -(-args.steps // copies))
     with torch.cuda.stream(stream):
         for s in range(args.warmup):
-            pv.pvmvmd_server_mvm(W[s % copies], Xd, Yhat=Y, stream=stream)
+            g.replay()
     stream.synchronize()
     clocks = ClockSampler(device.index)
     clocks.start()
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
+    clocks.region_started()
     with torch.cuda.stream(stream):
         t0.record(stream)
-        for s in range(args.steps):
-            pv.pvmvmd_server_mvm(W[s % copies], Xd, Yhat=Y, stream=stream)
+        for s in range(reps):
+            g.replay()
         t1.record(stream)
+        clock_tail(lambda i: g.replay(), 0.03 * copies)
     stream.synchronize()
     clk = clocks.stop()
     pv.pvmvmd_device_status(stream)
-    ms = t0.elapsed_time(t1) / args.steps
+    ms = t0.elapsed_time(t1) / (reps * copies)
     macs = m * K * B
     peaks, kind = measured_peaks()
     if B <= 16 and K % 16 == 0:
@@ -1445,7 +1497,7 @@ def run_server_shape(args):
         roof = {"bound": "tensor", "kernel": "k_batched (tcgen05 kind::f16 digit GEMM) + k_digit_tiles",
                 "achieved": flops / (ms / 1e3) / 1e12, "peak": peaks.get("bf16_tflops", 0.0), "unit": "TFLOP/s",
                 "peak_kind": f"{kind} bf16_tflops (burst)"}
-        launches = 2 * args.steps
+        launches = None  # k_digit_tiles_grouped + k_batched_grouped (+ k_split_finish when K is split)
     roof["frac"] = roof["achieved"] / roof["peak"] if roof["peak"] else None
     if rank == 0:
         print(json.dumps({
@@ -1455,6 +1507,7 @@ def run_server_shape(args):
             "dtype": ("u32 (F_q exact; int8 weights, dp4a digits)" if roof["bound"] == "hbm"
                       else "u32 (F_q exact; fp16 digit MMAs, fp32 TMEM accumulation)"), "data": "synthetic",
             "config": {"workload": "server-shape", "m": m, "K": K, "B": B, "weight_copies": copies,
+                       "calls_timed": reps * copies, "timing": "CUDA graph of one call per weight copy",
                        "l2": "weights rotated over copies larger than L2"},
             "roofline": roof, "gpu_launches": launches, "clocks": clk}), flush=True)
     return 0
@@ -1478,10 +1531,14 @@ def main(argv=None):
     ap.add_argument("--shape", default="4096x4096x64",
                     help="m x K x B for --workload server-shape, K x B for --workload encode-shape")
     ap.add_argument("--server-streams", type=int, default=4)
-    ap.add_argument("--schedule", choices=["phases", "projections"], default="projections",
+    ap.add_argument("--schedule", choices=["phases", "projections", "grouped"], default="grouped",
                     help="batched workloads: all encodes, then all products, then all decodes "
-                         "(phases), or each projection's three calls in order on one of "
-                         "--server-streams streams (projections)")
+                         "(phases); each projection's three calls in order on one of "
+                         "--server-streams streams (projections); or the encodes side by side on those "
+                         "streams, one grouped product call, the decodes side by side (grouped)")
+    ap.add_argument("--server-call", choices=["grouped", "per-projection"], default="grouped",
+                    help="batched workloads, server phase: one pvmvmd_server_mvm_grouped call for the layer, "
+                         "or one pvmvmd_server_mvm call per projection spread over --server-streams streams")
     ap.add_argument("--step-schedule", choices=["overlap", "serial"], default="overlap",
                     help="batch1-4096 standard mode: overlap the next batch's encode with this batch's "
                          "decode on a second stream, or run encode, server and decode in order")

@@ -163,6 +163,31 @@ typedef struct {
  * 1 <= count, each 1 <= K <= PVMVMD_MAX_K, 1 <= m. */
 int pvmvmd_server_mvm_multi(const pvmvmd_mvm_job *jobs, int count, void *stream);
 
+/* One product of pvmvmd_server_mvm_grouped: Yhat = W Xhat over F_q for a
+ * batch of B vectors (Xhat_dev B x K, Yhat_dev B x m). */
+typedef struct {
+    const int8_t *W_dev;      /* int8 m x K row-major                       */
+    const uint32_t *Xhat_dev; /* B x K field elements                       */
+    uint32_t *Yhat_dev;       /* B x m field elements (output)              */
+    int m, K, B;
+} pvmvmd_mvm_batch_job;
+
+/* The server's products for `count` independent batched requests, such as
+ * the projections of one decoder layer for a batch of masked vectors
+ * (Sec. 6.1: the server's online work is the product of each matrix with
+ * the masked vectors it receives).  Results equal `count` calls of
+ * pvmvmd_server_mvm.  Every job with B > 16, K a multiple of 16 and a
+ * 16-byte aligned W runs in one persistent tensor-core launch over all such
+ * jobs (up to 8 per launch): one pair of CTAs per pair of SMs walks a list
+ * of tiles of all the jobs, longest first, so that small matrices fill the
+ * GPU and the pipeline is set up once.  Other jobs take the path
+ * pvmvmd_server_mvm gives them (batch-1 requests together in one grouped
+ * GEMV).  `jobs` is a host array that may be freed on return; outputs must
+ * not overlap any input or each other.  1 <= count, each 1 <= K <=
+ * PVMVMD_MAX_K, 1 <= m, 1 <= B.  The digit operands live in library scratch
+ * held per stream, as for pvmvmd_server_mvm. */
+int pvmvmd_server_mvm_grouped(const pvmvmd_mvm_batch_job *jobs, int count, void *stream);
+
 /* Size of the fixed device buffer behind pvmvmd_server_mvm_noalloc. */
 #define PVMVMD_NOALLOC_SCRATCH_BYTES (16u << 20)
 

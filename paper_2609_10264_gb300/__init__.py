@@ -73,6 +73,11 @@ class pvmvmd_bv_view(ctypes.Structure):
                [("Qs", ctypes.c_void_p), ("QauxT", ctypes.c_void_p), ("chal2", ctypes.c_void_p)]
 
 
+class pvmvmd_mvm_batch_job(ctypes.Structure):
+    _fields_ = [("W_dev", ctypes.c_void_p), ("Xhat_dev", ctypes.c_void_p), ("Yhat_dev", ctypes.c_void_p),
+                ("m", ctypes.c_int), ("K", ctypes.c_int), ("B", ctypes.c_int)]
+
+
 class pvmvmd_mvm_job(ctypes.Structure):
     _fields_ = [("W_dev", ctypes.c_void_p), ("xhat_dev", ctypes.c_void_p), ("yhat_dev", ctypes.c_void_p),
                 ("m", ctypes.c_int), ("K", ctypes.c_int)]
@@ -89,6 +94,7 @@ SIGNATURES = {
     "pvmvmd_server_mvm": (_i, [_vp, _i, _i, _vp, _i, _vp, _vp]),
     "pvmvmd_server_mvm_multi": (_i, [ctypes.POINTER(pvmvmd_mvm_job), _i, _vp]),
     "pvmvmd_server_mvm_noalloc": (_i, [_vp, _i, _i, _vp, _i, _vp, _vp]),
+    "pvmvmd_server_mvm_grouped": (_i, [ctypes.POINTER(pvmvmd_mvm_batch_job), _i, _vp]),
     "pvmvmd_decode_verify": (_i, [_vp, _vp, _vp, _vp, _i, ctypes.POINTER(pvmvmd_key), _vp, _vp, _vp]),
     "pvmvmd_boost_prepare": (_i, [_vp, _i, ctypes.POINTER(pvmvmd_key), _vp, _vp, _vp, _vp]),
     "pvmvmd_boost_encode": (_i, [_vp, _vp, _i, _i, _vp, _vp]),
@@ -401,6 +407,30 @@ def pvmvmd_server_mvm_noalloc(W, Xhat, Yhat, stream=None) -> None:
                                           _dev_ptr(Xhat, "Xhat", _u32_types()), B,
                                           _dev_ptr(Yhat, "Yhat", _u32_types(), B * m), _stream_ptr(stream)),
            "pvmvmd_server_mvm_noalloc")
+
+
+def batch_jobs(triples):
+    """A ctypes job array for pvmvmd_server_mvm_grouped from (W, Xhat, Yhat)
+    tensors (Xhat B x K, Yhat B x m); reusable across calls while the tensors
+    live."""
+    import torch
+    arr = (pvmvmd_mvm_batch_job * len(triples))()
+    for i, (W, Xh, Yh) in enumerate(triples):
+        m, K = W.shape
+        B = _batch(Xh, K, "Xhat")
+        arr[i].W_dev = _dev_ptr(W, "W", (torch.int8,)).value
+        arr[i].Xhat_dev = _dev_ptr(Xh, "Xhat", _u32_types()).value
+        arr[i].Yhat_dev = _dev_ptr(Yh, "Yhat", _u32_types(), B * m).value
+        arr[i].m, arr[i].K, arr[i].B = m, K, B
+    return arr
+
+
+def pvmvmd_server_mvm_grouped(jobs, stream=None) -> None:
+    """Several independent server products in as few launches as possible:
+    `jobs` is a list of (W, Xhat, Yhat) tensors or an array from batch_jobs."""
+    if not isinstance(jobs, ctypes.Array):
+        jobs = batch_jobs(jobs)
+    _check(_lib.pvmvmd_server_mvm_grouped(jobs, len(jobs), _stream_ptr(stream)), "pvmvmd_server_mvm_grouped")
 
 
 def mvm_jobs(triples):

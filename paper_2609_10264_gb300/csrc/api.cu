@@ -667,6 +667,43 @@ int pvmvmd_server_mvm_multi(const pvmvmd_mvm_job *jobs, int count, void *stream)
     return PVMVMD_OK;
 }
 
+int pvmvmd_server_mvm_grouped(const pvmvmd_mvm_batch_job *jobs, int count, void *stream) {
+    if (!jobs || count < 1) return count < 1 ? PVMVMD_E_SHAPE : PVMVMD_E_ARG;
+    for (int i = 0; i < count; ++i) {
+        const pvmvmd_mvm_batch_job &j = jobs[i];
+        if (!j.W_dev || !j.Xhat_dev || !j.Yhat_dev) return PVMVMD_E_ARG;
+        if (j.m < 1 || j.K < 1 || j.K > PVMVMD_MAX_K || j.B < 1) return PVMVMD_E_SHAPE;
+    }
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    uint32_t *err = error_word();
+    if (!err) return PVMVMD_E_CUDA;
+    // the tensor-core products together in one persistent launch; every
+    // other job takes the path pvmvmd_server_mvm gives it
+    std::vector<BatchJob> grouped;
+    std::vector<MvmJob> single;
+    for (int i = 0; i < count; ++i) {
+        const pvmvmd_mvm_batch_job &j = jobs[i];
+        const bool small = j.B <= kSmallBatchMax && j.K % 16 == 0 &&
+                           ((reinterpret_cast<uintptr_t>(j.W_dev) | reinterpret_cast<uintptr_t>(j.Xhat_dev)) & 15u) == 0;
+        if (j.B > 1 && !small && batched_grouped_eligible(j.W_dev, j.m, j.K, j.B)) {
+            grouped.push_back(BatchJob{j.W_dev, j.Xhat_dev, j.Yhat_dev, j.m, j.K, j.B});
+            continue;
+        }
+        if (j.B == 1) {
+            MvmJob t{j.W_dev, j.Xhat_dev, j.Yhat_dev, j.m, j.K, (size_t)j.K, 0};
+            if (multi_eligible(t)) {
+                single.push_back(t);
+                continue;
+            }
+        }
+        const int st = pvmvmd_server_mvm(j.W_dev, j.m, j.K, j.Xhat_dev, j.B, j.Yhat_dev, stream);
+        if (st != PVMVMD_OK) return st;
+    }
+    if (!single.empty()) PV_CUDA(launch_gemv_multi(single.data(), (int)single.size(), s));
+    if (!grouped.empty()) PV_CUDA(launch_batched_grouped(grouped.data(), (int)grouped.size(), err, s));
+    return PVMVMD_OK;
+}
+
 namespace pv {
 namespace {
 // The verification of a call: challenges e_q <- E_{t_y}^{N_y} shared by the

@@ -126,6 +126,17 @@ cudaError_t launch_gemv(const int8_t *W, int m, int K, const uint32_t *xhat, uin
 cudaError_t launch_batched(const int8_t *W, int m, int K, const uint32_t *Xhat, int B,
                            uint32_t *Yhat, uint32_t *err, cudaStream_t s);
 
+// Several independent batched products in one persistent tensor-core launch
+// (jobs with K % 16 == 0 and 16-byte aligned W; outputs must not overlap).
+struct BatchJob {
+    const int8_t *W;
+    const uint32_t *Xhat;
+    uint32_t *Yhat;
+    int m, K, B;
+};
+bool batched_grouped_eligible(const int8_t *W, int m, int K, int B);
+cudaError_t launch_batched_grouped(const BatchJob *jobs, int count, uint32_t *err, cudaStream_t s);
+
 // Grow-only scratch of at least `need` bytes for `purpose` on the current
 // device, one buffer per stream (see scratch.cu).
 enum ScratchPurpose { kScratchDigitTiles = 0, kScratchDigitPlanes = 1 };

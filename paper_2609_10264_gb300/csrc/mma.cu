@@ -42,10 +42,12 @@
 #include <cudaTypedefs.h>
 #include <cuda_fp16.h>
 
+#include <algorithm>
 #include <cstring>
 #include <map>
 #include <mutex>
 #include <tuple>
+#include <vector>
 
 #include "common.cuh"
 #include "launch.h"
@@ -702,11 +704,563 @@ cudaError_t batched_launch(const int8_t *W, int m, int K, const uint32_t *Xhat, 
                               wait_ns);
 }
 
+// ---------------------------------------------------------------------------
+// Grouped persistent product: one launch over a list of independent batched
+// products (for example the projections of a decoder layer).  Work items are
+// (job, pair of 128-row tiles, 64-vector tile, K-split); one CTA pair of a
+// thread-block cluster stays resident and walks its items, its pipelines
+// (stages, raw ring, double-buffered TMEM accumulator) running on from one
+// item to the next, so that the pipeline fill, TMEM allocation and barrier
+// set-up are paid once per launch and an item's epilogue overlaps the next
+// item's MMAs.  Items are ordered longest first (jobs by blocks per item),
+// and within a job by row pair, then K-split, then vector tile, so that the
+// items that run at the same time read the same rows of M; pair c of C takes
+// items c, 2C - 1 - c, 2C + c, ... (a snake order, close to the greedy
+// longest-first assignment).  A job whose K is split over several items
+// adds its partial sums (each canonical, times R^2 already applied) into a
+// 64-bit buffer with atomics; a final kernel reduces them mod q.
+// ---------------------------------------------------------------------------
+constexpr int kMaxGroupJobs = 8;
+constexpr int kMaxSplit = 8;
+
+struct GroupJob {
+    const uint8_t *D;         // digit tiles: nvt x nkb blocks of kBTile bytes
+    uint32_t *Y;              // B x m, written directly when split == 1
+    unsigned long long *acc;  // B x m partial sums when split > 1
+    int m, K, B, nkb, nvt, mp, split, per, item0;
+    const uint32_t *Xhat;     // for the digit-tile kernel
+};
+struct GroupArgs {
+    CUtensorMap map[kMaxGroupJobs];  // M of each job as a K x m tensor of bytes
+    GroupJob job[kMaxGroupJobs];
+    int njobs, total_items;
+};
+
+struct Item {
+    int j, p, v, kb0, nblk;
+};
+__device__ __forceinline__ Item group_item(const GroupArgs &a, int idx) {
+    int j = 0;
+    while (j + 1 < a.njobs && idx >= a.job[j + 1].item0) ++j;
+    const GroupJob &g = a.job[j];
+    int t = idx - g.item0;
+    const int per_p = g.split * g.nvt;
+    Item it;
+    it.j = j;
+    it.p = t / per_p;
+    t -= it.p * per_p;
+    const int s = t / g.nvt;
+    it.v = t - s * g.nvt;
+    it.kb0 = s * g.per;
+    it.nblk = min(g.nkb, it.kb0 + g.per) - it.kb0;
+    return it;
+}
+// The r-th item of pair c among C pairs (snake order); -1 past the end.
+__device__ __forceinline__ int group_item_index(int r, int c, int C, int total) {
+    const int idx = r * C + ((r & 1) ? C - 1 - c : c);
+    return idx < total ? idx : -1;
+}
+
+// Digit tiles of every job (as k_digit_tiles, blockIdx.y = job) and zeroed
+// partial-sum buffers of the split jobs.
+__global__ void __launch_bounds__(256) k_digit_tiles_grouped(const __grid_constant__ GroupArgs args) {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    const GroupJob &g = args.job[blockIdx.y];
+    const size_t gid = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (g.split > 1) {
+        const size_t n = (size_t)g.B * g.m;
+        for (size_t i = gid; i < n; i += (size_t)gridDim.x * blockDim.x) g.acc[i] = 0ull;
+    }
+    const size_t per_vec = (size_t)g.nkb * 8;
+    const size_t total = (size_t)g.nvt * kBV * per_vec;
+    if (gid >= total) return;
+    const int v = (int)(gid / per_vec);
+    const int grp = (int)(gid % per_vec);
+    const int kb = grp >> 3, chunk = grp & 7;
+    const int k0 = kb * kBK + chunk * 8;
+    int d[4][8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+        const int k = k0 + e;
+        if (v < g.B && k < g.K) {
+            limb_split(g.Xhat[(size_t)v * g.K + k], d[0][e], d[1][e], d[2][e], d[3][e]);
+        } else {
+            d[0][e] = d[1][e] = d[2][e] = d[3][e] = 0;
+        }
+    }
+    const int nt = v / kBV, vl = v % kBV;
+    uint8_t *blk = const_cast<uint8_t *>(g.D) + ((size_t)nt * g.nkb + kb) * kBTile;
+#pragma unroll
+    for (int l = 0; l < 4; ++l) {
+        const uint32_t row = 4 * vl + l;
+        uint4 q;
+        q.x = f16x2_of_int(d[l][0], d[l][1]);
+        q.y = f16x2_of_int(d[l][2], d[l][3]);
+        q.z = f16x2_of_int(d[l][4], d[l][5]);
+        q.w = f16x2_of_int(d[l][6], d[l][7]);
+        *reinterpret_cast<uint4 *>(blk + sw128_off(row, chunk)) = q;
+    }
+}
+
+// Y = acc mod q for the split jobs (blockIdx.y = job).
+__global__ void __launch_bounds__(256) k_split_finish(const __grid_constant__ GroupArgs args) {
+    const GroupJob &g = args.job[blockIdx.y];
+    if (g.split <= 1) return;
+    const size_t n = (size_t)g.B * g.m;
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x)
+        g.Y[i] = fred(g.acc[i]);
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    k_batched_grouped(const __grid_constant__ GroupArgs args, uint32_t *__restrict__ err, int skip_report,
+                      uint64_t wait_ns) {
+    cg::cluster_group cluster = cg::this_cluster();
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ __align__(8) uint64_t full[kStages], empty_bar[kStages];
+    __shared__ __align__(8) uint64_t acc_full[2], acc_empty[2], mma_done;
+    __shared__ __align__(8) uint64_t raw_full[kRaw], raw_empty[kRaw];
+    __shared__ uint32_t s_tmem;
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const uint32_t base = (smem_addr(smem_raw) + 1023u) & ~1023u;
+    uint8_t *smem = smem_raw + (base - smem_addr(smem_raw));
+    const uint32_t half = cluster.block_rank() & 1u;  // 0: the even CTA, which issues the MMAs
+    const uint16_t pair_mask = 3u;
+    const int c = (int)(blockIdx.x >> 1), C = (int)(gridDim.x >> 1);
+    const int total = args.total_items;
+
+    if (tid == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(&full[s], kConvThreads / 64 + 1 + (half == 0 ? 1 : 0));
+            mbar_init(&empty_bar[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&acc_full[b], 1);
+            mbar_init(&acc_empty[b], 2 * kEpiThreads / 32);
+        }
+        mbar_init(&mma_done, 1);
+        for (int r = 0; r < kRaw; ++r) {
+            mbar_init(&raw_full[r], 1);
+            mbar_init(&raw_empty[r], kConvThreads / 64);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == kWarpMma) {
+        asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], 512;" ::"r"(
+                         smem_addr(&s_tmem)));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;");
+    }
+    tc_fence_before();
+    cluster.sync();
+    tc_fence_after();
+    const uint32_t tmem = s_tmem;
+
+    if (warp < 8) {
+        // ------------------------------------------------ converters (group = block parity)
+        const int grp = warp >> 2;
+        const int t = tid & 127;
+        const int r0 = t >> 2, qk = t & 3;
+        uint32_t g = 0;
+        bool ok = true;
+        for (int r = 0; ok; ++r) {
+            const int idx = group_item_index(r, c, C, total);
+            if (idx < 0) break;
+            const Item it = group_item(args, idx);
+            for (int i = 0; i < it.nblk; ++i, ++g) {
+                if ((int)(g & 1u) != grp) continue;
+                const int s = g % kStages, rs = g % kRaw;
+                const uint32_t ph = (g / kStages) & 1u, rph = (g / kRaw) & 1u;
+                if (!mbar_wait_warp(&raw_full[rs], rph, err, wait_ns) ||
+                    !mbar_wait_warp(&empty_bar[s], ph ^ 1u, err, wait_ns)) {
+                    ok = false;
+                    break;
+                }
+                const uint8_t *raw = smem + kRawOff + rs * kRawTile;
+                uint8_t *a = smem + s * kStageBytes;
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const uint4 w = *reinterpret_cast<const uint4 *>(raw + (r0 + 32 * j) * kBK + 16 * qk);
+                    uint32_t o[8];
+                    i8x4_to_f16x4(w.x, o[0], o[1]);
+                    i8x4_to_f16x4(w.y, o[2], o[3]);
+                    i8x4_to_f16x4(w.z, o[4], o[5]);
+                    i8x4_to_f16x4(w.w, o[6], o[7]);
+                    const int row = r0 + 32 * j;
+                    *reinterpret_cast<uint4 *>(a + sw128_off(row, 2 * qk)) = make_uint4(o[0], o[1], o[2], o[3]);
+                    *reinterpret_cast<uint4 *>(a + sw128_off(row, 2 * qk + 1)) = make_uint4(o[4], o[5], o[6], o[7]);
+                }
+                fence_async_smem();
+                __syncwarp();
+                if (lane == 0) {
+                    mbar_arrive(&full[s]);
+                    mbar_arrive(&raw_empty[rs]);
+                }
+            }
+        }
+    } else if (warp < 16) {
+        // ------------------------------------------------ epilogue: TMEM -> mod-q sums -> Y
+        const int q = warp & 3;
+        const int grp = (warp - 8) >> 2;
+        const uint32_t acc_empty_leader = cluster_addr(&acc_empty[0], 0);
+        uint32_t gc = 0;
+        bool ok = true;
+        for (int r = 0; ok; ++r) {
+            const int idx = group_item_index(r, c, C, total);
+            if (idx < 0) break;
+            const Item it = group_item(args, idx);
+            const GroupJob &job = args.job[it.j];
+            uint32_t run[32];
+#pragma unroll
+            for (int v = 0; v < 32; ++v) run[v] = 0u;
+            const int nch = (it.nblk + kChunkBlocks - 1) / kChunkBlocks;
+            for (int ch = 0; ch < nch; ++ch, ++gc) {
+                const int bsel = gc & 1u;
+                if (!mbar_wait_warp(&acc_full[bsel], (gc >> 1) & 1u, err, wait_ns)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    uint32_t rr[32];
+                    tmem_ld32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(bsel * kBN + 128 * grp + 32 * j), rr);
+#pragma unroll
+                    for (int v = 0; v < 8; ++v) {
+                        run[8 * j + v] = fadd(run[8 * j + v],
+                                              digits_redc(__float2int_rn(__uint_as_float(rr[4 * v])),
+                                                          __float2int_rn(__uint_as_float(rr[4 * v + 1])),
+                                                          __float2int_rn(__uint_as_float(rr[4 * v + 2])),
+                                                          __float2int_rn(__uint_as_float(rr[4 * v + 3]))));
+                    }
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive_cluster(acc_empty_leader + 8u * (uint32_t)bsel);
+            }
+            if (!ok) break;
+            const int row = it.p * (2 * kBM) + (int)half * kBM + 32 * q + lane;
+            if (row < job.m) {
+#pragma unroll
+                for (int v = 0; v < 32; ++v) {
+                    const int b = it.v * kBV + 32 * grp + v;
+                    if (b < job.B) {
+                        const uint32_t val = fmul_mont(run[v], kR2);
+                        const size_t o = (size_t)b * job.m + row;
+                        if (job.split > 1)
+                            atomicAdd(job.acc + o, (unsigned long long)val);
+                        else
+                            job.Y[o] = val;
+                    }
+                }
+            }
+        }
+    } else if (warp == kWarpLoader) {
+        // ------------------------------------------------ this CTA's half of the digit operand
+        if (lane == 0) {
+            // the digit tiles come from the kernel launched just before this one
+            asm volatile("griddepcontrol.wait;" ::: "memory");
+            uint32_t g = 0;
+            bool ok = true;
+            for (int r = 0; ok; ++r) {
+                const int idx = group_item_index(r, c, C, total);
+                if (idx < 0) break;
+                const Item it = group_item(args, idx);
+                const GroupJob &job = args.job[it.j];
+                const uint8_t *src = job.D + ((size_t)it.v * job.nkb + it.kb0) * kBTile + (size_t)half * kBHalf;
+                for (int i = 0; i < it.nblk; ++i, ++g) {
+                    const int s = g % kStages;
+                    if (!mbar_wait(&empty_bar[s], ((g / kStages) & 1u) ^ 1u, err, wait_ns)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_tx(&full[s], kBHalf);
+                    bulk_g2s(smem + s * kStageBytes + kATile, src + (size_t)i * kBTile, kBHalf, &full[s]);
+                }
+            }
+            // copies in flight complete before the CTA may exit
+            for (uint32_t i = g > (uint32_t)kStages ? g - kStages : 0u; i < g; ++i)
+                mbar_wait(&full[i % kStages], (i / kStages) & 1u, err, wait_ns);
+        }
+    } else if (warp == kWarpWLoad) {
+        // ------------------------------------------------ raw int8 tiles of M by TMA
+        if (lane == 0) {
+            uint32_t g = 0;
+            bool ok = true;
+            for (int r = 0; ok; ++r) {
+                const int idx = group_item_index(r, c, C, total);
+                if (idx < 0) break;
+                const Item it = group_item(args, idx);
+                const int m0 = it.p * (2 * kBM) + (int)half * kBM;
+                const CUtensorMap *map = &args.map[it.j];
+                for (int i = 0; i < it.nblk; ++i, ++g) {
+                    const int rs = g % kRaw;
+                    if (!mbar_wait(&raw_empty[rs], ((g / kRaw) & 1u) ^ 1u, err, wait_ns)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_tx(&raw_full[rs], kRawTile);
+                    tma_load_2d(smem + kRawOff + rs * kRawTile, map, (it.kb0 + i) * kBK, m0, &raw_full[rs]);
+                }
+            }
+            for (uint32_t i = g > (uint32_t)kRaw ? g - kRaw : 0u; i < g; ++i)
+                mbar_wait(&raw_full[i % kRaw], (i / kRaw) & 1u, err, wait_ns);
+        }
+    } else if (half == 0) {
+        // ------------------------------------------------ MMA issuer (even CTA)
+        if (lane == 0) {
+            uint32_t g = 0, gc = 0;
+            bool ok = true;
+            for (int r = 0; ok; ++r) {
+                const int idx = group_item_index(r, c, C, total);
+                if (idx < 0) break;
+                const Item it = group_item(args, idx);
+                const int nch = (it.nblk + kChunkBlocks - 1) / kChunkBlocks;
+                for (int ch = 0; ch < nch && ok; ++ch, ++gc) {
+                    const int bsel = gc & 1u;
+                    if (!mbar_wait(&acc_empty[bsel], ((gc >> 1) & 1u) ^ 1u, err, wait_ns)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t dcol = tmem + (uint32_t)(bsel * kBN);
+                    const int i_end = min(it.nblk, (ch + 1) * kChunkBlocks);
+                    for (int i = ch * kChunkBlocks; i < i_end; ++i, ++g) {
+                        const int s = g % kStages;
+                        if (!mbar_wait(&full[s], (g / kStages) & 1u, err, wait_ns)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint32_t a_addr = base + (uint32_t)(s * kStageBytes);
+                        const uint32_t b_addr = a_addr + kATile;
+#pragma unroll
+                        for (int k = 0; k < kBK / 16; ++k)
+                            mma_pair(dcol, sw128_desc(a_addr + 32u * k), sw128_desc(b_addr + 32u * k),
+                                     (i > ch * kChunkBlocks || k > 0) ? 1u : 0u);
+                        mma_commit_pair(&empty_bar[s], pair_mask);
+                    }
+                    mma_commit_pair(&acc_full[bsel], pair_mask);
+                }
+            }
+            mma_commit_pair(&mma_done, (uint16_t)1u);
+            mbar_wait(&mma_done, 0, err, wait_ns);
+        }
+    } else {
+        // ------------------------------------------------ stage relay (odd CTA)
+        if (lane == 0) {
+            const uint32_t full_leader = cluster_addr(&full[0], 0);
+            uint32_t g = 0;
+            bool ok = true;
+            for (int r = 0; ok; ++r) {
+                const int idx = group_item_index(r, c, C, total);
+                if (idx < 0) break;
+                const Item it = group_item(args, idx);
+                for (int i = 0; i < it.nblk; ++i, ++g) {
+                    const int s = g % kStages;
+                    if (!mbar_wait(&full[s], (g / kStages) & 1u, err, wait_ns)) {
+                        ok = false;
+                        break;
+                    }
+                    // a failure-path test withholds one report (off: skip_report < 0)
+                    if ((int)g == skip_report) continue;
+                    mbar_arrive_cluster(full_leader + 8u * (uint32_t)s);
+                }
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    cluster.sync();  // the peer is done too: no MMA reads this CTA's memory any more
+    if (warp == kWarpMma) {
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, 512;" ::"r"(tmem));
+    }
+}
+
+// A job of the grouped launch as the host plans it.
+struct PlanJob {
+    int src;  // index in the caller's list
+    int m, K, B, nkb, nvt, mp, split, per, items;
+};
+
+// Blocks per item for a target item size T (in K-blocks).
+void plan_splits(std::vector<PlanJob> &jobs, int T) {
+    for (PlanJob &j : jobs) {
+        int s = (j.nkb + T - 1) / T;
+        s = s < 1 ? 1 : (s > kMaxSplit ? kMaxSplit : s);
+        j.per = (j.nkb + s - 1) / s;
+        j.split = (j.nkb + j.per - 1) / j.per;
+        j.items = j.mp * j.split * j.nvt;
+    }
+}
+
+// Estimated makespan (K-blocks plus a per-item overhead) of the snake
+// assignment of the longest-first item list over C pairs.
+double plan_makespan(const std::vector<PlanJob> &jobs, int C) {
+    std::vector<double> load(C, 0.0);
+    int idx = 0;
+    for (const PlanJob &j : jobs) {
+        for (int p = 0; p < j.mp; ++p)
+            for (int s = 0; s < j.split; ++s) {
+                const int nb = std::min(j.nkb, (s + 1) * j.per) - s * j.per;
+                for (int v = 0; v < j.nvt; ++v, ++idx) {
+                    const int r = idx / C, cc = idx % C;
+                    load[(r & 1) ? C - 1 - cc : cc] += nb + 3.0 + (j.split > 1 ? 1.0 : 0.0);
+                }
+            }
+    }
+    return *std::max_element(load.begin(), load.end());
+}
+
 }  // namespace
+
+bool batched_grouped_eligible(const int8_t *W, int m, int K, int B) {
+    return m >= 1 && B >= 1 && K >= 1 && K % 16 == 0 && (reinterpret_cast<uintptr_t>(W) & 15u) == 0;
+}
+
+cudaError_t launch_batched_grouped(const BatchJob *jobs, int count, uint32_t *err, cudaStream_t s) {
+    for (int a = 0; a < count; a += kMaxGroupJobs) {
+        const int n = std::min(count - a, kMaxGroupJobs);
+        std::vector<PlanJob> plan;
+        for (int i = 0; i < n; ++i) {
+            const BatchJob &b = jobs[a + i];
+            PlanJob p{};
+            p.src = a + i;
+            p.m = b.m;
+            p.K = b.K;
+            p.B = b.B;
+            p.nkb = (b.K + kBK - 1) / kBK;
+            p.nvt = (b.B + kBV - 1) / kBV;
+            p.mp = (b.m + 2 * kBM - 1) / (2 * kBM);
+            plan.push_back(p);
+        }
+        const cudaError_t attr =
+            func_attr((const void *)k_batched_grouped, cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
+        if (attr != cudaSuccess) return attr;
+        const int cap = resident_clusters((const void *)k_batched_grouped, 1);
+        // the target item size with the smallest estimated makespan
+        static const int kTargets[] = {8, 12, 16, 24, 32, 48, 64, 96, 128, 192, 256, 384, 512, 1 << 20};
+        double best = 1e300;
+        int best_t = 1 << 20, best_c = cap;
+        for (int T : kTargets) {
+            plan_splits(plan, T);
+            std::sort(plan.begin(), plan.end(), [](const PlanJob &x, const PlanJob &y) {
+                return x.per != y.per ? x.per > y.per : x.src < y.src;
+            });
+            int items = 0;
+            for (const PlanJob &j : plan) items += j.items;
+            const int C = std::min(cap, items);
+            const double ms = plan_makespan(plan, C);
+            if (ms < best - 1e-9) {
+                best = ms;
+                best_t = T;
+                best_c = C;
+            }
+        }
+        plan_splits(plan, best_t);
+        std::sort(plan.begin(), plan.end(), [](const PlanJob &x, const PlanJob &y) {
+            return x.per != y.per ? x.per > y.per : x.src < y.src;
+        });
+        // scratch: digit tiles of every job, then the split jobs' partial sums
+        size_t dbytes = 0, abytes = 0;
+        for (const PlanJob &j : plan) {
+            dbytes += (size_t)j.nvt * j.nkb * kBTile;
+            if (j.split > 1) abytes += (size_t)j.B * j.m * 8;
+        }
+        void *buf = nullptr;
+        cudaError_t e = stream_scratch(kScratchDigitTiles, dbytes + abytes, s, &buf);
+        if (e != cudaSuccess) return e;
+        PFN_cuTensorMapEncodeTiled_v12000 encode = tensor_map_encoder();
+        if (!encode) return cudaErrorNotSupported;
+        GroupArgs args;
+        memset(&args, 0, sizeof(args));
+        uint8_t *dp = static_cast<uint8_t *>(buf);
+        unsigned long long *ap = reinterpret_cast<unsigned long long *>(dp + dbytes);
+        int item0 = 0, any_split = 0, max_threads = 0, max_acc = 0;
+        for (int i = 0; i < (int)plan.size(); ++i) {
+            const PlanJob &p = plan[i];
+            const BatchJob &b = jobs[p.src];
+            GroupJob &g = args.job[i];
+            g.D = dp;
+            dp += (size_t)p.nvt * p.nkb * kBTile;
+            g.Y = b.Yhat;
+            g.acc = nullptr;
+            if (p.split > 1) {
+                g.acc = ap;
+                ap += (size_t)p.B * p.m;
+                any_split = 1;
+                max_acc = std::max(max_acc, p.B * p.m);
+            }
+            g.m = p.m;
+            g.K = p.K;
+            g.B = p.B;
+            g.nkb = p.nkb;
+            g.nvt = p.nvt;
+            g.mp = p.mp;
+            g.split = p.split;
+            g.per = p.per;
+            g.item0 = item0;
+            g.Xhat = b.Xhat;
+            item0 += p.items;
+            max_threads = std::max(max_threads, p.nvt * kBV * p.nkb * 8);
+            const cuuint64_t gdim[2] = {(cuuint64_t)p.K, (cuuint64_t)p.m};
+            const cuuint64_t gstride[1] = {(cuuint64_t)p.K};
+            const cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)kBM};
+            const cuuint32_t estride[2] = {1, 1};
+            if (encode(&args.map[i], CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<int8_t *>(b.W), gdim, gstride,
+                       box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                       CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+                return cudaErrorInvalidValue;
+        }
+        args.njobs = (int)plan.size();
+        args.total_items = item0;
+        if (item0 == 0) continue;
+        // digit tiles (and zeroed partial sums); enough CTAs for the largest job
+        const int dblocks = std::max((max_threads + 255) / 256, any_split ? std::min(1024, (max_acc + 255) / 256) : 1);
+        k_digit_tiles_grouped<<<dim3((unsigned)dblocks, (unsigned)args.njobs), 256, 0, s>>>(args);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+        const int C = std::min(best_c, item0);
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(2 * C, 1, 1);
+        cfg.blockDim = dim3(kThreads, 1, 1);
+        cfg.dynamicSmemBytes = kMmaSmem;
+        cfg.stream = s;
+        cudaLaunchAttribute lattr[2];
+        lattr[0].id = cudaLaunchAttributeClusterDimension;
+        lattr[0].val.clusterDim.x = 2;
+        lattr[0].val.clusterDim.y = 1;
+        lattr[0].val.clusterDim.z = 1;
+        lattr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        lattr[1].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = lattr;
+        cfg.numAttrs = 2;
+        const DebugWait dbg = debug_wait();
+        const int skip_report = dbg.site == PVMVMD_DEBUG_WAIT_PRODUCT ? (int)dbg.index : -1;
+        const uint64_t wait_ns = dbg.site == PVMVMD_DEBUG_WAIT_PRODUCT ? dbg.limit : kWaitNs;
+        e = cudaLaunchKernelEx(&cfg, k_batched_grouped, args, err, skip_report, wait_ns);
+        if (e != cudaSuccess) return e;
+        if (any_split) {
+            int dev = 0, sms = 0;
+            cudaGetDevice(&dev);
+            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+            k_split_finish<<<dim3((unsigned)(2 * sms), (unsigned)args.njobs), 256, 0, s>>>(args);
+            e = cudaGetLastError();
+            if (e != cudaSuccess) return e;
+        }
+    }
+    return cudaSuccess;
+}
+
 
 cudaError_t launch_batched(const int8_t *W, int m, int K, const uint32_t *Xhat, int B,
                            uint32_t *Yhat, uint32_t *err, cudaStream_t s) {
     if (m <= 0 || K <= 0 || B <= 0) return cudaSuccess;
+    if (batched_grouped_eligible(W, m, K, B)) {
+        const BatchJob job{W, Xhat, Yhat, m, K, B};
+        return launch_batched_grouped(&job, 1, err, s);
+    }
     const int nkb = (K + kBK - 1) / kBK;
     const int nvt = (B + kBV - 1) / kBV;
     void *D = nullptr;

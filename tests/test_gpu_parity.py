@@ -666,3 +666,50 @@ def test_long_code_uses_three_kernel_path(pv, wl):
     W = wl.weights_uniform(16, 50000, 9)
     x = wl.int8_vectors(2, 50000, 10)
     _full_round_trip(pv, W, x, seeds=(31, 32, 33))
+
+
+@pytest.mark.parametrize("layer,B", [("8b", 64), ("70b", 256)])
+def test_server_mvm_grouped_layer(pv, wl, layer, B):
+    """A decoder layer's projections in one grouped call (one persistent
+    tensor-core launch over all of them, K split where that balances the
+    work): every output element equals the oracle's."""
+    import torch
+    shapes = list((wl.LAYER_8B if layer == "8b" else wl.LAYER_70B).values())
+    rng = np.random.default_rng(B + len(shapes))
+    ins = []
+    for j, (m, K) in enumerate(shapes):
+        W = wl.weights_gaussian(m, K, (12, j))
+        X = rng.integers(0, Q, size=(B, K)).astype(np.uint32)
+        ins.append((W, X, to_dev(W), to_dev(X), torch.empty((B, m), dtype=torch.int32, device="cuda")))
+    jobs = pv.batch_jobs([(Wd, Xd, Yd) for _, _, Wd, Xd, Yd in ins])
+    for rep in range(2):   # the second call must not depend on the first's scratch
+        for *_, Yd in ins:
+            Yd.fill_(-1)
+        pv.pvmvmd_server_mvm_grouped(jobs)
+        torch.cuda.synchronize()
+        for W, X, _, _, Yd in ins:
+            assert_equal_report(pv.as_u32(Yd), oracle.server_mvm_batch(W, X), f"rep {rep} {W.shape}")
+    assert pv.pvmvmd_device_status() == 0
+
+
+def test_server_mvm_grouped_mixed_jobs(pv):
+    """Ten jobs of every kind in one call: more tensor-core jobs than one
+    launch takes (8), ragged shapes, a K that is not a multiple of 16 (the
+    single-problem kernel), batch 1 and a small batch (the GEMVs)."""
+    import torch
+    rng = np.random.default_rng(77)
+    specs = [(300, 1024, 70), (513, 4144, 130), (64, 2048, 65), (1030, 8192, 257), (256, 512, 17),
+             (700, 1000, 40), (128, 16384, 64), (40, 4096, 1), (333, 2048, 9), (2000, 1024, 100),
+             (96, 256, 33), (4096, 4096, 64)]
+    ins = []
+    for m, K, B in specs:
+        W = rng.integers(-128, 128, size=(m, K), dtype=np.int8)
+        W[0] = -128
+        X = rng.integers(0, Q, size=(B, K)).astype(np.uint32)
+        X[0] = Q - 1
+        ins.append((W, X, to_dev(W), to_dev(X), torch.full((B, m), -1, dtype=torch.int32, device="cuda")))
+    pv.pvmvmd_server_mvm_grouped([(Wd, Xd, Yd) for _, _, Wd, Xd, Yd in ins])
+    torch.cuda.synchronize()
+    for W, X, _, _, Yd in ins:
+        assert_equal_report(pv.as_u32(Yd), oracle.server_mvm_batch(W, X), str((W.shape, X.shape[0])))
+    assert pv.pvmvmd_device_status() == 0

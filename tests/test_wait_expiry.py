@@ -63,14 +63,16 @@ def test_lookback_scan_wait_expires_and_recovers(pv):
     ctx.destroy()
 
 
-def test_tensor_core_pipeline_wait_expires_and_recovers(pv):
-    """The batched product (512 x 4096, 64 vectors) with the second CTA of
-    every pair withholding its report for K-block 3, and pipeline waits
-    limited to 20 ms."""
+@pytest.mark.parametrize("K", [4096, 4100])
+def test_tensor_core_pipeline_wait_expires_and_recovers(pv, K):
+    """The batched product (512 x K, 64 vectors; K = 4096 runs the persistent
+    kernel, K = 4100 the single-problem kernel's byte-load path) with the
+    second CTA of every pair withholding its report for K-block 3, and
+    pipeline waits limited to 20 ms."""
     import torch
     rng = np.random.default_rng(5)
-    W = rng.integers(-128, 128, size=(512, 4096), dtype=np.int8)
-    X = rng.integers(0, Q, size=(64, 4096)).astype(np.uint32)
+    W = rng.integers(-128, 128, size=(512, K), dtype=np.int8)
+    X = rng.integers(0, Q, size=(64, K)).astype(np.uint32)
     Wd, Xd = to_dev(W), to_dev(X)
     exp = oracle.server_mvm_batch(W, X)
     assert_equal_report(pv.as_u32(pv.pvmvmd_server_mvm(Wd, Xd)), exp, "before")
