@@ -161,6 +161,13 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, i
         "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
         : "memory");
 }
+// Ask L2 to fetch the same box ahead of its load (no shared memory used).
+__device__ __forceinline__ void tma_prefetch_2d(const CUtensorMap *map, int x, int y) {
+    asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
+                     reinterpret_cast<uint64_t>(map)),
+                 "r"(x), "r"(y)
+                 : "memory");
+}
 __device__ __forceinline__ void fence_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
@@ -718,7 +725,10 @@ cudaError_t batched_launch(const int8_t *W, int m, int K, const uint32_t *Xhat, 
 // items c, 2C - 1 - c, 2C + c, ... (a snake order, close to the greedy
 // longest-first assignment).  A job whose K is split over several items
 // adds its partial sums (each canonical, times R^2 already applied) into a
-// 64-bit buffer with atomics; a final kernel reduces them mod q.
+// 64-bit buffer with atomics; a final kernel reduces them mod q.  (Having
+// the epilogue warp that adds the last part reduce its block instead, behind
+// a fence and a counter, held the epilogue up and was slower: 8B layer
+// 84 -> 97 us.)
 // ---------------------------------------------------------------------------
 constexpr int kMaxGroupJobs = 8;
 constexpr int kMaxSplit = 8;
@@ -778,27 +788,36 @@ __global__ void __launch_bounds__(256) k_digit_tiles_grouped(const __grid_consta
     const int grp = (int)(gid % per_vec);
     const int kb = grp >> 3, chunk = grp & 7;
     const int k0 = kb * kBK + chunk * 8;
-    int d[4][8];
+    // u = centred x_hat + 0x80808080: byte l of u is digit l plus 128 (the
+    // signed base-256 digits of limb_split, since 128 (1 + 2^8 + 2^16 + 2^24)
+    // added to sum_l 2^(8l) d_l carries nowhere), and the fp16 pattern
+    // 0x6400 | (d + 128) is 1024 + d + 128, so one byte permute and one packed
+    // add give two digits as exact fp16 values.  K is a multiple of 16 here.
+    uint32_t u[8];
+    if (v < g.B && k0 < g.K) {
+        const uint4 *src = reinterpret_cast<const uint4 *>(g.Xhat + (size_t)v * g.K + k0);
+        const uint4 a = src[0], b = src[1];
+        const uint32_t x[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
 #pragma unroll
-    for (int e = 0; e < 8; ++e) {
-        const int k = k0 + e;
-        if (v < g.B && k < g.K) {
-            limb_split(g.Xhat[(size_t)v * g.K + k], d[0][e], d[1][e], d[2][e], d[3][e]);
-        } else {
-            d[0][e] = d[1][e] = d[2][e] = d[3][e] = 0;
-        }
+        for (int e = 0; e < 8; ++e) u[e] = (x[e] > kHalfQ ? x[e] - kQ : x[e]) + 0x80808080u;
+    } else {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) u[e] = 0x80808080u;  // digits 0
     }
     const int nt = v / kBV, vl = v % kBV;
     uint8_t *blk = const_cast<uint8_t *>(g.D) + ((size_t)nt * g.nkb + kb) * kBTile;
+    const __half2 off = __halves2half2(__ushort_as_half(0xE480u), __ushort_as_half(0xE480u));  // -1152
 #pragma unroll
     for (int l = 0; l < 4; ++l) {
-        const uint32_t row = 4 * vl + l;
-        uint4 q;
-        q.x = f16x2_of_int(d[l][0], d[l][1]);
-        q.y = f16x2_of_int(d[l][2], d[l][3]);
-        q.z = f16x2_of_int(d[l][4], d[l][5]);
-        q.w = f16x2_of_int(d[l][6], d[l][7]);
-        *reinterpret_cast<uint4 *>(blk + sw128_off(row, chunk)) = q;
+        uint32_t w[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const uint32_t t = __byte_perm(u[2 * e], u[2 * e + 1], (uint32_t)(l | ((4 + l) << 4)));
+            const uint32_t h = __byte_perm(t, 0x64646464u, 0x5140);
+            const __half2 d = __hadd2(*reinterpret_cast<const __half2 *>(&h), off);
+            w[e] = *reinterpret_cast<const uint32_t *>(&d);
+        }
+        *reinterpret_cast<uint4 *>(blk + sw128_off(4 * vl + l, chunk)) = make_uint4(w[0], w[1], w[2], w[3]);
     }
 }
 
@@ -811,14 +830,27 @@ __global__ void __launch_bounds__(256) k_split_finish(const __grid_constant__ Gr
         g.Y[i] = fred(g.acc[i]);
 }
 
+// Stages of the grouped kernel hold two K-blocks each (A0 A1 B0 B1), so that
+// the MMA thread waits for a stage and commits it once per eight MMAs; the
+// two converter groups fill the two blocks of a stage side by side.
+constexpr int kGStageBlocks = 2;
+constexpr int kGStages = 3;
+constexpr int kGRaw = 4;
+constexpr int kGPrefetch = 12;   // blocks of M asked of L2 ahead of their load
+constexpr int kGStageBytes = kGStageBlocks * (kATile + kBHalf);  // 64 KiB
+constexpr int kGRawOff = kGStages * kGStageBytes;                  // 192 KiB
+constexpr int kGSmem = kGRawOff + kGRaw * kRawTile + 1024;          // + alignment slack
+static_assert(kGSmem <= 232448, "shared memory per CTA");
+static_assert(kChunkBlocks % kGStageBlocks == 0, "chunks end on stage boundaries");
+
 __global__ void __launch_bounds__(kThreads, 1)
     k_batched_grouped(const __grid_constant__ GroupArgs args, uint32_t *__restrict__ err, int skip_report,
                       uint64_t wait_ns) {
     cg::cluster_group cluster = cg::this_cluster();
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t full[kStages], empty_bar[kStages];
+    __shared__ __align__(8) uint64_t full[kGStages], empty_bar[kGStages];
     __shared__ __align__(8) uint64_t acc_full[2], acc_empty[2], mma_done;
-    __shared__ __align__(8) uint64_t raw_full[kRaw], raw_empty[kRaw];
+    __shared__ __align__(8) uint64_t raw_full[kGRaw], raw_empty[kGRaw];
     __shared__ uint32_t s_tmem;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -830,8 +862,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int total = args.total_items;
 
     if (tid == 0) {
-        for (int s = 0; s < kStages; ++s) {
-            mbar_init(&full[s], kConvThreads / 64 + 1 + (half == 0 ? 1 : 0));
+        for (int s = 0; s < kGStages; ++s) {
+            // every converter warp (both groups), the digit copies' arrival
+            // and, in the even CTA, the odd CTA's report
+            mbar_init(&full[s], kConvThreads / 32 + 1 + (half == 0 ? 1 : 0));
             mbar_init(&empty_bar[s], 1);
         }
         for (int b = 0; b < 2; ++b) {
@@ -839,7 +873,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(&acc_empty[b], 2 * kEpiThreads / 32);
         }
         mbar_init(&mma_done, 1);
-        for (int r = 0; r < kRaw; ++r) {
+        for (int r = 0; r < kGRaw; ++r) {
             mbar_init(&raw_full[r], 1);
             mbar_init(&raw_empty[r], kConvThreads / 64);
         }
@@ -856,44 +890,58 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tmem = s_tmem;
 
     if (warp < 8) {
-        // ------------------------------------------------ converters (group = block parity)
+        // ------------------------------------------------ converters: group j fills block j of each stage
         const int grp = warp >> 2;
         const int t = tid & 127;
         const int r0 = t >> 2, qk = t & 3;
-        uint32_t g = 0;
+        uint32_t gs = 0, gb = 0;
         bool ok = true;
         for (int r = 0; ok; ++r) {
             const int idx = group_item_index(r, c, C, total);
             if (idx < 0) break;
             const Item it = group_item(args, idx);
-            for (int i = 0; i < it.nblk; ++i, ++g) {
-                if ((int)(g & 1u) != grp) continue;
-                const int s = g % kStages, rs = g % kRaw;
-                const uint32_t ph = (g / kStages) & 1u, rph = (g / kRaw) & 1u;
-                if (!mbar_wait_warp(&raw_full[rs], rph, err, wait_ns) ||
-                    !mbar_wait_warp(&empty_bar[s], ph ^ 1u, err, wait_ns)) {
-                    ok = false;
-                    break;
-                }
-                const uint8_t *raw = smem + kRawOff + rs * kRawTile;
-                uint8_t *a = smem + s * kStageBytes;
+            for (int b0 = 0; b0 < it.nblk; b0 += kGStageBlocks, ++gs) {
+                const int nb = min(kGStageBlocks, it.nblk - b0);
+                const int s = gs % kGStages;
+                const uint32_t ph = (gs / kGStages) & 1u;
+                const uint32_t rb = gb + (uint32_t)grp;
+                gb += (uint32_t)nb;
+                if (grp < nb) {
+                    const int rs = rb % kGRaw;
+                    if (!mbar_wait_warp(&raw_full[rs], (rb / kGRaw) & 1u, err, wait_ns) ||
+                        !mbar_wait_warp(&empty_bar[s], ph ^ 1u, err, wait_ns)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint8_t *raw = smem + kGRawOff + rs * kRawTile;
+                    uint8_t *a = smem + s * kGStageBytes + grp * kATile;
 #pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    const uint4 w = *reinterpret_cast<const uint4 *>(raw + (r0 + 32 * j) * kBK + 16 * qk);
-                    uint32_t o[8];
-                    i8x4_to_f16x4(w.x, o[0], o[1]);
-                    i8x4_to_f16x4(w.y, o[2], o[3]);
-                    i8x4_to_f16x4(w.z, o[4], o[5]);
-                    i8x4_to_f16x4(w.w, o[6], o[7]);
-                    const int row = r0 + 32 * j;
-                    *reinterpret_cast<uint4 *>(a + sw128_off(row, 2 * qk)) = make_uint4(o[0], o[1], o[2], o[3]);
-                    *reinterpret_cast<uint4 *>(a + sw128_off(row, 2 * qk + 1)) = make_uint4(o[4], o[5], o[6], o[7]);
-                }
-                fence_async_smem();
-                __syncwarp();
-                if (lane == 0) {
-                    mbar_arrive(&full[s]);
-                    mbar_arrive(&raw_empty[rs]);
+                    for (int j = 0; j < 4; ++j) {
+                        const uint4 w = *reinterpret_cast<const uint4 *>(raw + (r0 + 32 * j) * kBK + 16 * qk);
+                        uint32_t o[8];
+                        i8x4_to_f16x4(w.x, o[0], o[1]);
+                        i8x4_to_f16x4(w.y, o[2], o[3]);
+                        i8x4_to_f16x4(w.z, o[4], o[5]);
+                        i8x4_to_f16x4(w.w, o[6], o[7]);
+                        const int row = r0 + 32 * j;
+                        *reinterpret_cast<uint4 *>(a + sw128_off(row, 2 * qk)) = make_uint4(o[0], o[1], o[2], o[3]);
+                        *reinterpret_cast<uint4 *>(a + sw128_off(row, 2 * qk + 1)) =
+                            make_uint4(o[4], o[5], o[6], o[7]);
+                    }
+                    fence_async_smem();
+                    __syncwarp();
+                    if (lane == 0) {
+                        mbar_arrive(&full[s]);
+                        mbar_arrive(&raw_empty[rs]);
+                    }
+                } else {
+                    // no block for this group in the stage (an item's odd
+                    // last block): arrive in the stage's current phase
+                    if (!mbar_wait_warp(&empty_bar[s], ph ^ 1u, err, wait_ns)) {
+                        ok = false;
+                        break;
+                    }
+                    if (lane == 0) mbar_arrive(&full[s]);
                 }
             }
         }
@@ -959,7 +1007,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {
             // the digit tiles come from the kernel launched just before this one
             asm volatile("griddepcontrol.wait;" ::: "memory");
-            uint32_t g = 0;
+            uint32_t gs = 0;
             bool ok = true;
             for (int r = 0; ok; ++r) {
                 const int idx = group_item_index(r, c, C, total);
@@ -967,48 +1015,70 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const Item it = group_item(args, idx);
                 const GroupJob &job = args.job[it.j];
                 const uint8_t *src = job.D + ((size_t)it.v * job.nkb + it.kb0) * kBTile + (size_t)half * kBHalf;
-                for (int i = 0; i < it.nblk; ++i, ++g) {
-                    const int s = g % kStages;
-                    if (!mbar_wait(&empty_bar[s], ((g / kStages) & 1u) ^ 1u, err, wait_ns)) {
+                for (int b0 = 0; b0 < it.nblk; b0 += kGStageBlocks, ++gs) {
+                    const int nb = min(kGStageBlocks, it.nblk - b0);
+                    const int s = gs % kGStages;
+                    if (!mbar_wait(&empty_bar[s], ((gs / kGStages) & 1u) ^ 1u, err, wait_ns)) {
                         ok = false;
                         break;
                     }
-                    mbar_arrive_tx(&full[s], kBHalf);
-                    bulk_g2s(smem + s * kStageBytes + kATile, src + (size_t)i * kBTile, kBHalf, &full[s]);
+                    mbar_arrive_tx(&full[s], (uint32_t)nb * kBHalf);
+                    uint8_t *dst = smem + s * kGStageBytes + kGStageBlocks * kATile;
+                    for (int j = 0; j < nb; ++j)
+                        bulk_g2s(dst + j * kBHalf, src + (size_t)(b0 + j) * kBTile, kBHalf, &full[s]);
                 }
             }
             // copies in flight complete before the CTA may exit
-            for (uint32_t i = g > (uint32_t)kStages ? g - kStages : 0u; i < g; ++i)
-                mbar_wait(&full[i % kStages], (i / kStages) & 1u, err, wait_ns);
+            for (uint32_t i = gs > (uint32_t)kGStages ? gs - kGStages : 0u; i < gs; ++i)
+                mbar_wait(&full[i % kGStages], (i / kGStages) & 1u, err, wait_ns);
         }
     } else if (warp == kWarpWLoad) {
         // ------------------------------------------------ raw int8 tiles of M by TMA
         if (lane == 0) {
-            uint32_t g = 0;
+            uint32_t gb = 0;
             bool ok = true;
+            // L2 prefetches run kGPrefetch blocks ahead of the loads, into the
+            // next item near the end of this one: the raw ring alone holds too
+            // few blocks to cover the latency of HBM when the weights stream
+            // at the rate a 64-vector tile consumes them
+            const int idx0 = group_item_index(0, c, C, total);
+            Item nxt = idx0 >= 0 ? group_item(args, idx0) : Item{0, 0, 0, 0, 0};
+            int nxt_idx = idx0;
+            auto prefetch = [&](const Item &t, int i) {
+                const int y = t.p * (2 * kBM) + (int)half * kBM;
+                if (i < t.nblk && y < args.job[t.j].m) tma_prefetch_2d(&args.map[t.j], (t.kb0 + i) * kBK, y);
+            };
+            if (idx0 >= 0)
+                for (int i = 0; i < kGPrefetch; ++i) prefetch(nxt, i);
             for (int r = 0; ok; ++r) {
-                const int idx = group_item_index(r, c, C, total);
+                const int idx = nxt_idx;
                 if (idx < 0) break;
-                const Item it = group_item(args, idx);
+                const Item it = nxt;
+                nxt_idx = group_item_index(r + 1, c, C, total);
+                if (nxt_idx >= 0) nxt = group_item(args, nxt_idx);
                 const int m0 = it.p * (2 * kBM) + (int)half * kBM;
                 const CUtensorMap *map = &args.map[it.j];
-                for (int i = 0; i < it.nblk; ++i, ++g) {
-                    const int rs = g % kRaw;
-                    if (!mbar_wait(&raw_empty[rs], ((g / kRaw) & 1u) ^ 1u, err, wait_ns)) {
+                for (int i = 0; i < it.nblk; ++i, ++gb) {
+                    if (i + kGPrefetch < it.nblk)
+                        prefetch(it, i + kGPrefetch);
+                    else if (nxt_idx >= 0)
+                        prefetch(nxt, i + kGPrefetch - it.nblk);
+                    const int rs = gb % kGRaw;
+                    if (!mbar_wait(&raw_empty[rs], ((gb / kGRaw) & 1u) ^ 1u, err, wait_ns)) {
                         ok = false;
                         break;
                     }
                     mbar_arrive_tx(&raw_full[rs], kRawTile);
-                    tma_load_2d(smem + kRawOff + rs * kRawTile, map, (it.kb0 + i) * kBK, m0, &raw_full[rs]);
+                    tma_load_2d(smem + kGRawOff + rs * kRawTile, map, (it.kb0 + i) * kBK, m0, &raw_full[rs]);
                 }
             }
-            for (uint32_t i = g > (uint32_t)kRaw ? g - kRaw : 0u; i < g; ++i)
-                mbar_wait(&raw_full[i % kRaw], (i / kRaw) & 1u, err, wait_ns);
+            for (uint32_t i = gb > (uint32_t)kGRaw ? gb - kGRaw : 0u; i < gb; ++i)
+                mbar_wait(&raw_full[i % kGRaw], (i / kGRaw) & 1u, err, wait_ns);
         }
     } else if (half == 0) {
         // ------------------------------------------------ MMA issuer (even CTA)
         if (lane == 0) {
-            uint32_t g = 0, gc = 0;
+            uint32_t gs = 0, gc = 0;
             bool ok = true;
             for (int r = 0; ok; ++r) {
                 const int idx = group_item_index(r, c, C, total);
@@ -1024,19 +1094,23 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tc_fence_after();
                     const uint32_t dcol = tmem + (uint32_t)(bsel * kBN);
                     const int i_end = min(it.nblk, (ch + 1) * kChunkBlocks);
-                    for (int i = ch * kChunkBlocks; i < i_end; ++i, ++g) {
-                        const int s = g % kStages;
-                        if (!mbar_wait(&full[s], (g / kStages) & 1u, err, wait_ns)) {
+                    for (int b0 = ch * kChunkBlocks; b0 < i_end; b0 += kGStageBlocks, ++gs) {
+                        const int nb = min(kGStageBlocks, i_end - b0);
+                        const int s = gs % kGStages;
+                        if (!mbar_wait(&full[s], (gs / kGStages) & 1u, err, wait_ns)) {
                             ok = false;
                             break;
                         }
                         tc_fence_after();
-                        const uint32_t a_addr = base + (uint32_t)(s * kStageBytes);
-                        const uint32_t b_addr = a_addr + kATile;
+                        const uint32_t st = base + (uint32_t)(s * kGStageBytes);
+                        for (int j = 0; j < nb; ++j) {
+                            const uint32_t a_addr = st + (uint32_t)(j * kATile);
+                            const uint32_t b_addr = st + (uint32_t)(kGStageBlocks * kATile + j * kBHalf);
 #pragma unroll
-                        for (int k = 0; k < kBK / 16; ++k)
-                            mma_pair(dcol, sw128_desc(a_addr + 32u * k), sw128_desc(b_addr + 32u * k),
-                                     (i > ch * kChunkBlocks || k > 0) ? 1u : 0u);
+                            for (int k = 0; k < kBK / 16; ++k)
+                                mma_pair(dcol, sw128_desc(a_addr + 32u * k), sw128_desc(b_addr + 32u * k),
+                                         (b0 > ch * kChunkBlocks || j > 0 || k > 0) ? 1u : 0u);
+                        }
                         mma_commit_pair(&empty_bar[s], pair_mask);
                     }
                     mma_commit_pair(&acc_full[bsel], pair_mask);
@@ -1049,20 +1123,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ------------------------------------------------ stage relay (odd CTA)
         if (lane == 0) {
             const uint32_t full_leader = cluster_addr(&full[0], 0);
-            uint32_t g = 0;
+            uint32_t gs = 0;
             bool ok = true;
             for (int r = 0; ok; ++r) {
                 const int idx = group_item_index(r, c, C, total);
                 if (idx < 0) break;
                 const Item it = group_item(args, idx);
-                for (int i = 0; i < it.nblk; ++i, ++g) {
-                    const int s = g % kStages;
-                    if (!mbar_wait(&full[s], (g / kStages) & 1u, err, wait_ns)) {
+                for (int b0 = 0; b0 < it.nblk; b0 += kGStageBlocks, ++gs) {
+                    const int s = gs % kGStages;
+                    if (!mbar_wait(&full[s], (gs / kGStages) & 1u, err, wait_ns)) {
                         ok = false;
                         break;
                     }
                     // a failure-path test withholds one report (off: skip_report < 0)
-                    if ((int)g == skip_report) continue;
+                    if ((int)gs == skip_report) continue;
                     mbar_arrive_cluster(full_leader + 8u * (uint32_t)s);
                 }
             }
@@ -1136,7 +1210,7 @@ cudaError_t launch_batched_grouped(const BatchJob *jobs, int count, uint32_t *er
             plan.push_back(p);
         }
         const cudaError_t attr =
-            func_attr((const void *)k_batched_grouped, cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
+            func_attr((const void *)k_batched_grouped, cudaFuncAttributeMaxDynamicSharedMemorySize, kGSmem);
         if (attr != cudaSuccess) return attr;
         const int cap = resident_clusters((const void *)k_batched_grouped, 1);
         // the target item size with the smallest estimated makespan
@@ -1225,7 +1299,7 @@ cudaError_t launch_batched_grouped(const BatchJob *jobs, int count, uint32_t *er
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(2 * C, 1, 1);
         cfg.blockDim = dim3(kThreads, 1, 1);
-        cfg.dynamicSmemBytes = kMmaSmem;
+        cfg.dynamicSmemBytes = kGSmem;
         cfg.stream = s;
         cudaLaunchAttribute lattr[2];
         lattr[0].id = cudaLaunchAttributeClusterDimension;
