@@ -190,11 +190,17 @@ class ClockSampler:
                                               "same steps queued after it (clock tail)"}
 
 
-def clock_tail(replay, ms_per_call: float, seconds: float = 0.5) -> int:
+CLOCK_TAIL_S = 0.5
+
+
+def clock_tail(replay, ms_per_call: float, seconds: float | None = None) -> int:
     """Queue untimed calls of `replay` after the timed region's stop event, so
     that the clock sampler (100 ms period) sees the GPU under the same load
     for `seconds` even when the timed region itself is only milliseconds
     long.  Returns the number of calls queued."""
+    seconds = CLOCK_TAIL_S if seconds is None else seconds
+    if seconds <= 0:
+        return 0
     n = max(1, int(seconds * 1e3 / max(ms_per_call, 1e-3)))
     for i in range(n):
         replay(i)
@@ -1513,6 +1519,128 @@ def run_server_shape(args):
     return 0
 
 
+def run_server_layer(args):
+    """The server's products of one layer alone (``--shape`` = a batched
+    workload name: layer8b-b64, layer70b-b256, layerqwen4b-b8), as one
+    pvmvmd_server_mvm_grouped call, timed inside a CUDA graph.  Only the
+    weights and the masked vectors are on the device (no client context), so
+    the launch also serves as a small case for a profiler."""
+    import torch
+    rank, world, local = dist_env()
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    import paper_2609_10264_gb300 as pv
+    Q = pv.PVMVMD_Q
+    spec = BATCHED[args.shape]
+    B = spec["B"]
+    gen = torch.Generator(device=device)
+    gen.manual_seed(91)
+    ins = []
+    for name, m, K in spec["shapes"]:
+        W = (torch.randn((m, K), generator=gen, device=device) * 32.0).round_().clamp_(-127, 127).to(torch.int8)
+        X = torch.randint(0, Q, (B, K), generator=gen, device=device, dtype=torch.int64).to(torch.int32)
+        ins.append((W, X, torch.empty((B, m), dtype=torch.int32, device=device)))
+    torch.cuda.synchronize(device)
+    stream = torch.cuda.Stream(device)
+    jobs = pv.batch_jobs(ins)
+    with torch.cuda.stream(stream):
+        pv.pvmvmd_server_mvm_grouped(jobs, stream=stream)
+    stream.synchronize()
+    assert pv.pvmvmd_device_status(stream) == 0
+    for W, X, Y in ins:   # sampled rows against an exact int64 product
+        rows = [0, W.shape[0] // 2, W.shape[0] - 1]
+        exp = (W[rows].cpu().numpy().astype(np.int64) @ pv.as_u32(X).astype(np.int64).T) % Q
+        assert np.array_equal(pv.as_u32(Y)[:, rows].T.astype(np.int64), exp)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        pv.pvmvmd_server_mvm_grouped(jobs, stream=stream)
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            g.replay()
+        t0.record(stream)
+        for _ in range(args.steps):
+            g.replay()
+        t1.record(stream)
+    stream.synchronize()
+    ms = t0.elapsed_time(t1) / args.steps
+    macs = sum(m * K for _, m, K in spec["shapes"]) * B
+    peaks, kind = measured_peaks()
+    if rank == 0:
+        tf = 8 * macs / (ms / 1e3) / 1e12
+        print(json.dumps({
+            "metric": "server_field_mac_per_s", "value": macs / (ms / 1e3), "unit": "field-MAC/s", "n_gpus": 1,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "u32 (F_q exact; fp16 digit MMAs)", "data": "synthetic",
+            "config": {"workload": "server-layer", "layer": args.shape, "B": B,
+                       "projections": [list(x) for x in spec["shapes"]],
+                       "timing": "CUDA graph of one pvmvmd_server_mvm_grouped call per step"},
+            "roofline": {"bound": "tensor", "kernel": "k_digit_tiles_grouped + k_batched_grouped (+ k_split_finish)",
+                         "achieved": tf, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                         "frac": tf / peaks["bf16_tflops"], "peak_kind": f"{kind} bf16_tflops (burst)"},
+            "gpu_launches": None}), flush=True)
+    return 0
+
+
+def run_decode_shape(args):
+    """pvmvmd_decode_verify alone (``--shape mxKxB``): preprocessing, one
+    encode and one server product first, then --steps decode calls with fresh
+    challenge keys.  4096x8192x256 holds 2 GiB of P^T and Q, a small case of
+    the 70B-class decode for a profiler."""
+    import torch
+    rank, world, local = dist_env()
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    import paper_2609_10264_gb300 as pv
+    from paper_2609_10264_gb300 import workloads as wl
+    m, K, B = (int(v) for v in args.shape.lower().split("x"))
+    W = torch.from_numpy(wl.weights_gaussian(m, K, (13, 0))).to(device)
+    x = wl.int8_vectors(B, K, (13, 1))
+    X = torch.from_numpy(np.mod(x, pv.PVMVMD_Q).astype(np.uint32).view(np.int32)).to(device)
+    params = pv.pvmvmd_params()
+    params.scratch_batch = B
+    ctx = pv.pvmvmd_preprocess(W, key=131, params=params)
+    torch.cuda.synchronize(device)
+    stream = torch.cuda.Stream(device)
+    with torch.cuda.stream(stream):
+        Xh, st = pv.pvmvmd_encode(ctx, X, key=132, stream=stream)
+        Yh = pv.pvmvmd_server_mvm(W, Xh, stream=stream)
+        Y, acc = pv.pvmvmd_decode_verify(ctx, st, Xh, Yh, 133, stream=stream)
+    stream.synchronize()
+    assert int(acc.sum()) == B
+    supp = pv.as_u32(st)[:, :ctx.t_x]
+    distinct = len(np.unique(supp))
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        for s_ in range(args.warmup):
+            pv.pvmvmd_decode_verify(ctx, st, Xh, Yh, 200 + s_, Y=Y, accept=acc, stream=stream)
+        t0.record(stream)
+        for s_ in range(args.steps):
+            pv.pvmvmd_decode_verify(ctx, st, Xh, Yh, 300 + s_, Y=Y, accept=acc, stream=stream)
+        t1.record(stream)
+    stream.synchronize()
+    assert pv.pvmvmd_device_status(stream) == 0 and int(acc.sum()) == B
+    ms = t0.elapsed_time(t1) / args.steps
+    peaks, kind = measured_peaks()
+    # the decrypt's bytes when every needed row of P^T is read once (the
+    # distinct rows of the batch's supports), plus y_hat read and y written
+    nbytes = distinct * 4 * m + 8 * B * m
+    if rank == 0:
+        print(json.dumps({
+            "metric": "decoded vectors/s", "value": B / (ms / 1e3), "unit": "vectors/s", "n_gpus": 1,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "u32 (F_q exact)", "data": "synthetic",
+            "config": {"workload": "decode-shape", "m": m, "K": K, "B": B, "t_x": ctx.t_x,
+                       "support_draws": int(supp.size), "distinct_rows": distinct,
+                       "bytes_distinct_rows": nbytes, "bytes_per_vector_rows": int(supp.size) * 4 * m + 8 * B * m},
+            "roofline": {"bound": "hbm", "kernel": "pvmvmd_decode_verify call (k_decrypt dominant)",
+                         "achieved": nbytes / (ms / 1e3) / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                         "frac": nbytes / (ms / 1e3) / 1e9 / peaks["hbm_gbs"], "peak_kind": f"{kind} hbm_gbs"},
+            "gpu_launches": None}), flush=True)
+    ctx.destroy()
+    return 0
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
@@ -1520,16 +1648,21 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--clock-tail-s", type=float, default=0.5,
+                    help="seconds of untimed steps queued after each timed region so that the clock "
+                         "sampler sees the load (0 under a profiler)")
     ap.add_argument("--no-extra-configs", action="store_true",
                     help="default workload: skip the 70B-class batched and 8B-class token sub-records")
     ap.add_argument("--cpu-vectors", type=int, default=150)
     ap.add_argument("--server-mode", choices=["multi", "calls"], default="multi")
-    ap.add_argument("--workload", choices=["batch1-4096", "server-shape", "encode-shape", "encoder-shape",
+    ap.add_argument("--workload", choices=["batch1-4096", "server-shape", "server-layer", "decode-shape",
+                                           "encode-shape", "encoder-shape",
                                            "preprocess-shape", "token8b-b1", "bv-b8-1024"]
                     + sorted(BATCHED),
                     default="batch1-4096")
     ap.add_argument("--shape", default="4096x4096x64",
-                    help="m x K x B for --workload server-shape, K x B for --workload encode-shape")
+                    help="m x K x B for --workload server-shape and decode-shape, K x B for --workload "
+                         "encode-shape, a batched workload name for --workload server-layer")
     ap.add_argument("--server-streams", type=int, default=4)
     ap.add_argument("--schedule", choices=["phases", "projections", "grouped"], default="grouped",
                     help="batched workloads: all encodes, then all products, then all decodes "
@@ -1547,6 +1680,8 @@ def main(argv=None):
                          "the step), boost (masks prepared ahead, untimed) or pipelined (standard mode "
                          "with the next step's masks prepared on a second stream, timed)")
     args = ap.parse_args(argv)
+    global CLOCK_TAIL_S
+    CLOCK_TAIL_S = args.clock_tail_s
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
     if args.impl == "reference":
@@ -1555,6 +1690,10 @@ def main(argv=None):
         return run_batched(args)
     if args.workload == "server-shape":
         return run_server_shape(args)
+    if args.workload == "server-layer":
+        return run_server_layer(args)
+    if args.workload == "decode-shape":
+        return run_decode_shape(args)
     if args.workload == "token8b-b1":
         return run_token(args)
     if args.workload == "bv-b8-1024":
