@@ -131,7 +131,9 @@ int pvmvmd_encode(pvmvmd_ctx *ctx, const uint32_t *X_dev, int B, const pvmvmd_ke
  * online work).  W_dev int8 m x K row-major, Xhat_dev B x K, Yhat_dev B x m.
  * Needs no context and no secret.  B == 1 runs the bandwidth-bound GEMV;
  * 2 <= B <= 16 (K a multiple of 16, 16-byte aligned W and Xhat) a GEMV that
- * reads M once per four vectors; larger B the byte-limb tensor-core product.
+ * reads M once per four vectors, or, for B >= 8 and m K B >= 2^27, the
+ * tensor-core product with 16-vector tiles; larger B the byte-limb
+ * tensor-core product.
  * 1 <= K <= PVMVMD_MAX_K.  The batch-1 GEMV and the 2 <= B <= 16 GEMV may
  * start reading M while the kernel before it on the stream finishes, when
  * that kernel signals its
@@ -176,13 +178,13 @@ typedef struct {
  * the projections of one decoder layer for a batch of masked vectors
  * (Sec. 6.1: the server's online work is the product of each matrix with
  * the masked vectors it receives).  Results equal `count` calls of
- * pvmvmd_server_mvm.  Every job with B > 16, K a multiple of 16 and a
- * 16-byte aligned W runs in one persistent tensor-core launch over all such
- * jobs (up to 8 per launch): one pair of CTAs per pair of SMs walks a list
- * of tiles of all the jobs, longest first, so that small matrices fill the
- * GPU and the pipeline is set up once.  Other jobs take the path
- * pvmvmd_server_mvm gives them (batch-1 requests together in one grouped
- * GEMV).  `jobs` is a host array that may be freed on return; outputs must
+ * pvmvmd_server_mvm.  Every job with B >= 2, K a multiple of 16 and a
+ * 16-byte aligned W runs on the tensor cores in one persistent launch per
+ * tile width (16-vector tiles for B <= 16, 64-vector tiles above; up to 8
+ * jobs per launch): one pair of CTAs per pair of SMs walks a list of tiles
+ * of all the jobs, longest first, so that small matrices fill the GPU and
+ * the pipeline is set up once.  Other jobs take the path pvmvmd_server_mvm
+ * gives them (batch-1 requests together in one grouped GEMV).  `jobs` is a host array that may be freed on return; outputs must
  * not overlap any input or each other.  1 <= count, each 1 <= K <=
  * PVMVMD_MAX_K, 1 <= m, 1 <= B.  The digit operands live in library scratch
  * held per stream, as for pvmvmd_server_mvm. */

@@ -632,9 +632,13 @@ int pvmvmd_server_mvm(const int8_t *W_dev, int m, int K, const uint32_t *Xhat_de
         PV_CUDA(launch_gemv(W_dev, m, K, Xhat_dev, Yhat_dev, err, s));
         return PVMVMD_OK;
     }
-    // a few vectors: one pass over M per four vectors (the tensor-core
-    // product's tiles hold 64 vectors)
-    if (B <= kSmallBatchMax && K % 16 == 0 &&
+    // a few vectors: one pass over M per four vectors with dp4a, unless the
+    // problem is large enough for the tensor-core product with 16-vector
+    // tiles to win (measured: 14336 x 4096 with 8 vectors 41.0 against
+    // 27.1 us, with 4 vectors 23.8 against 26.0 us; 4096 x 2560 with 8
+    // vectors 12.1 against 12.9 us)
+    const bool tensor_small = B >= 8 && (double)m * K * B >= 128.0 * 1024 * 1024;
+    if (B <= kSmallBatchMax && !tensor_small && K % 16 == 0 &&
         ((reinterpret_cast<uintptr_t>(W_dev) | reinterpret_cast<uintptr_t>(Xhat_dev)) & 15u) == 0) {
         PV_CUDA(launch_gemv_small_batch(W_dev, m, K, Xhat_dev, B, Yhat_dev, s));
         return PVMVMD_OK;
@@ -683,9 +687,7 @@ int pvmvmd_server_mvm_grouped(const pvmvmd_mvm_batch_job *jobs, int count, void 
     std::vector<MvmJob> single;
     for (int i = 0; i < count; ++i) {
         const pvmvmd_mvm_batch_job &j = jobs[i];
-        const bool small = j.B <= kSmallBatchMax && j.K % 16 == 0 &&
-                           ((reinterpret_cast<uintptr_t>(j.W_dev) | reinterpret_cast<uintptr_t>(j.Xhat_dev)) & 15u) == 0;
-        if (j.B > 1 && !small && batched_grouped_eligible(j.W_dev, j.m, j.K, j.B)) {
+        if (j.B > 1 && batched_grouped_eligible(j.W_dev, j.m, j.K, j.B)) {
             grouped.push_back(BatchJob{j.W_dev, j.Xhat_dev, j.Yhat_dev, j.m, j.K, j.B});
             continue;
         }

@@ -732,9 +732,42 @@ cudaError_t batched_launch(const int8_t *W, int m, int K, const uint32_t *Xhat, 
 // ---------------------------------------------------------------------------
 constexpr int kMaxGroupJobs = 8;
 constexpr int kMaxSplit = 8;
+constexpr int kNarrowMaxB = 16;  // batches up to this size use 16-vector tiles
+constexpr int kGPrefetch = 12;   // blocks of M asked of L2 ahead of their load
+
+// Tile geometry of the grouped kernel for V vectors per tile: 64 (N = 256
+// digit rows, the batched configurations) or 16 (N = 64, small batches,
+// where a 64-vector tile would leave three quarters of the MMA idle).  A
+// stage holds two K-blocks (A0 A1 B0 B1); the smaller digit operand of
+// V = 16 leaves room for four stages and eight raw tiles.
+template <int V>
+struct GTile {
+    static constexpr int kBV = V;
+    static constexpr int kBN = 4 * V;                      // MMA N (digit rows)
+    static constexpr int kBTile = kBN * kBK * 2;           // digit bytes per K-block (pair)
+    static constexpr int kBHalf = kBTile / 2;              // one CTA's half
+    static constexpr int kStages = V == 64 ? 3 : 4;
+    static constexpr int kRaw = V == 64 ? 4 : 8;
+    static constexpr int kStageBytes = 2 * (kATile + kBHalf);
+    static constexpr int kRawOff = kStages * kStageBytes;
+    static constexpr int kSmem = kRawOff + kRaw * kRawTile + 1024;  // + alignment slack
+    static constexpr int kTmemCols = 2 * kBN;              // double-buffered accumulator
+    static constexpr int kVecs = V / 2;                    // vectors per epilogue thread
+    static constexpr uint32_t kIdesc = (1u << 4) | ((uint32_t)(kBN >> 3) << 17) | ((uint32_t)(2 * kBM >> 4) << 24);
+    static_assert(kSmem <= 232448, "shared memory per CTA");
+    static_assert(kTmemCols == 128 || kTmemCols == 512, "TMEM allocation");
+};
+
+template <uint32_t IDESC>
+__device__ __forceinline__ void mma_pair_n(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+        "l"(adesc), "l"(bdesc), "r"(IDESC), "r"(accumulate));
+}
 
 struct GroupJob {
-    const uint8_t *D;         // digit tiles: nvt x nkb blocks of kBTile bytes
+    const uint8_t *D;         // digit tiles: nvt x nkb blocks of GTile<V>::kBTile bytes
     uint32_t *Y;              // B x m, written directly when split == 1
     unsigned long long *acc;  // B x m partial sums when split > 1
     int m, K, B, nkb, nvt, mp, split, per, item0;
@@ -773,7 +806,9 @@ __device__ __forceinline__ int group_item_index(int r, int c, int C, int total) 
 
 // Digit tiles of every job (as k_digit_tiles, blockIdx.y = job) and zeroed
 // partial-sum buffers of the split jobs.
+template <int V>
 __global__ void __launch_bounds__(256) k_digit_tiles_grouped(const __grid_constant__ GroupArgs args) {
+    using T = GTile<V>;
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const GroupJob &g = args.job[blockIdx.y];
     const size_t gid = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -782,7 +817,7 @@ __global__ void __launch_bounds__(256) k_digit_tiles_grouped(const __grid_consta
         for (size_t i = gid; i < n; i += (size_t)gridDim.x * blockDim.x) g.acc[i] = 0ull;
     }
     const size_t per_vec = (size_t)g.nkb * 8;
-    const size_t total = (size_t)g.nvt * kBV * per_vec;
+    const size_t total = (size_t)g.nvt * T::kBV * per_vec;
     if (gid >= total) return;
     const int v = (int)(gid / per_vec);
     const int grp = (int)(gid % per_vec);
@@ -804,8 +839,8 @@ __global__ void __launch_bounds__(256) k_digit_tiles_grouped(const __grid_consta
 #pragma unroll
         for (int e = 0; e < 8; ++e) u[e] = 0x80808080u;  // digits 0
     }
-    const int nt = v / kBV, vl = v % kBV;
-    uint8_t *blk = const_cast<uint8_t *>(g.D) + ((size_t)nt * g.nkb + kb) * kBTile;
+    const int nt = v / T::kBV, vl = v % T::kBV;
+    uint8_t *blk = const_cast<uint8_t *>(g.D) + ((size_t)nt * g.nkb + kb) * T::kBTile;
     const __half2 off = __halves2half2(__ushort_as_half(0xE480u), __ushort_as_half(0xE480u));  // -1152
 #pragma unroll
     for (int l = 0; l < 4; ++l) {
@@ -830,22 +865,15 @@ __global__ void __launch_bounds__(256) k_split_finish(const __grid_constant__ Gr
         g.Y[i] = fred(g.acc[i]);
 }
 
-// Stages of the grouped kernel hold two K-blocks each (A0 A1 B0 B1), so that
-// the MMA thread waits for a stage and commits it once per eight MMAs; the
-// two converter groups fill the two blocks of a stage side by side.
-constexpr int kGStageBlocks = 2;
-constexpr int kGStages = 3;
-constexpr int kGRaw = 4;
-constexpr int kGPrefetch = 12;   // blocks of M asked of L2 ahead of their load
-constexpr int kGStageBytes = kGStageBlocks * (kATile + kBHalf);  // 64 KiB
-constexpr int kGRawOff = kGStages * kGStageBytes;                  // 192 KiB
-constexpr int kGSmem = kGRawOff + kGRaw * kRawTile + 1024;          // + alignment slack
-static_assert(kGSmem <= 232448, "shared memory per CTA");
-static_assert(kChunkBlocks % kGStageBlocks == 0, "chunks end on stage boundaries");
-
+template <int V>
 __global__ void __launch_bounds__(kThreads, 1)
     k_batched_grouped(const __grid_constant__ GroupArgs args, uint32_t *__restrict__ err, int skip_report,
                       uint64_t wait_ns) {
+    using T = GTile<V>;
+    constexpr int kGStageBlocks = 2;
+    constexpr int kGStages = T::kStages, kGRaw = T::kRaw, kGStageBytes = T::kStageBytes, kGRawOff = T::kRawOff;
+    constexpr int kBHalfG = T::kBHalf, kBTileG = T::kBTile, kBNG = T::kBN, kBVG = T::kBV;
+    static_assert(kChunkBlocks % kGStageBlocks == 0, "chunks end on stage boundaries");
     cg::cluster_group cluster = cg::this_cluster();
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t full[kGStages], empty_bar[kGStages];
@@ -880,8 +908,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == kWarpMma) {
-        asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], 512;" ::"r"(
-                         smem_addr(&s_tmem)));
+        asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_addr(&s_tmem)), "n"(T::kTmemCols));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;");
     }
     tc_fence_before();
@@ -957,9 +985,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (idx < 0) break;
             const Item it = group_item(args, idx);
             const GroupJob &job = args.job[it.j];
-            uint32_t run[32];
+            uint32_t run[T::kVecs];
 #pragma unroll
-            for (int v = 0; v < 32; ++v) run[v] = 0u;
+            for (int v = 0; v < T::kVecs; ++v) run[v] = 0u;
             const int nch = (it.nblk + kChunkBlocks - 1) / kChunkBlocks;
             for (int ch = 0; ch < nch; ++ch, ++gc) {
                 const int bsel = gc & 1u;
@@ -969,9 +997,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 tc_fence_after();
 #pragma unroll
-                for (int j = 0; j < 4; ++j) {
+                for (int j = 0; j < T::kVecs / 8; ++j) {
                     uint32_t rr[32];
-                    tmem_ld32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(bsel * kBN + 128 * grp + 32 * j), rr);
+                    tmem_ld32(tmem + ((uint32_t)(32 * q) << 16) +
+                                  (uint32_t)(bsel * kBNG + (kBNG / 2) * grp + 32 * j), rr);
 #pragma unroll
                     for (int v = 0; v < 8; ++v) {
                         run[8 * j + v] = fadd(run[8 * j + v],
@@ -989,8 +1018,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int row = it.p * (2 * kBM) + (int)half * kBM + 32 * q + lane;
             if (row < job.m) {
 #pragma unroll
-                for (int v = 0; v < 32; ++v) {
-                    const int b = it.v * kBV + 32 * grp + v;
+                for (int v = 0; v < T::kVecs; ++v) {
+                    const int b = it.v * kBVG + T::kVecs * grp + v;
                     if (b < job.B) {
                         const uint32_t val = fmul_mont(run[v], kR2);
                         const size_t o = (size_t)b * job.m + row;
@@ -1014,7 +1043,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (idx < 0) break;
                 const Item it = group_item(args, idx);
                 const GroupJob &job = args.job[it.j];
-                const uint8_t *src = job.D + ((size_t)it.v * job.nkb + it.kb0) * kBTile + (size_t)half * kBHalf;
+                const uint8_t *src = job.D + ((size_t)it.v * job.nkb + it.kb0) * kBTileG + (size_t)half * kBHalfG;
                 for (int b0 = 0; b0 < it.nblk; b0 += kGStageBlocks, ++gs) {
                     const int nb = min(kGStageBlocks, it.nblk - b0);
                     const int s = gs % kGStages;
@@ -1022,10 +1051,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                         ok = false;
                         break;
                     }
-                    mbar_arrive_tx(&full[s], (uint32_t)nb * kBHalf);
+                    mbar_arrive_tx(&full[s], (uint32_t)nb * kBHalfG);
                     uint8_t *dst = smem + s * kGStageBytes + kGStageBlocks * kATile;
                     for (int j = 0; j < nb; ++j)
-                        bulk_g2s(dst + j * kBHalf, src + (size_t)(b0 + j) * kBTile, kBHalf, &full[s]);
+                        bulk_g2s(dst + j * kBHalfG, src + (size_t)(b0 + j) * kBTileG, kBHalfG, &full[s]);
                 }
             }
             // copies in flight complete before the CTA may exit
@@ -1092,7 +1121,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t dcol = tmem + (uint32_t)(bsel * kBN);
+                    const uint32_t dcol = tmem + (uint32_t)(bsel * kBNG);
                     const int i_end = min(it.nblk, (ch + 1) * kChunkBlocks);
                     for (int b0 = ch * kChunkBlocks; b0 < i_end; b0 += kGStageBlocks, ++gs) {
                         const int nb = min(kGStageBlocks, i_end - b0);
@@ -1105,11 +1134,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const uint32_t st = base + (uint32_t)(s * kGStageBytes);
                         for (int j = 0; j < nb; ++j) {
                             const uint32_t a_addr = st + (uint32_t)(j * kATile);
-                            const uint32_t b_addr = st + (uint32_t)(kGStageBlocks * kATile + j * kBHalf);
+                            const uint32_t b_addr = st + (uint32_t)(kGStageBlocks * kATile + j * kBHalfG);
 #pragma unroll
                             for (int k = 0; k < kBK / 16; ++k)
-                                mma_pair(dcol, sw128_desc(a_addr + 32u * k), sw128_desc(b_addr + 32u * k),
-                                         (b0 > ch * kChunkBlocks || j > 0 || k > 0) ? 1u : 0u);
+                                mma_pair_n<T::kIdesc>(dcol, sw128_desc(a_addr + 32u * k),
+                                                      sw128_desc(b_addr + 32u * k),
+                                                      (b0 > ch * kChunkBlocks || j > 0 || k > 0) ? 1u : 0u);
                         }
                         mma_commit_pair(&empty_bar[s], pair_mask);
                     }
@@ -1148,7 +1178,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     cluster.sync();  // the peer is done too: no MMA reads this CTA's memory any more
     if (warp == kWarpMma) {
         tc_fence_after();
-        asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, 512;" ::"r"(tmem));
+        asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem), "n"(T::kTmemCols));
     }
 }
 
@@ -1193,7 +1223,9 @@ bool batched_grouped_eligible(const int8_t *W, int m, int K, int B) {
     return m >= 1 && B >= 1 && K >= 1 && K % 16 == 0 && (reinterpret_cast<uintptr_t>(W) & 15u) == 0;
 }
 
-cudaError_t launch_batched_grouped(const BatchJob *jobs, int count, uint32_t *err, cudaStream_t s) {
+template <int V>
+cudaError_t launch_grouped_v(const BatchJob *jobs, int count, uint32_t *err, cudaStream_t s) {
+    using T = GTile<V>;
     for (int a = 0; a < count; a += kMaxGroupJobs) {
         const int n = std::min(count - a, kMaxGroupJobs);
         std::vector<PlanJob> plan;
@@ -1205,14 +1237,14 @@ cudaError_t launch_batched_grouped(const BatchJob *jobs, int count, uint32_t *er
             p.K = b.K;
             p.B = b.B;
             p.nkb = (b.K + kBK - 1) / kBK;
-            p.nvt = (b.B + kBV - 1) / kBV;
+            p.nvt = (b.B + T::kBV - 1) / T::kBV;
             p.mp = (b.m + 2 * kBM - 1) / (2 * kBM);
             plan.push_back(p);
         }
         const cudaError_t attr =
-            func_attr((const void *)k_batched_grouped, cudaFuncAttributeMaxDynamicSharedMemorySize, kGSmem);
+            func_attr((const void *)k_batched_grouped<V>, cudaFuncAttributeMaxDynamicSharedMemorySize, T::kSmem);
         if (attr != cudaSuccess) return attr;
-        const int cap = resident_clusters((const void *)k_batched_grouped, 1);
+        const int cap = resident_clusters((const void *)k_batched_grouped<V>, 1);
         // the target item size with the smallest estimated makespan
         static const int kTargets[] = {8, 12, 16, 24, 32, 48, 64, 96, 128, 192, 256, 384, 512, 1 << 20};
         double best = 1e300;
@@ -1239,7 +1271,7 @@ cudaError_t launch_batched_grouped(const BatchJob *jobs, int count, uint32_t *er
         // scratch: digit tiles of every job, then the split jobs' partial sums
         size_t dbytes = 0, abytes = 0;
         for (const PlanJob &j : plan) {
-            dbytes += (size_t)j.nvt * j.nkb * kBTile;
+            dbytes += (size_t)j.nvt * j.nkb * T::kBTile;
             if (j.split > 1) abytes += (size_t)j.B * j.m * 8;
         }
         void *buf = nullptr;
@@ -1257,7 +1289,7 @@ cudaError_t launch_batched_grouped(const BatchJob *jobs, int count, uint32_t *er
             const BatchJob &b = jobs[p.src];
             GroupJob &g = args.job[i];
             g.D = dp;
-            dp += (size_t)p.nvt * p.nkb * kBTile;
+            dp += (size_t)p.nvt * p.nkb * T::kBTile;
             g.Y = b.Yhat;
             g.acc = nullptr;
             if (p.split > 1) {
@@ -1277,7 +1309,7 @@ cudaError_t launch_batched_grouped(const BatchJob *jobs, int count, uint32_t *er
             g.item0 = item0;
             g.Xhat = b.Xhat;
             item0 += p.items;
-            max_threads = std::max(max_threads, p.nvt * kBV * p.nkb * 8);
+            max_threads = std::max(max_threads, p.nvt * T::kBV * p.nkb * 8);
             const cuuint64_t gdim[2] = {(cuuint64_t)p.K, (cuuint64_t)p.m};
             const cuuint64_t gstride[1] = {(cuuint64_t)p.K};
             const cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)kBM};
@@ -1292,14 +1324,14 @@ cudaError_t launch_batched_grouped(const BatchJob *jobs, int count, uint32_t *er
         if (item0 == 0) continue;
         // digit tiles (and zeroed partial sums); enough CTAs for the largest job
         const int dblocks = std::max((max_threads + 255) / 256, any_split ? std::min(1024, (max_acc + 255) / 256) : 1);
-        k_digit_tiles_grouped<<<dim3((unsigned)dblocks, (unsigned)args.njobs), 256, 0, s>>>(args);
+        k_digit_tiles_grouped<V><<<dim3((unsigned)dblocks, (unsigned)args.njobs), 256, 0, s>>>(args);
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
         const int C = std::min(best_c, item0);
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(2 * C, 1, 1);
         cfg.blockDim = dim3(kThreads, 1, 1);
-        cfg.dynamicSmemBytes = kGSmem;
+        cfg.dynamicSmemBytes = T::kSmem;
         cfg.stream = s;
         cudaLaunchAttribute lattr[2];
         lattr[0].id = cudaLaunchAttributeClusterDimension;
@@ -1313,7 +1345,7 @@ cudaError_t launch_batched_grouped(const BatchJob *jobs, int count, uint32_t *er
         const DebugWait dbg = debug_wait();
         const int skip_report = dbg.site == PVMVMD_DEBUG_WAIT_PRODUCT ? (int)dbg.index : -1;
         const uint64_t wait_ns = dbg.site == PVMVMD_DEBUG_WAIT_PRODUCT ? dbg.limit : kWaitNs;
-        e = cudaLaunchKernelEx(&cfg, k_batched_grouped, args, err, skip_report, wait_ns);
+        e = cudaLaunchKernelEx(&cfg, k_batched_grouped<V>, args, err, skip_report, wait_ns);
         if (e != cudaSuccess) return e;
         if (any_split) {
             int dev = 0, sms = 0;
@@ -1325,6 +1357,16 @@ cudaError_t launch_batched_grouped(const BatchJob *jobs, int count, uint32_t *er
         }
     }
     return cudaSuccess;
+}
+
+cudaError_t launch_batched_grouped(const BatchJob *jobs, int count, uint32_t *err, cudaStream_t s) {
+    // small batches in 16-vector tiles, the rest in 64-vector tiles
+    std::vector<BatchJob> narrow, wide;
+    for (int i = 0; i < count; ++i) (jobs[i].B <= kNarrowMaxB ? narrow : wide).push_back(jobs[i]);
+    cudaError_t e = cudaSuccess;
+    if (!wide.empty()) e = launch_grouped_v<64>(wide.data(), (int)wide.size(), err, s);
+    if (e == cudaSuccess && !narrow.empty()) e = launch_grouped_v<16>(narrow.data(), (int)narrow.size(), err, s);
+    return e;
 }
 
 

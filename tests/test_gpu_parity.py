@@ -713,3 +713,29 @@ def test_server_mvm_grouped_mixed_jobs(pv):
     for W, X, _, _, Yd in ins:
         assert_equal_report(pv.as_u32(Yd), oracle.server_mvm_batch(W, X), str((W.shape, X.shape[0])))
     assert pv.pvmvmd_device_status() == 0
+
+
+@pytest.mark.parametrize("specs", [
+    [(300, 1024, 5), (513, 4144, 16), (1030, 2048, 2), (65, 16384, 11)],
+    [(4096, 2560, 8), (1024, 2560, 8), (2560, 4096, 8), (9728, 2560, 8), (2560, 9728, 8)],
+])
+def test_server_mvm_grouped_small_batches(pv, specs):
+    """Batches of 2 to 16 vectors in one grouped call run the tensor-core
+    kernel with 16-vector tiles (N = 64): every output equals the oracle's,
+    on ragged shapes and on the Qwen3-4B block's projections with 8 vectors."""
+    import torch
+    rng = np.random.default_rng(len(specs) * 31 + specs[0][0])
+    ins = []
+    for m, K, B in specs:
+        W = rng.integers(-128, 128, size=(m, K), dtype=np.int8)
+        W[m - 1] = -128
+        X = rng.integers(0, Q, size=(B, K)).astype(np.uint32)
+        X[B - 1] = (Q + 1) // 2
+        ins.append((W, X, to_dev(W), to_dev(X), torch.full((B, m), -1, dtype=torch.int32, device="cuda")))
+    jobs = pv.batch_jobs([(Wd, Xd, Yd) for _, _, Wd, Xd, Yd in ins])
+    for rep in range(2):
+        pv.pvmvmd_server_mvm_grouped(jobs)
+        torch.cuda.synchronize()
+        for W, X, _, _, Yd in ins:
+            assert_equal_report(pv.as_u32(Yd), oracle.server_mvm_batch(W, X), f"rep {rep} {W.shape} B={X.shape[0]}")
+    assert pv.pvmvmd_device_status() == 0
