@@ -861,13 +861,79 @@ def measure_batched(args, workload, device, rank=0, world=1, with_cpu=True, with
         pv.pvmvmd_server_mvm_grouped(grouped_jobs, stream=stream)
         forked(d)
 
-    step_fn = {"projections": pipelined, "phases": phases, "grouped": grouped}[args.schedule]
+    # --schedule pipeline: three batches in flight.  Step k encodes batch
+    # k + 1, runs the server products of batch k (one grouped call) and
+    # decodes batch k - 1, the three branches side by side on their own
+    # streams; every step still encodes, multiplies and decodes one batch of
+    # every projection.  Three sets of buffers rotate (an encode and a decode
+    # of one context may overlap; two of either never do).
+    nsets = 3
+    # zero-filled: the first two eager steps decode sets that hold no batch
+    # yet, and a zero mask state indexes row 0 of P^T, which exists
+    for p in projs:
+        p["sets"] = [dict(Xh=torch.zeros_like(p["X"]), st=torch.zeros_like(p["st"]), Yh=torch.zeros_like(p["Yh"]),
+                          Y=torch.zeros_like(p["Y"]), acc=torch.zeros_like(p["acc"])) for _ in range(nsets)]
+    set_jobs = [pv.batch_jobs([(p["W"], p["sets"][i]["Xh"], p["sets"][i]["Yh"]) for p in projs])
+                for i in range(nsets)]
+    srv_stream = torch.cuda.Stream(device)
+    dec_streams = [torch.cuda.Stream(device) for _ in range(max(1, args.server_streams))]
+
+    def pipeline_step(k, host=None):
+        se, sv, sd = (k + 1) % nsets, k % nsets, (k - 1) % nsets
+        fork = torch.cuda.Event()
+        fork.record(stream)
+        branches = proj_streams + dec_streams + [srv_stream]
+        for ss in branches:
+            ss.wait_event(fork)
+        for j, p in enumerate(projs):
+            ss = proj_streams[j % len(proj_streams)]
+            with torch.cuda.stream(ss):
+                src, b = p["X"], p["sets"][se]
+                if host is not None:
+                    b["Xin"].copy_(p["Xhost"], non_blocking=True)
+                    src = b["Xin"]
+                pv.pvmvmd_encode(p["ctx"], src, 21, Xhat=b["Xh"], st=b["st"], stream=ss)
+        pv.pvmvmd_server_mvm_grouped(set_jobs[sv], stream=srv_stream)
+        for j, p in enumerate(projs):
+            ss = dec_streams[j % len(dec_streams)]
+            with torch.cuda.stream(ss):
+                b = p["sets"][sd]
+                pv.pvmvmd_decode_verify(p["ctx"], b["st"], b["Xh"], b["Yh"], 22, Y=b["Y"], accept=b["acc"],
+                                        stream=ss)
+                if host is not None:
+                    b["Yhost"].copy_(b["Y"], non_blocking=True)
+                    b["Ahost"].copy_(b["acc"], non_blocking=True)
+        for ss in branches:
+            join = torch.cuda.Event()
+            join.record(ss)
+            stream.wait_event(join)
+
+    if args.schedule == "pipeline":
+        # fill the pipeline eagerly: after steps -1, 0, 1 batch 0 is decoded
+        with torch.cuda.stream(stream):
+            for k in (-1, 0, 1):
+                pipeline_step(k)
+        stream.synchronize()
+        for p in projs:
+            b = p["sets"][0]
+            p["Y"].copy_(b["Y"])
+            p["acc"].copy_(b["acc"])
+        torch.cuda.synchronize(device)
+
+    step_fn = {"projections": pipelined, "phases": phases, "grouped": grouped, "pipeline": None}[args.schedule]
     # eager runs of every schedule that is captured below (the first call on
     # a stream sizes its scratch, which a capture may not do)
     with torch.cuda.stream(stream):
-        enc(); srv(); dec()
-        step_fn()
+        if step_fn is not None:
+            enc(); srv(); dec()
+            step_fn()
+        else:   # the pipeline's output was checked out above; the phases still run eagerly once
+            Ysave = [(p["Y"].clone(), p["acc"].clone()) for p in projs]
+            enc(); srv(); dec()
     stream.synchronize()
+    if step_fn is None:
+        for p, (yv, av) in zip(projs, Ysave):
+            assert torch.equal(yv, p["Y"]) and torch.equal(av, p["acc"]), "pipelined batch differs from the phases"
     assert pv.pvmvmd_device_status(stream) == 0
     for p in projs:
         assert int(p["acc"].sum()) == B
@@ -883,19 +949,29 @@ def measure_batched(args, workload, device, rank=0, world=1, with_cpu=True, with
         graphs.append(g)
     # the whole step as one graph (what `value` times); the per-phase graphs
     # give the phase split
-    g_step = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(g_step, stream=stream):
-        step_fn()
+    if step_fn is not None:
+        g_step = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g_step, stream=stream):
+            step_fn()
+        step_graphs = [g_step]
+    else:
+        step_graphs = []
+        for k in range(nsets):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                pipeline_step(k)
+            step_graphs.append(g)
+    nsg = len(step_graphs)
     w0, w1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with torch.cuda.stream(stream):
         for g in graphs:
             g.replay()
         w0.record(stream)
-        for _ in range(args.warmup):
-            g_step.replay()
+        for w in range(args.warmup * nsg):
+            step_graphs[w % nsg].replay()
         w1.record(stream)
     stream.synchronize()
-    ms_est = w0.elapsed_time(w1) / args.warmup
+    ms_est = w0.elapsed_time(w1) / (args.warmup * nsg)
     clocks = ClockSampler(device.index)
     clocks.start()
     barrier(device)
@@ -905,11 +981,16 @@ def measure_batched(args, workload, device, rank=0, world=1, with_cpu=True, with
     clocks.region_started()
     with torch.cuda.stream(stream):
         t0.record(stream)
-        for s in range(args.steps):
-            g_step.replay()
+        for s_ in range(args.steps):
+            step_graphs[s_ % nsg].replay()
         t1.record(stream)
-        clock_tail(lambda i: g_step.replay(), ms_est)
+        clock_tail(lambda i: step_graphs[(args.steps + i) % nsg].replay(), ms_est)
     stream.synchronize()
+    if step_fn is None:
+        # the batch decoded by the last timed step completed its three steps
+        last = (args.steps - 2) % nsets
+        for p in projs:
+            assert int(p["sets"][last]["acc"].sum()) == B, "pipelined batch rejected"
     torch.cuda.synchronize(device)
     clk = clocks.stop()
     barrier(device)
@@ -981,31 +1062,54 @@ def measure_batched(args, workload, device, rank=0, world=1, with_cpu=True, with
             p["Xin"] = torch.empty_like(p["X"])
             p["Yhost"] = torch.empty((B, p["m"]), dtype=torch.int32).pin_memory()
             p["Ahost"] = torch.empty(B, dtype=torch.int32).pin_memory()
-        e2e_fn = grouped if args.schedule == "grouped" else pipelined
+        if args.schedule == "pipeline":
+            for p in projs:
+                for b in p["sets"]:
+                    b["Xin"] = torch.empty_like(p["X"])
+                    b["Yhost"] = torch.empty((B, p["m"]), dtype=torch.int32).pin_memory()
+                    b["Ahost"] = torch.empty(B, dtype=torch.int32).pin_memory()
+            with torch.cuda.stream(stream):
+                for k in (-1, 0, 1):
+                    pipeline_step(k, host=True)
+            stream.synchronize()
+            e2e_graphs = []
+            for k in range(nsets):
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=stream):
+                    pipeline_step(k, host=True)
+                e2e_graphs.append(g)
+        else:
+            e2e_fn = grouped if args.schedule == "grouped" else pipelined
+            with torch.cuda.stream(stream):
+                e2e_fn(host=True)
+            stream.synchronize()
+            g_e2e = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g_e2e, stream=stream):
+                e2e_fn(host=True)
+            e2e_graphs = [g_e2e]
+        ne = len(e2e_graphs)
         with torch.cuda.stream(stream):
-            e2e_fn(host=True)
-        stream.synchronize()
-        g_e2e = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g_e2e, stream=stream):
-            e2e_fn(host=True)
-        with torch.cuda.stream(stream):
-            for _ in range(args.warmup):
-                g_e2e.replay()
+            for w in range(args.warmup * ne):
+                e2e_graphs[w % ne].replay()
         stream.synchronize()
         barrier(device)
-        n_e2e = max(2, args.steps)
+        n_e2e = max(3, args.steps)
         te = time.perf_counter()
         with torch.cuda.stream(stream):
-            for _ in range(n_e2e):
-                g_e2e.replay()
+            for i in range(n_e2e):
+                e2e_graphs[i % ne].replay()
         stream.synchronize()
         e2e_s = max_over_ranks(time.perf_counter() - te, device)
         for p in projs:
-            assert int(p["Ahost"].sum()) == B
+            hosts = [b["Ahost"] for b in p["sets"]] if args.schedule == "pipeline" else [p["Ahost"]]
+            assert any(int(h.sum()) == B for h in hosts)
         e2e = {"value": world * macs * n_e2e / e2e_s, "unit": UNIT,
                "h2d_bytes_per_step": int(sum(p["Xhost"].numel() * 4 for p in projs)),
                "d2h_bytes_per_step": int(sum(p["Yhost"].numel() * 4 + p["Ahost"].numel() * 4 for p in projs)),
-               "how": ("CUDA graph of the public calls (the encodes side by side on "
+               "how": ("CUDA graphs of the public calls, three batches in flight (batch k + 1's encodes, "
+                       "batch k's grouped product call and batch k - 1's decodes side by side)"
+                       if args.schedule == "pipeline" else
+                       "CUDA graph of the public calls (the encodes side by side on "
                        f"{len(proj_streams)} streams, one grouped product call, the decodes side by side)"
                        if args.schedule == "grouped" else
                        "CUDA graph of the public calls (each projection's encode, product, decode on one of "
@@ -1664,11 +1768,13 @@ def main(argv=None):
                     help="m x K x B for --workload server-shape and decode-shape, K x B for --workload "
                          "encode-shape, a batched workload name for --workload server-layer")
     ap.add_argument("--server-streams", type=int, default=4)
-    ap.add_argument("--schedule", choices=["phases", "projections", "grouped"], default="grouped",
+    ap.add_argument("--schedule", choices=["phases", "projections", "grouped", "pipeline"], default="grouped",
                     help="batched workloads: all encodes, then all products, then all decodes "
                          "(phases); each projection's three calls in order on one of "
                          "--server-streams streams (projections); or the encodes side by side on those "
-                         "streams, one grouped product call, the decodes side by side (grouped)")
+                         "streams, one grouped product call, the decodes side by side (grouped); or three "
+                         "batches in flight, batch k+1's encodes beside batch k's products and batch k-1's "
+                         "decodes (pipeline)")
     ap.add_argument("--server-call", choices=["grouped", "per-projection"], default="grouped",
                     help="batched workloads, server phase: one pvmvmd_server_mvm_grouped call for the layer, "
                          "or one pvmvmd_server_mvm call per projection spread over --server-streams streams")

@@ -226,7 +226,8 @@ int pvmvmd_server_mvm_noalloc(const int8_t *W_dev, int m, int K, const uint32_t 
  * vector b is accepted iff (e_q^T Q) x_hat_b == e_q^T (G_y^T y_hat_b) for every q.
  * The right side is evaluated as (G_y e_q)^T y_hat_b, the same number by
  * transposition.  Decrypt: Y_b = y_hat_b - P e_x,b.  st_dev as written by
- * pvmvmd_encode; Xhat_dev B x K; Yhat_dev B x m; Y_dev B x m (may alias
+ * pvmvmd_encode (another state gives unspecified results, but every read
+ * stays inside P); Xhat_dev B x K; Yhat_dev B x m; Y_dev B x m (may alias
  * Yhat_dev); accept_dev B int32, each 1 (accept) or 0 (reject).  A rejection
  * is data, not an error.  Y is written for rejected vectors too. */
 int pvmvmd_decode_verify(pvmvmd_ctx *ctx, const void *st_dev, const uint32_t *Xhat_dev,

@@ -760,8 +760,8 @@ int decode_verify_batch(pvmvmd_ctx *ctx, const void *st_dev, const uint32_t *mas
     }
     int st = verify_chain(ctx, challenge_key, Xhat_dev, Yhat_dev, B, accept_dev, cs);
     if (st) return st;
-    PV_CUDA(launch_decrypt(ctx->PT, ctx->m, static_cast<const uint32_t *>(st_dev), ctx->t_x, Yhat_dev, B,
-                           Y_dev, s, mask_out_dev));
+    PV_CUDA(launch_decrypt(ctx->PT, ctx->m, static_cast<const uint32_t *>(st_dev), ctx->t_x, (uint32_t)ctx->Nx,
+                           Yhat_dev, B, Y_dev, s, mask_out_dev));
     if (!in_place) {
         PV_CUDA(cudaEventRecord(ctx->join, ctx->side));
         PV_CUDA(cudaStreamWaitEvent(s, ctx->join, 0));

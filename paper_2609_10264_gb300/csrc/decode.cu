@@ -166,7 +166,7 @@ constexpr int kDecCols = 4 * kDecColThreads;              // 512 columns per CTA
 template <bool kBoost>
 __global__ void __launch_bounds__(kDecThreads) k_decrypt(const uint32_t *__restrict__ PT, int m,
                                                         const uint32_t *__restrict__ st, uint32_t t_x,
-                                                        const uint32_t *Yhat, uint32_t *Y,
+                                                        uint32_t Nx, const uint32_t *Yhat, uint32_t *Y,
                                                         const uint32_t *__restrict__ mask, bool vec) {
     extern __shared__ uint32_t sm[];  // support[t_x], values[t_x]
     __shared__ uint4 s_part[kDecGroups > 1 ? kDecGroups - 1 : 1][kDecColThreads];
@@ -178,7 +178,12 @@ __global__ void __launch_bounds__(kDecThreads) k_decrypt(const uint32_t *__restr
     uint32_t pe[4] = {0u, 0u, 0u, 0u};
     if (!kBoost) {
         const uint32_t *stb = st + b * 2 * t_x;
-        for (uint32_t j = tid; j < 2 * t_x; j += kDecThreads) sm[j] = stb[j];
+        // a support index past the code (a state the encode did not write)
+        // reads row 0 instead: the result is then wrong, never out of bounds
+        for (uint32_t j = tid; j < 2 * t_x; j += kDecThreads) {
+            const uint32_t v = stb[j];
+            sm[j] = (j < t_x && v >= Nx) ? 0u : v;
+        }
         __syncthreads();
         const uint32_t per = (t_x + kDecGroups - 1) / kDecGroups;
         const uint32_t j0 = min(t_x, (uint32_t)grp * per), j1 = min(t_x, j0 + per);
@@ -373,7 +378,7 @@ cudaError_t launch_verify_u(const uint32_t *Qm, int K, const uint32_t *chal, uin
     return cudaLaunchKernelEx(&cfg, k_verify_u, Qm, K, chal, t_y, u);
 }
 
-cudaError_t launch_decrypt(const uint32_t *PT, int m, const uint32_t *st, uint32_t t_x,
+cudaError_t launch_decrypt(const uint32_t *PT, int m, const uint32_t *st, uint32_t t_x, uint32_t Nx,
                            const uint32_t *Yhat, int B, uint32_t *Y, cudaStream_t s, const uint32_t *mask) {
     if (B <= 0 || m <= 0) return cudaSuccess;
     const bool vec = (m % 4 == 0) &&
@@ -385,9 +390,9 @@ cudaError_t launch_decrypt(const uint32_t *PT, int m, const uint32_t *st, uint32
     const dim3 grid((unsigned)B, (m + kDecCols - 1) / kDecCols);
     const dim3 grid_mask((unsigned)B, (m + 4 * kDecThreads - 1) / (4 * kDecThreads));
     if (mask)
-        k_decrypt<true><<<grid_mask, kDecThreads, 0, s>>>(PT, m, nullptr, t_x, Yhat, Y, mask, vec);
+        k_decrypt<true><<<grid_mask, kDecThreads, 0, s>>>(PT, m, nullptr, t_x, Nx, Yhat, Y, mask, vec);
     else
-        k_decrypt<false><<<grid, kDecThreads, smem, s>>>(PT, m, st, t_x, Yhat, Y, nullptr, vec);
+        k_decrypt<false><<<grid, kDecThreads, smem, s>>>(PT, m, st, t_x, Nx, Yhat, Y, nullptr, vec);
     return cudaGetLastError();
 }
 

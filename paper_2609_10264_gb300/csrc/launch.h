@@ -163,10 +163,11 @@ DebugWait debug_wait();
 cudaError_t launch_verify_u(const uint32_t *Qm, int K, const uint32_t *chal, uint32_t t_y,
                             uint32_t ell, uint32_t *u, cudaStream_t s);
 
-// Decrypt: Y[b] = Y_hat[b] - P e_x,b for B vectors (st [B][2t_x]); with
+// Decrypt: Y[b] = Y_hat[b] - P e_x,b for B vectors (st [B][2t_x], support
+// indices below Nx; others read row 0); with
 // mask non-null (boost mode) Y = Y_hat - mask, mask [B][m] = P e_x per
 // vector, and st is not read.  Y may alias Y_hat.
-cudaError_t launch_decrypt(const uint32_t *PT, int m, const uint32_t *st, uint32_t t_x,
+cudaError_t launch_decrypt(const uint32_t *PT, int m, const uint32_t *st, uint32_t t_x, uint32_t Nx,
                            const uint32_t *Yhat, int B, uint32_t *Y, cudaStream_t s,
                            const uint32_t *mask = nullptr);
 // Verify: accept[b] = AND_q (u_q . Xhat[b] == g_q . Yhat[b]) for the ell

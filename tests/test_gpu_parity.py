@@ -739,3 +739,25 @@ def test_server_mvm_grouped_small_batches(pv, specs):
         for W, X, _, _, Yd in ins:
             assert_equal_report(pv.as_u32(Yd), oracle.server_mvm_batch(W, X), f"rep {rep} {W.shape} B={X.shape[0]}")
     assert pv.pvmvmd_device_status() == 0
+
+
+def test_decode_with_foreign_state_stays_in_bounds(pv, wl):
+    """A mask state the encode did not write (support indices at and past
+    N_x) gives wrong outputs for that vector only: every read stays inside
+    P^T, the call completes, and the other vectors decode exactly."""
+    W = wl.weights_uniform(256, 512, 61)
+    x = wl.int8_vectors(3, 512, 62)
+    ctx = pv.pvmvmd_preprocess(to_dev(W), key=63)
+    Xh, st = pv.pvmvmd_encode(ctx, to_dev(field(x)), key=64)
+    Yh = pv.pvmvmd_server_mvm(to_dev(W), Xh)
+    bad = st.clone()
+    bad[1, 0] = ctx.N_x
+    bad[1, 1] = -1            # 0xFFFFFFFF as a support index
+    Y, acc = pv.pvmvmd_decode_verify(ctx, bad, Xh, Yh, challenge_key=65)
+    assert pv.pvmvmd_device_status() == 0
+    Y_h = oracle.centered(pv.as_u32(Y))
+    exp = exact_product(W, x)
+    assert np.array_equal(Y_h[0], exp[0]) and np.array_equal(Y_h[2], exp[2])
+    assert not np.array_equal(Y_h[1], exp[1])
+    assert pv.as_u32(acc).tolist() == [1, 1, 1]   # verification reads x_hat and y_hat only
+    ctx.destroy()
