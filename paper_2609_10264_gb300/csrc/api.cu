@@ -188,8 +188,9 @@ struct pvmvmd_ctx {
     unsigned long long *status = nullptr, *status_y = nullptr;
     // lane-parallel encode scratch (null when scratch_batch < kLaneMinBatch)
     uint32_t *S = nullptr, *laux = nullptr;
-    // decode: the challenge kernels run on `side`, forked from and joined
-    // back to the caller's stream, while the decrypt streams P^T
+    // decode: the challenge kernels run on `side` (highest stream priority),
+    // forked from and joined back to the caller's stream, while the decrypt
+    // streams P^T
     cudaStream_t side = nullptr;
     cudaEvent_t fork = nullptr, join = nullptr;
     std::vector<void *> owned;
@@ -204,7 +205,8 @@ struct pvmvmd_bv_ctx {
     uint32_t *QauxT = nullptr; // N' x N: Qaux transposed
     uint32_t *Yt = nullptr, *Z = nullptr;  // m x B, N x B
     uint32_t *chal2 = nullptr, *R = nullptr, *F2 = nullptr;
-    uint32_t *eS = nullptr, *eagg = nullptr, *eincl = nullptr, *eflags = nullptr;  // encode scratch
+    uint32_t *eS = nullptr, *eticket = nullptr;  // encode scratch: S, scan ticket
+    unsigned long long *estatus = nullptr;       // and scan status words
     unsigned long long *status = nullptr;
     std::vector<void *> owned;
 };
@@ -246,18 +248,19 @@ int upload_code(Ctx *c, CodeDev &d, const pvmvmd_key &key, int which, uint32_t N
 
 // Y (N x L lanes, row stride ldy) = G^T applied to the L lanes of X (n x L,
 // row stride ldx; row i holds message entry i of every lane), in lane chunks.
-// One chunk of lanes with caller-provided scratch (S: N x nl, agg / incl /
-// flags sized by encode_scan_*_words(N, nl)); no allocation, no sync.
+// One chunk of lanes with caller-provided scratch (S: N x nl; status:
+// encode_scan_status_words(N, nl) 64-bit words; ticket: one word); no
+// allocation, no sync.
 int encode_lanes_into(const CodeDev &d, uint32_t n, uint32_t r, const void *X, bool x_is_i8, size_t ldx,
-                      uint32_t nl, uint32_t *Y, size_t ldy, uint32_t *S, uint32_t *agg, uint32_t *incl,
-                      uint32_t *flags, uint32_t *err, cudaStream_t s) {
+                      uint32_t nl, uint32_t *Y, size_t ldy, uint32_t *S, unsigned long long *status,
+                      uint32_t *ticket, uint32_t *err, cudaStream_t s) {
     const uint32_t N = n * r;
-    cudaError_t e = cudaMemsetAsync(flags, 0, encode_scan_flag_words(N, nl) * 4, s);
+    cudaError_t e = encode_scan_clear(status, ticket, N, nl, s);
     if (e == cudaSuccess)  // S = A^T V1 Pi1^T R^T X
-        e = launch_encode_scan(X, x_is_i8, ldx, d.pi1, r, d.v1m, N, nl, S, nl, agg, incl, flags, err, s);
-    if (e == cudaSuccess) e = cudaMemsetAsync(flags, 0, encode_scan_flag_words(N, nl) * 4, s);
+        e = launch_encode_scan(X, x_is_i8, ldx, d.pi1, r, d.v1m, N, nl, S, nl, status, ticket, err, s);
+    if (e == cudaSuccess) e = encode_scan_clear(status, ticket, N, nl, s);
     if (e == cudaSuccess)  // Y = A^T V2 Pi2^T S
-        e = launch_encode_scan(S, false, nl, d.pi2, 1, d.v2m, N, nl, Y, ldy, agg, incl, flags, err, s);
+        e = launch_encode_scan(S, false, nl, d.pi2, 1, d.v2m, N, nl, Y, ldy, status, ticket, err, s);
     return e == cudaSuccess ? PVMVMD_OK : PVMVMD_E_CUDA;
 }
 
@@ -271,26 +274,25 @@ int encode_lanes(const CodeDev &d, uint32_t n, uint32_t r, const void *X, bool x
     lc = (lc / 256) * 256;
     if (lc < 256) lc = 256;
     if (lc > L) lc = L;
-    uint32_t *S = nullptr, *agg = nullptr, *incl = nullptr, *flags = nullptr;
-    const size_t fw = encode_scan_flag_words(N, (uint32_t)lc);
-    const size_t vw = encode_scan_value_words(N, (uint32_t)lc);
-    int status = PVMVMD_OK;
-    if (dev_alloc(&S, (size_t)N * lc) != cudaSuccess || dev_alloc(&agg, vw) != cudaSuccess ||
-        dev_alloc(&incl, vw) != cudaSuccess || dev_alloc(&flags, fw) != cudaSuccess) {
-        status = PVMVMD_E_NOMEM;
+    uint32_t *S = nullptr, *ticket = nullptr;
+    unsigned long long *status = nullptr;
+    const size_t sw = encode_scan_status_words(N, (uint32_t)lc);
+    int status_code = PVMVMD_OK;
+    if (dev_alloc(&S, (size_t)N * lc) != cudaSuccess || dev_alloc(&status, sw) != cudaSuccess ||
+        dev_alloc(&ticket, 1) != cudaSuccess) {
+        status_code = PVMVMD_E_NOMEM;
     }
-    for (uint32_t l0 = 0; status == PVMVMD_OK && l0 < L; l0 += (uint32_t)lc) {
+    for (uint32_t l0 = 0; status_code == PVMVMD_OK && l0 < L; l0 += (uint32_t)lc) {
         const uint32_t nl = (uint32_t)((L - l0) < lc ? (L - l0) : lc);
         const void *Xl = x_is_i8 ? static_cast<const void *>(static_cast<const int8_t *>(X) + l0)
                                  : static_cast<const void *>(static_cast<const uint32_t *>(X) + l0);
-        status = encode_lanes_into(d, n, r, Xl, x_is_i8, ldx, nl, Y + l0, ldy, S, agg, incl, flags, err, s);
+        status_code = encode_lanes_into(d, n, r, Xl, x_is_i8, ldx, nl, Y + l0, ldy, S, status, ticket, err, s);
     }
-    if (cudaStreamSynchronize(s) != cudaSuccess) status = PVMVMD_E_CUDA;
+    if (cudaStreamSynchronize(s) != cudaSuccess) status_code = PVMVMD_E_CUDA;
     cudaFree(S);
-    cudaFree(agg);
-    cudaFree(incl);
-    cudaFree(flags);
-    return status;
+    cudaFree(status);
+    cudaFree(ticket);
+    return status_code;
 }
 
 int read_and_clear_error() {
@@ -457,7 +459,12 @@ int preprocess_impl(const void *W_dev, bool w16, int m, int K, const pvmvmd_para
         ctx_alloc(c, &c->status, scan_status_words(c->Nx, c->sb)) != cudaSuccess ||
         ctx_alloc(c, &c->status_y, scan_status_words(c->Ny, c->ell)) != cudaSuccess)
         return fail(PVMVMD_E_NOMEM);
-    if (cudaStreamCreateWithFlags(&c->side, cudaStreamNonBlocking) != cudaSuccess ||
+    // the challenge kernels are few and short; at the highest priority their
+    // blocks take SMs as the decrypt's blocks drain instead of queueing
+    // behind the rest of the decrypt's grid
+    int prio_least = 0, prio_greatest = 0;
+    if (cudaDeviceGetStreamPriorityRange(&prio_least, &prio_greatest) != cudaSuccess ||
+        cudaStreamCreateWithPriority(&c->side, cudaStreamNonBlocking, prio_greatest) != cudaSuccess ||
         cudaEventCreateWithFlags(&c->fork, cudaEventDisableTiming) != cudaSuccess ||
         cudaEventCreateWithFlags(&c->join, cudaEventDisableTiming) != cudaSuccess)
         return fail(PVMVMD_E_CUDA);
@@ -794,19 +801,18 @@ int pvmvmd_boost_decode_verify(pvmvmd_ctx *ctx, const uint32_t *mask_out_dev,
 
 namespace pv {
 namespace {
-// Scratch of pvmvmd_code_encode_lanes: S (N x L), agg, incl (value words),
-// flags, each at a 16-byte aligned offset.
+// Scratch of pvmvmd_code_encode_lanes: S (N x L), the scan's 64-bit status
+// words and its ticket word, each at a 16-byte aligned offset.
 struct EncodeScratch {
-    size_t s_off, agg_off, incl_off, flag_off, bytes;
+    size_t s_off, status_off, ticket_off, bytes;
 };
 EncodeScratch encode_scratch_layout(uint32_t N, uint32_t L) {
     auto up = [](size_t b) { return (b + 15) & ~(size_t)15; };
     EncodeScratch e;
     e.s_off = 0;
-    e.agg_off = up((size_t)N * L * 4);
-    e.incl_off = e.agg_off + up(encode_scan_value_words(N, L) * 4);
-    e.flag_off = e.incl_off + up(encode_scan_value_words(N, L) * 4);
-    e.bytes = e.flag_off + up(encode_scan_flag_words(N, L) * 4);
+    e.status_off = up((size_t)N * L * 4);
+    e.ticket_off = e.status_off + up(encode_scan_status_words(N, L) * 8);
+    e.bytes = e.ticket_off + 16;
     return e;
 }
 }  // namespace
@@ -833,9 +839,8 @@ int pvmvmd_code_encode_lanes(const pvmvmd_ctx *ctx, int which, const uint32_t *X
     uint8_t *base = static_cast<uint8_t *>(scratch_dev);
     return encode_lanes_into(d, n, (uint32_t)ctx->rate, X_dev, false, (size_t)L, (uint32_t)L, Y_dev, (size_t)L,
                              reinterpret_cast<uint32_t *>(base + lay.s_off),
-                             reinterpret_cast<uint32_t *>(base + lay.agg_off),
-                             reinterpret_cast<uint32_t *>(base + lay.incl_off),
-                             reinterpret_cast<uint32_t *>(base + lay.flag_off), err,
+                             reinterpret_cast<unsigned long long *>(base + lay.status_off),
+                             reinterpret_cast<uint32_t *>(base + lay.ticket_off), err,
                              static_cast<cudaStream_t>(stream));
 }
 
@@ -928,8 +933,7 @@ int pvmvmd_bv_preprocess(const int8_t *W_dev, int B, int m, int n, const pvmvmd_
     const uint32_t Bn = (uint32_t)B * n;
     if ((st = upload_code(c, c->g, *key, 3, (uint32_t)N, s))) return fail(st);
     if ((st = upload_code(c, c->g2, *key, 4, (uint32_t)N2, s))) return fail(st);
-    const size_t fw = encode_scan_flag_words((uint32_t)N, (uint32_t)B);
-    const size_t vw = encode_scan_value_words((uint32_t)N, (uint32_t)B);
+    const size_t sw = encode_scan_status_words((uint32_t)N, (uint32_t)B);
     if (ctx_alloc(c, &c->Qs, (size_t)N * Bn) != cudaSuccess ||
         ctx_alloc(c, &c->QauxT, (size_t)N2 * N) != cudaSuccess ||
         ctx_alloc(c, &c->Yt, (size_t)m * B) != cudaSuccess ||
@@ -937,8 +941,8 @@ int pvmvmd_bv_preprocess(const int8_t *W_dev, int B, int m, int n, const pvmvmd_
         ctx_alloc(c, &c->chal2, (size_t)ell2 * 2 * t2) != cudaSuccess ||
         ctx_alloc(c, &c->R, (size_t)ell2 * Bn) != cudaSuccess ||
         ctx_alloc(c, &c->F2, (size_t)ell2 * N2) != cudaSuccess ||
-        ctx_alloc(c, &c->eS, (size_t)N * B) != cudaSuccess || ctx_alloc(c, &c->eagg, vw) != cudaSuccess ||
-        ctx_alloc(c, &c->eincl, vw) != cudaSuccess || ctx_alloc(c, &c->eflags, fw) != cudaSuccess ||
+        ctx_alloc(c, &c->eS, (size_t)N * B) != cudaSuccess || ctx_alloc(c, &c->estatus, sw) != cudaSuccess ||
+        ctx_alloc(c, &c->eticket, 1) != cudaSuccess ||
         ctx_alloc(c, &c->status, scan_status_words((uint32_t)N2, (uint32_t)ell2)) != cudaSuccess)
         return fail(PVMVMD_E_NOMEM);
     // Q_b = G^T M_b into the column block b n of Qs (the lanes are M_b's columns)
@@ -991,8 +995,8 @@ int pvmvmd_bv_check(pvmvmd_bv_ctx *ctx, const uint32_t *X_dev, const uint32_t *Y
     // z_b = G^T y_b (the B outputs as lanes)
     PV_CUDA(launch_transpose_u32(Y_dev, ctx->B, ctx->m, ctx->Yt, s));
     int st = encode_lanes_into(ctx->g, (uint32_t)ctx->m, (uint32_t)ctx->rate, ctx->Yt, false, (size_t)ctx->B,
-                               (uint32_t)ctx->B, ctx->Z, (size_t)ctx->B, ctx->eS, ctx->eagg, ctx->eincl,
-                               ctx->eflags, err, s);
+                               (uint32_t)ctx->B, ctx->Z, (size_t)ctx->B, ctx->eS, ctx->estatus, ctx->eticket,
+                               err, s);
     if (st) return st;
     // secondary challenges, drawn after the responses, and r^(j) = G' e'^(j)
     const CodeDev &d = ctx->g2;

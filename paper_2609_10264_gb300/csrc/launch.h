@@ -83,15 +83,17 @@ cudaError_t launch_syndrome_gather(const uint32_t *pi1inv, uint32_t n, uint32_t 
 // One accumulate stage of the encoding G^T w over L lanes (App. B, encoding
 // direction): Y[j][l] = sum_{j' <= j} vscale[j'] * X[perm[j'] / div][l] for
 // j < N, with vscale_m = vscale R mod q (Montgomery form, R = 2^32).  X is
-// int8 (lifted to F_q) when x_is_i8, else uint32.  The scratch
-// `flags` holds ceil(L/256) * ceil(N/kEncTile) + 1 words and must be zero.
+// int8 (lifted to F_q) when x_is_i8, else uint32.  Scratch: `status` holds
+// encode_scan_status_words(N, L) 64-bit words and `ticket` one 32-bit word,
+// all zero at launch (encode_scan_clear).
 constexpr int kEncTile = 32;
-size_t encode_scan_flag_words(uint32_t N, uint32_t L);
-size_t encode_scan_value_words(uint32_t N, uint32_t L);
+size_t encode_scan_status_words(uint32_t N, uint32_t L);
+cudaError_t encode_scan_clear(unsigned long long *status, uint32_t *ticket, uint32_t N, uint32_t L,
+                              cudaStream_t s);
 cudaError_t launch_encode_scan(const void *X, bool x_is_i8, size_t ldx, const uint32_t *perm,
                                uint32_t div, const uint32_t *vscale_m, uint32_t N, uint32_t L,
-                               uint32_t *Y, size_t ldy, uint32_t *agg, uint32_t *incl,
-                               uint32_t *flags, uint32_t *err, cudaStream_t s);
+                               uint32_t *Y, size_t ldy, unsigned long long *status, uint32_t *ticket,
+                               uint32_t *err, cudaStream_t s);
 
 // int8 transpose: out[c][r] = in[r][c] for an R x C matrix.
 cudaError_t launch_transpose_i8(const int8_t *in, int R, int C, int8_t *out, cudaStream_t s);

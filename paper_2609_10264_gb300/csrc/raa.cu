@@ -747,31 +747,39 @@ __global__ void __launch_bounds__(kFusedThreads) k_syndrome_fused(
 // (pi2, 1, v2) it is A^T V2 Pi2^T.  vscale_m holds vscale in Montgomery form
 // (v R mod q).  A CTA owns 256 lanes and kEncTile positions: the source row
 // and scale of each position are looked up once per CTA (in shared memory),
-// every thread then issues all kEncTile row loads of its lane before the
-// arithmetic, and tiles of one lane block are chained by a decoupled
-// look-back over per-lane aggregates (flags: 1 = aggregate, 2 = inclusive
-// prefix).  At 32 positions per tile the kernel is held to 64 registers, four
-// CTAs per SM: 0.755 against 0.823 ms per 4096 x 4096 encoding at three CTAs
-// (80 registers); 16-position tiles, twice as many per chain, took 1.16 ms,
-// and 64-position tiles (two halves of 32, the first half's sums in shared
-// memory) 0.864 ms at 80 registers and 1.49 ms held to 64.
+// and every thread issues all kEncTile row loads of its lane before the
+// arithmetic.  Tiles of one lane block are chained by a decoupled look-back
+// that each lane walks on its own: per (tile, lane) one 64-bit status word
+// holds a state in its high half (1: the tile's own sum, 2: the inclusive
+// prefix through the tile) and the value in its low half, so a reader gets
+// state and value in one load and no fence or block barrier is needed.
+// Tiles are numbered in the order CTAs start (a global ticket), so every
+// predecessor of a tile is already running.  (The earlier form, one flag per
+// tile and the lanes' values in separate arrays behind a fence and block
+// barriers, with warp 0 reading 32 flags at a time, took 0.755 ms per
+// 4096 x 4096 encoding.)  At 32 positions per tile the kernel is held to 64
+// registers, four CTAs per SM.
 // -----------------------------------------------------------------------------
+__device__ __forceinline__ unsigned long long enc_status(uint32_t state, uint32_t v) {
+    return ((unsigned long long)state << 32) | v;
+}
+
 template <bool kI8>
 __global__ void __launch_bounds__(256, 4) k_encode_scan(const void *__restrict__ Xv, size_t ldx,
                                                     const uint32_t *__restrict__ perm, uint32_t div,
                                                     const uint32_t *__restrict__ vscale_m, uint32_t N,
                                                     uint32_t L, uint32_t *__restrict__ Y, size_t ldy,
-                                                    uint32_t *agg, uint32_t *incl, uint32_t *flags,
+                                                    unsigned long long *status, uint32_t *ticket_ctr,
                                                     uint32_t *__restrict__ err) {
-    __shared__ uint32_t s_ticket, s_nagg, s_state;
+    __shared__ uint32_t s_ticket;
     __shared__ uint32_t s_src[kEncTile], s_vs[kEncTile];
     const int tid = threadIdx.x;
     const uint32_t nlb = (L + 255) / 256;
     const uint32_t ntiles = (N + kEncTile - 1) / kEncTile;
-    if (tid == 0) s_ticket = atomicAdd(flags, 1u);
+    if (tid == 0) s_ticket = atomicAdd(ticket_ctr, 1u);
     __syncthreads();
     const uint32_t ticket = s_ticket;
-    if (ticket >= nlb * ntiles) {  // flags not cleared: never index past the data
+    if (ticket >= nlb * ntiles) {  // ticket not cleared: never index past the data
         if (tid == 0) record_error(err, kErrScanTimeout);
         return;
     }
@@ -803,69 +811,30 @@ __global__ void __launch_bounds__(256, 4) k_encode_scan(const void *__restrict__
         v[u] = run;
     }
 
-    const size_t slot = (size_t)lb * ntiles + tile;
-    uint32_t *fl = flags + 1;
+    // this lane's status word of tile 0 of the lane block; tile p is p * 256 on
+    unsigned long long *sw = status + (size_t)lb * ntiles * 256 + tid;
     uint32_t prefix = 0;
     if (tile == 0) {
-        incl[slot * 256 + tid] = run;
-        __threadfence();
-        __syncthreads();
-        if (tid == 0) st_release_u32(fl + slot, 2u);
+        st_relaxed_u64(sw, enc_status(2u, run));
     } else {
-        agg[slot * 256 + tid] = run;
-        __threadfence();
-        __syncthreads();
-        if (tid == 0) st_release_u32(fl + slot, 1u);
-        // Look back over windows of 32 predecessors at once: warp 0 reads
-        // their flags (lane i: tile hi - i) until every tile newer than the
-        // nearest inclusive one has published its aggregate, then all
-        // threads add those aggregates and that inclusive prefix for their
-        // lanes with independent loads.  Tile 0 is always inclusive, so the
-        // walk ends there at the latest.
-        const size_t base = (size_t)lb * ntiles;
-        int32_t hi = (int32_t)tile - 1;  // newest predecessor not yet added
-        for (;;) {
-            if (tid < 32) {
-                const int32_t j = hi - tid;
-                uint32_t spins = 0, nagg = 32, state = 0;  // 0: go on, 1: inclusive found, 2: gave up
-                for (;;) {
-                    const uint32_t f = j >= 0 ? ld_acquire_u32(fl + base + j) : 2u;
-                    const unsigned incl_mask = __ballot_sync(kFull, f == 2u);
-                    const unsigned zero_mask = __ballot_sync(kFull, f == 0u);
-                    nagg = incl_mask ? (uint32_t)(__ffs(incl_mask) - 1) : 32u;
-                    const unsigned need = nagg >= 32u ? kFull : ((1u << nagg) - 1u);
-                    if ((zero_mask & need) == 0u) {
-                        state = incl_mask ? 1u : 0u;
-                        break;
-                    }
-                    if (++spins > kSpinLimit) {
-                        if (tid == 0) record_error(err, kErrScanTimeout);
-                        nagg = 0;
-                        state = 2;
-                        break;
-                    }
-                    __nanosleep(32);
+        st_relaxed_u64(sw + (size_t)tile * 256, enc_status(1u, run));
+        uint32_t spins = 0;
+        for (uint32_t p = tile - 1;;) {
+            const unsigned long long w = ld_relaxed_u64(sw + (size_t)p * 256);
+            const uint32_t state = (uint32_t)(w >> 32);
+            if (state == 0u) {
+                if (++spins > kSpinLimit) {
+                    record_error(err, kErrScanTimeout);
+                    break;
                 }
-                if (tid == 0) {
-                    s_nagg = nagg;
-                    s_state = state;
-                }
+                __nanosleep(32);
+                continue;
             }
-            __syncthreads();
-            const int nagg = (int)s_nagg;
-            const uint32_t state = s_state;
-            __syncthreads();  // s_nagg / s_state are rewritten for the next window
-#pragma unroll 8
-            for (int c = 0; c < nagg; ++c) prefix = fadd(prefix, ld_cg_u32(agg + (base + hi - c) * 256 + tid));
-            if (state == 1u && hi - nagg >= 0)
-                prefix = fadd(prefix, ld_cg_u32(incl + (base + hi - nagg) * 256 + tid));
-            if (state != 0u) break;
-            hi -= 32;
+            prefix = fadd(prefix, (uint32_t)w);
+            if (state == 2u || p == 0u) break;  // tile 0 is always inclusive
+            --p;
         }
-        incl[slot * 256 + tid] = fadd(run, prefix);
-        __threadfence();
-        __syncthreads();
-        if (tid == 0) st_release_u32(fl + slot, 2u);
+        st_relaxed_u64(sw + (size_t)tile * 256, enc_status(2u, fadd(run, prefix)));
     }
     if (lane_ok) {
 #pragma unroll
@@ -1304,26 +1273,30 @@ cudaError_t launch_syndrome_gather(const uint32_t *pi1inv, uint32_t n, uint32_t 
     return cudaGetLastError();
 }
 
-size_t encode_scan_flag_words(uint32_t N, uint32_t L) {
-    return 1 + (size_t)((L + 255) / 256) * ((N + kEncTile - 1) / kEncTile);
-}
-size_t encode_scan_value_words(uint32_t N, uint32_t L) {
+size_t encode_scan_status_words(uint32_t N, uint32_t L) {
     return (size_t)((L + 255) / 256) * ((N + kEncTile - 1) / kEncTile) * 256;
+}
+
+cudaError_t encode_scan_clear(unsigned long long *status, uint32_t *ticket, uint32_t N, uint32_t L,
+                              cudaStream_t s) {
+    cudaError_t e = cudaMemsetAsync(status, 0, encode_scan_status_words(N, L) * sizeof(unsigned long long), s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(ticket, 0, sizeof(uint32_t), s);
+    return e;
 }
 
 cudaError_t launch_encode_scan(const void *X, bool x_is_i8, size_t ldx, const uint32_t *perm,
                                uint32_t div, const uint32_t *vscale_m, uint32_t N, uint32_t L,
-                               uint32_t *Y, size_t ldy, uint32_t *agg, uint32_t *incl,
-                               uint32_t *flags, uint32_t *err, cudaStream_t s) {
-    const size_t ctas = encode_scan_flag_words(N, L) - 1;
+                               uint32_t *Y, size_t ldy, unsigned long long *status, uint32_t *ticket,
+                               uint32_t *err, cudaStream_t s) {
+    const size_t ctas = encode_scan_status_words(N, L) / 256;
     if (ctas == 0) return cudaSuccess;
     if (ctas > 0x7fffffffu) return cudaErrorInvalidValue;
     if (x_is_i8)
         k_encode_scan<true><<<(unsigned)ctas, 256, 0, s>>>(X, ldx, perm, div, vscale_m, N, L, Y, ldy,
-                                                           agg, incl, flags, err);
+                                                           status, ticket, err);
     else
         k_encode_scan<false><<<(unsigned)ctas, 256, 0, s>>>(X, ldx, perm, div, vscale_m, N, L, Y, ldy,
-                                                            agg, incl, flags, err);
+                                                            status, ticket, err);
     return cudaGetLastError();
 }
 
