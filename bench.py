@@ -509,15 +509,20 @@ def run_ours(args):
         with torch.cuda.stream(stream):
             pv.pvmvmd_encode(ctx, Xd, 21 + rank, Xhat=Xh_sets[0], st=st_sets[0], stream=stream)
         stream.synchronize()
+        n_launch0 = pv.pvmvmd_kernel_launches()
         g_steps = [capture(lambda k=k: overlapped_step(k), stream) for k in range(2)]
     else:
+        n_launch0 = pv.pvmvmd_kernel_launches()
         g_steps = [capture(lambda k=k: whole_step(k), stream) for k in range(nsets)]
+    # kernels the library enqueued into the step graphs (each replay launches them again)
+    counted_per_step = (pv.pvmvmd_kernel_launches() - n_launch0) / len(g_steps)
     cur[0] = 0
     # encode: the fused syndrome kernel (standard), or k_field_add with masks
     # prepared ahead (boost; pipelined adds the preparation: fused syndrome +
     # k_output_mask); decode: challenge syndrome, k_verify_u, k_decrypt, k_check
     enc_launches = {"standard": 1, "boost": 1, "pipelined": 1 + 2}[args.mode]
     launches_per_step = enc_launches + (1 if args.server_mode == "multi" else VECTORS) + 4
+    assert counted_per_step == launches_per_step, (counted_per_step, launches_per_step)
     step_no = [0]
 
     def step(record=None):
@@ -948,7 +953,10 @@ def measure_batched(args, workload, device, rank=0, world=1, with_cpu=True, with
             fn()
         graphs.append(g)
     # the whole step as one graph (what `value` times); the per-phase graphs
-    # give the phase split
+    # give the phase split.  The library counts the kernels it enqueues, also
+    # while a stream is captured: the count around the step captures is the
+    # kernels every replay of those graphs launches.
+    n_launch0 = pv.pvmvmd_kernel_launches()
     if step_fn is not None:
         g_step = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g_step, stream=stream):
@@ -962,6 +970,7 @@ def measure_batched(args, workload, device, rank=0, world=1, with_cpu=True, with
                 pipeline_step(k)
             step_graphs.append(g)
     nsg = len(step_graphs)
+    launches_per_graph = (pv.pvmvmd_kernel_launches() - n_launch0) / nsg
     w0, w1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with torch.cuda.stream(stream):
         for g in graphs:
@@ -1028,7 +1037,15 @@ def measure_batched(args, workload, device, rank=0, world=1, with_cpu=True, with
     stream.synchronize()
     big_ms = k0.elapsed_time(k1) / reps
 
-    if B <= 16 and all(p["K"] % 16 == 0 for p in projs):
+    if B <= 16 and args.server_call == "grouped":
+        # a few vectors in 16-vector tensor-core tiles: one pass over M per
+        # call, so the product is bound by HBM, not by the tensor pipe
+        nbytes = sum(p["m"] * p["K"] + 4 * B * (p["K"] + p["m"]) for p in projs)
+        roof = {"bound": "hbm", "kernel": "k_batched_grouped<16> (tcgen05, 16-vector tiles), server phase",
+                "achieved": nbytes / (ph[1] / 1e3) / 1e9, "peak": peaks.get("hbm_gbs", 0.0), "unit": "GB/s",
+                "peak_kind": f"{kind} hbm_gbs", "bytes_per_step": nbytes, "traffic": None}
+        dtype = "u32 (F_q exact; fp16 digit MMAs, fp32 TMEM accumulation)"
+    elif B <= 16 and all(p["K"] % 16 == 0 for p in projs):
         # a few vectors run the dp4a GEMV over four vectors' digit planes: one
         # pass over M per four vectors, x_hat read and y_hat written once
         nbytes = sum(p["m"] * p["K"] * ((B + 3) // 4) + 4 * B * (p["K"] + p["m"]) for p in projs)
@@ -1040,9 +1057,9 @@ def measure_batched(args, workload, device, rank=0, world=1, with_cpu=True, with
         peak = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"])
         big_flops = 2 * 4 * big["m"] * big["K"] * B
         roof = {"bound": "tensor",
-                "kernel": f"k_batched (tcgen05 kind::f16 digit GEMM) on {big['name']} "
-                          f"{big['m']}x{big['K']}x{B}, one pvmvmd_server_mvm call (k_digit_tiles + k_batched) "
-                          "timed alone by CUDA events",
+                "kernel": f"k_batched_grouped (tcgen05 kind::f16 digit GEMM) on {big['name']} "
+                          f"{big['m']}x{big['K']}x{B}, one pvmvmd_server_mvm call (k_digit_tiles_grouped + "
+                          "k_batched_grouped, + k_split_finish when K is split) timed alone by CUDA events",
                 "achieved": big_flops / (big_ms / 1e3) / 1e12, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
                 "peak_kind": f"{kind} bf16_tflops (burst; the kernel timed alone)", "traffic": None,
                 "flops_per_launch": big_flops, "launch_ms": big_ms,
@@ -1141,7 +1158,7 @@ def measure_batched(args, workload, device, rank=0, world=1, with_cpu=True, with
                    "l2": "weights, P^T and Q of the layer exceed L2"},
         "phases_ms": {"encode": ph[0], "server_batched": ph[1], "decode_verify": ph[2]},
         "roofline": roof, "e2e": e2e, "cpu_baseline": cpu,
-        "gpu_launches": None, "clocks": clk}
+        "gpu_launches": int(round(launches_per_graph * args.steps)), "clocks": clk}
     for p in projs:
         p["ctx"].destroy()
     projs.clear()

@@ -338,6 +338,15 @@ int pvmvmd_code_encode_scratch(const pvmvmd_ctx *ctx, int which, int L, size_t *
 int pvmvmd_code_encode_lanes(const pvmvmd_ctx *ctx, int which, const uint32_t *X_dev, int L,
                              uint32_t *Y_dev, void *scratch_dev, void *stream);
 
+/* The number of kernels the library has enqueued in this process since it
+ * was loaded, on every device and stream: each launch counts once when it is
+ * enqueued, also while a stream is being captured.  Replaying a captured CUDA
+ * graph launches its kernels again without passing through the library, so a
+ * caller that replays a graph multiplies the count taken around the capture
+ * by the replays.  (Introspection for benchmarks and tests; the paper has no
+ * counterpart.) */
+unsigned long long pvmvmd_kernel_launches(void);
+
 /* Synchronise `stream`, then read and clear the library's device error word:
  * PVMVMD_E_DEVICE_TIMEOUT if any kernel gave up a bounded wait since the last
  * call, else PVMVMD_OK (or PVMVMD_E_CUDA if synchronisation failed). */

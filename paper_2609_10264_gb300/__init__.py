@@ -114,6 +114,7 @@ SIGNATURES = {
     "pvmvmd_code_encode_scratch": (_i, [_vp, _i, _i, ctypes.POINTER(_sz)]),
     "pvmvmd_code_encode_lanes": (_i, [_vp, _i, _vp, _i, _vp, _vp, _vp]),
     "pvmvmd_device_status": (_i, [_vp]),
+    "pvmvmd_kernel_launches": (ctypes.c_ulonglong, []),
     "pvmvmd_debug_expire_wait": (_i, [_i, ctypes.c_uint32, ctypes.c_uint64]),
     "pvmvmd_ctx_info": (_i, [_vp, ctypes.POINTER(pvmvmd_ctx_view)]),
     "pvmvmd_destroy": (None, [_vp]),
@@ -618,6 +619,12 @@ def pvmvmd_device_status(stream=None) -> int:
     s = _lib.pvmvmd_device_status(_stream_ptr(stream))
     _check(s, "pvmvmd_device_status")
     return s
+
+
+def pvmvmd_kernel_launches() -> int:
+    """Kernels the library has enqueued in this process so far (launches
+    captured into a CUDA graph count once, at capture)."""
+    return int(_lib.pvmvmd_kernel_launches())
 
 
 def pvmvmd_destroy(ctx: Ctx) -> None:

@@ -5,6 +5,7 @@
 #include <cmath>
 #include <cstdlib>
 #include <cstring>
+#include <atomic>
 #include <mutex>
 #include <new>
 #include <vector>
@@ -136,6 +137,11 @@ int check_device() {
     return (major == 10 && minor == 3) ? PVMVMD_OK : PVMVMD_E_NODEVICE;
 }
 
+std::atomic<unsigned long long> g_kernel_launches{0};
+unsigned long long kernel_launches() { return g_kernel_launches.load(std::memory_order_relaxed); }
+}  // namespace
+void note_launch() { g_kernel_launches.fetch_add(1, std::memory_order_relaxed); }
+namespace {
 uint32_t *error_word() {
     static std::mutex mu;
     static uint32_t *addr[64] = {nullptr};
@@ -854,6 +860,8 @@ int pvmvmd_debug_expire_wait(int site, uint32_t index, uint64_t limit) {
     g_debug.limit = site == PVMVMD_DEBUG_WAIT_OFF ? 0u : limit;
     return PVMVMD_OK;
 }
+
+unsigned long long pvmvmd_kernel_launches(void) { return pv::kernel_launches(); }
 
 int pvmvmd_device_status(void *stream) {
     if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) {

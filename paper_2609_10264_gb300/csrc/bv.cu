@@ -83,7 +83,7 @@ cudaError_t launch_transpose_u32(const uint32_t *in, int R, int C, uint32_t *out
     if (R <= 0 || C <= 0) return cudaSuccess;
     dim3 grid((C + 31) / 32, (R + 31) / 32), block(32, 8);
     if (grid.y > 65535u) return cudaErrorInvalidValue;
-    k_transpose_u32<<<grid, block, 0, s>>>(in, R, C, out);
+    k_transpose_u32<<<grid, block, 0, s>>>(in, R, C, out); note_launch();
     return cudaGetLastError();
 }
 
@@ -91,12 +91,12 @@ cudaError_t launch_bv_checks(const uint32_t *QauxT, int N, int Bn, int n, int B,
                              uint32_t t, uint32_t ell, const uint32_t *chal2, uint32_t t2, uint32_t ell2,
                              const uint32_t *u, const uint32_t *R, const uint32_t *X, const uint32_t *Z,
                              int32_t *accept, cudaStream_t s) {
-    k_set_i32<<<1, 1, 0, s>>>(accept, 1);
+    k_set_i32<<<1, 1, 0, s>>>(accept, 1); note_launch();
     const size_t blocks = (size_t)ell * ell2 + (size_t)B * ell;
     if (blocks == 0) return cudaGetLastError();
     if (blocks > 0x7fffffffu) return cudaErrorInvalidValue;
     k_bv_checks<<<(unsigned)blocks, kBvThreads, 0, s>>>(QauxT, N, Bn, n, B, chal, t, ell, chal2, t2, ell2, u,
-                                                        R, X, Z, accept);
+                                                        R, X, Z, accept); note_launch();
     return cudaGetLastError();
 }
 

@@ -345,7 +345,7 @@ cudaError_t launch_field_add(const uint32_t *a, const uint32_t *b, size_t n, uin
                        reinterpret_cast<uintptr_t>(out)) & 15u) == 0;
     const size_t blocks = (n + 1023) / 1024;
     if (blocks > 0x7fffffffu) return cudaErrorInvalidValue;
-    k_field_add<<<(unsigned)blocks, 256, 0, s>>>(a, b, n, out, vec);
+    k_field_add<<<(unsigned)blocks, 256, 0, s>>>(a, b, n, out, vec); note_launch();
     return cudaGetLastError();
 }
 
@@ -357,7 +357,7 @@ cudaError_t launch_output_mask(const uint32_t *PT, int m, const uint32_t *st, ui
         const int nb = B - b0 < 65535 ? B - b0 : 65535;
         dim3 grid((m + kDecThreads * 4 - 1) / (kDecThreads * 4), nb);
         k_output_mask<<<grid, kDecThreads, 2 * (size_t)t_x * sizeof(uint32_t), s>>>(
-            PT, m, st + (size_t)b0 * 2 * t_x, t_x, out + (size_t)b0 * m, vec);
+            PT, m, st + (size_t)b0 * 2 * t_x, t_x, out + (size_t)b0 * m, vec); note_launch();
     }
     return cudaGetLastError();
 }
@@ -375,7 +375,7 @@ cudaError_t launch_verify_u(const uint32_t *Qm, int K, const uint32_t *chal, uin
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, k_verify_u, Qm, K, chal, t_y, u);
+    return counted_launch(cudaLaunchKernelEx(&cfg, k_verify_u, Qm, K, chal, t_y, u));
 }
 
 cudaError_t launch_decrypt(const uint32_t *PT, int m, const uint32_t *st, uint32_t t_x, uint32_t Nx,
@@ -393,13 +393,14 @@ cudaError_t launch_decrypt(const uint32_t *PT, int m, const uint32_t *st, uint32
         k_decrypt<true><<<grid_mask, kDecThreads, 0, s>>>(PT, m, nullptr, t_x, Nx, Yhat, Y, mask, vec);
     else
         k_decrypt<false><<<grid, kDecThreads, smem, s>>>(PT, m, st, t_x, Nx, Yhat, Y, nullptr, vec);
+    note_launch();
     return cudaGetLastError();
 }
 
 cudaError_t launch_check(const uint32_t *Xhat, int K, const uint32_t *Yhat, int m, const uint32_t *g,
                          const uint32_t *u, uint32_t ell, int B, int32_t *accept, cudaStream_t s) {
     if (B <= 0) return cudaSuccess;
-    k_check<<<(unsigned)B, kCheckThreads, 0, s>>>(Xhat, K, Yhat, m, g, u, ell, accept);
+    k_check<<<(unsigned)B, kCheckThreads, 0, s>>>(Xhat, K, Yhat, m, g, u, ell, accept); note_launch();
     return cudaGetLastError();
 }
 

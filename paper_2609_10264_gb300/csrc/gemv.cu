@@ -385,7 +385,7 @@ cudaError_t run_gemv_multi(const MvmJob *jobs, int count, cudaStream_t s) {
     attrs[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attrs;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, k_gemv_multi<2, 4>, args);
+    return counted_launch(cudaLaunchKernelEx(&cfg, k_gemv_multi<2, 4>, args));
 }
 
 template <int ROWS, int UNROLL, bool kVec>
@@ -403,7 +403,7 @@ cudaError_t run_gemv(const int8_t *W, size_t ldw, int m, int K, const uint32_t *
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int ngroups = (m + ROWS - 1) / ROWS;
     const int grid = ngroups < sms ? ngroups : sms;
-    kern<<<grid, kGemvThreads, smem, s>>>(W, ldw, m, K, xhat, y, accumulate);
+    kern<<<grid, kGemvThreads, smem, s>>>(W, ldw, m, K, xhat, y, accumulate); note_launch();
     return cudaGetLastError();
 }
 

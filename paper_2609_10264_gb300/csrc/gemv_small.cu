@@ -266,7 +266,7 @@ cudaError_t run_gemv_nb(const NbJob *jobs, int count, cudaStream_t s) {
     attrs[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attrs;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, k_gemv_nb<2, 2>, args);
+    return counted_launch(cudaLaunchKernelEx(&cfg, k_gemv_nb<2, 2>, args));
 }
 
 }  // namespace
@@ -292,7 +292,7 @@ cudaError_t launch_gemv_small_batch(const int8_t *W, int m, int K, const uint32_
         attrs[0].val.programmaticStreamSerializationAllowed = 1;
         cfg.attrs = attrs;
         cfg.numAttrs = 1;
-        if ((e = cudaLaunchKernelEx(&cfg, k_nb_planes, Xhat, B, K, Bp, planes)) != cudaSuccess) return e;
+        if ((e = counted_launch(cudaLaunchKernelEx(&cfg, k_nb_planes, Xhat, B, K, Bp, planes))) != cudaSuccess) return e;
     }
     // groups of four vectors; K in segments whose planes fit shared memory,
     // later segments accumulating

@@ -80,6 +80,15 @@ cudaError_t launch_syndrome_gather(const uint32_t *pi1inv, uint32_t n, uint32_t 
                                    const uint32_t *F, uint32_t N, const uint32_t *addend,
                                    uint32_t *out, uint32_t count, cudaStream_t s);
 
+// Every kernel launch site calls note_launch() (or wraps a cudaLaunchKernelEx
+// in counted_launch), so that pvmvmd_kernel_launches counts what the library
+// enqueued.
+void note_launch();
+inline cudaError_t counted_launch(cudaError_t e) {
+    if (e == cudaSuccess) note_launch();
+    return e;
+}
+
 // One accumulate stage of the encoding G^T w over L lanes (App. B, encoding
 // direction): Y[j][l] = sum_{j' <= j} vscale[j'] * X[perm[j'] / div][l] for
 // j < N, with vscale_m = vscale R mod q (Montgomery form, R = 2^32).  X is

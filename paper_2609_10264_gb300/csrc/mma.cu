@@ -660,7 +660,7 @@ cudaError_t batched_launch(const int8_t *W, int m, int K, const uint32_t *Xhat, 
     const int nkb = (K + kBK - 1) / kBK;
     const int nvt = (B + kBV - 1) / kBV;
     const size_t threads = (size_t)nvt * kBV * nkb * 8;
-    k_digit_tiles<<<(unsigned)((threads + 255) / 256), 256, 0, s>>>(Xhat, B, K, nkb, nvt, D);
+    k_digit_tiles<<<(unsigned)((threads + 255) / 256), 256, 0, s>>>(Xhat, B, K, nkb, nvt, D); note_launch();
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const int mp = (m + 2 * kBM - 1) / (2 * kBM);  // CTA pairs along M
@@ -707,8 +707,8 @@ cudaError_t batched_launch(const int8_t *W, int m, int K, const uint32_t *Xhat, 
     const DebugWait dbg = debug_wait();
     const int skip_report = dbg.site == PVMVMD_DEBUG_WAIT_PRODUCT ? (int)dbg.index : -1;
     const uint64_t wait_ns = dbg.site == PVMVMD_DEBUG_WAIT_PRODUCT ? dbg.limit : kWaitNs;
-    return cudaLaunchKernelEx(&cfg, kern, tmap, W, m, K, (const uint8_t *)D, nkb, B, Yhat, err, skip_report,
-                              wait_ns);
+    return counted_launch(cudaLaunchKernelEx(&cfg, kern, tmap, W, m, K, (const uint8_t *)D, nkb, B, Yhat, err, skip_report,
+                              wait_ns));
 }
 
 // ---------------------------------------------------------------------------
@@ -1324,7 +1324,7 @@ cudaError_t launch_grouped_v(const BatchJob *jobs, int count, uint32_t *err, cud
         if (item0 == 0) continue;
         // digit tiles (and zeroed partial sums); enough CTAs for the largest job
         const int dblocks = std::max((max_threads + 255) / 256, any_split ? std::min(1024, (max_acc + 255) / 256) : 1);
-        k_digit_tiles_grouped<V><<<dim3((unsigned)dblocks, (unsigned)args.njobs), 256, 0, s>>>(args);
+        k_digit_tiles_grouped<V><<<dim3((unsigned)dblocks, (unsigned)args.njobs), 256, 0, s>>>(args); note_launch();
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
         const int C = std::min(best_c, item0);
@@ -1345,13 +1345,13 @@ cudaError_t launch_grouped_v(const BatchJob *jobs, int count, uint32_t *err, cud
         const DebugWait dbg = debug_wait();
         const int skip_report = dbg.site == PVMVMD_DEBUG_WAIT_PRODUCT ? (int)dbg.index : -1;
         const uint64_t wait_ns = dbg.site == PVMVMD_DEBUG_WAIT_PRODUCT ? dbg.limit : kWaitNs;
-        e = cudaLaunchKernelEx(&cfg, k_batched_grouped<V>, args, err, skip_report, wait_ns);
+        e = counted_launch(cudaLaunchKernelEx(&cfg, k_batched_grouped<V>, args, err, skip_report, wait_ns));
         if (e != cudaSuccess) return e;
         if (any_split) {
             int dev = 0, sms = 0;
             cudaGetDevice(&dev);
             cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-            k_split_finish<<<dim3((unsigned)(2 * sms), (unsigned)args.njobs), 256, 0, s>>>(args);
+            k_split_finish<<<dim3((unsigned)(2 * sms), (unsigned)args.njobs), 256, 0, s>>>(args); note_launch();
             e = cudaGetLastError();
             if (e != cudaSuccess) return e;
         }

@@ -1245,7 +1245,7 @@ cudaError_t launch_sample_sparse(const pvmvmd_key &key, uint32_t tag, uint64_t i
     const cudaError_t attr = func_attr((const void *)k_sample_sparse, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)kSampleMaxSmem);
     if (attr != cudaSuccess) return attr;
-    k_sample_sparse<<<count, 32, smem, s>>>(key, tag, idx0, N, t, out, clear, clear_words);
+    k_sample_sparse<<<count, 32, smem, s>>>(key, tag, idx0, N, t, out, clear, clear_words); note_launch();
     return cudaGetLastError();
 }
 
@@ -1260,7 +1260,7 @@ cudaError_t launch_syndrome_scan(const uint32_t *pi2inv, const uint32_t *v2p, co
     const bool inject = dbg.site == PVMVMD_DEBUG_WAIT_SCAN;
     k_syndrome_scan<<<grid, kScanThreads, smem, s>>>(pi2inv, v2p, v1, N, sparse, t, count, F, status,
                                                      err, inject ? dbg.index : 0xFFFFFFFFu,
-                                                     inject ? (uint32_t)dbg.limit : kSpinLimit);
+                                                     inject ? (uint32_t)dbg.limit : kSpinLimit); note_launch();
     return cudaGetLastError();
 }
 
@@ -1269,7 +1269,7 @@ cudaError_t launch_syndrome_gather(const uint32_t *pi1inv, uint32_t n, uint32_t 
                                    uint32_t *out, uint32_t count, cudaStream_t s) {
     if (count == 0 || n == 0) return cudaSuccess;
     dim3 grid((n + 255) / 256, count);
-    k_syndrome_gather<<<grid, 256, 0, s>>>(pi1inv, n, r, F, N, addend, out);
+    k_syndrome_gather<<<grid, 256, 0, s>>>(pi1inv, n, r, F, N, addend, out); note_launch();
     return cudaGetLastError();
 }
 
@@ -1297,6 +1297,7 @@ cudaError_t launch_encode_scan(const void *X, bool x_is_i8, size_t ldx, const ui
     else
         k_encode_scan<false><<<(unsigned)ctas, 256, 0, s>>>(X, ldx, perm, div, vscale_m, N, L, Y, ldy,
                                                             status, ticket, err);
+    note_launch();
     return cudaGetLastError();
 }
 
@@ -1304,7 +1305,7 @@ cudaError_t launch_transpose_i8(const int8_t *in, int R, int C, int8_t *out, cud
     if (R <= 0 || C <= 0) return cudaSuccess;
     dim3 grid((C + 31) / 32, (R + 31) / 32), block(32, 8);
     if (grid.y > 65535u) return cudaErrorInvalidValue;
-    k_transpose_i8<<<grid, block, 0, s>>>(in, R, C, out);
+    k_transpose_i8<<<grid, block, 0, s>>>(in, R, C, out); note_launch();
     return cudaGetLastError();
 }
 
@@ -1426,11 +1427,11 @@ cudaError_t launch_syndrome_fused(const pvmvmd_key &key, uint32_t tag, uint64_t 
         attr1[1].val.programmaticStreamSerializationAllowed = 1;
         cfg.attrs = attr1;
         cfg.numAttrs = pdl ? 2 : 1;
-        cudaError_t e = cudaLaunchKernelEx(&cfg, k_syndrome_fused, key, tag, idx0 + c0, N, t, slice,
+        cudaError_t e = counted_launch(cudaLaunchKernelEx(&cfg, k_syndrome_fused, key, tag, idx0 + c0, N, t, slice,
                                            pi2inv, v2p, v1, pi1inv, n, r,
                                            sparse_out + (size_t)c0 * 2 * t,
                                            addend ? addend + (size_t)c0 * n : nullptr,
-                                           out + (size_t)c0 * n, pi2, v2m, v1pm);
+                                           out + (size_t)c0 * n, pi2, v2m, v1pm));
         if (e != cudaSuccess) return e;
     }
     return cudaSuccess;
@@ -1448,7 +1449,7 @@ cudaError_t launch_pdl(const void *fn, dim3 grid, dim3 block, size_t smem, cudaS
     a[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = a;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelExC(&cfg, fn, args);
+    return counted_launch(cudaLaunchKernelExC(&cfg, fn, args));
 }
 }  // namespace
 

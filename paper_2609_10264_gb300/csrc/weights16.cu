@@ -40,21 +40,21 @@ static unsigned grid_of(size_t n) { return (unsigned)((n + 255) / 256); }
 cudaError_t launch_split_i16(const int16_t *W, size_t n, int8_t *hi, int8_t *lo, cudaStream_t s) {
     if (n == 0) return cudaSuccess;
     if ((n + 255) / 256 > 0x7fffffffu) return cudaErrorInvalidValue;
-    k_split_i16<<<grid_of(n), 256, 0, s>>>(W, n, hi, lo);
+    k_split_i16<<<grid_of(n), 256, 0, s>>>(W, n, hi, lo); note_launch();
     return cudaGetLastError();
 }
 
 cudaError_t launch_lift_i16(const int16_t *W, size_t n, uint32_t *out, cudaStream_t s) {
     if (n == 0) return cudaSuccess;
     if ((n + 255) / 256 > 0x7fffffffu) return cudaErrorInvalidValue;
-    k_lift_i16<<<grid_of(n), 256, 0, s>>>(W, n, out);
+    k_lift_i16<<<grid_of(n), 256, 0, s>>>(W, n, out); note_launch();
     return cudaGetLastError();
 }
 
 cudaError_t launch_combine_256(uint32_t *y, const uint32_t *ylo, size_t n, cudaStream_t s) {
     if (n == 0) return cudaSuccess;
     if ((n + 255) / 256 > 0x7fffffffu) return cudaErrorInvalidValue;
-    k_combine_256<<<grid_of(n), 256, 0, s>>>(y, ylo, n);
+    k_combine_256<<<grid_of(n), 256, 0, s>>>(y, ylo, n); note_launch();
     return cudaGetLastError();
 }
 

@@ -761,3 +761,41 @@ def test_decode_with_foreign_state_stays_in_bounds(pv, wl):
     assert not np.array_equal(Y_h[1], exp[1])
     assert pv.as_u32(acc).tolist() == [1, 1, 1]   # verification reads x_hat and y_hat only
     ctx.destroy()
+
+
+def test_kernel_launch_counter(pv, wl):
+    """pvmvmd_kernel_launches counts the kernels each call enqueues: one
+    grouped GEMV launch for a batch-1 product, four for a decode (challenge
+    syndrome, e^T Q, decrypt, check), and launches captured into a graph
+    once, at capture."""
+    import torch
+    W = wl.weights_uniform(64, 96, 3)
+    X = field(wl.int8_vectors(2, 96, 4))
+    Wd, Xd = to_dev(W), to_dev(X)
+    ctx = pv.pvmvmd_preprocess(Wd, key=5)
+    Xh, st = pv.pvmvmd_encode(ctx, Xd, key=6)
+    torch.cuda.synchronize()
+    n0 = pv.pvmvmd_kernel_launches()
+    Yh = pv.pvmvmd_server_mvm(Wd, Xh[0])
+    assert pv.pvmvmd_kernel_launches() - n0 == 1
+    Yb = torch.stack([Yh, pv.pvmvmd_server_mvm(Wd, Xh[1])])
+    n1 = pv.pvmvmd_kernel_launches()
+    Y, acc = pv.pvmvmd_decode_verify(ctx, st, Xh, Yb, challenge_key=7)
+    assert pv.pvmvmd_kernel_launches() - n1 == 4
+    assert pv.as_u32(acc).tolist() == [1, 1]
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        pv.pvmvmd_server_mvm(Wd, Xh[0], Yhat=Yh, stream=s)
+    s.synchronize()
+    n2 = pv.pvmvmd_kernel_launches()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        pv.pvmvmd_server_mvm(Wd, Xh[0], Yhat=Yh, stream=s)
+    n3 = pv.pvmvmd_kernel_launches()
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    assert n3 - n2 == 1 and pv.pvmvmd_kernel_launches() == n3
+    assert np.array_equal(pv.as_u32(Yh), oracle.server_mvm(W, pv.as_u32(Xh)[0]))
+    assert pv.pvmvmd_device_status() == 0
+    ctx.destroy()
