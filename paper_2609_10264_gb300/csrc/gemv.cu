@@ -200,7 +200,8 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
 // own matrix once.  The bytes of all matrices are split evenly over the CTAs
 // (whole rows); a CTA walks its share job by job, splitting that job's x_hat
 // into digit planes once, and its warps stream row pairs with the loads of
-// the next batch issued before the arithmetic of the current one.  A single
+// the next batch issued before the arithmetic of the current one (and, on
+// long streams, a bulk L2 prefetch of its next row group).  A single
 // launch over many matrices keeps every SM's loads in flight for the whole
 // stream instead of paying the ramp-up and drain of one launch per matrix.
 // Launched with programmatic dependent launch; it waits for the preceding
@@ -215,7 +216,8 @@ struct MultiArgs {
     MvmJob job[kMultiMaxJobs];
 };
 
-template <int ROWS, int UNROLL>
+// kPrefetch: warps ask L2 for their next group of rows (long streams only).
+template <int ROWS, int UNROLL, bool kPrefetch>
 __global__ void __launch_bounds__(kMultiThreads, 2) k_gemv_multi(const __grid_constant__ MultiArgs args) {
     extern __shared__ uint4 s_planes[];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -287,6 +289,15 @@ __global__ void __launch_bounds__(kMultiThreads, 2) k_gemv_multi(const __grid_co
                     *P3 = s_planes + 3 * nchunks;
 
         for (; g < ngroups; g += kMultiWarps) {
+            if (kPrefetch && lane < ROWS && g + kMultiWarps < ngroups) {
+                // the rows of this warp's next group, whole, into L2 while
+                // this group streams through the registers
+                const int row = row_a + (g + kMultiWarps) * ROWS + lane;
+                if (row < row_b)
+                    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(job.W + (size_t)row * job.ldw),
+                                 "r"((uint32_t)K)
+                                 : "memory");
+            }
             int acc[ROWS][4];
 #pragma unroll
             for (int r = 0; r < ROWS; ++r) acc[r][0] = acc[r][1] = acc[r][2] = acc[r][3] = 0;
@@ -367,14 +378,22 @@ cudaError_t run_gemv_multi(const MvmJob *jobs, int count, cudaStream_t s) {
     long long rows = 0;
     for (int j = 0; j < count; ++j) rows += jobs[j].m;
     if (rows == 0) return cudaSuccess;
-    const cudaError_t attr = func_attr((const void *)k_gemv_multi<2, 4>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, 4 * kMultiMaxK);
-    if (attr != cudaSuccess) return attr;
+    for (const void *f : {(const void *)k_gemv_multi<2, 4, false>, (const void *)k_gemv_multi<2, 4, true>}) {
+        const cudaError_t attr = func_attr(f, cudaFuncAttributeMaxDynamicSharedMemorySize, 4 * kMultiMaxK);
+        if (attr != cudaSuccess) return attr;
+    }
     int dev = 0, sms = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     long long grid = 2LL * sms;
     if (grid > rows) grid = rows;
+    // The L2 prefetch of each warp's next row group pays on long streams
+    // (100 requests of 4096 x 4096 per launch: GEMV 269.7 -> 261.2 us) and
+    // costs on short ones, whose launches are mostly ramp-up (one token
+    // through 32 8B-class layers, 128 launches of 4-117 MB: 1.59 -> 1.85 ms),
+    // so it is on only when a CTA streams at least 1 MiB of M.
+    const bool prefetch = args.base[count] / grid >= (1LL << 20);
+    const auto kern = prefetch ? k_gemv_multi<2, 4, true> : k_gemv_multi<2, 4, false>;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)grid, 1, 1);
     cfg.blockDim = dim3(kMultiThreads, 1, 1);
@@ -385,7 +404,7 @@ cudaError_t run_gemv_multi(const MvmJob *jobs, int count, cudaStream_t s) {
     attrs[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attrs;
     cfg.numAttrs = 1;
-    return counted_launch(cudaLaunchKernelEx(&cfg, k_gemv_multi<2, 4>, args));
+    return counted_launch(cudaLaunchKernelEx(&cfg, kern, args));
 }
 
 template <int ROWS, int UNROLL, bool kVec>
