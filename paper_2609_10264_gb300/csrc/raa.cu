@@ -1319,42 +1319,6 @@ size_t fused_smem(uint32_t slice, uint32_t t) {
 }
 constexpr size_t kFusedMaxSmem = 180 * 1024;
 
-// Largest cluster the fused kernel may use on this device: 16 CTAs where the
-// device schedules clusters of that (non-portable) size, else 8.
-int fused_max_cluster() {
-    static std::mutex mu;
-    static std::map<int, int> cache;
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) {
-        cudaGetLastError();
-        return 8;
-    }
-    std::lock_guard<std::mutex> lock(mu);
-    auto it = cache.find(dev);
-    if (it != cache.end()) return it->second;
-    int cmax = 8;
-    if (func_attr((const void *)k_syndrome_fused, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) ==
-            cudaSuccess &&
-        func_attr((const void *)k_syndrome_fused, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                  (int)kFusedMaxSmem) == cudaSuccess) {
-        cudaLaunchConfig_t cfg = {};
-        cfg.gridDim = dim3(16, 1, 1);
-        cfg.blockDim = dim3(kFusedThreads, 1, 1);
-        cfg.dynamicSmemBytes = kFusedMaxSmem / 2;
-        cudaLaunchAttribute a[1];
-        a[0].id = cudaLaunchAttributeClusterDimension;
-        a[0].val.clusterDim.x = 16;
-        a[0].val.clusterDim.y = 1;
-        a[0].val.clusterDim.z = 1;
-        cfg.attrs = a;
-        cfg.numAttrs = 1;
-        int n = 0;
-        if (cudaOccupancyMaxActiveClusters(&n, k_syndrome_fused, &cfg) == cudaSuccess && n > 0) cmax = 16;
-    }
-    cudaGetLastError();
-    cache[dev] = cmax;
-    return cmax;
-}
 }  // namespace
 
 // Cluster size and slice for the fused syndrome; false if N is too long for
@@ -1377,17 +1341,23 @@ bool syndrome_fused_plan(uint32_t N, uint32_t t, int *C_out, uint32_t *slice_out
 // The cluster size one launch of `count` vectors uses: the smallest that
 // holds the intermediate, and for a batch that leaves most SMs idle (at most
 // a quarter busy) doubled while count * C CTAs still fit the SMs and every
-// CTA keeps at least one position per thread.  A small batch (the ell
-// shared challenges, a few encodes) then spreads each vector's serial work
-// over up to 16 SMs instead of one; larger batches keep the cheaper
-// per-position work of the smallest cluster.
+// CTA keeps at least one position per thread, up to 8 CTAs.  A small batch
+// (the ell shared challenges, a few encodes) then spreads each vector's
+// serial work over up to 8 SMs instead of one; larger batches keep the
+// cheaper per-position work of the smallest cluster.  (Up to 16 CTAs, a
+// non-portable size, made one decode call alone slightly faster, 0.3228
+// against 0.3242 ms per batch-1 step, but a layer's decodes side by side
+// fit only seven 16-CTA clusters at once: 8B layer, 64 vectors, 0.528
+// against 0.506 ms per step; Qwen3-4B block, 8 vectors, 0.324 against
+// 0.266 ms.)
+constexpr int kFusedClusterMax = 8;
 static void syndrome_fused_launch_plan(uint32_t N, uint32_t t, uint32_t count, int *C, uint32_t *slice,
                                        size_t *smem) {
     int dev = 0, sms = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if ((uint64_t)count * (uint64_t)*C * 4 > (uint64_t)sms) return;
-    const int cmax = fused_max_cluster();
+    const int cmax = kFusedClusterMax;
     while (*C < cmax && (uint64_t)count * (uint64_t)(2 * *C) <= (uint64_t)sms &&
            (uint64_t)(2 * *C) * kFusedThreads <= (uint64_t)N) {
         *C *= 2;
