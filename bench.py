@@ -708,11 +708,13 @@ def run_ours(args):
     if world == 1 and not args.no_extra_configs:
         # the other configurations the metric is quoted on, as sub-records of
         # this line: the 70B-class batched pipeline (the tensor-core half of
-        # the metric) and one 8B-class token at batch 1
+        # the metric) and one 8B-class token at batch 1, the server's chain
+        # alone and with the client's encodes and decodes of every call
         line["configs"] = {
             "layer70b-b256": measure_batched(args, "layer70b-b256", device, rank, world,
                                              with_cpu=not args.no_cpu_baseline),
             "token8b-b1": measure_token(args, device, rank),
+            "token8b-b1-client": measure_token_client(args, device, rank),
         }
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -1333,6 +1335,132 @@ def measure_token(args, device, rank=0):
         "gpu_launches": 4 * nlayers * args.steps, "clocks": clk}
 
 
+def measure_token_client(args, device, rank=0):
+    """One token through 32 8B-class layers at batch 1 with the client's work
+    of every call in the chain: per layer, {q,k,v} -> o -> {gate,up} -> down,
+    each group as the encodes of its inputs, one grouped server call and the
+    decodes (verify + decrypt) of its outputs, the group's projections side by
+    side, so every server call waits for its encodes and the next group for
+    the decodes (224 encodes, 128 server calls and 224 decodes per token, one
+    CUDA graph).  The client needs P^T and Q per matrix (13.8 GB for one
+    layer), so the 32 layers share one layer's weights and contexts; part of
+    each layer's 218 MB of weights then stays in the 126 MB L2, which the
+    same chain without the client work (reported beside it) shows."""
+    import torch
+    import paper_2609_10264_gb300 as pv
+    from paper_2609_10264_gb300 import workloads as wl
+    Q = pv.PVMVMD_Q
+    nlayers = 32
+    projs = {}
+    for j, (name, (m, K)) in enumerate(wl.LAYER_8B.items()):
+        W = wl.weights_gaussian(m, K, (11, j))
+        x = wl.int8_vectors(1, K, (12, j))
+        Wd = torch.from_numpy(W).to(device)
+        Xd = torch.from_numpy(np.mod(x, Q).astype(np.uint32).view(np.int32)).to(device)
+        ctx = pv.pvmvmd_preprocess(Wd, key=300 + j)
+        projs[name] = dict(W=Wd, Wh=W, x=x, X=Xd, ctx=ctx, Xh=torch.empty_like(Xd),
+                           st=torch.empty((1, 2 * ctx.t_x), dtype=torch.int32, device=device),
+                           Yh=torch.empty((1, m), dtype=torch.int32, device=device),
+                           Y=torch.empty((1, m), dtype=torch.int32, device=device),
+                           acc=torch.empty(1, dtype=torch.int32, device=device))
+    torch.cuda.synchronize(device)
+    jobs = [pv.mvm_jobs([(projs[n]["W"], projs[n]["Xh"][0], projs[n]["Yh"][0]) for n in grp])
+            for grp in TOKEN_GROUPS]
+    stream = torch.cuda.Stream(device)
+    # a group's projections are independent: their encodes (and decodes) run
+    # side by side, one side stream each, joined before the next step
+    side = [torch.cuda.Stream(device) for _ in range(3)]
+
+    def side_by_side(grp, call):
+        if len(grp) == 1:
+            call(projs[grp[0]], stream)
+            return
+        fork = torch.cuda.Event()
+        fork.record(stream)
+        for i, n in enumerate(grp):
+            side[i].wait_event(fork)
+            with torch.cuda.stream(side[i]):
+                call(projs[n], side[i])
+            join = torch.cuda.Event()
+            join.record(side[i])
+            stream.wait_event(join)
+
+    def token(client=True):
+        for l in range(nlayers):
+            for g, grp in enumerate(TOKEN_GROUPS):
+                if client:
+                    side_by_side(grp, lambda p, on: pv.pvmvmd_encode(p["ctx"], p["X"], 4 * l + g + 1, Xhat=p["Xh"],
+                                                                     st=p["st"], stream=on))
+                pv.pvmvmd_server_mvm_multi(jobs[g], stream=stream)
+                if client:
+                    side_by_side(grp, lambda p, on: pv.pvmvmd_decode_verify(p["ctx"], p["st"], p["Xh"], p["Yh"],
+                                                                            1000 + 4 * l + g, Y=p["Y"],
+                                                                            accept=p["acc"], stream=on))
+
+    with torch.cuda.stream(stream):
+        token()
+    stream.synchronize()
+    assert pv.pvmvmd_device_status(stream) == 0
+    for n, p in projs.items():   # every decoded output equals W x over the integers
+        assert int(p["acc"].sum()) == 1, n
+        y = pv.as_u32(p["Y"])[0].astype(np.int64)
+        y = np.where(y > (Q - 1) // 2, y - Q, y)
+        assert np.array_equal(y, p["Wh"].astype(np.int64) @ p["x"][0].astype(np.int64)), n
+    graphs, launches = {}, {}
+    for key, client in (("client", True), ("server", False)):
+        n0 = pv.pvmvmd_kernel_launches()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            token(client)
+        launches[key] = pv.pvmvmd_kernel_launches() - n0
+        graphs[key] = g
+    steps = max(3, min(args.steps, 20))
+    ms = {}
+    clk = None
+    for key in ("client", "server"):
+        with torch.cuda.stream(stream):
+            for _ in range(args.warmup):
+                graphs[key].replay()
+        stream.synchronize()
+        clocks = ClockSampler(device.index) if key == "client" else None
+        if clocks:
+            clocks.start()
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        if clocks:
+            clocks.region_started()
+        with torch.cuda.stream(stream):
+            t0.record(stream)
+            for _ in range(steps):
+                graphs[key].replay()
+            t1.record(stream)
+        stream.synchronize()
+        if clocks:
+            clk = clocks.stop()
+        ms[key] = t0.elapsed_time(t1) / steps
+    assert pv.pvmvmd_device_status(stream) == 0 and all(int(p["acc"].sum()) == 1 for p in projs.values())
+    macs = nlayers * sum(m * K for (m, K) in wl.LAYER_8B.values())
+    for p in projs.values():
+        p["ctx"].destroy()
+    projs.clear()
+    del graphs
+    torch.cuda.synchronize(device)
+    torch.cuda.empty_cache()
+    return {
+        "metric": METRIC, "value": macs / (ms["client"] / 1e3), "unit": UNIT, "n_gpus": 1, "steps": steps,
+        "warmup": args.warmup, "ms_per_step": ms["client"], "ms_per_token": ms["client"], "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "u32 (F_q exact; int8 weights, dp4a digits)",
+        "data": "synthetic",
+        "config": {"workload": "token8b-b1-client", "layers": nlayers, "projections": list(wl.LAYER_8B),
+                   "schedule": "per layer {q,k,v} -> o -> {gate,up} -> down; each group: the encodes of its "
+                               "inputs side by side, one pvmvmd_server_mvm_multi call, the decodes of its outputs "
+                               "side by side; the groups in order (224 encodes, 128 server calls, 224 decodes per "
+                               "token)",
+                   "weights": "one 8B-class layer's weights and client contexts shared by the 32 layers"},
+        "server_only_ms_per_token": ms["server"],
+        "client_ms_per_token": ms["client"] - ms["server"],
+        "gpu_launches": launches["client"] * steps,
+        "launches_per_token": launches, "clocks": clk}
+
 def run_token(args):
     import torch
     rank, world, local = dist_env()
@@ -1794,7 +1922,7 @@ def main(argv=None):
     ap.add_argument("--server-mode", choices=["multi", "calls"], default="multi")
     ap.add_argument("--workload", choices=["batch1-4096", "server-shape", "server-layer", "decode-shape",
                                            "encode-shape", "encoder-shape",
-                                           "preprocess-shape", "token8b-b1", "bv-b8-1024"]
+                                           "preprocess-shape", "token8b-b1", "token8b-b1-client", "bv-b8-1024"]
                     + sorted(BATCHED),
                     default="batch1-4096")
     ap.add_argument("--shape", default="4096x4096x64",
@@ -1833,6 +1961,15 @@ def main(argv=None):
         return run_server_layer(args)
     if args.workload == "decode-shape":
         return run_decode_shape(args)
+    if args.workload == "token8b-b1-client":
+        import torch
+        rank, world, local = dist_env()
+        device = torch.device("cuda", local)
+        torch.cuda.set_device(device)
+        rec = measure_token_client(args, device, rank)
+        if rank == 0:
+            print(json.dumps(rec), flush=True)
+        return 0
     if args.workload == "token8b-b1":
         return run_token(args)
     if args.workload == "bv-b8-1024":
