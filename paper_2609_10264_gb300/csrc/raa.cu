@@ -772,7 +772,8 @@ __global__ void __launch_bounds__(256, 4) k_encode_scan(const void *__restrict__
                                                     unsigned long long *status, uint32_t *ticket_ctr,
                                                     uint32_t *__restrict__ err) {
     __shared__ uint32_t s_ticket;
-    __shared__ uint32_t s_src[kEncTile], s_vs[kEncTile];
+    __shared__ unsigned long long s_off[kEncTile];  // source row offset (row * ldx) of each position
+    __shared__ uint32_t s_vs[kEncTile];
     const int tid = threadIdx.x;
     const uint32_t nlb = (L + 255) / 256;
     const uint32_t ntiles = (N + kEncTile - 1) / kEncTile;
@@ -789,7 +790,7 @@ __global__ void __launch_bounds__(256, 4) k_encode_scan(const void *__restrict__
     const uint32_t j0 = tile * kEncTile;
     if (tid < kEncTile) {
         const uint32_t j = j0 + tid;
-        s_src[tid] = j < N ? __ldg(perm + j) / div : 0u;
+        s_off[tid] = (unsigned long long)(j < N ? __ldg(perm + j) / div : 0u) * ldx;
         s_vs[tid] = j < N ? __ldg(vscale_m + j) : 0u;  // 0 past N: adds nothing
     }
     __syncthreads();
@@ -798,7 +799,7 @@ __global__ void __launch_bounds__(256, 4) k_encode_scan(const void *__restrict__
 #pragma unroll
     for (int u = 0; u < kEncTile; ++u) {
         const bool ok = lane_ok && j0 + u < N;
-        const size_t src = (size_t)s_src[u] * ldx + l;
+        const size_t src = (size_t)s_off[u] + l;
         if (kI8)
             v[u] = ok ? flift_i8(static_cast<const int8_t *>(Xv)[src]) : 0u;
         else
@@ -837,11 +838,11 @@ __global__ void __launch_bounds__(256, 4) k_encode_scan(const void *__restrict__
         st_relaxed_u64(sw + (size_t)tile * 256, enc_status(2u, fadd(run, prefix)));
     }
     if (lane_ok) {
+        uint32_t *yp = Y + (size_t)j0 * ldy + l;
+        const uint32_t nu = N - j0 < (uint32_t)kEncTile ? N - j0 : (uint32_t)kEncTile;
 #pragma unroll
-        for (int u = 0; u < kEncTile; ++u) {
-            const uint32_t j = j0 + u;
-            if (j < N) Y[j * ldy + l] = fadd(v[u], prefix);
-        }
+        for (int u = 0; u < kEncTile; ++u, yp += ldy)
+            if ((uint32_t)u < nu) *yp = fadd(v[u], prefix);
     }
 }
 
