@@ -24,6 +24,7 @@ namespace {
 // and the challenges each read their own keystream.
 constexpr uint32_t kTagCodeX = 1;       // G_x: pi1 = 1, pi2 = 2, v1 = 3, v2 = 4
 constexpr uint32_t kTagCodeY = 5;       // G_y: pi1 = 5, pi2 = 6, v1 = 7, v2 = 8
+static_assert(kTagCodeY == kTagCodeX + 4, "code `which` reads tags kTagCodeX + 4 which + 0..3");
 constexpr uint32_t kTagMask = 9;
 constexpr uint32_t kTagChallenge = 10;
 constexpr uint32_t kTagBvPrimary = 21;    // batch verification challenges
