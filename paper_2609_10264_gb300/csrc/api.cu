@@ -616,7 +616,7 @@ int encode_batch(pvmvmd_ctx *ctx, const uint32_t *X_dev, int B, const pvmvmd_key
         // sample, scan and gather in one launch per batch, no scratch
         PV_CUDA(launch_syndrome_fused(*key, kTagMask, 0, ctx->Nx, ctx->t_x, (uint32_t)B, d.pi2inv,
                                       d.v2p, d.v1, d.pi1inv, d.pi2, d.v2m, d.v1pm, ctx->K, ctx->rate,
-                                      stp, X_dev, Xhat_dev, s, /*pdl=*/true));
+                                      stp, X_dev, Xhat_dev, s, /*pdl=*/true, kSpreadEncode));
         return PVMVMD_OK;
     }
     for (int b0 = 0; b0 < B; b0 += ctx->sb) {
@@ -736,7 +736,8 @@ int verify_chain(pvmvmd_ctx *ctx, const pvmvmd_key *challenge_key, const uint32_
     if (syndrome_fused_plan(ctx->Ny, ctx->t_y, &C, &slice, &smem)) {
         PV_CUDA(launch_syndrome_fused(*challenge_key, kTagChallenge, 0, ctx->Ny, ctx->t_y,
                                       (uint32_t)ctx->ell, d.pi2inv, d.v2p, d.v1, d.pi1inv, d.pi2,
-                                      d.v2m, d.v1pm, ctx->m, ctx->rate, ctx->chal, nullptr, ctx->g, cs));
+                                      d.v2m, d.v1pm, ctx->m, ctx->rate, ctx->chal, nullptr, ctx->g, cs, false,
+                                      B >= kChallengeLargeBatch ? kSpreadChallenge : kSpreadChallengeSmallBatch));
     } else {
         PV_CUDA(launch_sample_sparse(*challenge_key, kTagChallenge, 0, ctx->Ny, ctx->t_y, ctx->ell,
                                      ctx->chal, ctx->status_y, scan_status_words(ctx->Ny, ctx->ell), cs));

@@ -39,6 +39,16 @@ cudaError_t launch_syndrome_scan(const uint32_t *pi2inv, const uint32_t *v2p, co
                                  uint32_t *F, unsigned long long *status, uint32_t *err,
                                  cudaStream_t s);
 
+// Cluster spread of the fused syndrome (how far a small batch's clusters
+// grow): encodes of a few vectors, and the few shared challenges of a
+// verification, each measured best at a different setting.  The challenges
+// of a large batch run beside a large decrypt and keep their clusters
+// small; those of a small batch are the decode's critical path.
+constexpr int kSpreadEncode = 4;
+constexpr int kSpreadChallenge = 16;
+constexpr int kSpreadChallengeSmallBatch = 4;
+constexpr int kChallengeLargeBatch = 32;
+
 // Fused syndrome for `count` freshly sampled sparse vectors (as
 // launch_sample_sparse, then out = addend + G e) in one launch with the
 // intermediate in cluster shared memory.  sparse_out: [count][2t];
@@ -57,7 +67,7 @@ cudaError_t launch_syndrome_fused(const pvmvmd_key &key, uint32_t tag, uint64_t 
                                   const uint32_t *pi2, const uint32_t *v2m, const uint32_t *v1pm,
                                   uint32_t n, uint32_t r, uint32_t *sparse_out,
                                   const uint32_t *addend, uint32_t *out, cudaStream_t s,
-                                  bool pdl = false);
+                                  bool pdl = false, int spread = kSpreadChallenge);
 
 // Lane-parallel syndrome for L vectors (vector b uses index idx0 + b, as
 // launch_sample_sparse): sparse_out [L][2t] as there, S lane_state_words(t,

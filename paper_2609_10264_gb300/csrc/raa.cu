@@ -1341,11 +1341,19 @@ bool syndrome_fused_plan(uint32_t N, uint32_t t, int *C_out, uint32_t *slice_out
 
 // The cluster size one launch of `count` vectors uses: the smallest that
 // holds the intermediate, and for a batch that leaves most SMs idle (at most
-// a quarter busy) doubled while count * C CTAs still fit the SMs and every
-// CTA keeps at least one position per thread, up to 8 CTAs.  A small batch
-// (the ell shared challenges, a few encodes) then spreads each vector's
-// serial work over up to 8 SMs instead of one; larger batches keep the
-// cheaper per-position work of the smallest cluster.  (Up to 16 CTAs, a
+// a quarter busy) doubled while count * C * spread CTAs still fit the SMs
+// and every CTA keeps at least one position per thread, up to 8 CTAs.  A
+// small batch then spreads each vector's serial work over a few SMs instead
+// of one; larger batches keep the cheaper per-position work of the smallest
+// cluster.  The callers' spread (launch_syndrome_fused) was measured: 4 for
+// encodes (8 vectors per call: Qwen3-4B block 0.265 -> 0.227 ms per step
+// against spread 1; 2 gave 0.275, 8 gave 0.255); for the ell = 2 shared
+// challenges 16 when the batch is large (a cluster of at most 2 CTAs at
+// N_y = 32768, taking few SMs from the decrypt beside it: batch-1 workload of
+// 100 vectors 0.3256 -> 0.3220 ms per step against spread 4), else 4 (the
+// challenges are then the decode's critical path: Qwen3-4B block, 8
+// vectors, 0.227 against 0.235 ms; one token with its 448 single-vector
+// encodes and decodes, client part 9.7 against 10.2 ms).  (Up to 16 CTAs, a
 // non-portable size, made one decode call alone slightly faster, 0.3228
 // against 0.3242 ms per batch-1 step, but a layer's decodes side by side
 // fit only seven 16-CTA clusters at once: 8B layer, 64 vectors, 0.528
@@ -1353,13 +1361,13 @@ bool syndrome_fused_plan(uint32_t N, uint32_t t, int *C_out, uint32_t *slice_out
 // 0.266 ms.)
 constexpr int kFusedClusterMax = 8;
 static void syndrome_fused_launch_plan(uint32_t N, uint32_t t, uint32_t count, int *C, uint32_t *slice,
-                                       size_t *smem) {
+                                       size_t *smem, int spread) {
     int dev = 0, sms = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if ((uint64_t)count * (uint64_t)*C * 4 > (uint64_t)sms) return;
     const int cmax = kFusedClusterMax;
-    while (*C < cmax && (uint64_t)count * (uint64_t)(2 * *C) <= (uint64_t)sms &&
+    while (*C < cmax && (uint64_t)count * (uint64_t)(2 * *C) * (uint64_t)spread <= (uint64_t)sms &&
            (uint64_t)(2 * *C) * kFusedThreads <= (uint64_t)N) {
         *C *= 2;
         *slice = fused_slice(N, *C);
@@ -1372,7 +1380,8 @@ cudaError_t launch_syndrome_fused(const pvmvmd_key &key, uint32_t tag, uint64_t 
                                   const uint32_t *v2p, const uint32_t *v1, const uint32_t *pi1inv,
                                   const uint32_t *pi2, const uint32_t *v2m, const uint32_t *v1pm,
                                   uint32_t n, uint32_t r, uint32_t *sparse_out,
-                                  const uint32_t *addend, uint32_t *out, cudaStream_t s, bool pdl) {
+                                  const uint32_t *addend, uint32_t *out, cudaStream_t s, bool pdl,
+                                  int spread) {
     if (count == 0) return cudaSuccess;
     int C = 0;
     uint32_t slice = 0;
@@ -1381,7 +1390,7 @@ cudaError_t launch_syndrome_fused(const pvmvmd_key &key, uint32_t tag, uint64_t 
     const cudaError_t attr = func_attr((const void *)k_syndrome_fused, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)kFusedMaxSmem);
     if (attr != cudaSuccess) return attr;
-    syndrome_fused_launch_plan(N, t, count < 65535 ? count : 65535, &C, &slice, &smem);
+    syndrome_fused_launch_plan(N, t, count < 65535 ? count : 65535, &C, &slice, &smem, spread < 1 ? 1 : spread);
     for (uint32_t c0 = 0; c0 < count; c0 += 65535) {
         const uint32_t nb = count - c0 < 65535 ? count - c0 : 65535;
         cudaLaunchConfig_t cfg = {};
