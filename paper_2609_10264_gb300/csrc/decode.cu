@@ -13,6 +13,10 @@
 //                       R_q = e_q^T (G_y^T y_hat_b) by transposition.
 //  * k_output_mask      the output masks P e_x,b alone (boost mode's
 //                       offline step).
+#include <cmath>
+#include <map>
+#include <mutex>
+
 #include "common.cuh"
 #include "launch.h"
 
@@ -148,26 +152,23 @@ __device__ __forceinline__ void pe_cols(const uint32_t *__restrict__ PT, int m, 
 // (128 column threads x 4 columns, so each row of P^T is read in 2 KiB
 // segments) and splits the t_x rows over kDecGroups = 2 row groups, so each
 // thread streams about t_x / 2 row segments (rounds of 8 loads in flight)
-// and the grid holds many short CTAs whatever m and B are.  The groups'
-// partial sums meet in shared memory.  (256 columns and 4 groups, or 1024
-// columns and 1 group, were 6 and 13 % slower at m = K = 8192, B = 256.
-// At m = K = 4096, B = 100, where 800 CTAs are 1.3 waves of the 608
-// resident ones, 256 columns left the decode call at 54.6 us: its check
-// waits for the challenge kernels that run beside the decrypt.)
+// and the grid holds many short CTAs whatever m and B are; or 256 columns
+// over 4 row groups when that fills the last wave of resident CTAs better.
+// The groups' partial sums meet in shared memory.  (256 columns everywhere,
+// or 1024 columns and 1 group, were 6 and 13 % slower at m = K = 8192,
+// B = 256.)
 // In boost mode (Sec. 7.2) P e_x,b was prepared ahead: Y_b = y_hat_b - mask_b.
 // The grid runs vectors fastest (blockIdx.x = b, blockIdx.y = column block),
 // so the CTAs in flight share a few column blocks and a row of P^T drawn by
 // several vectors' supports is read from HBM once and then from L2.
 // ---------------------------------------------------------------------------
-constexpr int kDecGroups = 2;
-constexpr int kDecColThreads = kDecThreads / kDecGroups;  // 128
-constexpr int kDecCols = 4 * kDecColThreads;              // 512 columns per CTA
-
-template <bool kBoost>
+template <bool kBoost, int kDecGroups>
 __global__ void __launch_bounds__(kDecThreads) k_decrypt(const uint32_t *__restrict__ PT, int m,
                                                         const uint32_t *__restrict__ st, uint32_t t_x,
                                                         uint32_t Nx, const uint32_t *Yhat, uint32_t *Y,
                                                         const uint32_t *__restrict__ mask, bool vec) {
+    constexpr int kDecColThreads = kDecThreads / kDecGroups;
+    constexpr int kDecCols = 4 * kDecColThreads;
     extern __shared__ uint32_t sm[];  // support[t_x], values[t_x]
     __shared__ uint4 s_part[kDecGroups > 1 ? kDecGroups - 1 : 1][kDecColThreads];
     const int tid = threadIdx.x;
@@ -378,6 +379,28 @@ cudaError_t launch_verify_u(const uint32_t *Qm, int K, const uint32_t *chal, uin
     return counted_launch(cudaLaunchKernelEx(&cfg, k_verify_u, Qm, K, chal, t_y, u));
 }
 
+// Resident k_decrypt CTAs on the current device (cached per device).
+int decrypt_slots() {
+    static std::mutex mu;
+    static std::map<int, int> cache;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        (void)cudaGetLastError();
+        return 0;
+    }
+    std::lock_guard<std::mutex> lock(mu);
+    auto it = cache.find(dev);
+    if (it != cache.end()) return it->second;
+    int per_sm = 0, sms = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_decrypt<false, 2>, kDecThreads, 1024) !=
+            cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+        (void)cudaGetLastError();
+        per_sm = 0;
+    }
+    return cache[dev] = per_sm * sms;
+}
+
 cudaError_t launch_decrypt(const uint32_t *PT, int m, const uint32_t *st, uint32_t t_x, uint32_t Nx,
                            const uint32_t *Yhat, int B, uint32_t *Y, cudaStream_t s, const uint32_t *mask) {
     if (B <= 0 || m <= 0) return cudaSuccess;
@@ -386,13 +409,32 @@ cudaError_t launch_decrypt(const uint32_t *PT, int m, const uint32_t *st, uint32
                        reinterpret_cast<uintptr_t>(Y)) & 15u) == 0;
     const size_t smem = mask ? 0 : 2 * (size_t)t_x * sizeof(uint32_t);
     if (smem > 48 * 1024) return cudaErrorInvalidValue;
-    if ((m + kDecCols - 1) / kDecCols > 65535) return cudaErrorInvalidValue;
-    const dim3 grid((unsigned)B, (m + kDecCols - 1) / kDecCols);
     const dim3 grid_mask((unsigned)B, (m + 4 * kDecThreads - 1) / (4 * kDecThreads));
-    if (mask)
-        k_decrypt<true><<<grid_mask, kDecThreads, 0, s>>>(PT, m, nullptr, t_x, Nx, Yhat, Y, mask, vec);
+    if (mask) {
+        k_decrypt<true, 2><<<grid_mask, kDecThreads, 0, s>>>(PT, m, nullptr, t_x, Nx, Yhat, Y, mask, vec);
+        note_launch();
+        return cudaGetLastError();
+    }
+    // Every CTA streams the same t_x row segments, so a last wave that is a
+    // third full costs as much as a full one: 256-column CTAs are used when
+    // they fill the last wave of resident CTAs clearly better than 512
+    // (4096 x 4096, 100 vectors: 800 CTAs are 1.32 waves of 608, 1600 are
+    // 2.63; decrypt 47 -> 41 us, step 0.3221 -> 0.3202 ms).  Where both
+    // fill alike the wider CTAs stay (70B-class shapes, 256 vectors: 256
+    // columns everywhere took 2.221 -> 2.272 ms per step).
+    const int slots = decrypt_slots();
+    auto fill = [&](int cols) {
+        const double waves = (double)B * (double)((m + cols - 1) / cols) / slots;
+        return waves / std::ceil(waves);
+    };
+    const bool narrow = slots > 0 && fill(256) > fill(512) + 0.1;
+    const int cols = narrow ? 256 : 512;
+    if ((m + cols - 1) / cols > 65535) return cudaErrorInvalidValue;
+    const dim3 grid((unsigned)B, (m + cols - 1) / cols);
+    if (narrow)
+        k_decrypt<false, 4><<<grid, kDecThreads, smem, s>>>(PT, m, st, t_x, Nx, Yhat, Y, nullptr, vec);
     else
-        k_decrypt<false><<<grid, kDecThreads, smem, s>>>(PT, m, st, t_x, Nx, Yhat, Y, nullptr, vec);
+        k_decrypt<false, 2><<<grid, kDecThreads, smem, s>>>(PT, m, st, t_x, Nx, Yhat, Y, nullptr, vec);
     note_launch();
     return cudaGetLastError();
 }
