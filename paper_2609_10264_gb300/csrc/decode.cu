@@ -229,8 +229,13 @@ __global__ void __launch_bounds__(kDecThreads) k_decrypt(const uint32_t *__restr
 // e_q^T Q and g_q = G_y e_q from the challenge kernels.  One CTA per vector;
 // the repetitions run one after the other over the (cached) vectors.
 // ---------------------------------------------------------------------------
-constexpr int kCheckThreads = 1024;
-constexpr int kCheckBatch = 4;  // loads in flight per operand and thread
+// 512 threads with eight loads of each operand in flight (1024 threads with
+// four, an SM's whole register file per CTA, waited longer for SMs beside
+// the decrypts: 8B layer 0.500 -> 0.492 ms, 70B layer 2.218 -> 2.191 ms per
+// step, the batch-1 workload unchanged at 0.320 ms; 256 threads were
+// slower)
+constexpr int kCheckThreads = 512;
+constexpr int kCheckBatch = 8;  // loads in flight per operand and thread
 
 __global__ void __launch_bounds__(kCheckThreads) k_check(const uint32_t *__restrict__ Xhat, int K,
                                                         const uint32_t *__restrict__ Yhat, int m,
@@ -267,18 +272,22 @@ __global__ void __launch_bounds__(kCheckThreads) k_check(const uint32_t *__restr
                 c1[v] = ky ? __ldg(g1 + k) : 0u;
             }
             // four products of values below q stay below 2^64 with the
-            // reduced running sum
+            // reduced running sum, so the sums are reduced every four
 #pragma unroll
-            for (int v = 0; v < kCheckBatch; ++v) {
-                l0 += (uint64_t)a0[v] * x[v];
-                l1 += (uint64_t)a1[v] * x[v];
-                r0 += (uint64_t)c0[v] * y[v];
-                r1 += (uint64_t)c1[v] * y[v];
+            for (int v0 = 0; v0 < kCheckBatch; v0 += 4) {
+#pragma unroll
+                for (int v = v0; v < v0 + 4; ++v) {
+                    l0 += (uint64_t)a0[v] * x[v];
+                    l1 += (uint64_t)a1[v] * x[v];
+                    r0 += (uint64_t)c0[v] * y[v];
+                    r1 += (uint64_t)c1[v] * y[v];
+                }
+                l0 = fred(l0);
+                l1 = fred(l1);
+                r0 = fred(r0);
+                r1 = fred(r1);
             }
-            l0 = fred(l0);
-            l1 = fred(l1);
-            r0 = fred(r0);
-            r1 = fred(r1);
+            static_assert(kCheckBatch % 4 == 0, "sums reduced every four products");
         }
         const uint32_t w0 = warp_fsum((uint32_t)l0), w1 = warp_fsum((uint32_t)l1);
         const uint32_t w2 = warp_fsum((uint32_t)r0), w3 = warp_fsum((uint32_t)r1);
