@@ -712,10 +712,12 @@ def run_ours(args):
     torch.cuda.empty_cache()
     if world == 1 and not args.no_extra_configs:
         # the other configurations the metric is quoted on, as sub-records of
-        # this line: the 70B-class batched pipeline (the tensor-core half of
-        # the metric) and one 8B-class token at batch 1, the server's chain
-        # alone and with the client's encodes and decodes of every call
+        # this line: the 8B- and 70B-class batched pipelines (the tensor-core
+        # half of the metric) and one 8B-class token at batch 1, the server's
+        # chain alone and with the client's encodes and decodes of every call
         line["configs"] = {
+            "layer8b-b64": measure_batched(args, "layer8b-b64", device, rank, world,
+                                           with_cpu=not args.no_cpu_baseline),
             "layer70b-b256": measure_batched(args, "layer70b-b256", device, rank, world,
                                              with_cpu=not args.no_cpu_baseline),
             "token8b-b1": measure_token(args, device, rank),
@@ -1040,14 +1042,24 @@ def measure_batched(args, workload, device, rank=0, world=1, with_cpu=True, with
     flops = 2 * 4 * macs
     peaks, kind = measured_peaks()
 
-    # the dominant projection's product alone, by CUDA events on its stream
+    # the dominant kernel as the step launches it, alone, by CUDA events on
+    # its stream: the layer's products in one grouped call (one launch of
+    # k_batched_grouped), or the largest projection's product when the
+    # products are separate calls
     big = max(projs, key=lambda p: p["m"] * p["K"])
+    grouped_call = args.server_call == "grouped"
+
+    def one_product():
+        if grouped_call:
+            pv.pvmvmd_server_mvm_grouped(grouped_jobs, stream=stream)
+        else:
+            pv.pvmvmd_server_mvm(big["W"], big["Xh"], Yhat=big["Yh"], stream=stream)
     with torch.cuda.stream(stream):   # sizes this stream's scratch before the capture
-        pv.pvmvmd_server_mvm(big["W"], big["Xh"], Yhat=big["Yh"], stream=stream)
+        one_product()
     stream.synchronize()
     g_big = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g_big, stream=stream):
-        pv.pvmvmd_server_mvm(big["W"], big["Xh"], Yhat=big["Yh"], stream=stream)
+        one_product()
     k0, k1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     reps = max(args.steps, 5)
     with torch.cuda.stream(stream):
@@ -1078,11 +1090,14 @@ def measure_batched(args, workload, device, rank=0, world=1, with_cpu=True, with
         dtype = "u32 (F_q exact; int8 weights, dp4a digits)"
     else:
         peak = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"])
-        big_flops = 2 * 4 * big["m"] * big["K"] * B
+        big_flops = 2 * 4 * (macs if grouped_call else big["m"] * big["K"] * B)
         roof = {"bound": "tensor",
-                "kernel": f"k_batched_grouped (tcgen05 kind::f16 digit GEMM) on {big['name']} "
-                          f"{big['m']}x{big['K']}x{B}, one pvmvmd_server_mvm call (k_digit_tiles_grouped + "
-                          "k_batched_grouped, + k_split_finish when K is split) timed alone by CUDA events",
+                "kernel": ("k_batched_grouped (tcgen05 kind::f16 digit GEMM) over the layer's products, one "
+                           "pvmvmd_server_mvm_grouped call as the step makes it" if grouped_call else
+                           f"k_batched_grouped (tcgen05 kind::f16 digit GEMM) on {big['name']} "
+                           f"{big['m']}x{big['K']}x{B}, one pvmvmd_server_mvm call") +
+                          " (k_digit_tiles_grouped + k_batched_grouped, + k_split_finish when K is split), "
+                          "timed alone by CUDA events",
                 "achieved": big_flops / (big_ms / 1e3) / 1e12, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
                 "peak_kind": f"{kind} bf16_tflops (burst; the kernel timed alone)", "traffic": None,
                 "flops_per_launch": big_flops, "launch_ms": big_ms,
