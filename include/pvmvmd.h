@@ -111,7 +111,9 @@ int pvmvmd_params_resolve(const pvmvmd_params *in, int m, int K, pvmvmd_params *
  * not stay alive afterwards.  params may be NULL (all defaults).
  * 1 <= m, 1 <= K <= PVMVMD_MAX_K.  Allocates about 8*rate*m*K bytes of device
  * memory plus code tables and scratch; the call synchronises `stream` before
- * returning.  On error *out is NULL. */
+ * returning.  The context also owns one CUDA stream, created at the device's
+ * highest stream priority, on which pvmvmd_decode_verify runs its short
+ * verification kernels beside the decrypt.  On error *out is NULL. */
 int pvmvmd_preprocess(const int8_t *W_dev, int m, int K, const pvmvmd_params *params,
                       const pvmvmd_key *key, void *stream, pvmvmd_ctx **out);
 
