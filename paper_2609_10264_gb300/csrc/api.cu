@@ -725,8 +725,11 @@ namespace {
 // The verification of a call: challenges e_q <- E_{t_y}^{N_y} shared by the
 // B vectors, g_q = G_y e_q, u_q = e_q^T Q, and accept_b from x_hat_b and
 // y_hat_b, all on stream cs.
+// beside_decrypt: a decrypt of t_x rows per vector runs beside the chain
+// (standard mode), so a large batch keeps its challenge clusters small; in
+// boost mode the chain is the whole decode and gets the wider clusters.
 int verify_chain(pvmvmd_ctx *ctx, const pvmvmd_key *challenge_key, const uint32_t *Xhat_dev,
-                 const uint32_t *Yhat_dev, int B, int32_t *accept_dev, cudaStream_t cs) {
+                 const uint32_t *Yhat_dev, int B, int32_t *accept_dev, cudaStream_t cs, bool beside_decrypt) {
     uint32_t *err = error_word();
     if (!err) return PVMVMD_E_CUDA;
     const CodeDev &d = ctx->gy;
@@ -737,7 +740,8 @@ int verify_chain(pvmvmd_ctx *ctx, const pvmvmd_key *challenge_key, const uint32_
         PV_CUDA(launch_syndrome_fused(*challenge_key, kTagChallenge, 0, ctx->Ny, ctx->t_y,
                                       (uint32_t)ctx->ell, d.pi2inv, d.v2p, d.v1, d.pi1inv, d.pi2,
                                       d.v2m, d.v1pm, ctx->m, ctx->rate, ctx->chal, nullptr, ctx->g, cs, false,
-                                      B >= kChallengeLargeBatch ? kSpreadChallenge : kSpreadChallengeSmallBatch));
+                                      beside_decrypt && B >= kChallengeLargeBatch ? kSpreadChallenge
+                                                                                 : kSpreadChallengeSmallBatch));
     } else {
         PV_CUDA(launch_sample_sparse(*challenge_key, kTagChallenge, 0, ctx->Ny, ctx->t_y, ctx->ell,
                                      ctx->chal, ctx->status_y, scan_status_words(ctx->Ny, ctx->ell), cs));
@@ -773,7 +777,7 @@ int decode_verify_batch(pvmvmd_ctx *ctx, const void *st_dev, const uint32_t *mas
         PV_CUDA(cudaEventRecord(ctx->fork, s));
         PV_CUDA(cudaStreamWaitEvent(ctx->side, ctx->fork, 0));
     }
-    int st = verify_chain(ctx, challenge_key, Xhat_dev, Yhat_dev, B, accept_dev, cs);
+    int st = verify_chain(ctx, challenge_key, Xhat_dev, Yhat_dev, B, accept_dev, cs, mask_out_dev == nullptr);
     if (st) return st;
     PV_CUDA(launch_decrypt(ctx->PT, ctx->m, static_cast<const uint32_t *>(st_dev), ctx->t_x, (uint32_t)ctx->Nx,
                            Yhat_dev, B, Y_dev, s, mask_out_dev));

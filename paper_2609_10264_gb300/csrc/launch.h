@@ -43,7 +43,8 @@ cudaError_t launch_syndrome_scan(const uint32_t *pi2inv, const uint32_t *v2p, co
 // grow): encodes of a few vectors, and the few shared challenges of a
 // verification, each measured best at a different setting.  The challenges
 // of a large batch run beside a large decrypt and keep their clusters
-// small; those of a small batch are the decode's critical path.
+// small; those of a small batch, and those of boost mode (no decrypt of
+// P^T rows beside them), are the decode's critical path.
 constexpr int kSpreadEncode = 4;
 constexpr int kSpreadChallenge = 16;
 constexpr int kSpreadChallengeSmallBatch = 4;
